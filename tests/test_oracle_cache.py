@@ -1,0 +1,125 @@
+"""Pins of the expert-cache oracle (Section 4.1 "Simulation", Eq. metrics).
+
+Hand-traced sequences (tests/golden/lru_traces.txt), the paper's Table 2 values through the metric
+identity, invariants the rule implies, and agreement of the two independent formulations.
+"""
+import os
+
+import numpy as np
+import pytest
+
+from oracle import cache as C
+from paper_2609_34077_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load_traces():
+    traces, cur = [], None
+    for line in open(os.path.join(GOLDEN, "lru_traces.txt")):
+        line = line.strip()
+        if not line or line.startswith("#"):
+            continue
+        if line.startswith("trace"):
+            _, name, _, E, _, B = line.split()
+            cur = dict(name=name, E=int(E), B=int(B), steps=[])
+            traces.append(cur)
+        elif line.startswith("step"):
+            ids, hits, misses = [p.strip() for p in line[4:].split("|")]
+            ml = [tuple(int(v) for v in m.split(":")) for m in misses.split()[1:]]
+            cur["steps"].append(([int(v) for v in ids.split(",")], int(hits.split()[1]), ml))
+        elif line.startswith("total"):
+            f = line.split()
+            cur["total"] = dict(hits=int(f[2]), fetches=int(f[4]), bypass=int(f[6]))
+    return traces
+
+
+TRACES = _load_traces()
+
+
+@pytest.mark.parametrize("cls", [C.LRUStamps, C.LRUList])
+@pytest.mark.parametrize("tr", TRACES, ids=[t["name"] for t in TRACES])
+def test_hand_traces(cls, tr):
+    c = cls(tr["E"], tr["B"])
+    th = tf = tb = 0
+    for ids, hits, misses in tr["steps"]:
+        h, f, b, ml = c.step(ids)
+        assert h == hits
+        assert ml == misses
+        th, tf, tb = th + h, tf + f, tb + b
+    assert (th, tf, tb) == (tr["total"]["hits"], tr["total"]["fetches"], tr["total"]["bypass"])
+
+
+def test_table2_metric_identity():
+    """Every Table 2 row: Fetches/tok = L K (1 - HR) to the printed rounding; and the oracle's
+    Eq. metrics normalisation reproduces both printed numbers from consistent totals."""
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "table2_metrics.txt"))
+            if l.strip() and not l.startswith("#")]
+    assert len(rows) == 18
+    N = 10_000
+    for model, L, K, B, method, policy, hr, fpt in rows:
+        L, K, hr, fpt = int(L), int(K), float(hr) / 100, float(fpt)
+        # HR is printed to 0.01 %: the identity holds within L K * 0.005 % + 0.005
+        tol = L * K * 0.5e-4 + 0.005
+        assert C.fetches_per_token_from_hit_rate(hr, L, K) == pytest.approx(fpt, abs=tol)
+        hits = hr * N * L * K
+        fetches = N * L * K - hits
+        HR, FPT = C.metrics(hits, fetches, N, L, K)
+        assert HR == pytest.approx(hr, rel=1e-12)
+        assert FPT == pytest.approx(fpt, abs=tol)
+    # the headline reductions quoted in the abstract: -23.7 % (Mixtral LFU), -10.1 % (DeepSeek LFU)
+    v = {(r[0], r[4], r[5]): float(r[7]) for r in rows}
+    red = lambda m: 1 - v[(m, "maskcoft", "LFU")] / v[(m, "baseline", "LFU")]
+    assert round(100 * red("mixtral-8x7b"), 1) == 23.7
+    assert round(100 * red("deepseek-v2-lite"), 1) == 10.1
+
+
+@pytest.mark.parametrize("T,K,E,B", [(1, 2, 8, 4), (16, 2, 8, 4), (1, 6, 64, 12), (8, 6, 64, 12),
+                                     (64, 6, 64, 12), (4, 1, 5, 2)])
+def test_two_formulations_agree(T, K, E, B):
+    ids = inputs.random_ids(11, 300, T, K, E, hot=range(min(E, B + 2)), p_hot=0.7)
+    a, b = C.LRUStamps(E, B), C.LRUList(E, B)
+    for s in range(ids.shape[0]):
+        ra, rb = a.step(ids[s]), b.step(ids[s])
+        assert ra == rb
+        assert a.tag == b.state()
+
+
+def test_batch1_fetch_identity():
+    """At batch 1 with K distinct experts per step: f = K - h every step, and over the stream
+    Fetches/tok = L K (1 - HR) (Eq. metrics)."""
+    L, K, E, B, N = 3, 2, 8, 4, 200
+    th = tf = 0
+    for layer in range(L):
+        ids = inputs.random_ids(12 + layer, N, 1, K, E, hot=range(4), p_hot=0.6)
+        h, f, b, _ = C.simulate(ids, E, B)
+        assert np.all(f == K - h) and np.all(b == 0)
+        th, tf = th + h.sum(), tf + f.sum()
+    HR, FPT = C.metrics(th, tf, N, L, K)
+    assert FPT == pytest.approx(C.fetches_per_token_from_hit_rate(HR, L, K), rel=1e-12)
+
+
+def test_hard_mask_with_B_kept_experts_only_cold_misses():
+    """A hard mask keeping E' = B experts: every chosen expert is in the kept set, so the cache
+    never evicts and total fetches = number of distinct experts used (<= B)."""
+    E, K, B = 8, 2, 4
+    kept = [0, 1, 2, 3]
+    ids = inputs.random_ids(13, 64, 1, K, E, hot=kept, p_hot=1.0)
+    h, f, b, _ = C.simulate(ids, E, B)
+    assert f.sum() == len(np.unique(ids)) <= B
+
+
+def test_large_cache_only_cold_misses():
+    E, K, B = 16, 3, 15
+    ids = inputs.random_ids(14, 100, 2, K, E, hot=range(10), p_hot=1.0)
+    h, f, b, _ = C.simulate(ids, E, B)
+    assert f.sum() == len(np.unique(ids))
+    assert b.sum() == 0
+
+
+def test_invalid():
+    with pytest.raises(ValueError):
+        C.LRUStamps(4, 4)
+    c = C.LRUStamps(4, 2)
+    with pytest.raises(ValueError):
+        c.step([5])
