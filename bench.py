@@ -1,0 +1,470 @@
+#!/usr/bin/env python
+"""Benchmark of the masked MoE layer forward with its expert cache on GB300 (one JSON line).
+
+Workload (default): a Mixtral-8x7B-shaped MoE layer decoding (d = 4096, E = 8, K = 2, SwiGLU width
+14336, bf16) at batch 16 over a 512-step AR(1) hidden-state stream (rho = 0.8), routed with the soft
+prior of a random keep-4-of-8 mask (pi = softmax(2 m)), with a 4-slot LRU expert cache whose misses
+are fetched from pinned host memory. One step = routing + cache decision + fetch of missed experts
++ expert FFN + combine for one decode position of all 16 rows. Also reported: the same at batch 1,
+and the masked fine-tuning / prefill forward (T = 4096 tokens, hard mask keeping 4 of 8 experts).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mcft|reference]
+
+Under torchrun (N > 1) every rank runs an independent replica on its own GPU (weak scaling; the
+forward has no exchange step); rank 0 prints the line.
+"""
+from __future__ import annotations
+
+import os
+
+_CORES = os.cpu_count() or 1
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(_CORES))
+
+import argparse  # noqa: E402
+import json  # noqa: E402
+import statistics  # noqa: E402
+import subprocess  # noqa: E402
+import sys  # noqa: E402
+import threading  # noqa: E402
+import time  # noqa: E402
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_34077_gb300 import inputs as I  # noqa: E402
+
+STREAM_STEPS = 512
+METRIC = "masked MoE layer tokens/s"
+
+
+# ------------------------------------------------------------------------------------------------
+# host-side helpers (also exercised by the CPU multi-process tests)
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), \
+        int(os.environ.get("LOCAL_RANK", 0))
+
+
+def replica_seed(base: int, rank: int) -> int:
+    """Each replica decodes its own streams (weak scaling)."""
+    return base + 1000 * rank
+
+
+def aggregate(elapsed_s: float, units: float, world: int, group=None):
+    """Max elapsed over ranks and summed units (tokens) -> (max_elapsed, total_units)."""
+    if world == 1:
+        return elapsed_s, units
+    import torch.distributed as dist
+
+    t = torch.tensor([elapsed_s], dtype=torch.float64)
+    u = torch.tensor([units], dtype=torch.float64)
+    if dist.get_backend(group) == "nccl":
+        t, u = t.cuda(), u.cuda()
+    dist.all_reduce(t, op=dist.ReduceOp.MAX, group=group)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM, group=group)
+    return float(t.item()), float(u.item())
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sust=d.get("bf16_tflops_sustained"),
+                    src="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sust=1700.0, src="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi samples (SM clock, max, throttle reasons) during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.lines, self.proc = index, [], None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.th = threading.Thread(target=self._read, daemon=True)
+            self.th.start()
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        time.sleep(0.25)
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [v.strip() for v in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx = float(f[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------------
+
+class DecodeLayer:
+    """One MoE layer in decode: router + pinned host expert pool + device cache + workspace."""
+
+    def __init__(self, shape, batch, seed, dev):
+        from paper_2609_34077_gb300 import mcft as M
+
+        self.M, self.shape, self.batch, self.dev = M, shape, batch, dev
+        self.desc = M.desc_of(shape)
+        self.lw = I.layer_weights(seed, shape, pin=True)
+        self.prior = I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep))
+        self.x_host = I.ar1_streams(seed, shape, STREAM_STEPS, batch).pin_memory()
+        self.x = self.x_host.to(dev)
+        self.wr = self.lw.router.to(dev)
+        self.shared = [b.to(dev) for b in self.lw.shared]
+        self.cache = M.mcft_cache_create(1, shape.E, shape.cache_slots, shape.expert_bytes,
+                                         self.lw.experts, max_assign=batch * shape.K)
+        self.ws = torch.empty(M.mcft_moe_workspace_size(self.desc, batch), dtype=torch.uint8, device=dev)
+        self.idx = torch.empty((STREAM_STEPS, batch, shape.K), dtype=torch.int32, device=dev)
+        self.gate = torch.empty((STREAM_STEPS, batch, shape.K), dtype=torch.float32, device=dev)
+        self.y = torch.empty((batch, shape.d), dtype=torch.bfloat16, device=dev)
+        self.compute = torch.cuda.current_stream(dev)
+        self.copy = torch.cuda.Stream(dev)
+
+    def step(self, s, x=None):
+        M, p = self.M, s % STREAM_STEPS
+        x = self.x[p] if x is None else x
+        M.mcft_route(self.desc, x, self.wr, M.MCFT_ROUTE_SOFT_PRIOR, prior=self.prior,
+                     idx=self.idx[p], gate=self.gate[p], stream=self.compute)
+        M.mcft_cache_step(self.cache, 0, self.idx[p], stream=self.compute)
+        ptrs = M.mcft_fetch_experts(self.cache, 0, self.compute, self.copy)
+        M.mcft_moe_forward(self.desc, x, self.idx[p], self.gate[p], ptrs, self.shared, y=self.y,
+                           workspace=self.ws, stream=self.compute)
+        return self.y
+
+
+def time_steps(fn, first, steps, stream):
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for s in range(first, first + steps):
+        fn(s)
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / 1e3
+
+
+def host_link_probe(dev, nbytes):
+    """Pinned host -> device copy bandwidth (GB/s), best of 10."""
+    src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    best = 0.0
+    for _ in range(10):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        dst.copy_(src, non_blocking=True)
+        b.record()
+        torch.cuda.synchronize()
+        best = max(best, nbytes / (a.elapsed_time(b) / 1e3) / 1e9)
+    del src, dst
+    return best
+
+
+def unique_per_step(idx_steps):
+    return [len(torch.unique(i)) for i in idx_steps]
+
+
+def run_decode(shape, batch, steps, warmup, seed, dev, peaks, profile=True):
+    M = __import__("paper_2609_34077_gb300.mcft", fromlist=["x"])
+    L = DecodeLayer(shape, batch, seed, dev)
+    for s in range(warmup):
+        L.step(s)
+    torch.cuda.synchronize()
+    h0, f0, b0 = M.mcft_cache_stats(L.cache, 0)
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(profile)
+    elapsed = time_steps(L.step, warmup, steps, L.compute)
+    M.mcft_profile_enable(False)
+    prof = M.mcft_profile_read()
+    M.mcft_device_error()
+    h1, f1, b1 = M.mcft_cache_stats(L.cache, 0)
+    pos = [(s % STREAM_STEPS) for s in range(warmup, warmup + steps)]
+    U = unique_per_step([L.idx[p] for p in pos])
+    hits, fetches, byp = h1 - h0, f1 - f0, b1 - b0
+    # roofline of the dominant kernel (gate/up projection GEMV): bytes each launch must move
+    w13_bytes = 2 * shape.w * shape.d * 2
+    alg13 = sum(u * w13_bytes for u in U) + steps * (batch * shape.d * 2 + batch * shape.K * shape.w * 4)
+    n13, ms13 = prof["ffn13_rowwise"]
+    alg2 = sum(u * shape.w * shape.d * 2 for u in U) + steps * batch * shape.K * (shape.w * 4 + shape.d * 4)
+    n2, ms2 = prof["ffn2_rowwise"]
+    out = dict(
+        tokens_per_s=batch * steps / elapsed, ms_per_step=elapsed * 1e3 / steps, steps=steps,
+        hits=hits, fetches=fetches, bypass=byp,
+        fetches_per_step=fetches / steps, fetches_per_token=fetches / (steps * batch),
+        hit_rate=hits / max(1, hits + fetches), mean_experts_per_step=float(np.mean(U)),
+        fetch_bytes_per_step=fetches * shape.expert_bytes / steps,
+        kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
+        gpu_launches=int(sum(v[0] for v in prof.values())),
+    )
+    out["roofline"] = dict(bound="hbm", achieved=alg13 / (ms13 / 1e3) / 1e9 if ms13 else None,
+                           peak=peaks["hbm"], unit="GB/s", kernel="ffn13_rowwise",
+                           alg_bytes_per_launch=alg13 / max(1, n13), launches=n13)
+    out["roofline"]["frac"] = out["roofline"]["achieved"] / peaks["hbm"] if ms13 else None
+    out["ffn2_gbs"] = alg2 / (ms2 / 1e3) / 1e9 if ms2 else None
+    kernel_ms = sum(v[1] for v in prof.values())
+    out["kernel_ms_per_step"] = kernel_ms / steps
+    return L, out
+
+
+def run_decode_e2e(L, steps, first):
+    """Same decode steps through the public calls with the hidden states in pinned host memory:
+    each step copies its inputs host -> device and its output device -> host."""
+    xd = torch.empty((L.batch, L.shape.d), dtype=torch.bfloat16, device=L.dev)
+    y_host = torch.empty((L.batch, L.shape.d), dtype=torch.bfloat16).pin_memory()
+
+    def step(s):
+        xd.copy_(L.x_host[s % STREAM_STEPS], non_blocking=True)
+        y = L.step(s, x=xd)
+        y_host.copy_(y, non_blocking=True)
+
+    elapsed = time_steps(step, first, steps, L.compute)
+    nb = L.batch * L.shape.d * 2
+    return dict(value=L.batch * steps / elapsed, unit="tokens/s", h2d_bytes_per_step=nb,
+                d2h_bytes_per_step=nb)
+
+
+def run_prefill(steps, warmup, seed, dev, peaks):
+    from paper_2609_34077_gb300 import mcft as M
+
+    sh, T = I.MIXTRAL, 4096
+    desc = M.desc_of(sh)
+    mask = I.keep_mask(seed, sh.E, 4)
+    lw = I.layer_weights(seed, sh, experts=[int(e) for e in np.nonzero(mask)[0]])
+    experts = [None if b is None else b.to(dev) for b in lw.experts]
+    wr = lw.router.to(dev)
+    x = I.hidden_iid(seed, sh, T).to(dev)
+    ws = torch.empty(M.mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=dev)
+    y = torch.empty_like(x)
+    idx = torch.empty((T, sh.K), dtype=torch.int32, device=dev)
+    gate = torch.empty((T, sh.K), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(s):
+        M.mcft_route(desc, x, wr, M.MCFT_ROUTE_HARD_MASK, mask=mask, idx=idx, gate=gate, stream=stream)
+        M.mcft_moe_forward(desc, x, idx, gate, experts, y=y, workspace=ws, stream=stream)
+
+    for s in range(warmup):
+        step(s)
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(True)
+    elapsed = time_steps(step, 0, steps, stream)
+    M.mcft_profile_enable(False)
+    prof = M.mcft_profile_read()
+    M.mcft_device_error()
+    A = T * sh.K
+    f13 = 2.0 * A * sh.d * 2 * sh.w
+    f2 = 2.0 * A * sh.w * sh.d
+    n13, ms13 = prof["gemm13_tc"]
+    n2, ms2 = prof["gemm2_tc"]
+    peak = peaks["bf16"]
+    res = dict(workload="mixtral-8x7b prefill T=4096 hard mask keep 4/8", tokens_per_s=T * steps / elapsed,
+               ms_per_step=elapsed * 1e3 / steps, tflop_per_step=(f13 + f2) / 1e12,
+               kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
+               gpu_launches=int(sum(v[0] for v in prof.values())))
+    if ms13 and ms2:
+        a13 = f13 / (ms13 / n13 / 1e3) / 1e12
+        a2 = f2 / (ms2 / n2 / 1e3) / 1e12
+        res["roofline"] = dict(bound="tensor", kernel="gemm13_tc", achieved=a13, peak=peak,
+                               unit="TFLOP/s", frac=a13 / peak, flop_per_launch=f13)
+        res["gemm2_tflops"] = a2
+        res["gemm_frac_of_peak"] = (f13 + f2) / ((ms13 / n13 + ms2 / n2) / 1e3) / 1e12 / peak
+    return res
+
+
+# ------------------------------------------------------------------------------------------------
+# CPU oracle timing (the reported baseline, and the reference arm)
+
+def oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0, lw=None):
+    """The CPU oracle (routing + LRU accounting + fp64 SwiGLU combine) on decode steps of the same
+    stream until ~budget_s of work; returns (tokens/s, steps done)."""
+    import oracle
+
+    lw = lw or I.layer_weights(seed, shape)
+    prior = I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep))
+    xs = I.ar1_streams(seed, shape, STREAM_STEPS, batch)
+    wr = lw.router.double().numpy()
+    ex = [tuple(t.double().numpy() for t in I.split_expert(b, shape)) for b in lw.experts]
+    sh = [tuple(t.double().numpy() for t in I.split_expert(b, shape)) for b in lw.shared]
+    cache = oracle.cache.LRUStamps(shape.E, shape.cache_slots)
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        x = xs[n % STREAM_STEPS].double().numpy()
+        r = oracle.routing.route(x, wr, shape.K, oracle.routing.MODE_SOFT_PRIOR, shape.gate, prior=prior)
+        cache.step(r["idx"])
+        oracle.ffn.moe_layer(x, r["idx"], r["gate"], ex, sh)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or n >= STREAM_STEPS:
+            return batch * n / el, n
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return 0
+    shape, batch = I.MIXTRAL, 16
+    seed = replica_seed(0, 0)
+    lw = I.layer_weights(seed, shape)
+    budget = max(2.0, min(20.0, 6.0 * args.steps / max(1, args.steps)))
+    tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=budget, lw=lw)
+    line = dict(impl="reference", metric=METRIC, value=tps, unit="tokens/s", n_gpus=args.gpus,
+                steps=n, warmup=0, ms_per_step=1e3 * batch / tps, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+                config=_config(batch),
+                cpu_baseline=dict(value=tps, unit="tokens/s", cores=_CORES, kind="oracle",
+                                  sample=f"{n} decode steps x batch {batch} of the same stream"),
+                e2e=dict(value=tps, unit="tokens/s", h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def _config(batch):
+    return {"workload": f"mixtral-8x7b-shaped MoE layer decode, batch {batch}, 512-step AR(1) "
+                        "stream, soft prior keep-4-of-8, 4-slot LRU cache, host fetch",
+            "d": 4096, "E": 8, "K": 2, "w": 14336, "batch": batch, "cache_slots": 4,
+            "l2": "inputs larger than L2 (each step streams >= 0.7 GB of expert weights)",
+            "parallelism": "replicas"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", default="mcft", choices=["mcft", "reference"])
+    ap.add_argument("--batch", type=int, default=16)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
+    args = ap.parse_args()
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        return reference_arm(args, rank, world)
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+
+    import __graft_entry__
+
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    if rank == 0 or not os.path.exists(os.path.join(ROOT, "paper_2609_34077_gb300", "libmcft.so")):
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2609_34077_gb300 import mcft as M
+
+    M.lib()
+    peaks = load_peaks()
+    seed = replica_seed(0, rank)
+    shape, batch = I.MIXTRAL, args.batch
+
+    L = DecodeLayer(shape, batch, seed, dev)
+    for s in range(args.warmup):
+        L.step(s)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    h0, f0, b0 = M.mcft_cache_stats(L.cache, 0)
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(True)
+    with ClockSampler(local) as clk:
+        elapsed = time_steps(L.step, args.warmup, args.steps, L.compute)
+    M.mcft_profile_enable(False)
+    if world > 1:
+        dist.barrier()
+    prof = M.mcft_profile_read()
+    M.mcft_device_error()
+    h1, f1, b1 = M.mcft_cache_stats(L.cache, 0)
+    max_el, tokens = aggregate(elapsed, batch * args.steps, world)
+    pos = [s % STREAM_STEPS for s in range(args.warmup, args.warmup + args.steps)]
+    U = unique_per_step([L.idx[p] for p in pos])
+    w13_bytes = 2 * shape.w * shape.d * 2
+    alg13 = sum(u * w13_bytes for u in U) + args.steps * (batch * shape.d * 2 + batch * shape.K * shape.w * 4)
+    n13, ms13 = prof["ffn13_rowwise"]
+    achieved = alg13 / (ms13 / 1e3) / 1e9 if ms13 else None
+    hits, fetches, byp = h1 - h0, f1 - f0, b1 - b0
+
+    e2e = run_decode_e2e(L, args.steps, args.warmup + args.steps)
+    link = host_link_probe(dev, shape.expert_bytes)
+    line = dict(
+        metric=METRIC, value=tokens / max_el, unit="tokens/s", n_gpus=world, steps=args.steps,
+        warmup=args.warmup, ms_per_step=max_el * 1e3 / args.steps, higher_is_better=True,
+        scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic", config=_config(batch),
+        roofline=dict(bound="hbm", achieved=achieved, peak=peaks["hbm"], unit="GB/s",
+                      frac=achieved / peaks["hbm"] if achieved else None, traffic=None,
+                      kernel="ffn13_rowwise", peak_source=peaks["src"] + " hbm_gbs",
+                      alg_bytes_per_launch=alg13 / max(1, n13)),
+        e2e=e2e, gpu_launches=int(sum(v[0] for v in prof.values())), clocks=clk.summary(),
+        kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
+        cache=dict(hits=hits, fetches=fetches, bypass=byp, fetches_per_step=fetches / args.steps,
+                   fetches_per_token=fetches / (args.steps * batch),
+                   hit_rate=hits / max(1, hits + fetches), mean_experts_per_step=float(np.mean(U))),
+        fetch=dict(bytes_per_step=fetches * shape.expert_bytes / args.steps,
+                   host_link_probe_gbs=link,
+                   fetch_share_of_step=None),
+    )
+    kern_ms = sum(v[1] for v in prof.values()) / args.steps
+    line["fetch"]["fetch_share_of_step"] = max(0.0, 1 - kern_ms / line["ms_per_step"])
+    del L
+    torch.cuda.empty_cache()
+    if not args.no_extra:
+        _, b1 = run_decode(shape, 1, min(args.steps, 256), args.warmup, seed + 1, dev, peaks)
+        b1.pop("kernels", None)
+        line["batch1"] = b1
+        line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)
+    if rank == 0 and not args.no_cpu_baseline:
+        tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0)
+        line["cpu_baseline"] = dict(value=tps, unit="tokens/s", cores=_CORES, kind="oracle",
+                                    sample=f"{n} decode steps x batch {batch} of the same stream "
+                                           "(fp64 numpy, BLAS threads = cores)")
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,231 @@
+/*
+ * mcft.h - C ABI of libmcft: the masked MoE layer forward and the per-layer expert cache, on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * The method (MaskCoFT, arxiv 2609.34077) restricts or re-ranks the Top-K routing of each MoE layer
+ * with a per-layer mask, so that decoding touches fewer experts and an expert cache in GPU memory
+ * misses less often. This library computes, per layer:
+ *
+ *   z = W x,  p = softmax(z)                                   (Section 3.1)
+ *   A = TopK(p)            plain routing                        (Section 3.1, Eq. topk)
+ *   A = TopK(p * m)        hard binary mask, fine-tuning        (Section 3.2, Eq. stage1)
+ *   A = TopK(p * pi)       soft prior, inference                (Section 3.2, Eq. inference)
+ *   y = sum_{i in A} g_i F_i(x)  (+ shared experts)             (Section 3.1, Eq. topk)
+ *
+ * with g_i from p (renormalised over A for Mixtral, p_i for DeepSeek), F_i a SwiGLU expert, and the
+ * per-layer LRU cache of B experts of Section 4.1 ("Simulation"): misses counted per Eq. metrics and
+ * fetched from pinned host memory.
+ *
+ * Conventions for every call:
+ *  - Device pointers are caller-owned CUDA device memory; host pointers are caller-owned host
+ *    memory read (or written) before the call returns, unless stated otherwise.
+ *  - Calls are asynchronous on the given stream unless stated otherwise; a NULL stream is the
+ *    legacy default stream.
+ *  - Argument errors are found on the host and returned synchronously as MCFT_ERR_INVALID (or
+ *    MCFT_ERR_UNSUPPORTED for shapes this build does not handle); nothing is launched then.
+ *  - Errors found inside a kernel (an expert id out of range, a missing expert pointer, a wait that
+ *    ran out of time) set a device error word and make the remaining kernels of that call skip
+ *    their work; mcft_device_error() reads and clears it.
+ *  - No call throws; mcft_last_error() returns a message for the calling thread's last error.
+ *  - Layouts are row-major. dtype MCFT_BF16 means bf16 x, weights and y (fp32 accumulation);
+ *    MCFT_F32 means fp32 everywhere (CUDA-core arithmetic, no TF32).
+ */
+#ifndef MCFT_H
+#define MCFT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t, declared here so that this header needs no CUDA header. */
+typedef struct CUstream_st* mcft_stream_t;
+
+typedef enum {
+  MCFT_OK = 0,
+  MCFT_ERR_INVALID = 1,      /* bad argument (found on the host) or bad data (found on device) */
+  MCFT_ERR_OOM = 2,          /* a device or pinned host allocation failed */
+  MCFT_ERR_CUDA = 3,         /* a CUDA runtime call failed; mcft_last_error() has the text */
+  MCFT_ERR_TIMEOUT = 4,      /* a kernel's bounded wait ran out; the kernel returned early */
+  MCFT_ERR_UNSUPPORTED = 5   /* valid but outside what this build handles (e.g. E > 64) */
+} mcft_status;
+
+/* Routing rule. Section 3.1 Eq. topk / Section 3.2 Eq. stage1 / Section 3.2 Eq. inference. */
+typedef enum {
+  MCFT_ROUTE_TOPK = 0,        /* A = TopK(p) */
+  MCFT_ROUTE_HARD_MASK = 1,   /* A = TopK(p * m): only experts with m_e = 1 are eligible */
+  MCFT_ROUTE_SOFT_PRIOR = 2   /* A = TopK(p * pi), pi > 0: every expert stays eligible */
+} mcft_route_mode;
+
+/* Gate weights, always from p (Section 3.1, text after Eq. topk; Section 3.2 after Eq. inference). */
+typedef enum {
+  MCFT_GATE_RENORM = 0,  /* Mixtral:  g_i = p_i / sum_{j in A} p_j */
+  MCFT_GATE_PLAIN = 1    /* DeepSeek: g_i = p_i                      */
+} mcft_gate_mode;
+
+typedef enum { MCFT_F32 = 0, MCFT_BF16 = 1 } mcft_dtype;
+
+/* Shape of one MoE layer (Section 3.1; model sizes of Appendix A Table 4).
+ *   d        hidden size d_h; multiple of 64
+ *   E        routed experts, 1..64
+ *   K        active experts per token, 1..min(E, 8)
+ *   w        SwiGLU width of every expert (routed and shared); multiple of 64
+ *   n_shared shared experts (DeepSeek-V2-Lite: 2), each of width w, added un-gated, 0..8
+ *   gate     mcft_gate_mode
+ *   dtype    mcft_dtype of x, router and expert weights, and y */
+typedef struct {
+  int d, E, K, w, n_shared, gate, dtype;
+} mcft_layer_desc;
+
+/* Packed expert block: one contiguous allocation per expert, [W1 | W3 | W2] with
+ * W1, W3 of shape [w, d] (gate and up projections) and W2 of shape [d, w] (down projection),
+ * so that F(x) = W2 (silu(W1 x) * (W3 x)). Size: 3 * w * d elements of the layer dtype. One
+ * block is one unit of cache traffic (one copy per fetch). Base address 16-byte aligned. */
+
+/* ---------------------------------------------------------------------------------------------
+ * mcft_route: router GEMV/GEMM, mask or prior, Top-K, softmax gates.
+ * Section 3.1 (z = W x, p = softmax(z), Eq. topk), Section 3.2 Eq. stage1 (hard mask) and
+ * Eq. inference (soft prior); gate weights from p.
+ *
+ *   x        device [T, d], layer dtype
+ *   T        tokens, >= 0 (T = 0 is a no-op)
+ *   w_router device [E, d], layer dtype
+ *   mode     mcft_route_mode
+ *   mask     host [E] bytes, 0 or 1, at least K ones; read only in HARD_MASK mode (else may be NULL)
+ *   prior    host [E] fp32, every entry > 0 and finite; read only in SOFT_PRIOR mode
+ *   idx      device [T, K] int32 out: active experts, by descending score; equal scores go to the
+ *            lower expert index. SOFT_PRIOR ranks by z_e + log(pi_e), which orders experts exactly
+ *            as p_e * pi_e does.
+ *   gate     device [T, K] fp32 out: gate weight of each active expert
+ * Errors: MCFT_ERR_INVALID for a NULL pointer, bad desc, a mask with fewer than K ones, a prior
+ * entry <= 0 or not finite; MCFT_ERR_UNSUPPORTED for E > 64 or K > 8. */
+mcft_status mcft_route(const mcft_layer_desc* desc, const void* x, int T, const void* w_router,
+                       int mode, const uint8_t* mask, const float* prior, int32_t* idx, float* gate,
+                       mcft_stream_t stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * mcft_moe_workspace_size: bytes of device workspace mcft_moe_forward needs for up to T_max
+ * tokens of this layer shape. */
+mcft_status mcft_moe_workspace_size(const mcft_layer_desc* desc, int T_max, size_t* bytes);
+
+/* mcft_moe_forward: token permutation by expert, grouped SwiGLU expert FFN, weighted combine and
+ * shared experts: y[t] = sum_k gate[t,k] F_{idx[t,k]}(x[t]) + sum_s F^shared_s(x[t]).
+ * Section 3.1 Eq. topk (and the shared experts described after it).
+ *
+ *   x         device [T, d] layer dtype
+ *   idx, gate device [T, K] as written by mcft_route (any ids in [0, E) are accepted; an id out
+ *             of range sets the device error word and the call writes nothing to y)
+ *   experts   host array [E] of device pointers to packed expert blocks; an entry may be NULL if
+ *             no token of this call selects that expert (a NULL that is selected sets the device
+ *             error word). The array itself is read before the call returns.
+ *   shared    host array [n_shared] of device pointers to packed blocks (NULL if n_shared = 0)
+ *   y         device [T, d] layer dtype out (may not alias x)
+ *   workspace device, at least mcft_moe_workspace_size(desc, T) bytes, 256-byte aligned; used
+ *             by the call's kernels until they finish on the stream
+ * bf16 layers with T > 64 tokens run the expert GEMMs on tcgen05 tensor cores (TMA-fed, fp32
+ * accumulators in tensor memory, SiLU*up fused in the epilogue, hidden activation rounded to bf16);
+ * smaller bf16 batches run an HBM-streaming GEMV; fp32 layers run CUDA-core fp32 arithmetic.
+ * Errors: MCFT_ERR_INVALID for a NULL pointer, bad desc, workspace too small or misaligned. */
+mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, const int32_t* idx,
+                             const float* gate, const void* const* experts,
+                             const void* const* shared, void* y, void* workspace, size_t ws_bytes,
+                             mcft_stream_t stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Per-layer expert cache (Section 4.1 "Simulation"; Eq. metrics).
+ * L layers, each with B slots for routed experts, K <= B < E. Caches start empty and persist
+ * across calls; first fills count as misses. Per layer and decode step t:
+ *   U = distinct experts selected by the step's tokens; cached experts of U are hits and get
+ *   last_use = t; the others are misses, one fetch each, taken in ascending expert id: a miss
+ *   takes the lowest free slot, else evicts the slot with the smallest (last_use, expert id)
+ *   among slots not used at step t; if every slot was used at step t (possible only when |U| > B)
+ *   the expert is fetched into a staging buffer for this step only ("bypass") and not cached.
+ *   At batch size 1 this is the paper's LRU cache and f = K - h.
+ * Shared experts are not cached here (always resident, Section 4.1). */
+typedef struct mcft_cache mcft_cache;
+
+/* mcft_cache_create: allocate the device tag/timestamp/counter arrays, L*B device slots of
+ * expert_bytes each, and the bypass staging buffers (min(E - B, max_assign) of them).
+ *   host_experts  host array [L*E] of pinned host pointers to packed expert blocks (layer-major),
+ *                 read during the call and kept; the blocks themselves must stay valid and
+ *                 pinned until mcft_cache_destroy. NULL = accounting only: no slots are
+ *                 allocated and mcft_fetch_experts copies nothing.
+ *   max_assign    largest T*K any mcft_cache_step call will pass.
+ * Synchronous. Errors: MCFT_ERR_INVALID (B < 1, B >= E, E > 64, ...), MCFT_ERR_OOM. */
+mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
+                              const void* const* host_experts, int max_assign, mcft_cache** out);
+
+/* mcft_cache_step: one decode step of one layer. Reads idx (device [T, K] int32), decides hits,
+ * misses, evictions and bypasses on the device, updates the counters and writes the step's miss
+ * list to host-mapped memory for mcft_fetch_experts. Asynchronous on `stream`.
+ * Errors: MCFT_ERR_INVALID (layer out of range, T*K > max_assign, NULL idx); an id out of range
+ * sets the device error word and the step changes no state. */
+mcft_status mcft_cache_step(mcft_cache* cache, int layer, const int32_t* idx, int T, int K,
+                            mcft_stream_t stream);
+
+/* mcft_fetch_experts: complete the last mcft_cache_step of `layer`. The host waits until that
+ * step's miss list is written (the fetch cannot start before routing is known), issues one
+ * host-to-device copy per missed expert on `copy_stream` (from the pinned host block into its slot
+ * or staging buffer), and makes `compute_stream` wait for those copies. Writes, into the host
+ * array expert_ptrs [E], the device address of every expert the step selected (NULL for the
+ * others), ready to pass to mcft_moe_forward on compute_stream. In accounting mode the addresses
+ * are NULL and nothing is copied. Blocks the calling thread until the miss list is known. */
+mcft_status mcft_fetch_experts(mcft_cache* cache, int layer, mcft_stream_t compute_stream,
+                               mcft_stream_t copy_stream, const void** expert_ptrs);
+
+/* mcft_cache_last_misses: the miss list of the last mcft_cache_step of `layer`, after
+ * mcft_fetch_experts (or a synchronisation of its stream): n_out = number of fetches;
+ * experts[i], slots[i] for i < n_out in processing order, slot = -1 for a bypass fetch.
+ * Arrays are host [E]. */
+mcft_status mcft_cache_last_misses(const mcft_cache* cache, int layer, int* n_out, int32_t* experts,
+                                   int32_t* slots);
+
+/* mcft_cache_stats: cumulative hits, fetches (misses, bypasses included) and bypasses of one
+ * layer, or summed over all layers when layer = -1. Synchronises `stream` first. HR and
+ * Fetches/tok of Eq. metrics follow as hits / (hits + fetches) and fetches / tokens. */
+mcft_status mcft_cache_stats(const mcft_cache* cache, int layer, uint64_t* hits, uint64_t* fetches,
+                             uint64_t* bypass, mcft_stream_t stream);
+
+/* mcft_cache_tags: host [B] copy of the expert id held by each slot of `layer` (-1 = empty).
+ * Synchronises `stream` first. */
+mcft_status mcft_cache_tags(const mcft_cache* cache, int layer, int32_t* tags, mcft_stream_t stream);
+
+/* mcft_cache_export / mcft_cache_import: checkpoint of the whole cache state (tags, timestamps,
+ * step counters, counters); import into a cache created with the same L, E, B resumes a stream
+ * with identical decisions. Slot contents are not part of the state: after an import, the slots
+ * the tags name must be refilled by the caller (or the cache used in accounting mode).
+ * export with buf = NULL writes the needed size to *bytes. Both synchronise `stream`. */
+mcft_status mcft_cache_export(const mcft_cache* cache, void* buf, size_t* bytes, mcft_stream_t stream);
+mcft_status mcft_cache_import(mcft_cache* cache, const void* buf, size_t bytes, mcft_stream_t stream);
+
+/* mcft_cache_destroy: free everything mcft_cache_create allocated (synchronises the device). */
+void mcft_cache_destroy(mcft_cache* cache);
+
+/* ---------------------------------------------------------------------------------------------
+ * mcft_device_error: synchronise `stream`, return and clear the device error word of the current
+ * device: MCFT_OK, MCFT_ERR_INVALID (bad id, missing expert pointer) or MCFT_ERR_TIMEOUT. */
+mcft_status mcft_device_error(mcft_stream_t stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Kernel timing (no counterpart in the paper; used to measure the path). While enabled, every
+ * kernel the library launches is bracketed by two CUDA events on its stream.
+ * mcft_profile_read synchronises the recorded events and returns, per kernel of the library, its
+ * name (static string), launches and total milliseconds since the last mcft_profile_reset;
+ * n_out = number of kernels (arrays are host [max]). Not thread-safe against concurrent enabling. */
+mcft_status mcft_profile_enable(int on);
+mcft_status mcft_profile_reset(void);
+mcft_status mcft_profile_read(int max, const char** names, uint64_t* launches, double* ms, int* n_out);
+
+/* mcft_last_error: message for the calling thread's last failed call ("" if none). */
+const char* mcft_last_error(void);
+
+/* mcft_version: library version, major * 10000 + minor * 100 + patch. */
+int mcft_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MCFT_H */

@@ -1,0 +1,521 @@
+// C ABI of libmcft (include/mcft.h): argument validation, workspace layout, kernel launches,
+// the expert cache object and its fetch engine (one host-to-device copy per miss on a copy stream,
+// ordered against the compute stream with events).
+#include <cuda_runtime.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace mcft {
+namespace {
+
+thread_local std::string g_last_error;
+
+mcft_status fail(mcft_status st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+mcft_status fail(mcft_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+mcft_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(e == cudaErrorMemoryAllocation ? MCFT_ERR_OOM : MCFT_ERR_CUDA, "%s: %s", where,
+              cudaGetErrorString(e));
+}
+
+#define MCFT_CUDA(call)                                   \
+  do {                                                    \
+    cudaError_t e_ = (call);                              \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call);   \
+  } while (0)
+
+__device__ unsigned g_device_error;  // one per device that loads the library
+
+constexpr int kMaxDevices = 64;
+
+int current_device() {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  return dev;
+}
+
+int num_sms() {
+  static int cache[kMaxDevices] = {0};
+  const int dev = current_device();
+  if (dev < kMaxDevices && cache[dev]) return cache[dev];
+  int n = 0;
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  if (n <= 0) n = 1;
+  if (dev < kMaxDevices) cache[dev] = n;
+  return n;
+}
+
+size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
+
+mcft_status check_desc(const mcft_layer_desc* d) {
+  if (!d) return fail(MCFT_ERR_INVALID, "desc is NULL");
+  if (d->d <= 0 || d->d % 64) return fail(MCFT_ERR_INVALID, "d = %d must be a positive multiple of 64", d->d);
+  if (d->w <= 0 || d->w % 64) return fail(MCFT_ERR_INVALID, "w = %d must be a positive multiple of 64", d->w);
+  if (d->E <= 0) return fail(MCFT_ERR_INVALID, "E = %d must be positive", d->E);
+  if (d->K <= 0 || d->K > d->E) return fail(MCFT_ERR_INVALID, "K = %d must be in [1, E = %d]", d->K, d->E);
+  if (d->E > kMaxE) return fail(MCFT_ERR_UNSUPPORTED, "E = %d > %d", d->E, kMaxE);
+  if (d->K > kMaxK) return fail(MCFT_ERR_UNSUPPORTED, "K = %d > %d", d->K, kMaxK);
+  if (d->n_shared < 0) return fail(MCFT_ERR_INVALID, "n_shared = %d < 0", d->n_shared);
+  if (d->n_shared > kMaxShared) return fail(MCFT_ERR_UNSUPPORTED, "n_shared = %d > %d", d->n_shared, kMaxShared);
+  if (d->gate != MCFT_GATE_RENORM && d->gate != MCFT_GATE_PLAIN)
+    return fail(MCFT_ERR_INVALID, "unknown gate mode %d", d->gate);
+  if (d->dtype != MCFT_F32 && d->dtype != MCFT_BF16)
+    return fail(MCFT_ERR_INVALID, "unknown dtype %d", d->dtype);
+  return MCFT_OK;
+}
+
+}  // namespace
+
+unsigned* device_error_word() {
+  static unsigned* cache[kMaxDevices] = {nullptr};
+  static std::mutex mu;
+  const int dev = current_device();
+  std::lock_guard<std::mutex> lock(mu);
+  if (dev < kMaxDevices && cache[dev]) return cache[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_device_error) != cudaSuccess) return nullptr;
+  if (dev < kMaxDevices) cache[dev] = static_cast<unsigned*>(p);
+  return static_cast<unsigned*>(p);
+}
+
+WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T) {
+  WsLayout L{};
+  L.tc = dtype == MCFT_BF16 && T > 64 && d % 256 == 0 && w % 128 == 0;
+  L.pad = L.tc ? 128 : 1;
+  const int nseg = E + S;
+  L.mcap = T * K + S * T + (L.tc ? nseg * (L.pad - 1) : 0);
+  size_t o = 0;
+  L.hdr = o;  o = align256(o + sizeof(WsHeader));
+  L.cnt = o;  o = align256(o + sizeof(int) * nseg);
+  L.off = o;  o = align256(o + sizeof(int) * (nseg + 1));
+  L.pos = o;  o = align256(o + sizeof(int) * size_t(T) * K);
+  L.perm = o; o = align256(o + sizeof(int) * size_t(L.mcap));
+  L.xp = o;   o = align256(o + (L.tc ? size_t(L.mcap) * d * 2 : 0));
+  L.h = o;    o = align256(o + size_t(L.mcap) * w * (L.tc ? 2 : 4));
+  L.o = o;    o = align256(o + size_t(L.mcap) * d * 4);
+  L.total = o;
+  return L;
+}
+
+}  // namespace mcft
+
+using namespace mcft;
+
+// ------------------------------------------------------------------------------------------------
+// Expert cache object
+
+struct mcft_cache {
+  int L = 0, E = 0, B = 0, max_assign = 0, n_staging = 0, device = 0;
+  size_t expert_bytes = 0;
+  std::vector<const void*> host_experts;  // [L*E] pinned host blocks (empty: accounting only)
+  int32_t* d_tag = nullptr;
+  int64_t* d_last = nullptr;
+  int64_t* d_step = nullptr;
+  unsigned long long* d_cnt = nullptr;
+  int32_t* h_miss = nullptr;  // host-mapped [L][miss_stride]
+  int32_t* d_miss = nullptr;  // device alias of h_miss
+  int miss_stride = 0;
+  char* d_slots = nullptr;    // [L*B] expert blocks
+  char* d_staging = nullptr;  // [n_staging] expert blocks
+  std::vector<cudaEvent_t> ev_step;  // per layer: recorded after its cache step
+  cudaEvent_t ev_copy = nullptr;
+};
+
+namespace {
+
+void cache_free(mcft_cache* c) {
+  if (!c) return;
+  cudaFree(c->d_tag);
+  cudaFree(c->d_last);
+  cudaFree(c->d_step);
+  cudaFree(c->d_cnt);
+  if (c->h_miss) cudaFreeHost(c->h_miss);
+  cudaFree(c->d_slots);
+  cudaFree(c->d_staging);
+  for (cudaEvent_t e : c->ev_step)
+    if (e) cudaEventDestroy(e);
+  if (c->ev_copy) cudaEventDestroy(c->ev_copy);
+  delete c;
+}
+
+const char* loc_ptr(const mcft_cache* c, int layer, int loc) {
+  if (loc < 0 || !c->d_slots) return nullptr;
+  if (loc < c->B) return c->d_slots + (size_t(layer) * c->B + loc) * c->expert_bytes;
+  return c->d_staging + size_t(loc - c->B) * c->expert_bytes;
+}
+
+struct CacheStateHeader {
+  uint32_t magic, L, E, B;
+};
+constexpr uint32_t kStateMagic = 0x4d434654u;  // "MCFT"
+
+}  // namespace
+
+extern "C" {
+
+int mcft_version(void) { return 100; }
+
+const char* mcft_last_error(void) { return g_last_error.c_str(); }
+
+mcft_status mcft_device_error(mcft_stream_t stream) {
+  unsigned* p = device_error_word();
+  if (!p) return fail(MCFT_ERR_CUDA, "cannot locate the device error word");
+  unsigned v = 0;
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  MCFT_CUDA(cudaMemcpyAsync(&v, p, sizeof(v), cudaMemcpyDeviceToHost, stream));
+  MCFT_CUDA(cudaMemsetAsync(p, 0, sizeof(unsigned), stream));
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  if (v == 0) return MCFT_OK;
+  return fail(static_cast<mcft_status>(v), "device error %u reported by a kernel", v);
+}
+
+mcft_status mcft_route(const mcft_layer_desc* desc, const void* x, int T, const void* w_router,
+                       int mode, const uint8_t* mask, const float* prior, int32_t* idx, float* gate,
+                       mcft_stream_t stream) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
+  if (mode != MCFT_ROUTE_TOPK && mode != MCFT_ROUTE_HARD_MASK && mode != MCFT_ROUTE_SOFT_PRIOR)
+    return fail(MCFT_ERR_INVALID, "unknown routing mode %d", mode);
+  RouteArgs a{};
+  if (mode == MCFT_ROUTE_HARD_MASK) {
+    if (!mask) return fail(MCFT_ERR_INVALID, "hard-mask routing needs a mask");
+    int ones = 0;
+    for (int e = 0; e < desc->E; ++e) {
+      if (mask[e] > 1) return fail(MCFT_ERR_INVALID, "mask[%d] = %d is not 0 or 1", e, mask[e]);
+      ones += mask[e];
+      a.mask[e] = mask[e];
+    }
+    if (ones < desc->K)
+      return fail(MCFT_ERR_INVALID, "mask keeps %d experts, fewer than K = %d", ones, desc->K);
+  } else if (mode == MCFT_ROUTE_SOFT_PRIOR) {
+    if (!prior) return fail(MCFT_ERR_INVALID, "soft-prior routing needs a prior");
+    for (int e = 0; e < desc->E; ++e) {
+      const float v = prior[e];
+      if (!(v > 0.f) || v > 3.4e38f)
+        return fail(MCFT_ERR_INVALID, "prior[%d] = %g must be positive and finite", e, double(v));
+      a.prior[e] = v;
+    }
+  }
+  if (T == 0) return MCFT_OK;
+  if (!x || !w_router || !idx || !gate) return fail(MCFT_ERR_INVALID, "NULL tensor pointer");
+  if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(w_router)) & 15u)
+    return fail(MCFT_ERR_INVALID, "x and w_router must be 16-byte aligned");
+  a.x = x;
+  a.w_router = w_router;
+  a.T = T;
+  a.d = desc->d;
+  a.E = desc->E;
+  a.K = desc->K;
+  a.mode = mode;
+  a.gate_mode = desc->gate;
+  a.idx = idx;
+  a.gate = gate;
+  a.err = device_error_word();
+  cudaError_t e = launch_route(a, desc->dtype, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "route kernel launch");
+  return MCFT_OK;
+}
+
+mcft_status mcft_moe_workspace_size(const mcft_layer_desc* desc, int T_max, size_t* bytes) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T_max < 0 || !bytes) return fail(MCFT_ERR_INVALID, "T_max < 0 or bytes is NULL");
+  size_t best = 0;
+  for (int T : {T_max, T_max < 64 ? T_max : 64}) {
+    const WsLayout L = ws_layout(desc->d, desc->E, desc->K, desc->w, desc->n_shared, desc->dtype, T);
+    if (L.total > best) best = L.total;
+  }
+  *bytes = best;
+  return MCFT_OK;
+}
+
+mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, const int32_t* idx,
+                             const float* gate, const void* const* experts,
+                             const void* const* shared, void* y, void* workspace, size_t ws_bytes,
+                             mcft_stream_t stream) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
+  if (T == 0) return MCFT_OK;
+  if (!x || !idx || !gate || !experts || !y || !workspace)
+    return fail(MCFT_ERR_INVALID, "NULL pointer argument");
+  if (desc->n_shared > 0 && !shared) return fail(MCFT_ERR_INVALID, "shared is NULL");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+    return fail(MCFT_ERR_INVALID, "workspace must be 256-byte aligned");
+  if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15u)
+    return fail(MCFT_ERR_INVALID, "x and y must be 16-byte aligned");
+  const int E = desc->E, S = desc->n_shared, K = desc->K;
+  const WsLayout L = ws_layout(desc->d, E, K, desc->w, S, desc->dtype, T);
+  if (ws_bytes < L.total)
+    return fail(MCFT_ERR_INVALID, "workspace of %zu bytes < %zu needed", ws_bytes, L.total);
+  for (int e = 0; e < E; ++e)
+    if (reinterpret_cast<uintptr_t>(experts[e]) & 15u)
+      return fail(MCFT_ERR_INVALID, "expert %d block is not 16-byte aligned", e);
+  for (int s = 0; s < S; ++s)
+    if (!shared[s] || (reinterpret_cast<uintptr_t>(shared[s]) & 15u))
+      return fail(MCFT_ERR_INVALID, "shared expert %d block is NULL or misaligned", s);
+
+  char* ws = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(ws + L.hdr);
+  int* cnt = reinterpret_cast<int*>(ws + L.cnt);
+  int* off = reinterpret_cast<int*>(ws + L.off);
+  int* pos = reinterpret_cast<int*>(ws + L.pos);
+  int* perm = reinterpret_cast<int*>(ws + L.perm);
+  unsigned* err = device_error_word();
+
+  PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
+  cudaError_t e = launch_permute(pa, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
+
+  FfnArgs fa{};
+  fa.x = x;
+  fa.off = off;
+  fa.perm = perm;
+  fa.hdr = hdr;
+  for (int i = 0; i < E; ++i) fa.wblk[i] = experts[i];
+  for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
+  fa.h = ws + L.h;
+  fa.o = reinterpret_cast<float*>(ws + L.o);
+  fa.T = T;
+  fa.d = desc->d;
+  fa.w = desc->w;
+  fa.nseg = E + S;
+  fa.E = E;
+  fa.err = err;
+  if (L.tc) {
+    GatherArgs ga{x, perm, hdr, ws + L.xp, desc->d, L.mcap};
+    e = launch_gather(ga, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "gather kernel launch");
+    e = launch_ffn_tc(fa, ws + L.xp, L.mcap, num_sms(), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "tensor-core expert GEMM launch");
+  } else {
+    e = launch_ffn_rowwise(fa, desc->dtype, num_sms(), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
+  }
+  CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S};
+  e = launch_combine(ca, desc->dtype, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
+  return MCFT_OK;
+}
+
+// ------------------------------------------------------------------------------------------------
+
+mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
+                              const void* const* host_experts, int max_assign, mcft_cache** out) {
+  if (!out) return fail(MCFT_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  if (L <= 0) return fail(MCFT_ERR_INVALID, "L = %d must be positive", L);
+  if (E <= 1) return fail(MCFT_ERR_INVALID, "E = %d must be at least 2", E);
+  if (E > kMaxE) return fail(MCFT_ERR_UNSUPPORTED, "E = %d > %d", E, kMaxE);
+  if (B < 1 || B >= E) return fail(MCFT_ERR_INVALID, "need 1 <= B < E (B = %d, E = %d)", B, E);
+  if (max_assign < 1) return fail(MCFT_ERR_INVALID, "max_assign = %d must be positive", max_assign);
+  if (host_experts) {
+    if (expert_bytes == 0 || expert_bytes % 16)
+      return fail(MCFT_ERR_INVALID, "expert_bytes = %zu must be a positive multiple of 16", expert_bytes);
+    for (int i = 0; i < L * E; ++i)
+      if (!host_experts[i]) return fail(MCFT_ERR_INVALID, "host expert %d is NULL", i);
+  }
+  mcft_cache* c = new mcft_cache();
+  c->L = L;
+  c->E = E;
+  c->B = B;
+  c->max_assign = max_assign;
+  c->expert_bytes = expert_bytes;
+  c->device = current_device();
+  c->miss_stride = (1 + 3 * E + 3) & ~3;
+  const int stg = E - B < max_assign ? E - B : max_assign;
+#define MCFT_CACHE_CUDA(call)                    \
+  do {                                           \
+    cudaError_t e_ = (call);                     \
+    if (e_ != cudaSuccess) {                     \
+      cache_free(c);                             \
+      return cuda_fail(e_, #call);               \
+    }                                            \
+  } while (0)
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_tag, sizeof(int32_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_last, sizeof(int64_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_step, sizeof(int64_t) * L));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_cnt, sizeof(unsigned long long) * L * 3));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_tag, 0xff, sizeof(int32_t) * L * B));  // -1 = empty
+  MCFT_CACHE_CUDA(cudaMemset(c->d_last, 0xff, sizeof(int64_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_step, 0, sizeof(int64_t) * L));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_cnt, 0, sizeof(unsigned long long) * L * 3));
+  MCFT_CACHE_CUDA(cudaHostAlloc(&c->h_miss, sizeof(int32_t) * L * c->miss_stride, cudaHostAllocMapped));
+  memset(c->h_miss, 0, sizeof(int32_t) * L * c->miss_stride);
+  MCFT_CACHE_CUDA(cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->d_miss), c->h_miss, 0));
+  if (host_experts) {
+    c->host_experts.assign(host_experts, host_experts + size_t(L) * E);
+    c->n_staging = stg;
+    MCFT_CACHE_CUDA(cudaMalloc(&c->d_slots, expert_bytes * size_t(L) * B));
+    if (stg > 0) MCFT_CACHE_CUDA(cudaMalloc(&c->d_staging, expert_bytes * size_t(stg)));
+  }
+  c->ev_step.assign(L, nullptr);
+  for (int l = 0; l < L; ++l)
+    MCFT_CACHE_CUDA(cudaEventCreateWithFlags(&c->ev_step[l], cudaEventDisableTiming));
+  MCFT_CACHE_CUDA(cudaEventCreateWithFlags(&c->ev_copy, cudaEventDisableTiming));
+  MCFT_CACHE_CUDA(cudaDeviceSynchronize());
+#undef MCFT_CACHE_CUDA
+  *out = c;
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T, int K,
+                            mcft_stream_t stream) {
+  if (!c || !idx) return fail(MCFT_ERR_INVALID, "NULL cache or idx");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  if (T < 1 || K < 1 || K > c->E) return fail(MCFT_ERR_INVALID, "bad T = %d or K = %d", T, K);
+  if (T * K > c->max_assign)
+    return fail(MCFT_ERR_INVALID, "T*K = %d exceeds max_assign = %d", T * K, c->max_assign);
+  CacheStepArgs a{idx, T * K, c->E, c->B, layer, c->d_tag, c->d_last, c->d_step, c->d_cnt,
+                  c->d_miss + size_t(layer) * c->miss_stride, device_error_word()};
+  cudaError_t e = launch_cache_step(a, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cache step launch");
+  MCFT_CUDA(cudaEventRecord(c->ev_step[layer], stream));
+  return MCFT_OK;
+}
+
+mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_stream,
+                               mcft_stream_t copy_stream, const void** expert_ptrs) {
+  if (!c || !expert_ptrs) return fail(MCFT_ERR_INVALID, "NULL cache or expert_ptrs");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  // The miss list is known only once routing and the cache decision have run.
+  MCFT_CUDA(cudaEventSynchronize(c->ev_step[layer]));
+  const int32_t* m = c->h_miss + size_t(layer) * c->miss_stride;
+  const int E = c->E;
+  const int nm = m[0];
+  const int32_t* m_exp = m + 1;
+  const int32_t* loc_of = m + 1 + 2 * E;
+  for (int e = 0; e < E; ++e) expert_ptrs[e] = loc_ptr(c, layer, loc_of[e]);
+  if (c->d_slots && nm > 0) {
+    // Every earlier use of these slots finished before the cache step's event (same stream).
+    for (int i = 0; i < nm; ++i) {
+      const int e = m_exp[i];
+      if (e < 0 || e >= E) return fail(MCFT_ERR_INVALID, "corrupt miss list");
+      const char* dst = loc_ptr(c, layer, loc_of[e]);
+      MCFT_CUDA(cudaMemcpyAsync(const_cast<char*>(dst), c->host_experts[size_t(layer) * E + e],
+                                c->expert_bytes, cudaMemcpyHostToDevice, copy_stream));
+    }
+    MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
+    MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
+  }
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_last_misses(const mcft_cache* c, int layer, int* n_out, int32_t* experts,
+                                   int32_t* slots) {
+  if (!c || !n_out || !experts || !slots) return fail(MCFT_ERR_INVALID, "NULL argument");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  const int32_t* m = c->h_miss + size_t(layer) * c->miss_stride;
+  const int nm = m[0];
+  if (nm < 0 || nm > c->E) return fail(MCFT_ERR_INVALID, "corrupt miss list");
+  *n_out = nm;
+  for (int i = 0; i < nm; ++i) {
+    experts[i] = m[1 + i];
+    slots[i] = m[1 + c->E + i];
+  }
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_stats(const mcft_cache* c, int layer, uint64_t* hits, uint64_t* fetches,
+                             uint64_t* bypass, mcft_stream_t stream) {
+  if (!c || !hits || !fetches || !bypass) return fail(MCFT_ERR_INVALID, "NULL argument");
+  if (layer < -1 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  std::vector<unsigned long long> h(size_t(c->L) * 3);
+  MCFT_CUDA(cudaMemcpyAsync(h.data(), c->d_cnt, h.size() * sizeof(h[0]), cudaMemcpyDeviceToHost, stream));
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  uint64_t a = 0, b = 0, d = 0;
+  for (int l = 0; l < c->L; ++l) {
+    if (layer >= 0 && l != layer) continue;
+    a += h[size_t(l) * 3];
+    b += h[size_t(l) * 3 + 1];
+    d += h[size_t(l) * 3 + 2];
+  }
+  *hits = a;
+  *fetches = b;
+  *bypass = d;
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_tags(const mcft_cache* c, int layer, int32_t* tags, mcft_stream_t stream) {
+  if (!c || !tags) return fail(MCFT_ERR_INVALID, "NULL argument");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  MCFT_CUDA(cudaMemcpyAsync(tags, c->d_tag + size_t(layer) * c->B, sizeof(int32_t) * c->B,
+                            cudaMemcpyDeviceToHost, stream));
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_export(const mcft_cache* c, void* buf, size_t* bytes, mcft_stream_t stream) {
+  if (!c || !bytes) return fail(MCFT_ERR_INVALID, "NULL argument");
+  const size_t LB = size_t(c->L) * c->B;
+  const size_t need = sizeof(CacheStateHeader) + LB * 4 + LB * 8 + size_t(c->L) * 8 + size_t(c->L) * 24;
+  if (!buf) {
+    *bytes = need;
+    return MCFT_OK;
+  }
+  if (*bytes < need) return fail(MCFT_ERR_INVALID, "buffer of %zu bytes < %zu needed", *bytes, need);
+  char* p = static_cast<char*>(buf);
+  CacheStateHeader h{kStateMagic, uint32_t(c->L), uint32_t(c->E), uint32_t(c->B)};
+  memcpy(p, &h, sizeof(h));
+  p += sizeof(h);
+  MCFT_CUDA(cudaMemcpyAsync(p, c->d_tag, LB * 4, cudaMemcpyDeviceToHost, stream));
+  p += LB * 4;
+  MCFT_CUDA(cudaMemcpyAsync(p, c->d_last, LB * 8, cudaMemcpyDeviceToHost, stream));
+  p += LB * 8;
+  MCFT_CUDA(cudaMemcpyAsync(p, c->d_step, size_t(c->L) * 8, cudaMemcpyDeviceToHost, stream));
+  p += size_t(c->L) * 8;
+  MCFT_CUDA(cudaMemcpyAsync(p, c->d_cnt, size_t(c->L) * 24, cudaMemcpyDeviceToHost, stream));
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  *bytes = need;
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_import(mcft_cache* c, const void* buf, size_t bytes, mcft_stream_t stream) {
+  if (!c || !buf) return fail(MCFT_ERR_INVALID, "NULL argument");
+  const size_t LB = size_t(c->L) * c->B;
+  const size_t need = sizeof(CacheStateHeader) + LB * 4 + LB * 8 + size_t(c->L) * 8 + size_t(c->L) * 24;
+  if (bytes < need) return fail(MCFT_ERR_INVALID, "state of %zu bytes < %zu expected", bytes, need);
+  const char* p = static_cast<const char*>(buf);
+  CacheStateHeader h;
+  memcpy(&h, p, sizeof(h));
+  if (h.magic != kStateMagic || h.L != uint32_t(c->L) || h.E != uint32_t(c->E) || h.B != uint32_t(c->B))
+    return fail(MCFT_ERR_INVALID, "state was exported from a cache of another shape");
+  p += sizeof(h);
+  const int32_t* tags = reinterpret_cast<const int32_t*>(p);
+  for (size_t i = 0; i < LB; ++i)
+    if (tags[i] < -1 || tags[i] >= c->E) return fail(MCFT_ERR_INVALID, "corrupt tag in state");
+  MCFT_CUDA(cudaMemcpyAsync(c->d_tag, p, LB * 4, cudaMemcpyHostToDevice, stream));
+  p += LB * 4;
+  MCFT_CUDA(cudaMemcpyAsync(c->d_last, p, LB * 8, cudaMemcpyHostToDevice, stream));
+  p += LB * 8;
+  MCFT_CUDA(cudaMemcpyAsync(c->d_step, p, size_t(c->L) * 8, cudaMemcpyHostToDevice, stream));
+  p += size_t(c->L) * 8;
+  MCFT_CUDA(cudaMemcpyAsync(c->d_cnt, p, size_t(c->L) * 24, cudaMemcpyHostToDevice, stream));
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  return MCFT_OK;
+}
+
+void mcft_cache_destroy(mcft_cache* c) {
+  if (!c) return;
+  cudaDeviceSynchronize();
+  cache_free(c);
+}
+
+}  // extern "C"

@@ -1,0 +1,106 @@
+// Per-layer expert cache decision kernel (Section 4.1 "Simulation", Eq. metrics).
+//
+// One warp per call: the lanes gather the distinct experts of the step (a 64-bit set) from the
+// routing output, then lane 0 applies the LRU rule on the layer's device-resident tag and
+// timestamp arrays: hits refresh, misses in ascending expert id take the lowest free slot or evict
+// the smallest (last_use, expert id) among slots not used this step, else go to a staging buffer
+// for this step only (bypass). The miss list and the expert -> location map are written straight
+// into host-mapped pinned memory, so the host can issue the fetches as soon as the step's event
+// completes.
+#include "common.cuh"
+#include "internal.h"
+
+namespace mcft {
+namespace {
+
+__global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ CacheStepArgs a) {
+  const int lane = threadIdx.x;
+  unsigned long long mine = 0;
+  int bad = 0;
+  for (int i = lane; i < a.n; i += 32) {
+    const int e = a.idx[i];
+    if (e < 0 || e >= a.E) bad = 1;
+    else mine |= 1ull << e;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    mine |= __shfl_xor_sync(0xffffffffu, mine, o);
+    bad |= __shfl_xor_sync(0xffffffffu, bad, o);
+  }
+  if (lane != 0) return;
+  if (bad) {  // no state change on bad input
+    set_error(a.err, kErrInvalid);
+    a.miss_out[0] = 0;
+    __threadfence_system();
+    return;
+  }
+  const int B = a.B, E = a.E;
+  int32_t* tag = a.tag + size_t(a.layer) * B;
+  int64_t* last = a.last + size_t(a.layer) * B;
+  const int64_t t = a.step[a.layer];
+  int32_t* out = a.miss_out;
+  int32_t* m_exp = out + 1;
+  int32_t* m_loc = out + 1 + E;
+  int32_t* loc_of = out + 1 + 2 * E;
+  for (int e = 0; e < E; ++e) loc_of[e] = -1;
+
+  unsigned long long cached = 0;
+  int hits = 0;
+  for (int s = 0; s < B; ++s) {
+    const int e = tag[s];
+    if (e < 0) continue;
+    cached |= 1ull << e;
+    if ((mine >> e) & 1ull) {
+      last[s] = t;
+      loc_of[e] = s;
+      ++hits;
+    }
+  }
+  int nm = 0, nbyp = 0;
+  unsigned long long miss = mine & ~cached;
+  while (miss) {
+    const int e = __ffsll(static_cast<long long>(miss)) - 1;  // ascending expert id
+    miss &= miss - 1;
+    int slot = -1;
+    for (int s = 0; s < B; ++s)
+      if (tag[s] < 0) { slot = s; break; }
+    if (slot < 0) {
+      for (int s = 0; s < B; ++s) {
+        if (last[s] >= t) continue;
+        if (slot < 0 || last[s] < last[slot] || (last[s] == last[slot] && tag[s] < tag[slot]))
+          slot = s;
+      }
+    }
+    if (slot < 0) {
+      m_exp[nm] = e;
+      m_loc[nm] = -1;
+      loc_of[e] = B + nbyp;
+      ++nbyp;
+    } else {
+      tag[slot] = e;
+      last[slot] = t;
+      m_exp[nm] = e;
+      m_loc[nm] = slot;
+      loc_of[e] = slot;
+    }
+    ++nm;
+  }
+  out[0] = nm;
+  a.step[a.layer] = t + 1;
+  unsigned long long* c = a.counters + size_t(a.layer) * 3;
+  c[0] += hits;
+  c[1] += nm;
+  c[2] += nbyp;
+  __threadfence_system();
+}
+
+}  // namespace
+
+cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s) {
+  prof_begin(kProfCache, s);
+  cache_step_kernel<<<1, 32, 0, s>>>(a);
+  prof_end(kProfCache, s);
+  return cudaGetLastError();
+}
+
+}  // namespace mcft

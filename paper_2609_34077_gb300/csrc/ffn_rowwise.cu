@@ -1,0 +1,288 @@
+// Row-streaming expert FFN for decode batches (bf16) and for fp32 layers, plus the combine.
+//
+// F(x) = W2 (silu(W1 x) * (W3 x)) per expert segment (Section 3.1; SwiGLU experts). Each weight
+// row is read once per call from HBM with 16-byte loads and dotted with every token of its segment
+// (up to 8 at a time from L1), so the kernel streams the selected experts' weights at the rate of
+// the memory system when segments hold few tokens. Work items are (segment, 16-row block), spread
+// over a persistent grid sized to the SMs.
+//
+// combine: y[t] = sum_k gate[t,k] o[pos(t,k)] + sum_s o[shared row of t in segment E+s], summed in
+// k order then shared-expert order (deterministic).
+#include "common.cuh"
+#include "internal.h"
+
+namespace mcft {
+namespace {
+
+constexpr int kWarps = 8;
+constexpr int kRowsPerWarp = 2;
+constexpr int kRowsPerItem = kWarps * kRowsPerWarp;
+constexpr int kTokGroup = 8;
+
+template <typename TW>
+struct W16;  // one 16-byte chunk of a row
+template <>
+struct W16<__nv_bfloat16> {
+  static constexpr int n = 8;
+  __device__ static void cvt(const uint4& v, float* f) { unpack8(v, f); }
+};
+template <>
+struct W16<float> {
+  static constexpr int n = 4;
+  __device__ static void cvt(const uint4& v, float* f) {
+    f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
+    f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+  }
+};
+
+struct Items {
+  int nseg, total;
+  int off[kMaxSeg + 1];
+  int first[kMaxSeg + 1];  // first item of each segment
+};
+
+// Prefix of work items over non-empty segments (rows_per_seg / kRowsPerItem items each).
+__device__ void build_items(Items& it, const FfnArgs& a, int rows_per_seg) {
+  if (threadIdx.x == 0) {
+    const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
+    it.nseg = nseg;
+    int acc = 0;
+    for (int s = 0; s <= nseg; ++s) it.off[s] = a.off[s];
+    for (int s = 0; s < nseg; ++s) {
+      it.first[s] = acc;
+      const int n = it.off[s + 1] - it.off[s];
+      if (n > 0) {
+        if (a.wblk[s] == nullptr) {  // a selected expert without weights
+          set_error(a.err, kErrInvalid);
+          const_cast<WsHeader*>(a.hdr)->abort = 1;
+          continue;
+        }
+        acc += rows_per_seg / kRowsPerItem;
+      }
+    }
+    it.first[nseg] = acc;
+    it.total = acc;
+  }
+  __syncthreads();
+}
+
+__device__ __forceinline__ int find_seg(const Items& it, int item) {
+  int s = 0;
+  // the last segment whose first item is <= item; it is never empty (its end lies past item)
+  while (s + 1 < it.nseg && it.first[s + 1] <= item) ++s;
+  return s;
+}
+
+// h[q, r] = silu(W1[r] . x_t) * (W3[r] . x_t) for rows r = r0, r0 + 1 and NT tokens of a segment.
+template <typename TW, int NT>
+__device__ __forceinline__ void ffn13_tile(const FfnArgs& a, const char* blk, int r0, int q0,
+                                           int nt, const int* tok, int lane) {
+  using C = W16<TW>;
+  const size_t rowb = size_t(a.d) * sizeof(TW);
+  const char* w1a = blk + size_t(r0) * rowb;
+  const char* w1b = w1a + rowb;
+  const char* w3a = blk + size_t(a.w + r0) * rowb;
+  const char* w3b = w3a + rowb;
+  const char* xb = reinterpret_cast<const char*>(a.x);
+  const char* xr[NT];
+#pragma unroll
+  for (int j = 0; j < NT; ++j) xr[j] = xb + size_t(j < nt ? tok[j] : tok[0]) * rowb;
+  float g0[NT], u0[NT], g1[NT], u1[NT];
+#pragma unroll
+  for (int j = 0; j < NT; ++j) g0[j] = u0[j] = g1[j] = u1[j] = 0.f;
+  const int nch = int(rowb / 16);
+#pragma unroll 2
+  for (int c = lane; c < nch; c += 32) {
+    const size_t ob = size_t(c) * 16;
+    float fa[C::n], fb[C::n], fc[C::n], fd[C::n];
+    C::cvt(ld_stream16(w1a + ob), fa);
+    C::cvt(ld_stream16(w3a + ob), fb);
+    C::cvt(ld_stream16(w1b + ob), fc);
+    C::cvt(ld_stream16(w3b + ob), fd);
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+      if (j < nt) {
+        float xv[C::n];
+        C::cvt(ldg16(xr[j] + ob), xv);
+#pragma unroll
+        for (int i = 0; i < C::n; ++i) {
+          g0[j] = fmaf(fa[i], xv[i], g0[j]);
+          u0[j] = fmaf(fb[i], xv[i], u0[j]);
+          g1[j] = fmaf(fc[i], xv[i], g1[j]);
+          u1[j] = fmaf(fd[i], xv[i], u1[j]);
+        }
+      }
+    }
+  }
+  float* h = reinterpret_cast<float*>(a.h);
+#pragma unroll
+  for (int j = 0; j < NT; ++j) {
+    if (j < nt) {
+      const float ga = warp_sum(g0[j]), ua = warp_sum(u0[j]);
+      const float gb = warp_sum(g1[j]), ub = warp_sum(u1[j]);
+      if (lane == j) {
+        float2 v = make_float2(silu(ga) * ua, silu(gb) * ub);
+        *reinterpret_cast<float2*>(h + size_t(q0 + j) * a.w + r0) = v;
+      }
+    }
+  }
+}
+
+// o[q, j] = W2[j] . h_q for output rows j = r0, r0 + 1 and NT permuted rows q0.. of a segment.
+template <typename TW, int NT>
+__device__ __forceinline__ void ffn2_tile(const FfnArgs& a, const char* blk, int r0, int q0, int nt,
+                                          int lane) {
+  using C = W16<TW>;
+  const size_t rowb = size_t(a.w) * sizeof(TW);
+  const char* w2 = blk + size_t(2) * a.w * a.d * sizeof(TW);
+  const char* wa = w2 + size_t(r0) * rowb;
+  const char* wb = wa + rowb;
+  const float* h = reinterpret_cast<const float*>(a.h);
+  float s0[NT], s1[NT];
+#pragma unroll
+  for (int j = 0; j < NT; ++j) s0[j] = s1[j] = 0.f;
+  const int nch = int(rowb / 16);
+#pragma unroll 2
+  for (int c = lane; c < nch; c += 32) {
+    float fa[C::n], fb[C::n];
+    C::cvt(ld_stream16(wa + size_t(c) * 16), fa);
+    C::cvt(ld_stream16(wb + size_t(c) * 16), fb);
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+      if (j < nt) {
+        const float4* hp = reinterpret_cast<const float4*>(h + size_t(q0 + j) * a.w + size_t(c) * C::n);
+        float hv[C::n];
+#pragma unroll
+        for (int v = 0; v < C::n / 4; ++v) {
+          const float4 t4 = hp[v];
+          hv[4 * v] = t4.x; hv[4 * v + 1] = t4.y; hv[4 * v + 2] = t4.z; hv[4 * v + 3] = t4.w;
+        }
+#pragma unroll
+        for (int i = 0; i < C::n; ++i) {
+          s0[j] = fmaf(fa[i], hv[i], s0[j]);
+          s1[j] = fmaf(fb[i], hv[i], s1[j]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < NT; ++j) {
+    if (j < nt) {
+      const float va = warp_sum(s0[j]), vb = warp_sum(s1[j]);
+      if (lane == j) *reinterpret_cast<float2*>(a.o + size_t(q0 + j) * a.d + r0) = make_float2(va, vb);
+    }
+  }
+}
+
+template <typename TW>
+__global__ void __launch_bounds__(kWarps * 32) ffn13_kernel(const __grid_constant__ FfnArgs a) {
+  __shared__ Items it;
+  build_items(it, a, a.w);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
+    const int s = find_seg(it, item);
+    const int r0 = (item - it.first[s]) * kRowsPerItem + warp * kRowsPerWarp;
+    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    const int q_begin = it.off[s], q_end = it.off[s + 1];
+    for (int q0 = q_begin; q0 < q_end; q0 += kTokGroup) {
+      const int nt = min(kTokGroup, q_end - q0);
+      int tok[kTokGroup];
+#pragma unroll
+      for (int j = 0; j < kTokGroup; ++j) tok[j] = j < nt ? a.perm[q0 + j] : 0;
+      if (nt == 1) ffn13_tile<TW, 1>(a, blk, r0, q0, nt, tok, lane);
+      else if (nt == 2) ffn13_tile<TW, 2>(a, blk, r0, q0, nt, tok, lane);
+      else if (nt <= 4) ffn13_tile<TW, 4>(a, blk, r0, q0, nt, tok, lane);
+      else ffn13_tile<TW, 8>(a, blk, r0, q0, nt, tok, lane);
+    }
+  }
+}
+
+template <typename TW>
+__global__ void __launch_bounds__(kWarps * 32) ffn2_kernel(const __grid_constant__ FfnArgs a) {
+  __shared__ Items it;
+  build_items(it, a, a.d);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
+    const int s = find_seg(it, item);
+    const int r0 = (item - it.first[s]) * kRowsPerItem + warp * kRowsPerWarp;
+    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    const int q_begin = it.off[s], q_end = it.off[s + 1];
+    for (int q0 = q_begin; q0 < q_end; q0 += kTokGroup) {
+      const int nt = min(kTokGroup, q_end - q0);
+      if (nt == 1) ffn2_tile<TW, 1>(a, blk, r0, q0, nt, lane);
+      else if (nt == 2) ffn2_tile<TW, 2>(a, blk, r0, q0, nt, lane);
+      else if (nt <= 4) ffn2_tile<TW, 4>(a, blk, r0, q0, nt, lane);
+      else ffn2_tile<TW, 8>(a, blk, r0, q0, nt, lane);
+    }
+  }
+}
+
+template <typename TY>
+__global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineArgs a) {
+  if (a.hdr->abort) return;
+  const int nq = a.d / 4;  // float4 columns per row
+  const size_t total = size_t(a.T) * nq;
+  for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+       i += size_t(gridDim.x) * blockDim.x) {
+    const int t = int(i / nq), c = int(i % nq) * 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k = 0; k < a.K; ++k) {
+      const float g = a.gate[size_t(t) * a.K + k];
+      const float4 v = *reinterpret_cast<const float4*>(a.o + size_t(a.pos[size_t(t) * a.K + k]) * a.d + c);
+      acc.x = fmaf(g, v.x, acc.x); acc.y = fmaf(g, v.y, acc.y);
+      acc.z = fmaf(g, v.z, acc.z); acc.w = fmaf(g, v.w, acc.w);
+    }
+    for (int s = 0; s < a.S; ++s) {
+      const float4 v = *reinterpret_cast<const float4*>(a.o + size_t(a.off[a.E + s] + t) * a.d + c);
+      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    }
+    if constexpr (sizeof(TY) == 4) {
+      *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.y) + size_t(t) * a.d + c) = acc;
+    } else {
+      uint2 p = make_uint2(pack2bf(acc.x, acc.y), pack2bf(acc.z, acc.w));
+      *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(a.y) + size_t(t) * a.d + c) = p;
+    }
+  }
+}
+
+int resident_blocks(const void* fn, int threads) {
+  int nb = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, fn, threads, 0) != cudaSuccess || nb < 1) nb = 1;
+  return nb;
+}
+
+template <typename TW>
+cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s) {
+  static int nb13 = resident_blocks(reinterpret_cast<const void*>(ffn13_kernel<TW>), kWarps * 32);
+  static int nb2 = resident_blocks(reinterpret_cast<const void*>(ffn2_kernel<TW>), kWarps * 32);
+  prof_begin(kProfFfn13, s);
+  ffn13_kernel<TW><<<num_sms * nb13, kWarps * 32, 0, s>>>(a);
+  prof_end(kProfFfn13, s);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  prof_begin(kProfFfn2, s);
+  ffn2_kernel<TW><<<num_sms * nb2, kWarps * 32, 0, s>>>(a);
+  prof_end(kProfFfn2, s);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s) {
+  return dtype == MCFT_BF16 ? launch_rowwise_typed<__nv_bfloat16>(a, num_sms, s)
+                            : launch_rowwise_typed<float>(a, num_sms, s);
+}
+
+cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s) {
+  if (a.T == 0) return cudaSuccess;
+  const size_t total = size_t(a.T) * (a.d / 4);
+  size_t blocks = (total + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  prof_begin(kProfCombine, s);
+  if (dtype == MCFT_BF16) combine_kernel<uint16_t><<<unsigned(blocks), 256, 0, s>>>(a);
+  else combine_kernel<float><<<unsigned(blocks), 256, 0, s>>>(a);
+  prof_end(kProfCombine, s);
+  return cudaGetLastError();
+}
+
+}  // namespace mcft

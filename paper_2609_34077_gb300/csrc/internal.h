@@ -1,0 +1,110 @@
+// Internal launchers and the workspace layout shared by the C ABI (api.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/mcft.h"
+
+namespace mcft {
+
+struct RouteArgs {
+  const void* x;
+  const void* w_router;
+  int T, d, E, K, mode, gate_mode;
+  float prior[64];            // SOFT_PRIOR: pi_e (> 0)
+  unsigned char mask[64];     // HARD_MASK: m_e in {0, 1}
+  int32_t* idx;
+  float* gate;
+  unsigned* err;
+};
+cudaError_t launch_route(const RouteArgs& a, int dtype, cudaStream_t s);
+
+// Header at the start of the forward workspace.
+struct WsHeader {
+  int abort;     // set when a kernel of this call found bad data; later kernels skip their work
+  int nseg;      // E + n_shared
+  int mrows;     // total permuted rows (padded)
+  int pad0;
+};
+
+// Device workspace of one mcft_moe_forward call. Segments 0..E-1 are the routed experts,
+// E..E+S-1 the shared experts (every token). Offsets are in permuted rows.
+struct WsLayout {
+  bool tc;        // tensor-core path (bf16, large T)
+  int pad;        // rows per segment are padded to a multiple of this (128 on the TC path)
+  int mcap;       // capacity in permuted rows
+  size_t hdr, cnt, off, pos, perm, xp, h, o, total;
+};
+WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T);
+
+struct PermuteArgs {
+  const int32_t* idx;
+  int T, K, E, S, pad, mcap;
+  WsHeader* hdr;
+  int* cnt;    // [E+S] rows per segment (unpadded)
+  int* off;    // [E+S+1] padded segment offsets
+  int* pos;    // [T*K] permuted row of assignment (t, k)
+  int* perm;   // [mcap] token of each permuted row, -1 for padding
+  unsigned* err;
+};
+cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s);
+
+struct GatherArgs {
+  const void* x;  // [T, d] bf16
+  const int* perm;
+  const WsHeader* hdr;
+  void* xp;       // [mcap, d] bf16
+  int d, mcap;
+};
+cudaError_t launch_gather(const GatherArgs& a, cudaStream_t s);
+
+struct FfnArgs {
+  const void* x;                 // [T, d] (FFN13) activations
+  const int* off;
+  const int* perm;
+  const WsHeader* hdr;
+  const void* wblk[72];          // packed expert block of each segment
+  void* h;                       // [mcap, w] fp32 (rowwise) or bf16 (tensor cores)
+  float* o;                      // [mcap, d] fp32
+  int T, d, w, nseg, E;
+  unsigned* err;
+};
+cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s);
+cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s);
+
+struct CombineArgs {
+  const float* o;
+  const float* gate;
+  const int* pos;
+  const int* off;
+  const WsHeader* hdr;
+  void* y;
+  int T, d, K, E, S;
+};
+cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s);
+
+// Cache step kernel state (device arrays of one cache).
+struct CacheStepArgs {
+  const int32_t* idx;
+  int n;              // T*K ids
+  int E, B, layer;
+  int32_t* tag;       // [L*B]
+  int64_t* last;      // [L*B]
+  int64_t* step;      // [L]
+  unsigned long long* counters;  // [L*3] hits, fetches, bypass
+  int32_t* miss_out;  // host-mapped, per layer: [n_miss, expert[E], loc[E], loc_of[E]]
+  unsigned* err;
+};
+cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s);
+
+unsigned* device_error_word();  // device address of the current device's error word
+
+// Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
+enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
+       kProfGemm2, kProfCombine, kProfCount };
+void prof_begin(int kid, cudaStream_t s);
+void prof_end(int kid, cudaStream_t s);
+
+}  // namespace mcft

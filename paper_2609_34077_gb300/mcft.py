@@ -1,0 +1,269 @@
+"""Python binding of libmcft (C ABI in include/mcft.h): argument marshalling only.
+
+Every function here has the name of the C entry point it calls and does nothing but convert torch
+tensors and Python values into pointers and sizes. All computation runs in libmcft.so; if the
+library is missing this module raises instead of computing anything another way.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmcft.so")
+
+MCFT_OK, MCFT_ERR_INVALID, MCFT_ERR_OOM, MCFT_ERR_CUDA, MCFT_ERR_TIMEOUT, MCFT_ERR_UNSUPPORTED = range(6)
+MCFT_ROUTE_TOPK, MCFT_ROUTE_HARD_MASK, MCFT_ROUTE_SOFT_PRIOR = 0, 1, 2
+MCFT_GATE_RENORM, MCFT_GATE_PLAIN = 0, 1
+MCFT_F32, MCFT_BF16 = 0, 1
+
+# every exported entry point: name -> (restype, argtypes)
+_vp, _i, _sz = C.c_void_p, C.c_int, C.c_size_t
+SIGNATURES = {
+    "mcft_route": (_i, [_vp, _vp, _i, _vp, _i, _vp, _vp, _vp, _vp, _vp]),
+    "mcft_moe_workspace_size": (_i, [_vp, _i, C.POINTER(_sz)]),
+    "mcft_moe_forward": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, C.POINTER(_vp)]),
+    "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
+    "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
+    "mcft_cache_last_misses": (_i, [_vp, _i, C.POINTER(_i), _vp, _vp]),
+    "mcft_cache_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64),
+                              C.POINTER(C.c_uint64), _vp]),
+    "mcft_cache_tags": (_i, [_vp, _i, _vp, _vp]),
+    "mcft_cache_export": (_i, [_vp, _vp, C.POINTER(_sz), _vp]),
+    "mcft_cache_import": (_i, [_vp, _vp, _sz, _vp]),
+    "mcft_cache_destroy": (None, [_vp]),
+    "mcft_device_error": (_i, [_vp]),
+    "mcft_profile_enable": (_i, [_i]),
+    "mcft_profile_reset": (_i, []),
+    "mcft_profile_read": (_i, [_i, _vp, _vp, _vp, C.POINTER(_i)]),
+    "mcft_last_error": (C.c_char_p, []),
+    "mcft_version": (_i, []),
+}
+
+
+class MCFTError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"mcft status {status}: {msg}")
+        self.status = status
+
+
+class LayerDesc(C.Structure):
+    """mcft_layer_desc"""
+    _fields_ = [("d", C.c_int), ("E", C.c_int), ("K", C.c_int), ("w", C.c_int),
+                ("n_shared", C.c_int), ("gate", C.c_int), ("dtype", C.c_int)]
+
+
+_lib = None
+
+
+def lib():
+    """Load libmcft.so (built by paper_2609_34077_gb300.build); raise if it is not there."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(f"{_LIB_PATH} is missing: build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        L = C.CDLL(_LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(st):
+    if st != MCFT_OK:
+        raise MCFTError(st, lib().mcft_last_error().decode())
+
+
+def _stream(stream):
+    if stream is None:
+        return C.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return C.c_void_p(stream.cuda_stream)
+    return C.c_void_p(int(stream))
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return C.c_void_p(t)
+    assert t.is_contiguous(), "tensors passed to libmcft must be contiguous"
+    return C.c_void_p(t.data_ptr())
+
+
+def desc_of(shape) -> LayerDesc:
+    """mcft_layer_desc of an inputs.LayerShape."""
+    return LayerDesc(shape.d, shape.E, shape.K, shape.w, shape.n_shared, shape.gate, shape.dtype)
+
+
+def torch_dtype(desc: LayerDesc):
+    return torch.bfloat16 if desc.dtype == MCFT_BF16 else torch.float32
+
+
+def mcft_version() -> int:
+    return lib().mcft_version()
+
+
+def mcft_device_error(stream=None):
+    _check(lib().mcft_device_error(_stream(stream)))
+
+
+def mcft_route(desc: LayerDesc, x, w_router, mode, mask=None, prior=None, idx=None, gate=None,
+               stream=None):
+    """idx [T,K] int32 and gate [T,K] fp32 (allocated on x's device if not given)."""
+    T = x.shape[0]
+    if idx is None:
+        idx = torch.empty((T, desc.K), dtype=torch.int32, device=x.device)
+    if gate is None:
+        gate = torch.empty((T, desc.K), dtype=torch.float32, device=x.device)
+    m = None
+    if mask is not None:
+        mb = bytes(int(v) for v in mask)
+        m = C.create_string_buffer(mb, len(mb))
+    p = None
+    if prior is not None:
+        p = (C.c_float * desc.E)(*[float(v) for v in prior])
+    _check(lib().mcft_route(C.byref(desc), _ptr(x), T, _ptr(w_router), int(mode),
+                            C.cast(m, C.c_void_p) if m is not None else None,
+                            C.cast(p, C.c_void_p) if p is not None else None,
+                            _ptr(idx), _ptr(gate), _stream(stream)))
+    return idx, gate
+
+
+def mcft_moe_workspace_size(desc: LayerDesc, T_max: int) -> int:
+    n = C.c_size_t(0)
+    _check(lib().mcft_moe_workspace_size(C.byref(desc), int(T_max), C.byref(n)))
+    return n.value
+
+
+def _ptr_array(items, n):
+    arr = (C.c_void_p * max(n, 1))()
+    for i in range(n):
+        it = items[i] if items is not None and i < len(items) else None
+        arr[i] = None if it is None else (it if isinstance(it, int) else it.data_ptr())
+    return arr
+
+
+def mcft_moe_forward(desc: LayerDesc, x, idx, gate, experts, shared=(), y=None, workspace=None,
+                     stream=None):
+    """y [T,d] = sum_k gate F_idx(x) + shared experts. ``experts``: E tensors / device addresses /
+    None; ``workspace``: uint8 device tensor (allocated if not given)."""
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.empty(mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=x.device)
+    ex = _ptr_array(experts, desc.E)
+    sh = _ptr_array(shared, desc.n_shared)
+    _check(lib().mcft_moe_forward(C.byref(desc), _ptr(x), T, _ptr(idx), _ptr(gate),
+                                  C.cast(ex, C.c_void_p), C.cast(sh, C.c_void_p), _ptr(y),
+                                  _ptr(workspace), workspace.numel(), _stream(stream)))
+    return y
+
+
+class Cache:
+    """Handle of an mcft_cache (per-layer expert cache, Section 4.1)."""
+
+    def __init__(self, handle, L, E, B):
+        self.handle, self.L, self.E, self.B = handle, L, E, B
+
+    def __del__(self):
+        if getattr(self, "handle", None):
+            try:
+                mcft_cache_destroy(self)
+            except Exception:
+                pass
+
+
+def mcft_cache_create(L, E, B, expert_bytes=0, host_experts=None, max_assign=1024) -> Cache:
+    """host_experts: L*E pinned host tensors (layer-major) or None for accounting only."""
+    h = C.c_void_p()
+    arr = _ptr_array(host_experts, L * E) if host_experts is not None else None
+    _check(lib().mcft_cache_create(L, E, B, expert_bytes,
+                                   C.cast(arr, C.c_void_p) if arr is not None else None,
+                                   max_assign, C.byref(h)))
+    c = Cache(h.value, L, E, B)
+    c._host_experts = host_experts  # keep the pinned blocks alive
+    return c
+
+
+def mcft_cache_destroy(cache: Cache):
+    if cache.handle:
+        lib().mcft_cache_destroy(C.c_void_p(cache.handle))
+        cache.handle = None
+
+
+def mcft_cache_step(cache: Cache, layer, idx, stream=None):
+    T, K = idx.shape
+    _check(lib().mcft_cache_step(C.c_void_p(cache.handle), layer, _ptr(idx), T, K, _stream(stream)))
+
+
+def mcft_fetch_experts(cache: Cache, layer, compute_stream=None, copy_stream=None):
+    """Returns the E device addresses (0 for experts not selected this step)."""
+    out = (C.c_void_p * cache.E)()
+    _check(lib().mcft_fetch_experts(C.c_void_p(cache.handle), layer, _stream(compute_stream),
+                                    _stream(copy_stream), C.cast(out, C.c_void_p)))
+    return [v or 0 for v in out]
+
+
+def mcft_cache_last_misses(cache: Cache, layer):
+    n = C.c_int(0)
+    ex = (C.c_int32 * cache.E)()
+    sl = (C.c_int32 * cache.E)()
+    _check(lib().mcft_cache_last_misses(C.c_void_p(cache.handle), layer, C.byref(n),
+                                        C.cast(ex, C.c_void_p), C.cast(sl, C.c_void_p)))
+    return [(ex[i], sl[i]) for i in range(n.value)]
+
+
+def mcft_cache_stats(cache: Cache, layer=-1, stream=None):
+    h, f, b = C.c_uint64(), C.c_uint64(), C.c_uint64()
+    _check(lib().mcft_cache_stats(C.c_void_p(cache.handle), layer, C.byref(h), C.byref(f),
+                                  C.byref(b), _stream(stream)))
+    return h.value, f.value, b.value
+
+
+def mcft_cache_tags(cache: Cache, layer, stream=None):
+    t = (C.c_int32 * cache.B)()
+    _check(lib().mcft_cache_tags(C.c_void_p(cache.handle), layer, C.cast(t, C.c_void_p),
+                                 _stream(stream)))
+    return list(t)
+
+
+def mcft_cache_export(cache: Cache, stream=None) -> bytes:
+    n = C.c_size_t(0)
+    _check(lib().mcft_cache_export(C.c_void_p(cache.handle), None, C.byref(n), _stream(stream)))
+    buf = C.create_string_buffer(n.value)
+    _check(lib().mcft_cache_export(C.c_void_p(cache.handle), C.cast(buf, C.c_void_p), C.byref(n),
+                                   _stream(stream)))
+    return buf.raw[: n.value]
+
+
+def mcft_cache_import(cache: Cache, state: bytes, stream=None):
+    buf = C.create_string_buffer(state, len(state))
+    _check(lib().mcft_cache_import(C.c_void_p(cache.handle), C.cast(buf, C.c_void_p), len(state),
+                                   _stream(stream)))
+
+
+def mcft_profile_enable(on: bool = True):
+    _check(lib().mcft_profile_enable(1 if on else 0))
+
+
+def mcft_profile_reset():
+    _check(lib().mcft_profile_reset())
+
+
+def mcft_profile_read():
+    """{kernel name: (launches, total ms)} since the last reset (synchronises recorded events)."""
+    n = C.c_int(0)
+    _check(lib().mcft_profile_read(0, None, None, None, C.byref(n)))
+    names = (C.c_char_p * n.value)()
+    launches = (C.c_uint64 * n.value)()
+    ms = (C.c_double * n.value)()
+    _check(lib().mcft_profile_read(n.value, C.cast(names, C.c_void_p), C.cast(launches, C.c_void_p),
+                                   C.cast(ms, C.c_void_p), C.byref(n)))
+    return {names[i].decode(): (launches[i], ms[i]) for i in range(n.value)}

@@ -1,0 +1,77 @@
+"""End-to-end decode steps through the C ABI: route (soft prior) -> cache step -> fetch of missed
+experts from pinned host memory -> expert FFN + combine, against the oracle's routing, cache and
+layer output (Section 3.1, Eq. inference, Section 4.1)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_34077_gb300 import inputs as I
+from paper_2609_34077_gb300 import mcft as M
+from tests.gpu_helpers import NEAR_TIE, TOL_BF16, check_output, expert_triples, f64, shared_triples
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+SMALL_MIX = I.LayerShape("small-mix", d=256, E=8, K=2, w=256, n_shared=0, gate=I.GATE_RENORM,
+                         dtype=I.BF16, cache_slots=4, keep=4)
+SMALL_DS = I.LayerShape("small-ds-layer", d=256, E=64, K=6, w=128, n_shared=2, gate=I.GATE_PLAIN,
+                        dtype=I.BF16, cache_slots=12, keep=16)
+
+
+def _decode_stream(shape, batch, steps, seed, check_every=1):
+    lw = I.layer_weights(seed, shape, pin=True)
+    desc = M.desc_of(shape)
+    prior = I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep))
+    xs = I.ar1_streams(seed, shape, steps, batch)
+    cache = M.mcft_cache_create(1, shape.E, shape.cache_slots, shape.expert_bytes, lw.experts,
+                                max_assign=batch * shape.K)
+    ref_cache = oracle.cache.LRUStamps(shape.E, shape.cache_slots)
+    wr = lw.router.to(DEV)
+    shared = [b.to(DEV) for b in lw.shared]
+    ws = torch.empty(M.mcft_moe_workspace_size(desc, batch), dtype=torch.uint8, device=DEV)
+    copy = torch.cuda.Stream()
+    ex_ref = expert_triples(lw, shape)
+    sh_ref = shared_triples(lw, shape)
+    mism = 0
+    diverged = False  # once routing differs (a near tie), the two caches see different streams
+    for s in range(steps):
+        x = xs[s]
+        xd = x.to(DEV)
+        idx, gate = M.mcft_route(desc, xd, wr, M.MCFT_ROUTE_SOFT_PRIOR, prior=prior)
+        M.mcft_cache_step(cache, 0, idx)
+        ptrs = M.mcft_fetch_experts(cache, 0, torch.cuda.current_stream(), copy)
+        y = M.mcft_moe_forward(desc, xd, idx, gate, ptrs, shared, workspace=ws)
+        ref = oracle.routing.route(f64(x), f64(lw.router), shape.K, M.MCFT_ROUTE_SOFT_PRIOR,
+                                   shape.gate, prior=prior)
+        gi = idx.cpu().numpy()
+        rows = np.all(gi == ref["idx"], axis=1)
+        if not rows.all():
+            near = (ref["gap_k"] < NEAR_TIE) | (ref["gap_in"] < NEAR_TIE)
+            assert np.all(near[~rows]), f"step {s}: routing differs outside a near tie"
+            mism += 1
+            diverged = True
+        h, f, b, ml = ref_cache.step(ref["idx"])
+        if not diverged:
+            assert M.mcft_cache_last_misses(cache, 0) == ml, f"step {s}"
+        if s % check_every == 0 and rows.any():
+            yref = oracle.ffn.moe_layer(f64(x)[rows], ref["idx"][rows], ref["gate"][rows], ex_ref, sh_ref)
+            check_output(y[torch.from_numpy(np.nonzero(rows)[0]).to(DEV)], yref, TOL_BF16,
+                         f"{shape.name} step {s}")
+    M.mcft_device_error()
+    return cache, mism
+
+
+@pytest.mark.parametrize("shape,batch", [(SMALL_MIX, 1), (SMALL_MIX, 16), (SMALL_DS, 1),
+                                         (SMALL_DS, 8), (SMALL_DS, 64)],
+                         ids=["mix-b1", "mix-b16", "ds-b1", "ds-b8", "ds-b64"])
+def test_decode_stream_small(shape, batch):
+    _, mism = _decode_stream(shape, batch, 64, seed=20 + batch)
+    assert mism <= 2
+
+
+def test_decode_stream_mixtral_full_size():
+    """Mixtral-shaped layer, 8 experts of 352 MB in pinned host memory, 4 GPU slots: 12 decode
+    steps at batch 1 with real fetches; output checked every 4th step."""
+    _, mism = _decode_stream(I.MIXTRAL, 1, 12, seed=30, check_every=4)
+    assert mism <= 1
