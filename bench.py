@@ -40,6 +40,22 @@ from paper_2609_34077_gb300 import inputs as I  # noqa: E402
 STREAM_STEPS = 512
 METRIC = "masked MoE layer tokens/s"
 
+# DRAM traffic per launch / algorithmic bytes, from one ncu capture of the kernel (summary and
+# command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
+# the source has changed since the capture, the bench reports traffic as null.
+TRAFFIC = {"ffn13_rowwise": ("paper_2609_34077_gb300/csrc/ffn_rowwise.cu", "e3dfba3481a402f4", 1.006,
+                             "profiles/ffn13_rowwise_mixtral_decode_b16.md")}
+
+
+def traffic_ratio(kernel):
+    import hashlib
+
+    if kernel not in TRAFFIC:
+        return None
+    src, digest, ratio, _ = TRAFFIC[kernel]
+    cur = hashlib.sha256(open(os.path.join(ROOT, src), "rb").read()).hexdigest()[:16]
+    return ratio if cur == digest else None
+
 
 # ------------------------------------------------------------------------------------------------
 # host-side helpers (also exercised by the CPU multi-process tests)
@@ -364,6 +380,37 @@ def _config(batch):
             "parallelism": "replicas"}
 
 
+def profile_case(case: str, dev) -> int:
+    """A few forwards with every expert resident on the device (no cache, no fetch): the small
+    launch sequence that ncu captures. decode16: Mixtral-shaped decode, batch 16 (rowwise GEMV);
+    decode1: batch 1; prefill: T = 4096 tokens, hard mask keep 4 of 8 (tcgen05 GEMMs)."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    sh = I.MIXTRAL
+    desc = M.desc_of(sh)
+    if case == "prefill":
+        T, mode = 4096, M.MCFT_ROUTE_HARD_MASK
+        kw = dict(mask=I.keep_mask(7, sh.E, 4))
+        keep = [int(e) for e in np.nonzero(kw["mask"])[0]]
+        x = I.hidden_iid(7, sh, T).to(dev)
+    else:
+        T, mode = (16 if case == "decode16" else 1), M.MCFT_ROUTE_SOFT_PRIOR
+        kw = dict(prior=I.prior_from_mask(I.keep_mask(7, sh.E, sh.keep)))
+        keep = list(range(sh.E))
+        x = I.ar1_streams(7, sh, 1, T)[0].to(dev)
+    lw = I.layer_weights(7, sh, experts=keep)
+    experts = [None if b is None else b.to(dev) for b in lw.experts]
+    wr = lw.router.to(dev)
+    ws = torch.empty(M.mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        idx, gate = M.mcft_route(desc, x, wr, mode, **kw)
+        y = M.mcft_moe_forward(desc, x, idx, gate, experts, workspace=ws)
+    M.mcft_device_error()
+    torch.cuda.synchronize()
+    print(json.dumps({"case": case, "T": T, "y_abs_mean": float(y.float().abs().mean())}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -373,7 +420,15 @@ def main():
     ap.add_argument("--batch", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
+    ap.add_argument("--case", choices=["decode16", "decode1", "prefill"],
+                    help="run only a few resident-expert forwards (for profiler captures)")
     args = ap.parse_args()
+    if args.case:
+        import __graft_entry__
+
+        __graft_entry__.build()
+        torch.cuda.set_device(0)
+        return profile_case(args.case, torch.device("cuda", 0))
     rank, world, local = dist_env()
     if args.impl == "reference":
         return reference_arm(args, rank, world)
@@ -432,7 +487,9 @@ def main():
         warmup=args.warmup, ms_per_step=max_el * 1e3 / args.steps, higher_is_better=True,
         scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic", config=_config(batch),
         roofline=dict(bound="hbm", achieved=achieved, peak=peaks["hbm"], unit="GB/s",
-                      frac=achieved / peaks["hbm"] if achieved else None, traffic=None,
+                      frac=achieved / peaks["hbm"] if achieved else None,
+                      traffic=(traffic_ratio("ffn13_rowwise") * alg13 / max(1, n13)
+                               if traffic_ratio("ffn13_rowwise") else None),
                       kernel="ffn13_rowwise", peak_source=peaks["src"] + " hbm_gbs",
                       alg_bytes_per_launch=alg13 / max(1, n13)),
         e2e=e2e, gpu_launches=int(sum(v[0] for v in prof.values())), clocks=clk.summary(),
