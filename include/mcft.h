@@ -133,6 +133,21 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
                              const void* const* shared, void* y, void* workspace, size_t ws_bytes,
                              mcft_stream_t stream);
 
+/* mcft_moe_forward_noalloc: the same computation as mcft_moe_forward (same arguments, minus the
+ * workspace), for callers that cannot allocate device memory when they run a layer, such as a
+ * plugin inside an application that owns every device allocation, or a decode loop that cannot
+ * afford an allocation's implicit synchronisation. The paper has no counterpart: this is an
+ * interface for such callers only. Scratch comes from one static device array of 16 MiB inside
+ * the library (held by every GPU that loads it, until exit), enough for decode calls of up to 64
+ * tokens of the Mixtral- and DeepSeek-V2-Lite-shaped layers; a call needing more returns
+ * MCFT_ERR_UNSUPPORTED (use mcft_moe_forward). The first call on a device looks up the array's
+ * device address; make it before any stream capture. All calls share the array: calls whose
+ * kernels overlap on the GPU race and must be serialised by the caller. Allocates nothing. */
+mcft_status mcft_moe_forward_noalloc(const mcft_layer_desc* desc, const void* x, int T,
+                                     const int32_t* idx, const float* gate,
+                                     const void* const* experts, const void* const* shared,
+                                     void* y, mcft_stream_t stream);
+
 /* ---------------------------------------------------------------------------------------------
  * Per-layer expert cache (Section 4.1 "Simulation"; Eq. metrics).
  * L layers, each with B slots for routed experts, K <= B < E. Caches start empty and persist

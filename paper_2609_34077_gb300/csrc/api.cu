@@ -82,6 +82,8 @@ mcft_status check_desc(const mcft_layer_desc* d) {
 
 }  // namespace
 
+mcft_status set_error_message(mcft_status st, const char* msg) { return fail(st, "%s", msg); }
+
 unsigned* device_error_word() {
   static unsigned* cache[kMaxDevices] = {nullptr};
   static std::mutex mu;

@@ -100,6 +100,7 @@ struct CacheStepArgs {
 cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s);
 
 unsigned* device_error_word();  // device address of the current device's error word
+mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_error() text
 
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,

@@ -24,6 +24,7 @@ SIGNATURES = {
     "mcft_route": (_i, [_vp, _vp, _i, _vp, _i, _vp, _vp, _vp, _vp, _vp]),
     "mcft_moe_workspace_size": (_i, [_vp, _i, C.POINTER(_sz)]),
     "mcft_moe_forward": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "mcft_moe_forward_noalloc": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
     "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, C.POINTER(_vp)]),
     "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
     "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
@@ -163,6 +164,20 @@ def mcft_moe_forward(desc: LayerDesc, x, idx, gate, experts, shared=(), y=None, 
     _check(lib().mcft_moe_forward(C.byref(desc), _ptr(x), T, _ptr(idx), _ptr(gate),
                                   C.cast(ex, C.c_void_p), C.cast(sh, C.c_void_p), _ptr(y),
                                   _ptr(workspace), workspace.numel(), _stream(stream)))
+    return y
+
+
+def mcft_moe_forward_noalloc(desc: LayerDesc, x, idx, gate, experts, shared=(), y=None, stream=None):
+    """mcft_moe_forward without a workspace: the library's static scratch array is used instead
+    (for callers that cannot allocate device memory; decode-sized calls only)."""
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty_like(x)
+    ex = _ptr_array(experts, desc.E)
+    sh = _ptr_array(shared, desc.n_shared)
+    _check(lib().mcft_moe_forward_noalloc(C.byref(desc), _ptr(x), T, _ptr(idx), _ptr(gate),
+                                          C.cast(ex, C.c_void_p), C.cast(sh, C.c_void_p), _ptr(y),
+                                          _stream(stream)))
     return y
 
 
