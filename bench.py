@@ -43,8 +43,12 @@ METRIC = "masked MoE layer tokens/s"
 # DRAM traffic per launch / algorithmic bytes, from one ncu capture of the kernel (summary and
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
-TRAFFIC = {"ffn13_rowwise": ("paper_2609_34077_gb300/csrc/ffn_rowwise.cu", "e3dfba3481a402f4", 1.006,
-                             "profiles/ffn13_rowwise_mixtral_decode_b16.md")}
+TRAFFIC = {
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f4a9f9398fa959c3", 1.0015,
+                     "profiles/ffn_decode_mixtral_decode.md"),
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f4a9f9398fa959c3", 1.0042,
+                    "profiles/ffn_decode_mixtral_decode.md"),
+}
 
 
 def traffic_ratio(kernel):
@@ -218,6 +222,34 @@ def unique_per_step(idx_steps):
     return [len(torch.unique(i)) for i in idx_steps]
 
 
+def decode_roofline(prof, U, steps, batch, shape, peaks):
+    """HBM roofline of the decode FFN kernels. Algorithmic bytes per launch: the W1 and W3 rows
+    (GEMM13) or W2 rows (GEMM2) of every expert the step selected, read once, plus the token
+    activations in and out. Returns (dominant kernel's roofline dict, {kernel: GB/s})."""
+    sel = sum(U)
+    T, K, d, w = batch, shape.K, shape.d, shape.w
+    alg = {"ffn13_decode": sel * 2 * w * d * 2 + steps * (T * d * 2 + T * K * w * 2),
+           "ffn2_decode": sel * w * d * 2 + steps * T * K * (w * 2 + d * 4)}
+    rates, best = {}, None
+    for k, b in alg.items():
+        n, ms = prof.get(k, (0, 0.0))
+        if not ms:
+            continue
+        rates[k] = b / (ms / 1e3) / 1e9
+        if best is None or ms > prof[best][1]:
+            best = k
+    if best is None:
+        return None, rates
+    n, ms = prof[best]
+    per_launch = alg[best] / max(1, n)
+    tr = traffic_ratio(best)
+    roof = dict(bound="hbm", achieved=rates[best], peak=peaks["hbm"], unit="GB/s",
+                frac=rates[best] / peaks["hbm"], traffic=tr * per_launch if tr else None,
+                kernel=best, peak_source=peaks["src"] + " hbm_gbs", alg_bytes_per_launch=per_launch,
+                launches=n)
+    return roof, rates
+
+
 def run_decode(shape, batch, steps, warmup, seed, dev, peaks, profile=True):
     M = __import__("paper_2609_34077_gb300.mcft", fromlist=["x"])
     L = DecodeLayer(shape, batch, seed, dev)
@@ -235,12 +267,7 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, profile=True):
     pos = [(s % STREAM_STEPS) for s in range(warmup, warmup + steps)]
     U = unique_per_step([L.idx[p] for p in pos])
     hits, fetches, byp = h1 - h0, f1 - f0, b1 - b0
-    # roofline of the dominant kernel (gate/up projection GEMV): bytes each launch must move
-    w13_bytes = 2 * shape.w * shape.d * 2
-    alg13 = sum(u * w13_bytes for u in U) + steps * (batch * shape.d * 2 + batch * shape.K * shape.w * 4)
-    n13, ms13 = prof["ffn13_rowwise"]
-    alg2 = sum(u * shape.w * shape.d * 2 for u in U) + steps * batch * shape.K * (shape.w * 4 + shape.d * 4)
-    n2, ms2 = prof["ffn2_rowwise"]
+    roof, rates = decode_roofline(prof, U, steps, batch, shape, peaks)
     out = dict(
         tokens_per_s=batch * steps / elapsed, ms_per_step=elapsed * 1e3 / steps, steps=steps,
         hits=hits, fetches=fetches, bypass=byp,
@@ -248,13 +275,8 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, profile=True):
         hit_rate=hits / max(1, hits + fetches), mean_experts_per_step=float(np.mean(U)),
         fetch_bytes_per_step=fetches * shape.expert_bytes / steps,
         kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
-        gpu_launches=int(sum(v[0] for v in prof.values())),
+        gpu_launches=int(sum(v[0] for v in prof.values())), roofline=roof, kernel_gbs=rates,
     )
-    out["roofline"] = dict(bound="hbm", achieved=alg13 / (ms13 / 1e3) / 1e9 if ms13 else None,
-                           peak=peaks["hbm"], unit="GB/s", kernel="ffn13_rowwise",
-                           alg_bytes_per_launch=alg13 / max(1, n13), launches=n13)
-    out["roofline"]["frac"] = out["roofline"]["achieved"] / peaks["hbm"] if ms13 else None
-    out["ffn2_gbs"] = alg2 / (ms2 / 1e3) / 1e9 if ms2 else None
     kernel_ms = sum(v[1] for v in prof.values())
     out["kernel_ms_per_step"] = kernel_ms / steps
     return L, out
@@ -275,6 +297,80 @@ def run_decode_e2e(L, steps, first):
     nb = L.batch * L.shape.d * 2
     return dict(value=L.batch * steps / elapsed, unit="tokens/s", h2d_bytes_per_step=nb,
                 d2h_bytes_per_step=nb)
+
+
+class DecodeStack:
+    """L MoE layers decoding at batch 1, each with its own router, soft prior (random keep-k
+    mask), AR(1) hidden-state stream and B cache slots; layers are not chained. The pinned host
+    pool holds E distinct expert blocks that every layer aliases (a 32-layer Mixtral pool would be
+    90 GB): fetch counts and bytes are those of distinct per-layer experts."""
+
+    def __init__(self, shape, L, steps, seed, dev, policy="LRU"):
+        from paper_2609_34077_gb300 import mcft as M
+
+        self.M, self.shape, self.L, self.dev = M, shape, L, dev
+        self.desc = M.desc_of(shape)
+        pool = I.layer_weights(seed, shape, layer=0, pin=True)
+        self.pool = pool
+        self.shared = [b.to(dev) for b in pool.shared]
+        self.routers, self.priors, self.x = [], [], []
+        for l in range(L):
+            self.routers.append(I.router_weight(seed, shape, l).to(dev))
+            self.priors.append(I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep, l)))
+            self.x.append(I.ar1_streams(seed, shape, steps, 1, l)[:, 0].contiguous().to(dev))
+        host = [pool.experts[e] for _ in range(L) for e in range(shape.E)]
+        self.cache = M.mcft_cache_create(L, shape.E, shape.cache_slots, shape.expert_bytes, host,
+                                         max_assign=shape.K, policy=policy)
+        self.ws = torch.empty(M.mcft_moe_workspace_size(self.desc, 1), dtype=torch.uint8, device=dev)
+        self.idx = torch.empty((L, shape.K), dtype=torch.int32, device=dev)
+        self.gate = torch.empty((L, shape.K), dtype=torch.float32, device=dev)
+        self.y = torch.empty((L, shape.d), dtype=torch.bfloat16, device=dev)
+        self.compute = torch.cuda.current_stream(dev)
+        self.copy = torch.cuda.Stream(dev)
+
+    def step(self, s):
+        M = self.M
+        for l in range(self.L):
+            x = self.x[l][s:s + 1]
+            M.mcft_route(self.desc, x, self.routers[l], M.MCFT_ROUTE_SOFT_PRIOR, prior=self.priors[l],
+                         idx=self.idx[l:l + 1], gate=self.gate[l:l + 1], stream=self.compute)
+            M.mcft_cache_step(self.cache, l, self.idx[l:l + 1], stream=self.compute)
+            ptrs = M.mcft_fetch_experts(self.cache, l, self.compute, self.copy)
+            M.mcft_moe_forward(self.desc, x, self.idx[l:l + 1], self.gate[l:l + 1], ptrs, self.shared,
+                               y=self.y[l:l + 1], workspace=self.ws, stream=self.compute)
+
+
+def run_stack(shape, L, steps, warmup, seed, dev, policy="LRU"):
+    """Decode `warmup + steps` tokens through an L-layer stack; TPOT over the last `steps`."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    S = DecodeStack(shape, L, warmup + steps, seed, dev, policy)
+    for s in range(warmup):
+        S.step(s)
+    torch.cuda.synchronize()
+    h0, f0, b0 = M.mcft_cache_stats(S.cache, -1)
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(True)
+    elapsed = time_steps(S.step, warmup, steps, S.compute)
+    M.mcft_profile_enable(False)
+    prof = M.mcft_profile_read()
+    M.mcft_device_error()
+    h1, f1, b1 = M.mcft_cache_stats(S.cache, -1)
+    hits, fetches = h1 - h0, f1 - f0
+    res = dict(workload=f"{shape.name} decode stack, {L} layers, batch 1, {policy}",
+               layers=L, policy=policy, steps=steps, warmup=warmup,
+               tpot_ms=elapsed * 1e3 / steps, tokens_per_s=steps / elapsed,
+               fetches_per_token=fetches / steps, hit_rate=hits / max(1, hits + fetches),
+               fetches_per_token_whole_stream=f1 / (warmup + steps),
+               hit_rate_whole_stream=h1 / max(1, h1 + f1),
+               fetch_gb_per_token=fetches * shape.expert_bytes / steps / 1e9,
+               kernel_ms_per_token=sum(v[1] for v in prof.values()) / steps,
+               gpu_launches=int(sum(v[0] for v in prof.values())),
+               kernels={k: dict(launches=v[0], ms=round(v[1], 3)) for k, v in prof.items() if v[0]},
+               host_pool="E distinct pinned blocks aliased by every layer")
+    del S
+    torch.cuda.empty_cache()
+    return res
 
 
 def run_prefill(steps, warmup, seed, dev, peaks):
@@ -422,7 +518,21 @@ def main():
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
     ap.add_argument("--case", choices=["decode16", "decode1", "prefill"],
                     help="run only a few resident-expert forwards (for profiler captures)")
+    ap.add_argument("--workload", default="layer", choices=["layer", "stack-mixtral", "stack-dsv2"],
+                    help="layer: the single-layer decode line; stack-*: the full decode stack")
+    ap.add_argument("--policy", default="LRU", choices=["LRU", "LFU", "FIFO"])
     args = ap.parse_args()
+    if args.workload != "layer":
+        import __graft_entry__
+
+        __graft_entry__.build()
+        torch.cuda.set_device(0)
+        shape, L = (I.MIXTRAL, 32) if args.workload == "stack-mixtral" else (I.DSV2_LITE, 26)
+        res = run_stack(shape, L, args.steps, args.warmup, 60, torch.device("cuda", 0), args.policy)
+        res.update(metric="masked MoE decode stack tokens/s", value=res["tokens_per_s"],
+                   unit="tokens/s", higher_is_better=True, dtype="bf16", data="synthetic")
+        print(json.dumps(res), flush=True)
+        return 0
     if args.case:
         import __graft_entry__
 
@@ -474,10 +584,7 @@ def main():
     max_el, tokens = aggregate(elapsed, batch * args.steps, world)
     pos = [s % STREAM_STEPS for s in range(args.warmup, args.warmup + args.steps)]
     U = unique_per_step([L.idx[p] for p in pos])
-    w13_bytes = 2 * shape.w * shape.d * 2
-    alg13 = sum(u * w13_bytes for u in U) + args.steps * (batch * shape.d * 2 + batch * shape.K * shape.w * 4)
-    n13, ms13 = prof["ffn13_rowwise"]
-    achieved = alg13 / (ms13 / 1e3) / 1e9 if ms13 else None
+    roof, rates = decode_roofline(prof, U, args.steps, batch, shape, peaks)
     hits, fetches, byp = h1 - h0, f1 - f0, b1 - b0
 
     e2e = run_decode_e2e(L, args.steps, args.warmup + args.steps)
@@ -486,12 +593,7 @@ def main():
         metric=METRIC, value=tokens / max_el, unit="tokens/s", n_gpus=world, steps=args.steps,
         warmup=args.warmup, ms_per_step=max_el * 1e3 / args.steps, higher_is_better=True,
         scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic", config=_config(batch),
-        roofline=dict(bound="hbm", achieved=achieved, peak=peaks["hbm"], unit="GB/s",
-                      frac=achieved / peaks["hbm"] if achieved else None,
-                      traffic=(traffic_ratio("ffn13_rowwise") * alg13 / max(1, n13)
-                               if traffic_ratio("ffn13_rowwise") else None),
-                      kernel="ffn13_rowwise", peak_source=peaks["src"] + " hbm_gbs",
-                      alg_bytes_per_launch=alg13 / max(1, n13)),
+        roofline=roof, kernel_gbs=rates,
         e2e=e2e, gpu_launches=int(sum(v[0] for v in prof.values())), clocks=clk.summary(),
         kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
         cache=dict(hits=hits, fetches=fetches, bypass=byp, fetches_per_step=fetches / args.steps,

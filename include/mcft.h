@@ -13,8 +13,8 @@
  *   y = sum_{i in A} g_i F_i(x)  (+ shared experts)             (Section 3.1, Eq. topk)
  *
  * with g_i from p (renormalised over A for Mixtral, p_i for DeepSeek), F_i a SwiGLU expert, and the
- * per-layer LRU cache of B experts of Section 4.1 ("Simulation"): misses counted per Eq. metrics and
- * fetched from pinned host memory.
+ * per-layer cache of B experts of Section 4.1 ("Simulation", LRU / LFU / FIFO replacement): misses
+ * counted per Eq. metrics and fetched from pinned host memory.
  *
  * Conventions for every call:
  *  - Device pointers are caller-owned CUDA device memory; host pointers are caller-owned host
@@ -152,14 +152,21 @@ mcft_status mcft_moe_forward_noalloc(const mcft_layer_desc* desc, const void* x,
  * Per-layer expert cache (Section 4.1 "Simulation"; Eq. metrics).
  * L layers, each with B slots for routed experts, K <= B < E. Caches start empty and persist
  * across calls; first fills count as misses. Per layer and decode step t:
- *   U = distinct experts selected by the step's tokens; cached experts of U are hits and get
- *   last_use = t; the others are misses, one fetch each, taken in ascending expert id: a miss
- *   takes the lowest free slot, else evicts the slot with the smallest (last_use, expert id)
- *   among slots not used at step t; if every slot was used at step t (possible only when |U| > B)
- *   the expert is fetched into a staging buffer for this step only ("bypass") and not cached.
- *   At batch size 1 this is the paper's LRU cache and f = K - h.
+ *   U = distinct experts selected by the step's tokens, each counting one access; cached experts
+ *   of U are hits and get last_use = t; the others are misses, one fetch each, taken in ascending
+ *   expert id: a miss takes the lowest free slot, else evicts, among slots not used at step t, the
+ *   one with the smallest policy key
+ *     LRU  (last_use, expert id)
+ *     LFU  (accesses of the expert since the stream began, last_use, expert id)
+ *     FIFO (step the expert was inserted, expert id);
+ *   if every slot was used at step t (possible only when |U| > B) the expert is fetched into a
+ *   staging buffer for this step only ("bypass") and not cached.
+ *   At batch size 1 this is the paper's cache and f = K - h.
  * Shared experts are not cached here (always resident, Section 4.1). */
 typedef struct mcft_cache mcft_cache;
+
+/* Replacement policy (Section 4.1: LRU, LFU, FIFO; Table 2). */
+typedef enum { MCFT_CACHE_LRU = 0, MCFT_CACHE_LFU = 1, MCFT_CACHE_FIFO = 2 } mcft_cache_policy;
 
 /* mcft_cache_create: allocate the device tag/timestamp/counter arrays, L*B device slots of
  * expert_bytes each, and the bypass staging buffers (min(E - B, max_assign) of them).
@@ -168,9 +175,11 @@ typedef struct mcft_cache mcft_cache;
  *                 pinned until mcft_cache_destroy. NULL = accounting only: no slots are
  *                 allocated and mcft_fetch_experts copies nothing.
  *   max_assign    largest T*K any mcft_cache_step call will pass.
- * Synchronous. Errors: MCFT_ERR_INVALID (B < 1, B >= E, E > 64, ...), MCFT_ERR_OOM. */
+ *   policy        mcft_cache_policy.
+ * Synchronous. Errors: MCFT_ERR_INVALID (B < 1, B >= E, E > 64, unknown policy, ...), MCFT_ERR_OOM. */
 mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
-                              const void* const* host_experts, int max_assign, mcft_cache** out);
+                              const void* const* host_experts, int max_assign, int policy,
+                              mcft_cache** out);
 
 /* mcft_cache_step: one decode step of one layer. Reads idx (device [T, K] int32), decides hits,
  * misses, evictions and bypasses on the device, updates the counters and writes the step's miss
@@ -207,8 +216,9 @@ mcft_status mcft_cache_stats(const mcft_cache* cache, int layer, uint64_t* hits,
  * Synchronises `stream` first. */
 mcft_status mcft_cache_tags(const mcft_cache* cache, int layer, int32_t* tags, mcft_stream_t stream);
 
-/* mcft_cache_export / mcft_cache_import: checkpoint of the whole cache state (tags, timestamps,
- * step counters, counters); import into a cache created with the same L, E, B resumes a stream
+/* mcft_cache_export / mcft_cache_import: checkpoint of the whole cache state (tags, last-use and
+ * insertion steps, access counts, step counters, counters); import into a cache created with the
+ * same L, E, B and policy resumes a stream
  * with identical decisions. Slot contents are not part of the state: after an import, the slots
  * the tags name must be refilled by the caller (or the cache used in accounting mode).
  * export with buf = NULL writes the needed size to *bytes. Both synchronise `stream`. */

@@ -1,38 +1,64 @@
-"""Per-layer expert cache oracle: LRU replacement, fetch accounting and metrics.
+"""Per-layer expert cache oracle: LRU / LFU / FIFO replacement, fetch accounting and metrics.
 
 Section 4.1 "Simulation": each layer keeps B routed experts (K <= B < E); caches start empty and
 persist; first fills count as misses; each miss is one expert fetch plus, when the cache is full, an
-eviction; the hit rate and fetches per token follow Eq. metrics (f = K - h at batch size 1).
+eviction under LRU, LFU or FIFO; the hit rate and fetches per token follow Eq. metrics (f = K - h at
+batch size 1).
 
 The paper only runs batch size 1 with K distinct experts per step. The rule used for any batch, per
 layer and decode step t (it reduces to the paper's at batch 1):
 
-1. U = the distinct experts chosen by any token of the step.
+1. U = the distinct experts chosen by any token of the step; each expert of U counts one access.
 2. Every expert of U already cached is a hit and gets last_use = t.
 3. The other experts of U are misses, taken in ascending expert id. Each is one fetch. It goes to
-   the lowest-numbered free slot if there is one; otherwise it replaces the slot whose
-   (last_use, expert id) is smallest among slots with last_use < t; if every slot was used at step t
-   (only possible when |U| > B) the expert is fetched for this step only ("bypass") and not cached.
+   the lowest-numbered free slot if there is one; otherwise it replaces, among slots with
+   last_use < t (not used at this step), the one with the smallest policy key:
+     LRU:  (last_use, expert id)
+     LFU:  (accesses of the expert since the stream began, last_use, expert id)
+     FIFO: (step the expert was inserted, expert id)
+   If every slot was used at step t (only possible when |U| > B) the expert is fetched for this
+   step only ("bypass") and not cached.
 4. h = |U and cache|, f = |U| - h.
 
-Two independent formulations are given: ``LRUStamps`` (per-slot timestamps and an argmin) and
-``LRUList`` (a recency-ordered list). Tests require them to agree.
+Readings: LFU counts persist across evictions (the paper evicts "the least frequently accessed
+experts"); FIFO hits do not refresh the insertion order; ties always fall to the older use and
+then the lower expert id.
+
+Two independent formulations are given: ``SlotCache`` (per-slot arrays and an argmin of the policy
+key) and ``OrderedCache`` (an ordered list of cached experts kept in victim order). Tests require
+them to agree.
 """
 from __future__ import annotations
 
 import numpy as np
 
 
-class LRUStamps:
-    """LRU cache of B slots as tag/timestamp arrays; victim = argmin (last_use, expert id)."""
+POLICIES = ("LRU", "LFU", "FIFO")
 
-    def __init__(self, E: int, B: int):
+
+class SlotCache:
+    """B slots as tag / last-use / insertion arrays plus per-expert access counts; the victim is the
+    argmin of the policy key over slots not used at this step."""
+
+    def __init__(self, E: int, B: int, policy: str = "LRU"):
         if not (0 < B < E):
             raise ValueError("need 0 < B < E")
-        self.E, self.B = E, B
+        if policy not in POLICIES:
+            raise ValueError(f"unknown policy {policy}")
+        self.E, self.B, self.policy = E, B, policy
         self.tag = [-1] * B
         self.last = [-1] * B
+        self.ins = [-1] * B
+        self.freq = [0] * E
         self.t = 0
+
+    def _key(self, s):
+        e = self.tag[s]
+        if self.policy == "LRU":
+            return (self.last[s], e)
+        if self.policy == "LFU":
+            return (self.freq[e], self.last[s], e)
+        return (self.ins[s], e)
 
     def step(self, ids):
         """Process one decode step given every expert id chosen by its tokens.
@@ -45,6 +71,8 @@ class LRUStamps:
         for e in U:
             if not 0 <= e < self.E:
                 raise ValueError(f"expert id {e} out of range")
+        for e in U:
+            self.freq[e] += 1
         hits = 0
         for s in range(self.B):
             if self.tag[s] in U:
@@ -62,72 +90,129 @@ class LRUStamps:
                 if not cand:
                     misses.append((e, -1))
                     continue
-                slot = min(cand, key=lambda s: (self.last[s], self.tag[s]))
+                slot = min(cand, key=self._key)
             self.tag[slot] = e
             self.last[slot] = t
+            self.ins[slot] = t
             misses.append((e, slot))
         self.t += 1
         bypass = sum(1 for _, s in misses if s < 0)
         return hits, len(misses), bypass, misses
 
 
-class LRUList:
-    """LRU cache of B slots as a list ordered from least to most recently used.
-
-    Within one step, the experts touched are appended in ascending id, so among experts last used
-    in the same step the lower id is evicted first.
-    """
+class LRUStamps(SlotCache):
+    """SlotCache with LRU replacement."""
 
     def __init__(self, E: int, B: int):
+        super().__init__(E, B, "LRU")
+
+
+class OrderedCache:
+    """Cached experts kept in a list ordered by eviction preference (first = next victim).
+
+    LRU: touched experts move to the end; FIFO: only insertions append; LFU: the list is kept
+    sorted by (accesses, last use, id) by re-inserting an expert at its place (bisection) whenever
+    it is touched. Experts touched in the current step are never victims.
+    """
+
+    def __init__(self, E: int, B: int, policy: str = "LRU"):
         if not (0 < B < E):
             raise ValueError("need 0 < B < E")
-        self.E, self.B = E, B
-        self.order = []          # experts, least recently used first
+        if policy not in POLICIES:
+            raise ValueError(f"unknown policy {policy}")
+        self.E, self.B, self.policy = E, B, policy
+        self.order = []          # cached experts, next victim first
+        self.keys = []           # LFU only: sort keys parallel to order
         self.slot_of = {}        # expert -> slot
         self.free = list(range(B))
+        self.count = [0] * E
+        self.t = 0
+
+    def _place(self, e):
+        """(Re)insert e at its position in the victim order after it was touched at step t."""
+        if self.policy == "LFU":
+            k = (self.count[e], self.t, e)
+            lo, hi = 0, len(self.keys)
+            while lo < hi:
+                mid = (lo + hi) // 2
+                if self.keys[mid] < k:
+                    lo = mid + 1
+                else:
+                    hi = mid
+            self.keys.insert(lo, k)
+            self.order.insert(lo, e)
+        else:
+            self.order.append(e)
+
+    def _remove(self, e):
+        i = self.order.index(e)
+        self.order.pop(i)
+        if self.policy == "LFU":
+            self.keys.pop(i)
 
     def step(self, ids):
         U = sorted(set(int(e) for e in np.asarray(ids).reshape(-1)))
         for e in U:
             if not 0 <= e < self.E:
                 raise ValueError(f"expert id {e} out of range")
-        touched = [e for e in U if e in self.slot_of]
-        hits = len(touched)
-        for e in touched:
-            self.order.remove(e)
+        for e in U:
+            self.count[e] += 1
+        touched = set()
+        hits = 0
+        for e in U:
+            if e in self.slot_of:
+                hits += 1
+                touched.add(e)
+                if self.policy != "FIFO":
+                    self._remove(e)
+                    self._place(e)
         misses = []
         for e in U:
             if e in self.slot_of:
                 continue
             if self.free:
                 slot = self.free.pop(0)
-            elif self.order:
-                victim = self.order.pop(0)
-                slot = self.slot_of.pop(victim)
             else:
-                misses.append((e, -1))
-                continue
+                victim = next((v for v in self.order if v not in touched), None)
+                if victim is None:
+                    misses.append((e, -1))
+                    continue
+                self._remove(victim)
+                slot = self.slot_of.pop(victim)
             self.slot_of[e] = slot
-            touched.append(e)
+            touched.add(e)
+            self._place(e)
             misses.append((e, slot))
-        self.order.extend(sorted(touched))
+        if self.policy == "LRU":
+            # experts touched in one step: lower id first (older) among equal last use
+            tail = [v for v in self.order if v in touched]
+            head = [v for v in self.order if v not in touched]
+            self.order = head + sorted(tail)
+        self.t += 1
         bypass = sum(1 for _, s in misses if s < 0)
         return hits, len(misses), bypass, misses
 
     def state(self):
-        """(tag per slot) for comparison with LRUStamps."""
+        """(tag per slot) for comparison with SlotCache."""
         tag = [-1] * self.B
         for e, s in self.slot_of.items():
             tag[s] = e
         return tag
 
 
-def simulate(steps_ids, E: int, B: int, cls=LRUStamps):
+class LRUList(OrderedCache):
+    """OrderedCache with LRU replacement."""
+
+    def __init__(self, E: int, B: int):
+        super().__init__(E, B, "LRU")
+
+
+def simulate(steps_ids, E: int, B: int, cls=SlotCache, policy: str = "LRU"):
     """Run one layer's cache over a stream of steps; steps_ids[t] holds the ids chosen at step t.
 
     Returns per-step arrays hits, fetches, bypass and the list of per-step miss lists.
     """
-    c = cls(E, B)
+    c = cls(E, B, policy)
     h, f, b, ml = [], [], [], []
     for ids in steps_ids:
         hi, fi, bi, mi = c.step(ids)

@@ -99,6 +99,8 @@ unsigned* device_error_word() {
 WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T) {
   WsLayout L{};
   L.tc = dtype == MCFT_BF16 && T > 64 && d % 256 == 0 && w % 128 == 0;
+  L.decode = !L.tc && dtype == MCFT_BF16;
+  L.ks = L.decode ? decode_ksplit(T) : 1;
   L.pad = L.tc ? 128 : 1;
   const int nseg = E + S;
   L.mcap = T * K + S * T + (L.tc ? nseg * (L.pad - 1) : 0);
@@ -109,8 +111,8 @@ WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T) {
   L.pos = o;  o = align256(o + sizeof(int) * size_t(T) * K);
   L.perm = o; o = align256(o + sizeof(int) * size_t(L.mcap));
   L.xp = o;   o = align256(o + (L.tc ? size_t(L.mcap) * d * 2 : 0));
-  L.h = o;    o = align256(o + size_t(L.mcap) * w * (L.tc ? 2 : 4));
-  L.o = o;    o = align256(o + size_t(L.mcap) * d * 4);
+  L.h = o;    o = align256(o + size_t(L.mcap) * w * (dtype == MCFT_BF16 ? 2 : 4));
+  L.o = o;    o = align256(o + size_t(L.ks) * L.mcap * d * 4);
   L.total = o;
   return L;
 }
@@ -123,11 +125,13 @@ using namespace mcft;
 // Expert cache object
 
 struct mcft_cache {
-  int L = 0, E = 0, B = 0, max_assign = 0, n_staging = 0, device = 0;
+  int L = 0, E = 0, B = 0, max_assign = 0, n_staging = 0, device = 0, policy = 0;
   size_t expert_bytes = 0;
   std::vector<const void*> host_experts;  // [L*E] pinned host blocks (empty: accounting only)
   int32_t* d_tag = nullptr;
   int64_t* d_last = nullptr;
+  int64_t* d_ins = nullptr;
+  int64_t* d_freq = nullptr;
   int64_t* d_step = nullptr;
   unsigned long long* d_cnt = nullptr;
   int32_t* h_miss = nullptr;  // host-mapped [L][miss_stride]
@@ -145,6 +149,8 @@ void cache_free(mcft_cache* c) {
   if (!c) return;
   cudaFree(c->d_tag);
   cudaFree(c->d_last);
+  cudaFree(c->d_ins);
+  cudaFree(c->d_freq);
   cudaFree(c->d_step);
   cudaFree(c->d_cnt);
   if (c->h_miss) cudaFreeHost(c->h_miss);
@@ -163,9 +169,16 @@ const char* loc_ptr(const mcft_cache* c, int layer, int loc) {
 }
 
 struct CacheStateHeader {
-  uint32_t magic, L, E, B;
+  uint32_t magic, L, E, B, policy, pad;
 };
-constexpr uint32_t kStateMagic = 0x4d434654u;  // "MCFT"
+constexpr uint32_t kStateMagic = 0x4d434655u;
+
+// Bytes of the exported state: header, tag [L*B] i32, last and ins [L*B] i64, freq [L*E] i64,
+// step [L] i64, counters [L*3] u64.
+size_t state_bytes(const mcft_cache* c) {
+  const size_t LB = size_t(c->L) * c->B, LE = size_t(c->L) * c->E;
+  return sizeof(CacheStateHeader) + LB * 4 + LB * 8 * 2 + LE * 8 + size_t(c->L) * 8 + size_t(c->L) * 24;
+}
 
 }  // namespace
 
@@ -239,9 +252,12 @@ mcft_status mcft_moe_workspace_size(const mcft_layer_desc* desc, int T_max, size
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (T_max < 0 || !bytes) return fail(MCFT_ERR_INVALID, "T_max < 0 or bytes is NULL");
+  // the largest layout over every T <= T_max (the decode path's split depends on T)
   size_t best = 0;
-  for (int T : {T_max, T_max < 64 ? T_max : 64}) {
-    const WsLayout L = ws_layout(desc->d, desc->E, desc->K, desc->w, desc->n_shared, desc->dtype, T);
+  const int upto = T_max < 64 ? T_max : 64;
+  for (int T = 0; T <= upto + 1; ++T) {
+    const int t = T <= upto ? T : T_max;
+    const WsLayout L = ws_layout(desc->d, desc->E, desc->K, desc->w, desc->n_shared, desc->dtype, t);
     if (L.total > best) best = L.total;
   }
   *bytes = best;
@@ -295,6 +311,8 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
   for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
   fa.h = ws + L.h;
   fa.o = reinterpret_cast<float*>(ws + L.o);
+  fa.o_plane = size_t(L.mcap) * desc->d;
+  fa.ksplit = L.ks;
   fa.T = T;
   fa.d = desc->d;
   fa.w = desc->w;
@@ -307,11 +325,14 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
     if (e != cudaSuccess) return cuda_fail(e, "gather kernel launch");
     e = launch_ffn_tc(fa, ws + L.xp, L.mcap, num_sms(), stream);
     if (e != cudaSuccess) return cuda_fail(e, "tensor-core expert GEMM launch");
+  } else if (L.decode) {
+    e = launch_ffn_decode(fa, num_sms(), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "decode expert FFN launch");
   } else {
     e = launch_ffn_rowwise(fa, desc->dtype, num_sms(), stream);
     if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
   }
-  CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S};
+  CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S, L.ks, fa.o_plane};
   e = launch_combine(ca, desc->dtype, stream);
   if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
   return MCFT_OK;
@@ -320,7 +341,8 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
 // ------------------------------------------------------------------------------------------------
 
 mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
-                              const void* const* host_experts, int max_assign, mcft_cache** out) {
+                              const void* const* host_experts, int max_assign, int policy,
+                              mcft_cache** out) {
   if (!out) return fail(MCFT_ERR_INVALID, "out is NULL");
   *out = nullptr;
   if (L <= 0) return fail(MCFT_ERR_INVALID, "L = %d must be positive", L);
@@ -328,6 +350,8 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   if (E > kMaxE) return fail(MCFT_ERR_UNSUPPORTED, "E = %d > %d", E, kMaxE);
   if (B < 1 || B >= E) return fail(MCFT_ERR_INVALID, "need 1 <= B < E (B = %d, E = %d)", B, E);
   if (max_assign < 1) return fail(MCFT_ERR_INVALID, "max_assign = %d must be positive", max_assign);
+  if (policy != MCFT_CACHE_LRU && policy != MCFT_CACHE_LFU && policy != MCFT_CACHE_FIFO)
+    return fail(MCFT_ERR_INVALID, "unknown cache policy %d", policy);
   if (host_experts) {
     if (expert_bytes == 0 || expert_bytes % 16)
       return fail(MCFT_ERR_INVALID, "expert_bytes = %zu must be a positive multiple of 16", expert_bytes);
@@ -339,6 +363,7 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   c->E = E;
   c->B = B;
   c->max_assign = max_assign;
+  c->policy = policy;
   c->expert_bytes = expert_bytes;
   c->device = current_device();
   c->miss_stride = (1 + 3 * E + 3) & ~3;
@@ -353,10 +378,14 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   } while (0)
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_tag, sizeof(int32_t) * L * B));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_last, sizeof(int64_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_ins, sizeof(int64_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_freq, sizeof(int64_t) * L * E));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_step, sizeof(int64_t) * L));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_cnt, sizeof(unsigned long long) * L * 3));
   MCFT_CACHE_CUDA(cudaMemset(c->d_tag, 0xff, sizeof(int32_t) * L * B));  // -1 = empty
   MCFT_CACHE_CUDA(cudaMemset(c->d_last, 0xff, sizeof(int64_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_ins, 0xff, sizeof(int64_t) * L * B));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_freq, 0, sizeof(int64_t) * L * E));
   MCFT_CACHE_CUDA(cudaMemset(c->d_step, 0, sizeof(int64_t) * L));
   MCFT_CACHE_CUDA(cudaMemset(c->d_cnt, 0, sizeof(unsigned long long) * L * 3));
   MCFT_CACHE_CUDA(cudaHostAlloc(&c->h_miss, sizeof(int32_t) * L * c->miss_stride, cudaHostAllocMapped));
@@ -385,8 +414,9 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
   if (T < 1 || K < 1 || K > c->E) return fail(MCFT_ERR_INVALID, "bad T = %d or K = %d", T, K);
   if (T * K > c->max_assign)
     return fail(MCFT_ERR_INVALID, "T*K = %d exceeds max_assign = %d", T * K, c->max_assign);
-  CacheStepArgs a{idx, T * K, c->E, c->B, layer, c->d_tag, c->d_last, c->d_step, c->d_cnt,
-                  c->d_miss + size_t(layer) * c->miss_stride, device_error_word()};
+  CacheStepArgs a{idx, T * K, c->E, c->B, layer, c->policy, c->d_tag, c->d_last, c->d_ins,
+                  c->d_freq, c->d_step, c->d_cnt, c->d_miss + size_t(layer) * c->miss_stride,
+                  device_error_word()};
   cudaError_t e = launch_cache_step(a, stream);
   if (e != cudaSuccess) return cuda_fail(e, "cache step launch");
   MCFT_CUDA(cudaEventRecord(c->ev_step[layer], stream));
@@ -466,24 +496,24 @@ mcft_status mcft_cache_tags(const mcft_cache* c, int layer, int32_t* tags, mcft_
 
 mcft_status mcft_cache_export(const mcft_cache* c, void* buf, size_t* bytes, mcft_stream_t stream) {
   if (!c || !bytes) return fail(MCFT_ERR_INVALID, "NULL argument");
-  const size_t LB = size_t(c->L) * c->B;
-  const size_t need = sizeof(CacheStateHeader) + LB * 4 + LB * 8 + size_t(c->L) * 8 + size_t(c->L) * 24;
+  const size_t LB = size_t(c->L) * c->B, LE = size_t(c->L) * c->E;
+  const size_t need = state_bytes(c);
   if (!buf) {
     *bytes = need;
     return MCFT_OK;
   }
   if (*bytes < need) return fail(MCFT_ERR_INVALID, "buffer of %zu bytes < %zu needed", *bytes, need);
   char* p = static_cast<char*>(buf);
-  CacheStateHeader h{kStateMagic, uint32_t(c->L), uint32_t(c->E), uint32_t(c->B)};
+  CacheStateHeader h{kStateMagic, uint32_t(c->L), uint32_t(c->E), uint32_t(c->B), uint32_t(c->policy), 0};
   memcpy(p, &h, sizeof(h));
   p += sizeof(h);
-  MCFT_CUDA(cudaMemcpyAsync(p, c->d_tag, LB * 4, cudaMemcpyDeviceToHost, stream));
-  p += LB * 4;
-  MCFT_CUDA(cudaMemcpyAsync(p, c->d_last, LB * 8, cudaMemcpyDeviceToHost, stream));
-  p += LB * 8;
-  MCFT_CUDA(cudaMemcpyAsync(p, c->d_step, size_t(c->L) * 8, cudaMemcpyDeviceToHost, stream));
-  p += size_t(c->L) * 8;
-  MCFT_CUDA(cudaMemcpyAsync(p, c->d_cnt, size_t(c->L) * 24, cudaMemcpyDeviceToHost, stream));
+  const struct { const void* src; size_t n; } parts[] = {
+      {c->d_tag, LB * 4}, {c->d_last, LB * 8}, {c->d_ins, LB * 8}, {c->d_freq, LE * 8},
+      {c->d_step, size_t(c->L) * 8}, {c->d_cnt, size_t(c->L) * 24}};
+  for (const auto& part : parts) {
+    MCFT_CUDA(cudaMemcpyAsync(p, part.src, part.n, cudaMemcpyDeviceToHost, stream));
+    p += part.n;
+  }
   MCFT_CUDA(cudaStreamSynchronize(stream));
   *bytes = need;
   return MCFT_OK;
@@ -491,25 +521,26 @@ mcft_status mcft_cache_export(const mcft_cache* c, void* buf, size_t* bytes, mcf
 
 mcft_status mcft_cache_import(mcft_cache* c, const void* buf, size_t bytes, mcft_stream_t stream) {
   if (!c || !buf) return fail(MCFT_ERR_INVALID, "NULL argument");
-  const size_t LB = size_t(c->L) * c->B;
-  const size_t need = sizeof(CacheStateHeader) + LB * 4 + LB * 8 + size_t(c->L) * 8 + size_t(c->L) * 24;
+  const size_t LB = size_t(c->L) * c->B, LE = size_t(c->L) * c->E;
+  const size_t need = state_bytes(c);
   if (bytes < need) return fail(MCFT_ERR_INVALID, "state of %zu bytes < %zu expected", bytes, need);
   const char* p = static_cast<const char*>(buf);
   CacheStateHeader h;
   memcpy(&h, p, sizeof(h));
-  if (h.magic != kStateMagic || h.L != uint32_t(c->L) || h.E != uint32_t(c->E) || h.B != uint32_t(c->B))
-    return fail(MCFT_ERR_INVALID, "state was exported from a cache of another shape");
+  if (h.magic != kStateMagic || h.L != uint32_t(c->L) || h.E != uint32_t(c->E) ||
+      h.B != uint32_t(c->B) || h.policy != uint32_t(c->policy))
+    return fail(MCFT_ERR_INVALID, "state was exported from a cache of another shape or policy");
   p += sizeof(h);
   const int32_t* tags = reinterpret_cast<const int32_t*>(p);
   for (size_t i = 0; i < LB; ++i)
     if (tags[i] < -1 || tags[i] >= c->E) return fail(MCFT_ERR_INVALID, "corrupt tag in state");
-  MCFT_CUDA(cudaMemcpyAsync(c->d_tag, p, LB * 4, cudaMemcpyHostToDevice, stream));
-  p += LB * 4;
-  MCFT_CUDA(cudaMemcpyAsync(c->d_last, p, LB * 8, cudaMemcpyHostToDevice, stream));
-  p += LB * 8;
-  MCFT_CUDA(cudaMemcpyAsync(c->d_step, p, size_t(c->L) * 8, cudaMemcpyHostToDevice, stream));
-  p += size_t(c->L) * 8;
-  MCFT_CUDA(cudaMemcpyAsync(c->d_cnt, p, size_t(c->L) * 24, cudaMemcpyHostToDevice, stream));
+  const struct { void* dst; size_t n; } parts[] = {
+      {c->d_tag, LB * 4}, {c->d_last, LB * 8}, {c->d_ins, LB * 8}, {c->d_freq, LE * 8},
+      {c->d_step, size_t(c->L) * 8}, {c->d_cnt, size_t(c->L) * 24}};
+  for (const auto& part : parts) {
+    MCFT_CUDA(cudaMemcpyAsync(part.dst, p, part.n, cudaMemcpyHostToDevice, stream));
+    p += part.n;
+  }
   MCFT_CUDA(cudaStreamSynchronize(stream));
   return MCFT_OK;
 }

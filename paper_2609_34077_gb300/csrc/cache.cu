@@ -1,10 +1,12 @@
 // Per-layer expert cache decision kernel (Section 4.1 "Simulation", Eq. metrics).
 //
 // One warp per call: the lanes gather the distinct experts of the step (a 64-bit set) from the
-// routing output, then lane 0 applies the LRU rule on the layer's device-resident tag and
-// timestamp arrays: hits refresh, misses in ascending expert id take the lowest free slot or evict
-// the smallest (last_use, expert id) among slots not used this step, else go to a staging buffer
-// for this step only (bypass). The miss list and the expert -> location map are written straight
+// routing output, then lane 0 applies the replacement rule on the layer's device-resident tag,
+// last-use, insertion and access-count arrays: every expert of the step counts one access, hits
+// refresh their last use, misses in ascending expert id take the lowest free slot or evict, among
+// slots not used this step, the smallest key of the policy (LRU: last use, expert id; LFU: access
+// count, last use, expert id; FIFO: insertion step, expert id), else go to a staging buffer for
+// this step only (bypass). The miss list and the expert -> location map are written straight
 // into host-mapped pinned memory, so the host can issue the fetches as soon as the step's event
 // completes.
 #include "common.cuh"
@@ -12,6 +14,21 @@
 
 namespace mcft {
 namespace {
+
+// True when slot s precedes slot v in eviction order under the policy's key.
+__device__ __forceinline__ bool victim_before(int policy, int s, int v, const int32_t* tag,
+                                              const int64_t* last, const int64_t* ins,
+                                              const int64_t* freq) {
+  if (policy == MCFT_CACHE_LFU) {
+    const int64_t fs = freq[tag[s]], fv = freq[tag[v]];
+    if (fs != fv) return fs < fv;
+  } else if (policy == MCFT_CACHE_FIFO) {
+    if (ins[s] != ins[v]) return ins[s] < ins[v];
+    return tag[s] < tag[v];
+  }
+  if (last[s] != last[v]) return last[s] < last[v];
+  return tag[s] < tag[v];
+}
 
 __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ CacheStepArgs a) {
   const int lane = threadIdx.x;
@@ -37,12 +54,17 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
   const int B = a.B, E = a.E;
   int32_t* tag = a.tag + size_t(a.layer) * B;
   int64_t* last = a.last + size_t(a.layer) * B;
+  int64_t* ins = a.ins + size_t(a.layer) * B;
+  int64_t* freq = a.freq + size_t(a.layer) * E;
   const int64_t t = a.step[a.layer];
   int32_t* out = a.miss_out;
   int32_t* m_exp = out + 1;
   int32_t* m_loc = out + 1 + E;
   int32_t* loc_of = out + 1 + 2 * E;
-  for (int e = 0; e < E; ++e) loc_of[e] = -1;
+  for (int e = 0; e < E; ++e) {
+    loc_of[e] = -1;
+    if ((mine >> e) & 1ull) freq[e] += 1;
+  }
 
   unsigned long long cached = 0;
   int hits = 0;
@@ -66,9 +88,8 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
       if (tag[s] < 0) { slot = s; break; }
     if (slot < 0) {
       for (int s = 0; s < B; ++s) {
-        if (last[s] >= t) continue;
-        if (slot < 0 || last[s] < last[slot] || (last[s] == last[slot] && tag[s] < tag[slot]))
-          slot = s;
+        if (last[s] >= t) continue;  // used at this step: never a victim
+        if (slot < 0 || victim_before(a.policy, s, slot, tag, last, ins, freq)) slot = s;
       }
     }
     if (slot < 0) {
@@ -79,6 +100,7 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
     } else {
       tag[slot] = e;
       last[slot] = t;
+      ins[slot] = t;
       m_exp[nm] = e;
       m_loc[nm] = slot;
       loc_of[e] = slot;

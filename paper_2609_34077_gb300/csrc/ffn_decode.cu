@@ -1,0 +1,294 @@
+// Decode-batch expert FFN (bf16, at most 64 tokens per call): HBM-streaming, one CTA per block of
+// 16 weight rows, token products on the tensor cores with mma.sync m16n8k16.
+//
+// F(x) = W2 (silu(W1 x) * (W3 x)) for each expert segment (Section 3.1, SwiGLU experts). At
+// decode the selected experts' weights are the only large operand, so the kernels are built to
+// read every weight byte once, in whole lines, with many loads in flight:
+//  * a CTA item is 16 consecutive rows of W1 and W3 (GEMM13) or of W2 (GEMM2) of one segment; its
+//    8 warps split the contraction dimension into 8 slices and walk their slice 64 elements at a
+//    time; in each load instruction the 4 lanes of a quad read 64 contiguous bytes of one row;
+//  * the 16 x 64 weight slab is the A operand of four m16n8k16 MMAs (the contraction order inside
+//    a 64-wide chunk is permuted identically for A and B, which leaves every dot product intact);
+//    the B operand is 8 tokens of the segment, so one A fragment serves up to 32 tokens per pass
+//    (segments of more tokens take a second pass, whose weight reads hit L2);
+//  * the 8 partial sums are added in shared memory in a fixed order (deterministic); GEMM13 then
+//    applies silu(gate) * up and stores h in bf16; GEMM2 stores fp32 outputs. At small batches
+//    GEMM2 also splits the contraction across `ksplit` CTAs (partial planes of o, summed in the
+//    combine kernel) so that few selected experts still give every SM work.
+// Items are spread over a persistent grid.
+#include "common.cuh"
+#include "internal.h"
+
+namespace mcft {
+namespace {
+
+constexpr int kWarps = 8;
+constexpr int kRows = 16;        // weight rows per CTA item
+constexpr int kChunk = 64;       // contraction elements per step (128 bytes of a row)
+constexpr int kPassTokens = 32;  // tokens per pass (4 MMA column groups of 8)
+constexpr int kMaxNG = kPassTokens / 8;
+
+struct DecItems {
+  int nseg, total, ksplit;
+  int off[kMaxSeg + 1];
+  int first[kMaxSeg + 1];
+};
+
+__device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows_per_seg, int ksplit) {
+  if (threadIdx.x == 0) {
+    const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
+    it.nseg = nseg;
+    it.ksplit = ksplit;
+    int acc = 0;
+    for (int s = 0; s <= nseg; ++s) it.off[s] = a.off[s];
+    for (int s = 0; s < nseg; ++s) {
+      it.first[s] = acc;
+      if (it.off[s + 1] > it.off[s]) {
+        if (a.wblk[s] == nullptr) {  // a selected expert without weights
+          set_error(a.err, kErrInvalid);
+          const_cast<WsHeader*>(a.hdr)->abort = 1;
+          continue;
+        }
+        acc += rows_per_seg / kRows * ksplit;
+      }
+    }
+    it.first[nseg] = acc;
+    it.total = acc;
+  }
+  __syncthreads();
+}
+
+__device__ __forceinline__ int dec_seg(const DecItems& it, int item) {
+  int s = 0;
+  while (s + 1 < it.nseg && it.first[s + 1] <= item) ++s;
+  return s;
+}
+
+__device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// A lane of quad position c holds elements 8c..8c+7 (lo) and 32+8c..32+8c+7 (hi) of a 64-wide
+// chunk. MMA step j (0..3) uses 32-bit words 2j and 2j+1 of (lo, hi): for each c these are 4
+// elements, and over the 4 lanes of the quad and the 4 steps every element is used exactly once.
+__device__ __forceinline__ uint32_t word(const uint4& lo, const uint4& hi, int i) {
+  switch (i) {
+    case 0: return lo.x;
+    case 1: return lo.y;
+    case 2: return lo.z;
+    case 3: return lo.w;
+    case 4: return hi.x;
+    case 5: return hi.y;
+    case 6: return hi.z;
+    default: return hi.w;
+  }
+}
+
+// Chunks [c0, c1) of this warp's slice of a contraction of nch chunks.
+__device__ __forceinline__ void warp_slice(int nch, int parts, int part, int& c0, int& c1) {
+  const int per = (nch + parts - 1) / parts;
+  c0 = min(nch, part * per);
+  c1 = min(nch, c0 + per);
+}
+
+// GEMM13 + SwiGLU for 16 rows (r0..r0+15) and n <= 32 tokens of one segment starting at
+// permuted row q0. red: shared scratch [kWarps][kMaxNG][8][32] floats.
+template <int NG>
+__device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, int r0, int q0, int n,
+                                           float* red) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const size_t rowb = size_t(a.d) * 2;
+  const char* w1g = blk + size_t(r0 + g) * rowb + c * 16;
+  const char* w1h = w1g + 8 * rowb;
+  const char* w3g = blk + size_t(a.w + r0 + g) * rowb + c * 16;
+  const char* w3h = w3g + 8 * rowb;
+  const char* xr[NG];
+#pragma unroll
+  for (int G = 0; G < NG; ++G) {
+    const int j = G * 8 + g;
+    const int t = a.perm[q0 + (j < n ? j : 0)];
+    xr[G] = reinterpret_cast<const char*>(a.x) + size_t(t) * rowb + c * 16;
+  }
+  float accg[NG][4], accu[NG][4];
+#pragma unroll
+  for (int G = 0; G < NG; ++G)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) accg[G][i] = accu[G][i] = 0.f;
+
+  int c0, c1;
+  warp_slice(int(rowb / (kChunk * 2)), kWarps, warp, c0, c1);
+  for (int ch = c0; ch < c1; ++ch) {
+    const size_t k = size_t(ch) * kChunk * 2;
+    const uint4 ag0 = ld_stream16(w1g + k), ag1 = ld_stream16(w1g + k + 64);
+    const uint4 ah0 = ld_stream16(w1h + k), ah1 = ld_stream16(w1h + k + 64);
+    const uint4 bg0 = ld_stream16(w3g + k), bg1 = ld_stream16(w3g + k + 64);
+    const uint4 bh0 = ld_stream16(w3h + k), bh1 = ld_stream16(w3h + k + 64);
+#pragma unroll
+    for (int G = 0; G < NG; ++G) {
+      const uint4 x0 = ldg16(xr[G] + k), x1 = ldg16(xr[G] + k + 64);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t xb0 = word(x0, x1, 2 * j), xb1 = word(x0, x1, 2 * j + 1);
+        mma16816(accg[G], word(ag0, ag1, 2 * j), word(ah0, ah1, 2 * j), word(ag0, ag1, 2 * j + 1),
+                 word(ah0, ah1, 2 * j + 1), xb0, xb1);
+        mma16816(accu[G], word(bg0, bg1, 2 * j), word(bh0, bh1, 2 * j), word(bg0, bg1, 2 * j + 1),
+                 word(bh0, bh1, 2 * j + 1), xb0, xb1);
+      }
+    }
+  }
+#pragma unroll
+  for (int G = 0; G < NG; ++G)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      red[((warp * kMaxNG + G) * 8 + i) * 32 + lane] = accg[G][i];
+      red[((warp * kMaxNG + G) * 8 + 4 + i) * 32 + lane] = accu[G][i];
+    }
+  __syncthreads();
+  // warp G adds the 8 slices of column group G; accumulator element i: row g (i < 2) or g + 8,
+  // token column 2c + (i & 1)
+  if (warp < NG) {
+    const int G = warp;
+    uint16_t* h = reinterpret_cast<uint16_t*>(a.h);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float sg = 0.f, su = 0.f;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        sg += red[((w * kMaxNG + G) * 8 + i) * 32 + lane];
+        su += red[((w * kMaxNG + G) * 8 + 4 + i) * 32 + lane];
+      }
+      const int j = G * 8 + 2 * c + (i & 1);
+      if (j < n) h[size_t(q0 + j) * a.w + r0 + g + (i >= 2 ? 8 : 0)] = f2bf(silu(sg) * su);
+    }
+  }
+  __syncthreads();
+}
+
+// GEMM2 for 16 output rows (r0..r0+15 of W2), contraction part `kp` of `ks`, and n <= 32 tokens.
+// red: shared scratch [kWarps][kMaxNG][4][32] floats. Output plane kp of o.
+template <int NG>
+__device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, int r0, int q0, int n,
+                                          int kp, int ks, float* red) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const size_t rowb = size_t(a.w) * 2;
+  const char* w2 = blk + size_t(2) * a.w * a.d * 2;
+  const char* wg = w2 + size_t(r0 + g) * rowb + c * 16;
+  const char* wh = wg + 8 * rowb;
+  const char* hr[NG];
+#pragma unroll
+  for (int G = 0; G < NG; ++G) {
+    const int j = G * 8 + g;
+    hr[G] = reinterpret_cast<const char*>(a.h) + size_t(q0 + (j < n ? j : 0)) * rowb + c * 16;
+  }
+  float acc[NG][4];
+#pragma unroll
+  for (int G = 0; G < NG; ++G)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[G][i] = 0.f;
+
+  int p0, p1, c0, c1;
+  warp_slice(int(rowb / (kChunk * 2)), ks, kp, p0, p1);
+  warp_slice(p1 - p0, kWarps, warp, c0, c1);
+#pragma unroll 2
+  for (int ch = p0 + c0; ch < p0 + c1; ++ch) {
+    const size_t k = size_t(ch) * kChunk * 2;
+    const uint4 ag0 = ld_stream16(wg + k), ag1 = ld_stream16(wg + k + 64);
+    const uint4 ah0 = ld_stream16(wh + k), ah1 = ld_stream16(wh + k + 64);
+#pragma unroll
+    for (int G = 0; G < NG; ++G) {
+      const uint4 x0 = ldg16(hr[G] + k), x1 = ldg16(hr[G] + k + 64);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        mma16816(acc[G], word(ag0, ag1, 2 * j), word(ah0, ah1, 2 * j), word(ag0, ag1, 2 * j + 1),
+                 word(ah0, ah1, 2 * j + 1), word(x0, x1, 2 * j), word(x0, x1, 2 * j + 1));
+    }
+  }
+#pragma unroll
+  for (int G = 0; G < NG; ++G)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) red[((warp * kMaxNG + G) * 4 + i) * 32 + lane] = acc[G][i];
+  __syncthreads();
+  if (warp < NG) {
+    const int G = warp;
+    float* o = a.o + size_t(kp) * a.o_plane;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float sum = 0.f;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) sum += red[((w * kMaxNG + G) * 4 + i) * 32 + lane];
+      const int j = G * 8 + 2 * c + (i & 1);
+      if (j < n) o[size_t(q0 + j) * a.d + r0 + g + (i >= 2 ? 8 : 0)] = sum;
+    }
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_constant__ FfnArgs a) {
+  __shared__ DecItems it;
+  __shared__ float red[kWarps * kMaxNG * 8 * 32];
+  build_dec_items(it, a, a.w, 1);
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
+    const int s = dec_seg(it, item);
+    const int r0 = (item - it.first[s]) * kRows;
+    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    // passes of at most 32 tokens; a second pass re-reads the 16 rows from L2, not HBM
+    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
+      const int n = min(kPassTokens, it.off[s + 1] - q0);
+      if (n <= 8) dec13_item<1>(a, blk, r0, q0, n, red);
+      else if (n <= 16) dec13_item<2>(a, blk, r0, q0, n, red);
+      else dec13_item<4>(a, blk, r0, q0, n, red);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_constant__ FfnArgs a) {
+  __shared__ DecItems it;
+  __shared__ float red[kWarps * kMaxNG * 4 * 32];
+  build_dec_items(it, a, a.d, a.ksplit);
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
+    const int s = dec_seg(it, item);
+    const int local = item - it.first[s];
+    const int r0 = (local / it.ksplit) * kRows, kp = local % it.ksplit;
+    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
+      const int n = min(kPassTokens, it.off[s + 1] - q0);
+      if (n <= 8) dec2_item<1>(a, blk, r0, q0, n, kp, it.ksplit, red);
+      else if (n <= 16) dec2_item<2>(a, blk, r0, q0, n, kp, it.ksplit, red);
+      else dec2_item<4>(a, blk, r0, q0, n, kp, it.ksplit, red);
+    }
+  }
+}
+
+int blocks_per_sm(const void* fn) {
+  int nb = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, fn, kWarps * 32, 0) != cudaSuccess || nb < 1)
+    nb = 1;
+  return nb;
+}
+
+}  // namespace
+
+int decode_ksplit(int T) { return T <= 4 ? 4 : (T <= 16 ? 2 : 1); }
+
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s) {
+  static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel));
+  static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel));
+  prof_begin(kProfDec13, s);
+  dec13_kernel<<<num_sms * nb13, kWarps * 32, 0, s>>>(a);
+  prof_end(kProfDec13, s);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  prof_begin(kProfDec2, s);
+  dec2_kernel<<<num_sms * nb2, kWarps * 32, 0, s>>>(a);
+  prof_end(kProfDec2, s);
+  return cudaGetLastError();
+}
+
+}  // namespace mcft

@@ -1,4 +1,4 @@
-// Row-streaming expert FFN for decode batches (bf16) and for fp32 layers, plus the combine.
+// Row-streaming expert FFN for fp32 layers (CUDA-core fp32 arithmetic), plus the combine.
 //
 // F(x) = W2 (silu(W1 x) * (W3 x)) per expert segment (Section 3.1; SwiGLU experts). Each weight
 // row is read once per call from HBM with 16-byte loads and dotted with every token of its segment
@@ -217,6 +217,16 @@ __global__ void __launch_bounds__(kWarps * 32) ffn2_kernel(const __grid_constant
   }
 }
 
+// Four consecutive outputs of one permuted row, summed over the partial planes in plane order.
+__device__ __forceinline__ float4 row_sum(const CombineArgs& a, size_t at) {
+  float4 v = *reinterpret_cast<const float4*>(a.o + at);
+  for (int p = 1; p < a.ks; ++p) {
+    const float4 u = *reinterpret_cast<const float4*>(a.o + size_t(p) * a.o_plane + at);
+    v.x += u.x; v.y += u.y; v.z += u.z; v.w += u.w;
+  }
+  return v;
+}
+
 template <typename TY>
 __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineArgs a) {
   if (a.hdr->abort) return;
@@ -228,12 +238,12 @@ __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ Co
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int k = 0; k < a.K; ++k) {
       const float g = a.gate[size_t(t) * a.K + k];
-      const float4 v = *reinterpret_cast<const float4*>(a.o + size_t(a.pos[size_t(t) * a.K + k]) * a.d + c);
+      const float4 v = row_sum(a, size_t(a.pos[size_t(t) * a.K + k]) * a.d + c);
       acc.x = fmaf(g, v.x, acc.x); acc.y = fmaf(g, v.y, acc.y);
       acc.z = fmaf(g, v.z, acc.z); acc.w = fmaf(g, v.w, acc.w);
     }
     for (int s = 0; s < a.S; ++s) {
-      const float4 v = *reinterpret_cast<const float4*>(a.o + size_t(a.off[a.E + s] + t) * a.d + c);
+      const float4 v = row_sum(a, size_t(a.off[a.E + s] + t) * a.d + c);
       acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
     }
     if constexpr (sizeof(TY) == 4) {
@@ -269,8 +279,8 @@ cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s) 
 }  // namespace
 
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s) {
-  return dtype == MCFT_BF16 ? launch_rowwise_typed<__nv_bfloat16>(a, num_sms, s)
-                            : launch_rowwise_typed<float>(a, num_sms, s);
+  if (dtype != MCFT_F32) return cudaErrorInvalidValue;  // bf16 layers use the decode or TC path
+  return launch_rowwise_typed<float>(a, num_sms, s);
 }
 
 cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s) {

@@ -33,8 +33,10 @@ struct WsHeader {
 // E..E+S-1 the shared experts (every token). Offsets are in permuted rows.
 struct WsLayout {
   bool tc;        // tensor-core path (bf16, large T)
+  bool decode;    // bf16 decode path (T <= 64)
   int pad;        // rows per segment are padded to a multiple of this (128 on the TC path)
   int mcap;       // capacity in permuted rows
+  int ks;         // partial planes of o (contraction split of the decode GEMM2)
   size_t hdr, cnt, off, pos, perm, xp, h, o, total;
 };
 WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T);
@@ -66,12 +68,15 @@ struct FfnArgs {
   const int* perm;
   const WsHeader* hdr;
   const void* wblk[72];          // packed expert block of each segment
-  void* h;                       // [mcap, w] fp32 (rowwise) or bf16 (tensor cores)
-  float* o;                      // [mcap, d] fp32
-  int T, d, w, nseg, E;
+  void* h;                       // [mcap, w] fp32 (rowwise) or bf16 (tensor cores, decode)
+  float* o;                      // [ksplit][mcap, d] fp32
+  size_t o_plane;                // elements between partial planes of o
+  int T, d, w, nseg, E, ksplit;
   unsigned* err;
 };
-cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s);
+cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s);  // fp32
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s);  // bf16, T <= 64
+int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
 cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s);
 
 struct CombineArgs {
@@ -81,7 +86,8 @@ struct CombineArgs {
   const int* off;
   const WsHeader* hdr;
   void* y;
-  int T, d, K, E, S;
+  int T, d, K, E, S, ks;  // ks partial planes of o, o_plane elements apart
+  size_t o_plane;
 };
 cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s);
 
@@ -89,9 +95,11 @@ cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s);
 struct CacheStepArgs {
   const int32_t* idx;
   int n;              // T*K ids
-  int E, B, layer;
+  int E, B, layer, policy;
   int32_t* tag;       // [L*B]
-  int64_t* last;      // [L*B]
+  int64_t* last;      // [L*B] step of last use
+  int64_t* ins;       // [L*B] step of insertion (FIFO)
+  int64_t* freq;      // [L*E] accesses per expert since the stream began (LFU)
   int64_t* step;      // [L]
   unsigned long long* counters;  // [L*3] hits, fetches, bypass
   int32_t* miss_out;  // host-mapped, per layer: [n_miss, expert[E], loc[E], loc_of[E]]
@@ -104,7 +112,7 @@ mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_er
 
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
-       kProfGemm2, kProfCombine, kProfCount };
+       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

@@ -12,9 +12,9 @@
 namespace mcft {
 namespace {
 
-const char* const kNames[kProfCount] = {"route",    "cache_step", "permute",   "gather",
-                                        "ffn13_rowwise", "ffn2_rowwise", "gemm13_tc", "gemm2_tc",
-                                        "combine"};
+const char* const kNames[kProfCount] = {
+    "route",     "cache_step", "permute", "gather",       "ffn13_rowwise", "ffn2_rowwise",
+    "gemm13_tc", "gemm2_tc",   "combine", "ffn13_decode", "ffn2_decode"};
 
 struct Pending {
   int kid;

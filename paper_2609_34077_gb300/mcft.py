@@ -17,6 +17,8 @@ MCFT_OK, MCFT_ERR_INVALID, MCFT_ERR_OOM, MCFT_ERR_CUDA, MCFT_ERR_TIMEOUT, MCFT_E
 MCFT_ROUTE_TOPK, MCFT_ROUTE_HARD_MASK, MCFT_ROUTE_SOFT_PRIOR = 0, 1, 2
 MCFT_GATE_RENORM, MCFT_GATE_PLAIN = 0, 1
 MCFT_F32, MCFT_BF16 = 0, 1
+MCFT_CACHE_LRU, MCFT_CACHE_LFU, MCFT_CACHE_FIFO = 0, 1, 2
+POLICY = {"LRU": MCFT_CACHE_LRU, "LFU": MCFT_CACHE_LFU, "FIFO": MCFT_CACHE_FIFO}
 
 # every exported entry point: name -> (restype, argtypes)
 _vp, _i, _sz = C.c_void_p, C.c_int, C.c_size_t
@@ -25,7 +27,7 @@ SIGNATURES = {
     "mcft_moe_workspace_size": (_i, [_vp, _i, C.POINTER(_sz)]),
     "mcft_moe_forward": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "mcft_moe_forward_noalloc": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
-    "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, C.POINTER(_vp)]),
+    "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, _i, C.POINTER(_vp)]),
     "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
     "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
     "mcft_cache_last_misses": (_i, [_vp, _i, C.POINTER(_i), _vp, _vp]),
@@ -195,13 +197,16 @@ class Cache:
                 pass
 
 
-def mcft_cache_create(L, E, B, expert_bytes=0, host_experts=None, max_assign=1024) -> Cache:
-    """host_experts: L*E pinned host tensors (layer-major) or None for accounting only."""
+def mcft_cache_create(L, E, B, expert_bytes=0, host_experts=None, max_assign=1024,
+                      policy=MCFT_CACHE_LRU) -> Cache:
+    """host_experts: L*E pinned host tensors (layer-major) or None for accounting only;
+    policy: MCFT_CACHE_LRU / LFU / FIFO or the names "LRU" / "LFU" / "FIFO"."""
     h = C.c_void_p()
     arr = _ptr_array(host_experts, L * E) if host_experts is not None else None
+    pol = POLICY.get(policy, policy)
     _check(lib().mcft_cache_create(L, E, B, expert_bytes,
                                    C.cast(arr, C.c_void_p) if arr is not None else None,
-                                   max_assign, C.byref(h)))
+                                   max_assign, int(pol), C.byref(h)))
     c = Cache(h.value, L, E, B)
     c._host_experts = host_experts  # keep the pinned blocks alive
     return c

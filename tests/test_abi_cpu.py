@@ -72,5 +72,7 @@ def test_host_validation_without_gpu(libpath):
     assert st == mcft.MCFT_ERR_INVALID
     # cache: K <= B < E
     h = C.c_void_p()
-    assert L.mcft_cache_create(1, 8, 8, 0, None, 2, C.byref(h)) == mcft.MCFT_ERR_INVALID
-    assert L.mcft_cache_create(1, 8, 0, 0, None, 2, C.byref(h)) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_cache_create(1, 8, 8, 0, None, 2, 0, C.byref(h)) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_cache_create(1, 8, 0, 0, None, 2, 0, C.byref(h)) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_cache_create(1, 8, 4, 0, None, 2, 7, C.byref(h)) == mcft.MCFT_ERR_INVALID
+    assert b"policy" in L.mcft_last_error()

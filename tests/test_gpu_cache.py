@@ -18,13 +18,14 @@ def _stream_ids(E, K, T, steps, keep, seed):
     return I.random_ids(seed, steps, T, K, E, hot=range(keep), p_hot=0.75)
 
 
+@pytest.mark.parametrize("policy", ["LRU", "LFU", "FIFO"])
 @pytest.mark.parametrize("E,B,K,T", [(8, 4, 2, 1), (8, 4, 2, 16), (64, 12, 6, 1), (64, 12, 6, 8),
                                      (64, 12, 6, 64), (5, 2, 1, 3)])
-def test_cache_decisions_bit_exact(E, B, K, T):
+def test_cache_decisions_bit_exact(E, B, K, T, policy):
     steps = 512 if T < 64 else 128
     ids = _stream_ids(E, K, T, steps, max(B // 2, K), seed=E + B + K + T)
-    c = M.mcft_cache_create(1, E, B, max_assign=T * K)
-    ref = oracle.cache.LRUStamps(E, B)
+    c = M.mcft_cache_create(1, E, B, max_assign=T * K, policy=policy)
+    ref = oracle.cache.SlotCache(E, B, policy)
     d_ids = torch.from_numpy(ids).to(DEV)
     th = tf = tb = 0
     for s in range(steps):
@@ -83,26 +84,32 @@ def test_cache_fetch_copies_expert_bytes():
     M.mcft_device_error()
 
 
-def test_cache_export_import_resume():
+@pytest.mark.parametrize("policy", ["LRU", "LFU", "FIFO"])
+def test_cache_export_import_resume(policy):
+    """Run N steps == run n steps, export, import into a fresh cache, run the other N - n."""
     E, B, K, T = 64, 12, 6, 8
     ids = _stream_ids(E, K, T, 200, 16, seed=9)
     d_ids = torch.from_numpy(ids).to(DEV)
-    full = M.mcft_cache_create(1, E, B, max_assign=T * K)
+    full = M.mcft_cache_create(1, E, B, max_assign=T * K, policy=policy)
     for s in range(200):
         M.mcft_cache_step(full, 0, d_ids[s])
-    a = M.mcft_cache_create(1, E, B, max_assign=T * K)
+    a = M.mcft_cache_create(1, E, B, max_assign=T * K, policy=policy)
     for s in range(77):
         M.mcft_cache_step(a, 0, d_ids[s])
     state = M.mcft_cache_export(a)
-    b = M.mcft_cache_create(1, E, B, max_assign=T * K)
+    b = M.mcft_cache_create(1, E, B, max_assign=T * K, policy=policy)
     M.mcft_cache_import(b, state)
     for s in range(77, 200):
         M.mcft_cache_step(b, 0, d_ids[s])
     assert M.mcft_cache_stats(b, 0) == M.mcft_cache_stats(full, 0)
     assert M.mcft_cache_tags(b, 0) == M.mcft_cache_tags(full, 0)
-    other = M.mcft_cache_create(1, E, B + 1, max_assign=T * K)
+    other = M.mcft_cache_create(1, E, B + 1, max_assign=T * K, policy=policy)
     with pytest.raises(M.MCFTError):
         M.mcft_cache_import(other, state)
+    other_policy = M.mcft_cache_create(1, E, B, max_assign=T * K,
+                                       policy="FIFO" if policy != "FIFO" else "LRU")
+    with pytest.raises(M.MCFTError):
+        M.mcft_cache_import(other_policy, state)
 
 
 def test_cache_bad_id_changes_nothing():

@@ -21,8 +21,9 @@ def _load_traces():
         if not line or line.startswith("#"):
             continue
         if line.startswith("trace"):
-            _, name, _, E, _, B = line.split()
-            cur = dict(name=name, E=int(E), B=int(B), steps=[])
+            f = line.split()
+            cur = dict(name=f[1], E=int(f[3]), B=int(f[5]), policy=f[7] if len(f) > 7 else "LRU",
+                       steps=[])
             traces.append(cur)
         elif line.startswith("step"):
             ids, hits, misses = [p.strip() for p in line[4:].split("|")]
@@ -37,10 +38,10 @@ def _load_traces():
 TRACES = _load_traces()
 
 
-@pytest.mark.parametrize("cls", [C.LRUStamps, C.LRUList])
+@pytest.mark.parametrize("cls", [C.SlotCache, C.OrderedCache])
 @pytest.mark.parametrize("tr", TRACES, ids=[t["name"] for t in TRACES])
 def test_hand_traces(cls, tr):
-    c = cls(tr["E"], tr["B"])
+    c = cls(tr["E"], tr["B"], tr["policy"])
     th = tf = tb = 0
     for ids, hits, misses in tr["steps"]:
         h, f, b, ml = c.step(ids)
@@ -74,50 +75,72 @@ def test_table2_metric_identity():
     assert round(100 * red("deepseek-v2-lite"), 1) == 10.1
 
 
+@pytest.mark.parametrize("policy", C.POLICIES)
 @pytest.mark.parametrize("T,K,E,B", [(1, 2, 8, 4), (16, 2, 8, 4), (1, 6, 64, 12), (8, 6, 64, 12),
                                      (64, 6, 64, 12), (4, 1, 5, 2)])
-def test_two_formulations_agree(T, K, E, B):
+def test_two_formulations_agree(T, K, E, B, policy):
     ids = inputs.random_ids(11, 300, T, K, E, hot=range(min(E, B + 2)), p_hot=0.7)
-    a, b = C.LRUStamps(E, B), C.LRUList(E, B)
+    a, b = C.SlotCache(E, B, policy), C.OrderedCache(E, B, policy)
     for s in range(ids.shape[0]):
         ra, rb = a.step(ids[s]), b.step(ids[s])
         assert ra == rb
         assert a.tag == b.state()
 
 
-def test_batch1_fetch_identity():
+@pytest.mark.parametrize("policy", C.POLICIES)
+def test_batch1_fetch_identity(policy):
     """At batch 1 with K distinct experts per step: f = K - h every step, and over the stream
     Fetches/tok = L K (1 - HR) (Eq. metrics)."""
     L, K, E, B, N = 3, 2, 8, 4, 200
     th = tf = 0
     for layer in range(L):
         ids = inputs.random_ids(12 + layer, N, 1, K, E, hot=range(4), p_hot=0.6)
-        h, f, b, _ = C.simulate(ids, E, B)
+        h, f, b, _ = C.simulate(ids, E, B, policy=policy)
         assert np.all(f == K - h) and np.all(b == 0)
         th, tf = th + h.sum(), tf + f.sum()
     HR, FPT = C.metrics(th, tf, N, L, K)
     assert FPT == pytest.approx(C.fetches_per_token_from_hit_rate(HR, L, K), rel=1e-12)
 
 
-def test_hard_mask_with_B_kept_experts_only_cold_misses():
+@pytest.mark.parametrize("policy", C.POLICIES)
+def test_hard_mask_with_B_kept_experts_only_cold_misses(policy):
     """A hard mask keeping E' = B experts: every chosen expert is in the kept set, so the cache
     never evicts and total fetches = number of distinct experts used (<= B)."""
     E, K, B = 8, 2, 4
     kept = [0, 1, 2, 3]
     ids = inputs.random_ids(13, 64, 1, K, E, hot=kept, p_hot=1.0)
-    h, f, b, _ = C.simulate(ids, E, B)
+    h, f, b, _ = C.simulate(ids, E, B, policy=policy)
     assert f.sum() == len(np.unique(ids)) <= B
 
 
-def test_large_cache_only_cold_misses():
+@pytest.mark.parametrize("policy", C.POLICIES)
+def test_large_cache_only_cold_misses(policy):
     E, K, B = 16, 3, 15
     ids = inputs.random_ids(14, 100, 2, K, E, hot=range(10), p_hot=1.0)
-    h, f, b, _ = C.simulate(ids, E, B)
+    h, f, b, _ = C.simulate(ids, E, B, policy=policy)
     assert f.sum() == len(np.unique(ids))
     assert b.sum() == 0
 
 
+def test_policies_agree_without_evictions():
+    """Until the cache is full no policy has a choice: all three make identical decisions."""
+    ids = inputs.random_ids(15, 40, 1, 2, 16, hot=range(6), p_hot=1.0)
+    runs = [C.simulate(ids, 16, 8, policy=p) for p in C.POLICIES]
+    for r in runs[1:]:
+        assert r[3] == runs[0][3]
+
+
+def test_lfu_keeps_a_hot_expert_lru_does_not():
+    """A stream where one expert recurs often but not recently: LFU keeps it, LRU evicts it."""
+    ids = [[0]] * 5 + [[1], [2], [0], [3], [4], [0]]
+    lfu = C.simulate(ids, 5, 2, policy="LFU")
+    lru = C.simulate(ids, 5, 2, policy="LRU")
+    assert lfu[0].sum() > lru[0].sum()
+
+
 def test_invalid():
+    with pytest.raises(ValueError):
+        C.SlotCache(4, 2, "MRU")
     with pytest.raises(ValueError):
         C.LRUStamps(4, 4)
     c = C.LRUStamps(4, 2)
