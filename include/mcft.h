@@ -199,6 +199,26 @@ mcft_status mcft_cache_step(mcft_cache* cache, int layer, const int32_t* idx, in
 mcft_status mcft_fetch_experts(mcft_cache* cache, int layer, mcft_stream_t compute_stream,
                                mcft_stream_t copy_stream, const void** expert_ptrs);
 
+/* mcft_moe_forward_cached: mcft_moe_forward for a decode step of `layer` whose experts come from
+ * the cache, with the fetch driven by the device and overlapped with compute; no host round trip.
+ * Call it after mcft_cache_step(cache, layer, idx, ...) on compute_stream, instead of
+ * mcft_fetch_experts + mcft_moe_forward. On copy_stream (after that cache step) a kernel copies
+ * every missed expert's block from pinned host memory into the slot or staging buffer the cache
+ * step chose, reading the host memory directly over the host link; on compute_stream the
+ * permutation and the FFN of the experts that were hits (and of the shared experts) run at the
+ * same time; then compute_stream waits for the copies and computes the fetched experts and the
+ * combine. Results equal mcft_moe_forward's with the same experts.
+ * Section 3.1 Eq. topk (the layer) and Section 4.1 / P:L53, P:L106 (fetch on a miss).
+ *   cache  created with host blocks (not accounting-only); its E and expert size match desc
+ *   other arguments as for mcft_moe_forward (the routed expert addresses come from the cache)
+ * Supports the decode path (bf16 with T <= 64, or fp32); larger bf16 calls return
+ * MCFT_ERR_UNSUPPORTED (use mcft_fetch_experts + mcft_moe_forward). Asynchronous. */
+mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, int T,
+                                    const int32_t* idx, const float* gate, mcft_cache* cache,
+                                    int layer, const void* const* shared, void* y, void* workspace,
+                                    size_t ws_bytes, mcft_stream_t compute_stream,
+                                    mcft_stream_t copy_stream);
+
 /* mcft_cache_last_misses: the miss list of the last mcft_cache_step of `layer`, after
  * mcft_fetch_experts (or a synchronisation of its stream): n_out = number of fetches;
  * experts[i], slots[i] for i < n_out in processing order, slot = -1 for a bypass fetch.

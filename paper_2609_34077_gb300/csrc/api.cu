@@ -137,10 +137,15 @@ struct mcft_cache {
   int32_t* h_miss = nullptr;  // host-mapped [L][miss_stride]
   int32_t* d_miss = nullptr;  // device alias of h_miss
   int miss_stride = 0;
+  int32_t* d_miss_dev = nullptr;            // device-memory copy [L][miss_stride]
+  unsigned long long* d_ptr_tab = nullptr;  // [L*E] block address of each selected expert
+  unsigned long long* d_ready = nullptr;    // [L] hit mask of the last step
+  unsigned long long* d_host_src = nullptr; // [L*E] device-visible addresses of the host blocks
   char* d_slots = nullptr;    // [L*B] expert blocks
   char* d_staging = nullptr;  // [n_staging] expert blocks
   std::vector<cudaEvent_t> ev_step;  // per layer: recorded after its cache step
   cudaEvent_t ev_copy = nullptr;
+  bool device_fetch = false;  // every host block has a device-visible address
 };
 
 namespace {
@@ -156,6 +161,10 @@ void cache_free(mcft_cache* c) {
   if (c->h_miss) cudaFreeHost(c->h_miss);
   cudaFree(c->d_slots);
   cudaFree(c->d_staging);
+  cudaFree(c->d_miss_dev);
+  cudaFree(c->d_ptr_tab);
+  cudaFree(c->d_ready);
+  cudaFree(c->d_host_src);
   for (cudaEvent_t e : c->ev_step)
     if (e) cudaEventDestroy(e);
   if (c->ev_copy) cudaEventDestroy(c->ev_copy);
@@ -391,11 +400,32 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   MCFT_CACHE_CUDA(cudaHostAlloc(&c->h_miss, sizeof(int32_t) * L * c->miss_stride, cudaHostAllocMapped));
   memset(c->h_miss, 0, sizeof(int32_t) * L * c->miss_stride);
   MCFT_CACHE_CUDA(cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->d_miss), c->h_miss, 0));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_miss_dev, sizeof(int32_t) * L * c->miss_stride));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_miss_dev, 0, sizeof(int32_t) * L * c->miss_stride));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_ptr_tab, sizeof(unsigned long long) * L * E));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_ptr_tab, 0, sizeof(unsigned long long) * L * E));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_ready, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_ready, 0, sizeof(unsigned long long) * L));
   if (host_experts) {
     c->host_experts.assign(host_experts, host_experts + size_t(L) * E);
     c->n_staging = stg;
     MCFT_CACHE_CUDA(cudaMalloc(&c->d_slots, expert_bytes * size_t(L) * B));
     if (stg > 0) MCFT_CACHE_CUDA(cudaMalloc(&c->d_staging, expert_bytes * size_t(stg)));
+    // device-visible addresses of the pinned host blocks, for the device-driven fetch
+    std::vector<unsigned long long> src(size_t(L) * E);
+    for (size_t i = 0; i < src.size(); ++i) {
+      void* dp = nullptr;
+      if (cudaHostGetDevicePointer(&dp, const_cast<void*>(host_experts[i]), 0) != cudaSuccess) {
+        cudaGetLastError();
+        dp = nullptr;  // not mapped: only the copy-engine fetch can serve this cache
+      }
+      src[i] = reinterpret_cast<unsigned long long>(dp);
+    }
+    MCFT_CACHE_CUDA(cudaMalloc(&c->d_host_src, sizeof(unsigned long long) * L * E));
+    MCFT_CACHE_CUDA(cudaMemcpy(c->d_host_src, src.data(), sizeof(unsigned long long) * L * E,
+                               cudaMemcpyHostToDevice));
+    c->device_fetch = true;
+    for (auto v : src) c->device_fetch = c->device_fetch && v != 0;
   }
   c->ev_step.assign(L, nullptr);
   for (int l = 0; l < L; ++l)
@@ -416,7 +446,10 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
     return fail(MCFT_ERR_INVALID, "T*K = %d exceeds max_assign = %d", T * K, c->max_assign);
   CacheStepArgs a{idx, T * K, c->E, c->B, layer, c->policy, c->d_tag, c->d_last, c->d_ins,
                   c->d_freq, c->d_step, c->d_cnt, c->d_miss + size_t(layer) * c->miss_stride,
-                  device_error_word()};
+                  c->d_miss_dev + size_t(layer) * c->miss_stride,
+                  c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer,
+                  c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
+                  c->d_staging, c->expert_bytes, device_error_word()};
   cudaError_t e = launch_cache_step(a, stream);
   if (e != cudaSuccess) return cuda_fail(e, "cache step launch");
   MCFT_CUDA(cudaEventRecord(c->ev_step[layer], stream));
@@ -447,6 +480,88 @@ mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_s
     MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
     MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
   }
+  return MCFT_OK;
+}
+
+mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, int T,
+                                    const int32_t* idx, const float* gate, mcft_cache* c, int layer,
+                                    const void* const* shared, void* y, void* workspace,
+                                    size_t ws_bytes, mcft_stream_t compute_stream,
+                                    mcft_stream_t copy_stream) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (!c) return fail(MCFT_ERR_INVALID, "cache is NULL");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  if (!c->d_slots || !c->device_fetch)
+    return fail(MCFT_ERR_INVALID, "the cache has no slots or its host blocks are not mapped");
+  if (desc->E != c->E) return fail(MCFT_ERR_INVALID, "desc E = %d but the cache has E = %d", desc->E, c->E);
+  const size_t eb = size_t(3) * desc->w * desc->d * (desc->dtype == MCFT_BF16 ? 2 : 4);
+  if (eb != c->expert_bytes)
+    return fail(MCFT_ERR_INVALID, "expert blocks of %zu bytes but the cache holds %zu", eb, c->expert_bytes);
+  if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
+  if (T == 0) return MCFT_OK;
+  if (!x || !idx || !gate || !y || !workspace) return fail(MCFT_ERR_INVALID, "NULL pointer argument");
+  const int E = desc->E, S = desc->n_shared, K = desc->K;
+  if (S > 0 && !shared) return fail(MCFT_ERR_INVALID, "shared is NULL");
+  for (int s = 0; s < S; ++s)
+    if (!shared[s] || (reinterpret_cast<uintptr_t>(shared[s]) & 15u))
+      return fail(MCFT_ERR_INVALID, "shared expert %d block is NULL or misaligned", s);
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) ||
+      ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15u))
+    return fail(MCFT_ERR_INVALID, "misaligned x, y or workspace");
+  const WsLayout L = ws_layout(desc->d, E, K, desc->w, S, desc->dtype, T);
+  if (L.tc)
+    return fail(MCFT_ERR_UNSUPPORTED, "T = %d runs the tensor-core path; use mcft_fetch_experts + "
+                "mcft_moe_forward", T);
+  if (ws_bytes < L.total)
+    return fail(MCFT_ERR_INVALID, "workspace of %zu bytes < %zu needed", ws_bytes, L.total);
+
+  char* ws = static_cast<char*>(workspace);
+  WsHeader* hdr = reinterpret_cast<WsHeader*>(ws + L.hdr);
+  int* cnt = reinterpret_cast<int*>(ws + L.cnt);
+  int* off = reinterpret_cast<int*>(ws + L.off);
+  int* pos = reinterpret_cast<int*>(ws + L.pos);
+  int* perm = reinterpret_cast<int*>(ws + L.perm);
+  unsigned* err = device_error_word();
+  // 1. the missed experts stream in on the copy stream, after this layer's cache step
+  MCFT_CUDA(cudaStreamWaitEvent(copy_stream, c->ev_step[layer], 0));
+  FetchArgs fe{c->d_miss_dev + size_t(layer) * c->miss_stride, c->d_host_src + size_t(layer) * E,
+               c->d_ptr_tab + size_t(layer) * E, c->expert_bytes};
+  cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
+  MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
+  // 2. meanwhile: permutation and the experts that were hits (and the shared experts)
+  PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
+  e = launch_permute(pa, compute_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
+  FfnArgs fa{};
+  fa.x = x;
+  fa.off = off;
+  fa.perm = perm;
+  fa.hdr = hdr;
+  for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
+  fa.h = ws + L.h;
+  fa.o = reinterpret_cast<float*>(ws + L.o);
+  fa.o_plane = size_t(L.mcap) * desc->d;
+  fa.ksplit = L.ks;
+  fa.T = T;
+  fa.d = desc->d;
+  fa.w = desc->w;
+  fa.nseg = E + S;
+  fa.E = E;
+  fa.err = err;
+  fa.wtab = c->d_ptr_tab + size_t(layer) * E;
+  fa.ready = c->d_ready + layer;
+  for (int phase = 1; phase <= 2; ++phase) {
+    fa.phase = phase;
+    if (phase == 2) MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
+    e = L.decode ? launch_ffn_decode(fa, num_sms(), compute_stream)
+                 : launch_ffn_rowwise(fa, desc->dtype, num_sms(), compute_stream);
+    if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
+  }
+  CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S, L.ks, fa.o_plane};
+  e = launch_combine(ca, desc->dtype, compute_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
   return MCFT_OK;
 }
 

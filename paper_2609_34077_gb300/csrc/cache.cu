@@ -48,6 +48,9 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
   if (bad) {  // no state change on bad input
     set_error(a.err, kErrInvalid);
     a.miss_out[0] = 0;
+    a.miss_dev[0] = 0;
+    *a.ready = 0;
+    for (int e = 0; e < a.E; ++e) a.ptr_tab[e] = 0;
     __threadfence_system();
     return;
   }
@@ -108,6 +111,19 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
     ++nm;
   }
   out[0] = nm;
+  // device copies for the device-driven fetch and the forward that follows it
+  unsigned long long hitmask = 0;
+  for (int i = 0; i < 1 + 3 * E; ++i) a.miss_dev[i] = out[i];
+  for (int e = 0; e < E; ++e) {
+    const int loc = loc_of[e];
+    unsigned long long p = 0;
+    if (loc >= 0 && a.slots)
+      p = reinterpret_cast<unsigned long long>(loc < B ? a.slots + size_t(loc) * a.expert_bytes
+                                                       : a.staging + size_t(loc - B) * a.expert_bytes);
+    a.ptr_tab[e] = p;
+    if (loc >= 0 && loc < B && ((cached >> e) & 1ull)) hitmask |= 1ull << e;
+  }
+  *a.ready = hitmask;
   a.step[a.layer] = t + 1;
   unsigned long long* c = a.counters + size_t(a.layer) * 3;
   c[0] += hits;
@@ -116,7 +132,40 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
   __threadfence_system();
 }
 
+// Copy the missed experts' blocks host -> device with 16-byte loads over the host link. Work
+// units are 64 KB pieces of the missed blocks, spread over the grid.
+__global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ FetchArgs a) {
+  const int n = a.miss[0];
+  const size_t words = a.bytes / 16, piece = 4096;
+  const size_t per = (words + piece - 1) / piece;
+  const size_t units = size_t(n) * per;
+  for (size_t u = blockIdx.x; u < units; u += gridDim.x) {
+    const int e = a.miss[1 + int(u / per)];
+    const uint4* src = reinterpret_cast<const uint4*>(a.host_src[e]);
+    uint4* dst = reinterpret_cast<uint4*>(a.ptr_tab[e]);
+    const size_t w0 = (u % per) * piece;
+    const size_t w1 = w0 + piece < words ? w0 + piece : words;
+    const size_t stride = blockDim.x;
+    for (size_t w = w0 + threadIdx.x; w < w1; w += 4 * stride) {
+      uint4 v[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (w + j * stride < w1) v[j] = src[w + j * stride];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (w + j * stride < w1) dst[w + j * stride] = v[j];
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s) {
+  prof_begin(kProfFetch, s);
+  fetch_kernel<<<blocks, 256, 0, s>>>(a);
+  prof_end(kProfFetch, s);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s) {
   prof_begin(kProfCache, s);

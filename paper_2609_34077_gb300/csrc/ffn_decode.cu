@@ -32,6 +32,7 @@ struct DecItems {
   int nseg, total, ksplit;
   int off[kMaxSeg + 1];
   int first[kMaxSeg + 1];
+  const char* blk[kMaxSeg];
 };
 
 __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows_per_seg, int ksplit) {
@@ -40,11 +41,13 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows_per_seg
     it.nseg = nseg;
     it.ksplit = ksplit;
     int acc = 0;
+    const unsigned long long hits = a.ready ? *a.ready : 0ull;
     for (int s = 0; s <= nseg; ++s) it.off[s] = a.off[s];
     for (int s = 0; s < nseg; ++s) {
       it.first[s] = acc;
-      if (it.off[s + 1] > it.off[s]) {
-        if (a.wblk[s] == nullptr) {  // a selected expert without weights
+      it.blk[s] = reinterpret_cast<const char*>(seg_block(a, s));
+      if (it.off[s + 1] > it.off[s] && seg_in_phase(a, s, hits)) {
+        if (it.blk[s] == nullptr) {  // a selected expert without weights
           set_error(a.err, kErrInvalid);
           const_cast<WsHeader*>(a.hdr)->abort = 1;
           continue;
@@ -237,7 +240,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
     const int s = dec_seg(it, item);
     const int r0 = (item - it.first[s]) * kRows;
-    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    const char* blk = it.blk[s];
     // passes of at most 32 tokens; a second pass re-reads the 16 rows from L2, not HBM
     for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
       const int n = min(kPassTokens, it.off[s + 1] - q0);
@@ -256,7 +259,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
     const int s = dec_seg(it, item);
     const int local = item - it.first[s];
     const int r0 = (local / it.ksplit) * kRows, kp = local % it.ksplit;
-    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    const char* blk = it.blk[s];
     for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
       const int n = min(kPassTokens, it.off[s + 1] - q0);
       if (n <= 8) dec2_item<1>(a, blk, r0, q0, n, kp, it.ksplit, red);

@@ -39,6 +39,7 @@ struct Items {
   int nseg, total;
   int off[kMaxSeg + 1];
   int first[kMaxSeg + 1];  // first item of each segment
+  const char* blk[kMaxSeg];
 };
 
 // Prefix of work items over non-empty segments (rows_per_seg / kRowsPerItem items each).
@@ -47,12 +48,14 @@ __device__ void build_items(Items& it, const FfnArgs& a, int rows_per_seg) {
     const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
     it.nseg = nseg;
     int acc = 0;
+    const unsigned long long hits = a.ready ? *a.ready : 0ull;
     for (int s = 0; s <= nseg; ++s) it.off[s] = a.off[s];
     for (int s = 0; s < nseg; ++s) {
       it.first[s] = acc;
+      it.blk[s] = reinterpret_cast<const char*>(seg_block(a, s));
       const int n = it.off[s + 1] - it.off[s];
-      if (n > 0) {
-        if (a.wblk[s] == nullptr) {  // a selected expert without weights
+      if (n > 0 && seg_in_phase(a, s, hits)) {
+        if (it.blk[s] == nullptr) {  // a selected expert without weights
           set_error(a.err, kErrInvalid);
           const_cast<WsHeader*>(a.hdr)->abort = 1;
           continue;
@@ -182,7 +185,7 @@ __global__ void __launch_bounds__(kWarps * 32) ffn13_kernel(const __grid_constan
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
     const int s = find_seg(it, item);
     const int r0 = (item - it.first[s]) * kRowsPerItem + warp * kRowsPerWarp;
-    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    const char* blk = it.blk[s];
     const int q_begin = it.off[s], q_end = it.off[s + 1];
     for (int q0 = q_begin; q0 < q_end; q0 += kTokGroup) {
       const int nt = min(kTokGroup, q_end - q0);
@@ -205,7 +208,7 @@ __global__ void __launch_bounds__(kWarps * 32) ffn2_kernel(const __grid_constant
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
     const int s = find_seg(it, item);
     const int r0 = (item - it.first[s]) * kRowsPerItem + warp * kRowsPerWarp;
-    const char* blk = reinterpret_cast<const char*>(a.wblk[s]);
+    const char* blk = it.blk[s];
     const int q_begin = it.off[s], q_end = it.off[s + 1];
     for (int q0 = q_begin; q0 < q_end; q0 += kTokGroup) {
       const int nt = min(kTokGroup, q_end - q0);

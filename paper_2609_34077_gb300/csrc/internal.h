@@ -73,7 +73,23 @@ struct FfnArgs {
   size_t o_plane;                // elements between partial planes of o
   int T, d, w, nseg, E, ksplit;
   unsigned* err;
+  // Expert addresses written on the device by a cache step (NULL: use wblk), that step's hit
+  // mask, and which segments this launch computes: 0 all, 1 hit experts and shared experts,
+  // 2 routed experts that were not hits (fetched or bypassed at this step).
+  const unsigned long long* wtab;
+  const unsigned long long* ready;
+  int phase;
 };
+
+// Segment s of a forward: its block address and whether this launch computes it.
+__device__ __forceinline__ const void* seg_block(const FfnArgs& a, int s) {
+  return (a.wtab && s < a.E) ? reinterpret_cast<const void*>(a.wtab[s]) : a.wblk[s];
+}
+__device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned long long hits) {
+  if (a.phase == 0) return true;
+  const bool hit = s >= a.E || ((hits >> s) & 1ull);
+  return a.phase == 1 ? hit : !hit;
+}
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s);  // fp32
 cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s);  // bf16, T <= 64
 int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
@@ -103,16 +119,32 @@ struct CacheStepArgs {
   int64_t* step;      // [L]
   unsigned long long* counters;  // [L*3] hits, fetches, bypass
   int32_t* miss_out;  // host-mapped, per layer: [n_miss, expert[E], loc[E], loc_of[E]]
+  int32_t* miss_dev;  // device copy of the same list (read by the fetch kernel)
+  unsigned long long* ptr_tab;  // device [E]: block address of each selected expert, else 0
+  unsigned long long* ready;    // device: bit e set when expert e was a hit at this step
+  const char* slots;            // this layer's first slot block (NULL in accounting mode)
+  const char* staging;          // bypass staging blocks
+  size_t expert_bytes;
   unsigned* err;
 };
 cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s);
+
+// Device-driven fetch: copy the blocks of a layer's missed experts from pinned host memory
+// (device-visible addresses host_src[E]) into the addresses ptr_tab[E] chosen by the cache step.
+struct FetchArgs {
+  const int32_t* miss;                // device miss list of the layer [1 + 3E]
+  const unsigned long long* host_src; // [E]
+  const unsigned long long* ptr_tab;  // [E]
+  size_t bytes;                       // per expert block, multiple of 16
+};
+cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s);
 
 unsigned* device_error_word();  // device address of the current device's error word
 mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_error() text
 
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
-       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfCount };
+       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

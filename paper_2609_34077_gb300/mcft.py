@@ -30,6 +30,7 @@ SIGNATURES = {
     "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, _i, C.POINTER(_vp)]),
     "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
     "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
+    "mcft_moe_forward_cached": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _sz, _vp, _vp]),
     "mcft_cache_last_misses": (_i, [_vp, _i, C.POINTER(_i), _vp, _vp]),
     "mcft_cache_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64),
                               C.POINTER(C.c_uint64), _vp]),
@@ -229,6 +230,22 @@ def mcft_fetch_experts(cache: Cache, layer, compute_stream=None, copy_stream=Non
     _check(lib().mcft_fetch_experts(C.c_void_p(cache.handle), layer, _stream(compute_stream),
                                     _stream(copy_stream), C.cast(out, C.c_void_p)))
     return [v or 0 for v in out]
+
+
+def mcft_moe_forward_cached(desc: LayerDesc, x, idx, gate, cache: Cache, layer, shared=(), y=None,
+                            workspace=None, compute_stream=None, copy_stream=None):
+    """Decode forward of `layer` with experts from the cache, fetch driven on the device."""
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.empty(mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=x.device)
+    sh = _ptr_array(shared, desc.n_shared)
+    _check(lib().mcft_moe_forward_cached(C.byref(desc), _ptr(x), T, _ptr(idx), _ptr(gate),
+                                         C.c_void_p(cache.handle), layer, C.cast(sh, C.c_void_p),
+                                         _ptr(y), _ptr(workspace), workspace.numel(),
+                                         _stream(compute_stream), _stream(copy_stream)))
+    return y
 
 
 def mcft_cache_last_misses(cache: Cache, layer):

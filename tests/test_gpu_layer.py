@@ -1,6 +1,8 @@
 """End-to-end decode steps through the C ABI: route (soft prior) -> cache step -> fetch of missed
 experts from pinned host memory -> expert FFN + combine, against the oracle's routing, cache and
-layer output (Section 3.1, Eq. inference, Section 4.1)."""
+layer output (Section 3.1, Eq. inference, Section 4.1). Two fetch paths: the host reads the miss
+list and issues copies (mcft_fetch_experts + mcft_moe_forward), or the device copies the missed
+experts itself while the hit experts are computed (mcft_moe_forward_cached)."""
 import numpy as np
 import pytest
 import torch
@@ -19,14 +21,14 @@ SMALL_DS = I.LayerShape("small-ds-layer", d=256, E=64, K=6, w=128, n_shared=2, g
                         dtype=I.BF16, cache_slots=12, keep=16)
 
 
-def _decode_stream(shape, batch, steps, seed, check_every=1):
+def _decode_stream(shape, batch, steps, seed, check_every=1, path="host", policy="LRU"):
     lw = I.layer_weights(seed, shape, pin=True)
     desc = M.desc_of(shape)
     prior = I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep))
     xs = I.ar1_streams(seed, shape, steps, batch)
     cache = M.mcft_cache_create(1, shape.E, shape.cache_slots, shape.expert_bytes, lw.experts,
-                                max_assign=batch * shape.K)
-    ref_cache = oracle.cache.LRUStamps(shape.E, shape.cache_slots)
+                                max_assign=batch * shape.K, policy=policy)
+    ref_cache = oracle.cache.SlotCache(shape.E, shape.cache_slots, policy)
     wr = lw.router.to(DEV)
     shared = [b.to(DEV) for b in lw.shared]
     ws = torch.empty(M.mcft_moe_workspace_size(desc, batch), dtype=torch.uint8, device=DEV)
@@ -40,8 +42,13 @@ def _decode_stream(shape, batch, steps, seed, check_every=1):
         xd = x.to(DEV)
         idx, gate = M.mcft_route(desc, xd, wr, M.MCFT_ROUTE_SOFT_PRIOR, prior=prior)
         M.mcft_cache_step(cache, 0, idx)
-        ptrs = M.mcft_fetch_experts(cache, 0, torch.cuda.current_stream(), copy)
-        y = M.mcft_moe_forward(desc, xd, idx, gate, ptrs, shared, workspace=ws)
+        if path == "host":
+            ptrs = M.mcft_fetch_experts(cache, 0, torch.cuda.current_stream(), copy)
+            y = M.mcft_moe_forward(desc, xd, idx, gate, ptrs, shared, workspace=ws)
+        else:
+            y = M.mcft_moe_forward_cached(desc, xd, idx, gate, cache, 0, shared, workspace=ws,
+                                          copy_stream=copy)
+            torch.cuda.synchronize()
         ref = oracle.routing.route(f64(x), f64(lw.router), shape.K, M.MCFT_ROUTE_SOFT_PRIOR,
                                    shape.gate, prior=prior)
         gi = idx.cpu().numpy()
@@ -62,16 +69,36 @@ def _decode_stream(shape, batch, steps, seed, check_every=1):
     return cache, mism
 
 
+@pytest.mark.parametrize("path", ["host", "device"])
 @pytest.mark.parametrize("shape,batch", [(SMALL_MIX, 1), (SMALL_MIX, 16), (SMALL_DS, 1),
                                          (SMALL_DS, 8), (SMALL_DS, 64)],
                          ids=["mix-b1", "mix-b16", "ds-b1", "ds-b8", "ds-b64"])
-def test_decode_stream_small(shape, batch):
-    _, mism = _decode_stream(shape, batch, 64, seed=20 + batch)
+def test_decode_stream_small(shape, batch, path):
+    _, mism = _decode_stream(shape, batch, 64, seed=20 + batch, path=path)
     assert mism <= 2
 
 
-def test_decode_stream_mixtral_full_size():
+@pytest.mark.parametrize("policy", ["LFU", "FIFO"])
+def test_decode_stream_policies_device_fetch(policy):
+    _, mism = _decode_stream(SMALL_DS, 8, 48, seed=27, path="device", policy=policy)
+    assert mism <= 2
+
+
+@pytest.mark.parametrize("path", ["host", "device"])
+def test_decode_stream_mixtral_full_size(path):
     """Mixtral-shaped layer, 8 experts of 352 MB in pinned host memory, 4 GPU slots: 12 decode
     steps at batch 1 with real fetches; output checked every 4th step."""
-    _, mism = _decode_stream(I.MIXTRAL, 1, 12, seed=30, check_every=4)
+    _, mism = _decode_stream(I.MIXTRAL, 1, 12, seed=30, check_every=4, path=path)
     assert mism <= 1
+
+
+def test_forward_cached_rejects_prefill_and_accounting_caches():
+    sh = SMALL_MIX
+    desc = M.desc_of(sh)
+    acc = M.mcft_cache_create(1, sh.E, sh.cache_slots, max_assign=2)
+    x = torch.zeros((1, sh.d), dtype=torch.bfloat16, device=DEV)
+    idx = torch.zeros((1, 2), dtype=torch.int32, device=DEV)
+    idx[0, 1] = 1
+    g = torch.ones((1, 2), device=DEV)
+    with pytest.raises(M.MCFTError):
+        M.mcft_moe_forward_cached(desc, x, idx, g, acc, 0)

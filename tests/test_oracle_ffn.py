@@ -100,3 +100,52 @@ def test_rel_err_rows():
     row, fro = F.rel_err_rows(y, ref)
     np.testing.assert_allclose(row, [0.01, 0.01])
     assert fro == pytest.approx(np.hypot(0.02, 0.005) / np.linalg.norm(ref))
+
+
+def _lora(g, d, w, r):
+    return (g.standard_normal((r, d)), g.standard_normal((w, r)), g.standard_normal((r, d)),
+            g.standard_normal((w, r)), g.standard_normal((r, w)), g.standard_normal((d, r)))
+
+
+def test_lora_zero_b_is_base_expert():
+    g = np.random.default_rng(5)
+    d, w, r = 6, 4, 2
+    x = g.standard_normal((3, d))
+    ex = _experts(g, 1, d, w)[0]
+    a1, b1, a3, b3, a2, b2 = _lora(g, d, w, r)
+    z = (a1, 0 * b1, a3, 0 * b3, a2, 0 * b2)
+    np.testing.assert_allclose(F.expert_lora(x, *ex, z, 2.0), F.expert(x, *ex), rtol=1e-13)
+
+
+def test_lora_equals_merged_weights():
+    """W x + s B (A x) == (W + s B A) x: the adapter form against merged weights."""
+    g = np.random.default_rng(6)
+    d, w, r, s = 7, 5, 3, 2.0
+    x = g.standard_normal((4, d))
+    w1, w3, w2 = _experts(g, 1, d, w)[0]
+    a1, b1, a3, b3, a2, b2 = _lora(g, d, w, r)
+    merged = (w1 + s * b1 @ a1, w3 + s * b3 @ a3, w2 + s * b2 @ a2)
+    np.testing.assert_allclose(F.expert_lora(x, w1, w3, w2, (a1, b1, a3, b3, a2, b2), s),
+                               F.expert(x, *merged), rtol=1e-11)
+    for t in range(4):  # and against naive loops on the merged weights
+        np.testing.assert_allclose(F.expert(x[t:t + 1], *merged)[0], _naive_expert(x[t], *merged),
+                                   rtol=1e-11)
+
+
+def test_lora_in_layer_matches_per_expert_sum():
+    g = np.random.default_rng(7)
+    E, K, d, w, r, T = 3, 2, 5, 4, 2, 6
+    x = g.standard_normal((T, d))
+    ex = _experts(g, E, d, w)
+    sh = _experts(g, 1, d, w)
+    ad = [_lora(g, d, w, r), None, _lora(g, d, w, r)]
+    sad = [_lora(g, d, w, r)]
+    idx = np.array([[0, 1], [2, 0], [1, 2], [0, 2], [2, 1], [1, 0]], np.int32)
+    gate = g.uniform(size=(T, K))
+    y = F.moe_layer(x, idx, gate, ex, sh, lora=ad, shared_lora=sad, lora_scale=2.0)
+    for t in range(T):
+        ref = sum(gate[t, k] * (F.expert(x[t:t + 1], *ex[idx[t, k]]) if ad[idx[t, k]] is None else
+                                F.expert_lora(x[t:t + 1], *ex[idx[t, k]], ad[idx[t, k]], 2.0))[0]
+                  for k in range(K))
+        ref = ref + F.expert_lora(x[t:t + 1], *sh[0], sad[0], 2.0)[0]
+        np.testing.assert_allclose(y[t], ref, rtol=1e-11)
