@@ -133,6 +133,29 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
                              const void* const* shared, void* y, void* workspace, size_t ws_bytes,
                              mcft_stream_t stream);
 
+/* mcft_moe_forward_lora / mcft_moe_workspace_size_lora: the same layer forward with LoRA
+ * adapters on the experts, the Stage-2 co-adaptation forward (Section 3.2: routers and experts are
+ * fine-tuned under the fixed mask, the experts through LoRA; Appendix B: rank 8, alpha 16). Each
+ * projection of an adapted expert becomes W v + s B (A v), s = lora_scale (alpha / rank):
+ *   F(x) = (W2 + s B2 A2) (silu((W1 + s B1 A1) x) * ((W3 + s B3 A3) x)).
+ *   expert_lora  host array [E] of device pointers to packed adapter blocks, NULL for an expert
+ *                without an adapter; block layout (layer dtype, row-major), r = lora_rank:
+ *                [A1 (r x d) | B1 (w x r) | A3 (r x d) | B3 (w x r) | A2 (r x w) | B2 (d x r)],
+ *                3 r (d + w) elements, 16-byte aligned
+ *   shared_lora  host array [n_shared], same layout (NULL entries allowed; NULL if n_shared = 0)
+ *   lora_rank    8 or 16 (MCFT_ERR_UNSUPPORTED otherwise); lora_scale finite
+ * The workspace needs mcft_moe_workspace_size_lora(desc, lora_rank, T) bytes. The down
+ * projections A v run in a small kernel per stage; the up projections are added in the epilogue
+ * of the expert GEMM / GEMV of every path. No dropout (a forward whose output is compared). */
+mcft_status mcft_moe_workspace_size_lora(const mcft_layer_desc* desc, int lora_rank, int T_max,
+                                         size_t* bytes);
+mcft_status mcft_moe_forward_lora(const mcft_layer_desc* desc, const void* x, int T,
+                                  const int32_t* idx, const float* gate,
+                                  const void* const* experts, const void* const* shared,
+                                  const void* const* expert_lora, const void* const* shared_lora,
+                                  int lora_rank, float lora_scale, void* y, void* workspace,
+                                  size_t ws_bytes, mcft_stream_t stream);
+
 /* mcft_moe_forward_noalloc: the same computation as mcft_moe_forward (same arguments, minus the
  * workspace), for callers that cannot allocate device memory when they run a layer, such as a
  * plugin inside an application that owns every device allocation, or a decode loop that cannot

@@ -96,8 +96,9 @@ unsigned* device_error_word() {
   return static_cast<unsigned*>(p);
 }
 
-WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T) {
+WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lrank) {
   WsLayout L{};
+  L.lrank = lrank;
   L.tc = dtype == MCFT_BF16 && T > 64 && d % 256 == 0 && w % 128 == 0;
   L.decode = !L.tc && dtype == MCFT_BF16;
   L.ks = L.decode ? decode_ksplit(T) : 1;
@@ -113,6 +114,8 @@ WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T) {
   L.xp = o;   o = align256(o + (L.tc ? size_t(L.mcap) * d * 2 : 0));
   L.h = o;    o = align256(o + size_t(L.mcap) * w * (dtype == MCFT_BF16 ? 2 : 4));
   L.o = o;    o = align256(o + size_t(L.ks) * L.mcap * d * 4);
+  L.u13 = o;  o = align256(o + size_t(L.mcap) * 2 * lrank * 4);
+  L.u2 = o;   o = align256(o + size_t(L.mcap) * lrank * 4);
   L.total = o;
   return L;
 }
@@ -257,26 +260,43 @@ mcft_status mcft_route(const mcft_layer_desc* desc, const void* x, int T, const 
   return MCFT_OK;
 }
 
-mcft_status mcft_moe_workspace_size(const mcft_layer_desc* desc, int T_max, size_t* bytes) {
-  mcft_status st = check_desc(desc);
-  if (st != MCFT_OK) return st;
-  if (T_max < 0 || !bytes) return fail(MCFT_ERR_INVALID, "T_max < 0 or bytes is NULL");
+}  // extern "C"
+
+namespace {
+
+size_t workspace_bytes(const mcft_layer_desc* desc, int T_max, int lrank) {
   // the largest layout over every T <= T_max (the decode path's split depends on T)
   size_t best = 0;
   const int upto = T_max < 64 ? T_max : 64;
   for (int T = 0; T <= upto + 1; ++T) {
     const int t = T <= upto ? T : T_max;
-    const WsLayout L = ws_layout(desc->d, desc->E, desc->K, desc->w, desc->n_shared, desc->dtype, t);
+    const WsLayout L =
+        ws_layout(desc->d, desc->E, desc->K, desc->w, desc->n_shared, desc->dtype, t, lrank);
     if (L.total > best) best = L.total;
   }
-  *bytes = best;
+  return best;
+}
+
+mcft_status check_lora(int rank, float scale) {
+  if (rank != 8 && rank != 16)
+    return fail(MCFT_ERR_UNSUPPORTED, "LoRA rank %d (supported: 8, 16)", rank);
+  if (!(scale == scale) || scale > 3.4e38f || scale < -3.4e38f)
+    return fail(MCFT_ERR_INVALID, "LoRA scale must be finite");
   return MCFT_OK;
 }
 
-mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, const int32_t* idx,
-                             const float* gate, const void* const* experts,
-                             const void* const* shared, void* y, void* workspace, size_t ws_bytes,
-                             mcft_stream_t stream) {
+struct LoraArgs {
+  const void* const* expert;  // host [E] adapter blocks (NULL entries: no adapter)
+  const void* const* shared;  // host [S]
+  int rank;
+  float scale;
+};
+
+// Permutation, grouped SwiGLU FFN (optionally with LoRA adapters) and combine.
+mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, const int32_t* idx,
+                         const float* gate, const void* const* experts, const void* const* shared,
+                         const LoraArgs* lora, void* y, void* workspace, size_t ws_bytes,
+                         cudaStream_t stream) {
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
@@ -289,7 +309,8 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
   if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15u)
     return fail(MCFT_ERR_INVALID, "x and y must be 16-byte aligned");
   const int E = desc->E, S = desc->n_shared, K = desc->K;
-  const WsLayout L = ws_layout(desc->d, E, K, desc->w, S, desc->dtype, T);
+  const int lrank = lora ? lora->rank : 0;
+  const WsLayout L = ws_layout(desc->d, E, K, desc->w, S, desc->dtype, T, lrank);
   if (ws_bytes < L.total)
     return fail(MCFT_ERR_INVALID, "workspace of %zu bytes < %zu needed", ws_bytes, L.total);
   for (int e = 0; e < E; ++e)
@@ -298,6 +319,15 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
   for (int s = 0; s < S; ++s)
     if (!shared[s] || (reinterpret_cast<uintptr_t>(shared[s]) & 15u))
       return fail(MCFT_ERR_INVALID, "shared expert %d block is NULL or misaligned", s);
+  if (lora) {
+    if (!lora->expert || (S > 0 && !lora->shared))
+      return fail(MCFT_ERR_INVALID, "NULL adapter array");
+    for (int i = 0; i < E + S; ++i) {
+      const void* p = i < E ? lora->expert[i] : lora->shared[i - E];
+      if (reinterpret_cast<uintptr_t>(p) & 15u)
+        return fail(MCFT_ERR_INVALID, "adapter block %d is not 16-byte aligned", i);
+    }
+  }
 
   char* ws = static_cast<char*>(workspace);
   WsHeader* hdr = reinterpret_cast<WsHeader*>(ws + L.hdr);
@@ -328,23 +358,108 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
   fa.nseg = E + S;
   fa.E = E;
   fa.err = err;
+  LoraDownArgs la{};
+  if (lora) {
+    for (int i = 0; i < E; ++i) fa.lblk[i] = lora->expert[i];
+    for (int s = 0; s < S; ++s) fa.lblk[E + s] = lora->shared[s];
+    fa.lrank = lrank;
+    fa.lscale = lora->scale;
+    fa.u13 = reinterpret_cast<float*>(ws + L.u13);
+    fa.u2 = reinterpret_cast<float*>(ws + L.u2);
+    const LoraOffsets lo = lora_offsets(desc->d, desc->w, lrank);
+    la.row_tok = perm;
+    la.off = off;
+    la.hdr = hdr;
+    la.nseg = E + S;
+    for (int i = 0; i < E + S; ++i) la.lblk[i] = fa.lblk[i];
+    la.r = lrank;
+    // u13[q] = [A1 x ; A3 x] for the token of every permuted row
+    la.in = x;
+    la.in_stride = size_t(desc->d);
+    la.by_token = 1;
+    la.a_off0 = lo.a1;
+    la.a_off1 = lo.a3;
+    la.K = desc->d;
+    la.u = const_cast<float*>(fa.u13);
+    la.ustride = 2 * lrank;
+    e = launch_lora_down(la, desc->dtype, 2 * lrank, L.mcap, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "LoRA kernel launch");
+  }
+  auto ffn = [&](int stages) -> cudaError_t {
+    if (L.tc) return launch_ffn_tc(fa, ws + L.xp, L.mcap, num_sms(), stream, stages);
+    if (L.decode) return launch_ffn_decode(fa, num_sms(), stream, stages);
+    return launch_ffn_rowwise(fa, desc->dtype, num_sms(), stream, stages);
+  };
   if (L.tc) {
     GatherArgs ga{x, perm, hdr, ws + L.xp, desc->d, L.mcap};
     e = launch_gather(ga, stream);
     if (e != cudaSuccess) return cuda_fail(e, "gather kernel launch");
-    e = launch_ffn_tc(fa, ws + L.xp, L.mcap, num_sms(), stream);
-    if (e != cudaSuccess) return cuda_fail(e, "tensor-core expert GEMM launch");
-  } else if (L.decode) {
-    e = launch_ffn_decode(fa, num_sms(), stream);
-    if (e != cudaSuccess) return cuda_fail(e, "decode expert FFN launch");
-  } else {
-    e = launch_ffn_rowwise(fa, desc->dtype, num_sms(), stream);
+  }
+  e = ffn(lora ? 1 : 3);
+  if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
+  if (lora) {
+    // u2[q] = A2 h_q for every permuted row, then the down projection with its adapter
+    const LoraOffsets lo = lora_offsets(desc->d, desc->w, lrank);
+    la.in = fa.h;
+    la.in_stride = size_t(desc->w);
+    la.by_token = 0;
+    la.a_off0 = lo.a2;
+    la.a_off1 = 0;
+    la.K = desc->w;
+    la.u = const_cast<float*>(fa.u2);
+    la.ustride = lrank;
+    e = launch_lora_down(la, desc->dtype, lrank, L.mcap, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "LoRA kernel launch");
+    e = ffn(2);
     if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
   }
   CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S, L.ks, fa.o_plane};
   e = launch_combine(ca, desc->dtype, stream);
   if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
   return MCFT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+mcft_status mcft_moe_workspace_size(const mcft_layer_desc* desc, int T_max, size_t* bytes) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T_max < 0 || !bytes) return fail(MCFT_ERR_INVALID, "T_max < 0 or bytes is NULL");
+  *bytes = workspace_bytes(desc, T_max, 0);
+  return MCFT_OK;
+}
+
+mcft_status mcft_moe_workspace_size_lora(const mcft_layer_desc* desc, int lora_rank, int T_max,
+                                         size_t* bytes) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  st = check_lora(lora_rank, 1.f);
+  if (st != MCFT_OK) return st;
+  if (T_max < 0 || !bytes) return fail(MCFT_ERR_INVALID, "T_max < 0 or bytes is NULL");
+  *bytes = workspace_bytes(desc, T_max, lora_rank);
+  return MCFT_OK;
+}
+
+mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, const int32_t* idx,
+                             const float* gate, const void* const* experts,
+                             const void* const* shared, void* y, void* workspace, size_t ws_bytes,
+                             mcft_stream_t stream) {
+  return forward_impl(desc, x, T, idx, gate, experts, shared, nullptr, y, workspace, ws_bytes,
+                      stream);
+}
+
+mcft_status mcft_moe_forward_lora(const mcft_layer_desc* desc, const void* x, int T,
+                                  const int32_t* idx, const float* gate,
+                                  const void* const* experts, const void* const* shared,
+                                  const void* const* expert_lora, const void* const* shared_lora,
+                                  int lora_rank, float lora_scale, void* y, void* workspace,
+                                  size_t ws_bytes, mcft_stream_t stream) {
+  mcft_status st = check_lora(lora_rank, lora_scale);
+  if (st != MCFT_OK) return st;
+  const LoraArgs la{expert_lora, shared_lora, lora_rank, lora_scale};
+  return forward_impl(desc, x, T, idx, gate, experts, shared, &la, y, workspace, ws_bytes, stream);
 }
 
 // ------------------------------------------------------------------------------------------------

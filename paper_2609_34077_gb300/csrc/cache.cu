@@ -31,12 +31,16 @@ __device__ __forceinline__ bool victim_before(int policy, int s, int v, const in
 }
 
 __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ CacheStepArgs a) {
+  __shared__ int32_t s_tag[kMaxE];
+  __shared__ int64_t s_last[kMaxE], s_ins[kMaxE], s_freq[kMaxE];
+  __shared__ int32_t s_out[1 + 3 * kMaxE];  // n_miss, miss experts, miss locations, loc_of
   const int lane = threadIdx.x;
+  const int B = a.B, E = a.E;
   unsigned long long mine = 0;
   int bad = 0;
   for (int i = lane; i < a.n; i += 32) {
     const int e = a.idx[i];
-    if (e < 0 || e >= a.E) bad = 1;
+    if (e < 0 || e >= E) bad = 1;
     else mine |= 1ull << e;
   }
 #pragma unroll
@@ -44,91 +48,107 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
     mine |= __shfl_xor_sync(0xffffffffu, mine, o);
     bad |= __shfl_xor_sync(0xffffffffu, bad, o);
   }
-  if (lane != 0) return;
   if (bad) {  // no state change on bad input
-    set_error(a.err, kErrInvalid);
-    a.miss_out[0] = 0;
-    a.miss_dev[0] = 0;
-    *a.ready = 0;
-    for (int e = 0; e < a.E; ++e) a.ptr_tab[e] = 0;
+    if (lane == 0) {
+      set_error(a.err, kErrInvalid);
+      a.miss_out[0] = 0;
+      a.miss_dev[0] = 0;
+      *a.ready = 0;
+    }
+    for (int e = lane; e < E; e += 32) a.ptr_tab[e] = 0;
     __threadfence_system();
     return;
   }
-  const int B = a.B, E = a.E;
   int32_t* tag = a.tag + size_t(a.layer) * B;
   int64_t* last = a.last + size_t(a.layer) * B;
   int64_t* ins = a.ins + size_t(a.layer) * B;
   int64_t* freq = a.freq + size_t(a.layer) * E;
-  const int64_t t = a.step[a.layer];
-  int32_t* out = a.miss_out;
-  int32_t* m_exp = out + 1;
-  int32_t* m_loc = out + 1 + E;
-  int32_t* loc_of = out + 1 + 2 * E;
-  for (int e = 0; e < E; ++e) {
-    loc_of[e] = -1;
-    if ((mine >> e) & 1ull) freq[e] += 1;
+  // stage the layer's state in shared memory (one load per lane)
+  for (int i = lane; i < B; i += 32) {
+    s_tag[i] = tag[i];
+    s_last[i] = last[i];
+    s_ins[i] = ins[i];
   }
-
+  for (int e = lane; e < E; e += 32) s_freq[e] = freq[e] + ((mine >> e) & 1ull);
+  __syncwarp();
   unsigned long long cached = 0;
-  int hits = 0;
-  for (int s = 0; s < B; ++s) {
-    const int e = tag[s];
-    if (e < 0) continue;
-    cached |= 1ull << e;
-    if ((mine >> e) & 1ull) {
-      last[s] = t;
-      loc_of[e] = s;
-      ++hits;
-    }
-  }
-  int nm = 0, nbyp = 0;
-  unsigned long long miss = mine & ~cached;
-  while (miss) {
-    const int e = __ffsll(static_cast<long long>(miss)) - 1;  // ascending expert id
-    miss &= miss - 1;
-    int slot = -1;
-    for (int s = 0; s < B; ++s)
-      if (tag[s] < 0) { slot = s; break; }
-    if (slot < 0) {
-      for (int s = 0; s < B; ++s) {
-        if (last[s] >= t) continue;  // used at this step: never a victim
-        if (slot < 0 || victim_before(a.policy, s, slot, tag, last, ins, freq)) slot = s;
+  int hits = 0, nm = 0, nbyp = 0;
+  const int64_t t = a.step[a.layer];
+  if (lane == 0) {
+    int32_t* m_exp = s_out + 1;
+    int32_t* m_loc = s_out + 1 + E;
+    int32_t* loc_of = s_out + 1 + 2 * E;
+    for (int e = 0; e < E; ++e) loc_of[e] = -1;
+    for (int sl = 0; sl < B; ++sl) {
+      const int e = s_tag[sl];
+      if (e < 0) continue;
+      cached |= 1ull << e;
+      if ((mine >> e) & 1ull) {
+        s_last[sl] = t;
+        loc_of[e] = sl;
+        ++hits;
       }
     }
-    if (slot < 0) {
+    unsigned long long miss = mine & ~cached;
+    while (miss) {
+      const int e = __ffsll(static_cast<long long>(miss)) - 1;  // ascending expert id
+      miss &= miss - 1;
+      int slot = -1;
+      for (int sl = 0; sl < B; ++sl)
+        if (s_tag[sl] < 0) { slot = sl; break; }
+      if (slot < 0) {
+        for (int sl = 0; sl < B; ++sl) {
+          if (s_last[sl] >= t) continue;  // used at this step: never a victim
+          if (slot < 0 || victim_before(a.policy, sl, slot, s_tag, s_last, s_ins, s_freq)) slot = sl;
+        }
+      }
       m_exp[nm] = e;
-      m_loc[nm] = -1;
-      loc_of[e] = B + nbyp;
-      ++nbyp;
-    } else {
-      tag[slot] = e;
-      last[slot] = t;
-      ins[slot] = t;
-      m_exp[nm] = e;
-      m_loc[nm] = slot;
-      loc_of[e] = slot;
+      if (slot < 0) {
+        m_loc[nm] = -1;
+        loc_of[e] = B + nbyp;
+        ++nbyp;
+      } else {
+        s_tag[slot] = e;
+        s_last[slot] = t;
+        s_ins[slot] = t;
+        m_loc[nm] = slot;
+        loc_of[e] = slot;
+      }
+      ++nm;
     }
-    ++nm;
+    s_out[0] = nm;
+    a.step[a.layer] = t + 1;
+    unsigned long long* c = a.counters + size_t(a.layer) * 3;
+    c[0] += hits;
+    c[1] += nm;
+    c[2] += nbyp;
   }
-  out[0] = nm;
-  // device copies for the device-driven fetch and the forward that follows it
-  unsigned long long hitmask = 0;
-  for (int i = 0; i < 1 + 3 * E; ++i) a.miss_dev[i] = out[i];
-  for (int e = 0; e < E; ++e) {
-    const int loc = loc_of[e];
+  cached = __shfl_sync(0xffffffffu, cached, 0);
+  __syncwarp();
+  // write back the state and publish the step's miss list and expert table (all lanes)
+  for (int i = lane; i < B; i += 32) {
+    tag[i] = s_tag[i];
+    last[i] = s_last[i];
+    ins[i] = s_ins[i];
+  }
+  for (int e = lane; e < E; e += 32) freq[e] = s_freq[e];
+  for (int i = lane; i < 1 + 3 * E; i += 32) {
+    a.miss_out[i] = s_out[i];
+    a.miss_dev[i] = s_out[i];
+  }
+  unsigned long long hitbits = 0;
+  for (int e = lane; e < E; e += 32) {
+    const int loc = s_out[1 + 2 * E + e];
     unsigned long long p = 0;
     if (loc >= 0 && a.slots)
       p = reinterpret_cast<unsigned long long>(loc < B ? a.slots + size_t(loc) * a.expert_bytes
                                                        : a.staging + size_t(loc - B) * a.expert_bytes);
     a.ptr_tab[e] = p;
-    if (loc >= 0 && loc < B && ((cached >> e) & 1ull)) hitmask |= 1ull << e;
+    if (loc >= 0 && loc < B && ((cached >> e) & 1ull)) hitbits |= 1ull << e;
   }
-  *a.ready = hitmask;
-  a.step[a.layer] = t + 1;
-  unsigned long long* c = a.counters + size_t(a.layer) * 3;
-  c[0] += hits;
-  c[1] += nm;
-  c[2] += nbyp;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) hitbits |= __shfl_xor_sync(0xffffffffu, hitbits, o);
+  if (lane == 0) *a.ready = hitbits;
   __threadfence_system();
 }
 

@@ -4,9 +4,10 @@
 // F(x) = W2 (silu(W1 x) * (W3 x)) for each expert segment (Section 3.1, SwiGLU experts). At
 // decode the selected experts' weights are the only large operand, so the kernels are built to
 // read every weight byte once, in whole lines, with many loads in flight:
-//  * a CTA item is 16 consecutive rows of W1 and W3 (GEMM13) or of W2 (GEMM2) of one segment; its
-//    8 warps split the contraction dimension into 8 slices and walk their slice 64 elements at a
-//    time; in each load instruction the 4 lanes of a quad read 64 contiguous bytes of one row;
+//  * a CTA item is RB blocks of 16 consecutive rows of W1 and W3 (GEMM13) or of W2 (GEMM2) of
+//    one segment; its 8 warps are RB x KS (KS = 8 / RB contraction slices per row block, chosen
+//    so every warp walks at least 8 chunks), each walking its slice 64 elements at a time; in
+//    each load instruction the 4 lanes of a quad read 64 contiguous bytes of one row;
 //  * the 16 x 64 weight slab is the A operand of four m16n8k16 MMAs (the contraction order inside
 //    a 64-wide chunk is permuted identically for A and B, which leaves every dot product intact);
 //    the B operand is 8 tokens of the segment, so one A fragment serves up to 32 tokens per pass
@@ -35,28 +36,56 @@ struct DecItems {
   const char* blk[kMaxSeg];
 };
 
-__device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows_per_seg, int ksplit) {
-  if (threadIdx.x == 0) {
+// Work list of this launch: items_per_seg items for every non-empty segment of the phase. Warp 0
+// builds it with one lane per segment (segments s = lane, lane + 32, lane + 64) and a shuffle
+// prefix sum, so the setup costs a few loads of latency, not one per segment.
+__device__ void build_dec_items(DecItems& it, const FfnArgs& a, int items_per_seg, int ksplit) {
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
     const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
-    it.nseg = nseg;
-    it.ksplit = ksplit;
-    int acc = 0;
     const unsigned long long hits = a.ready ? *a.ready : 0ull;
-    for (int s = 0; s <= nseg; ++s) it.off[s] = a.off[s];
-    for (int s = 0; s < nseg; ++s) {
-      it.first[s] = acc;
-      it.blk[s] = reinterpret_cast<const char*>(seg_block(a, s));
-      if (it.off[s + 1] > it.off[s] && seg_in_phase(a, s, hits)) {
-        if (it.blk[s] == nullptr) {  // a selected expert without weights
-          set_error(a.err, kErrInvalid);
-          const_cast<WsHeader*>(a.hdr)->abort = 1;
-          continue;
+    int offs[3], cnt[3];
+    for (int j = 0; j < 3; ++j) {
+      const int s = lane + 32 * j;
+      offs[j] = s <= nseg ? a.off[s] : 0;
+      if (s <= nseg) it.off[s] = offs[j];
+    }
+    __syncwarp();
+    bool bad = false;
+    for (int j = 0; j < 3; ++j) {
+      const int s = lane + 32 * j;
+      cnt[j] = 0;
+      if (s < nseg) {
+        const char* b = reinterpret_cast<const char*>(seg_block(a, s));
+        it.blk[s] = b;
+        if (it.off[s + 1] > offs[j] && seg_in_phase(a, s, hits)) {
+          if (b == nullptr) bad = true;  // a selected expert without weights
+          else cnt[j] = items_per_seg * ksplit;
         }
-        acc += rows_per_seg / kRows * ksplit;
       }
     }
-    it.first[nseg] = acc;
-    it.total = acc;
+    int base = 0;
+    for (int j = 0; j < 3; ++j) {
+      int v = cnt[j];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += u;
+      }
+      const int s = lane + 32 * j;
+      if (s <= nseg) it.first[s] = base + v - cnt[j];
+      base += __shfl_sync(0xffffffffu, v, 31);
+    }
+    const bool any_bad = __any_sync(0xffffffffu, bad);
+    if (lane == 0) {
+      if (any_bad) {  // the other segments still run; later kernels of the call skip their work
+        set_error(a.err, kErrInvalid);
+        const_cast<WsHeader*>(a.hdr)->abort = 1;
+      }
+      it.nseg = nseg;
+      it.ksplit = ksplit;
+      it.total = base;
+    }
   }
   __syncthreads();
 }
@@ -99,17 +128,19 @@ __device__ __forceinline__ void warp_slice(int nch, int parts, int part, int& c0
   c1 = min(nch, c0 + per);
 }
 
-// GEMM13 + SwiGLU for 16 rows (r0..r0+15) and n <= 32 tokens of one segment starting at
-// permuted row q0. red: shared scratch [kWarps][kMaxNG][8][32] floats.
+// GEMM13 + SwiGLU for RB blocks of 16 rows starting at r0 and n <= 32 tokens of one segment
+// starting at permuted row q0; warp w owns row block w / KS and contraction slice w % KS.
+// red: shared scratch [kWarps][kMaxNG][8][32] floats.
 template <int NG>
-__device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, int r0, int q0, int n,
-                                           float* red) {
+__device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, const void* lblk,
+                                           int r0, int q0, int n, int RB, int KS, float* red) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
+  const int rw = r0 + (warp / KS) * kRows;
   const size_t rowb = size_t(a.d) * 2;
-  const char* w1g = blk + size_t(r0 + g) * rowb + c * 16;
+  const char* w1g = blk + size_t(rw + g) * rowb + c * 16;
   const char* w1h = w1g + 8 * rowb;
-  const char* w3g = blk + size_t(a.w + r0 + g) * rowb + c * 16;
+  const char* w3g = blk + size_t(a.w + rw + g) * rowb + c * 16;
   const char* w3h = w3g + 8 * rowb;
   const char* xr[NG];
 #pragma unroll
@@ -125,7 +156,7 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, in
     for (int i = 0; i < 4; ++i) accg[G][i] = accu[G][i] = 0.f;
 
   int c0, c1;
-  warp_slice(int(rowb / (kChunk * 2)), kWarps, warp, c0, c1);
+  warp_slice(int(rowb / (kChunk * 2)), KS, warp % KS, c0, c1);
   for (int ch = c0; ch < c1; ++ch) {
     const size_t k = size_t(ch) * kChunk * 2;
     const uint4 ag0 = ld_stream16(w1g + k), ag1 = ld_stream16(w1g + k + 64);
@@ -153,36 +184,48 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, in
       red[((warp * kMaxNG + G) * 8 + 4 + i) * 32 + lane] = accu[G][i];
     }
   __syncthreads();
-  // warp G adds the 8 slices of column group G; accumulator element i: row g (i < 2) or g + 8,
-  // token column 2c + (i & 1)
-  if (warp < NG) {
-    const int G = warp;
-    uint16_t* h = reinterpret_cast<uint16_t*>(a.h);
+  // (row block, column group) pairs over the warps; slices added in order. Accumulator element
+  // i: row g (i < 2) or g + 8, token column 2c + (i & 1)
+  uint16_t* h = reinterpret_cast<uint16_t*>(a.h);
+  for (int p = warp; p < RB * NG; p += kWarps) {
+    const int rb = p / NG, G = p % NG;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       float sg = 0.f, su = 0.f;
-#pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
+      for (int k = 0; k < KS; ++k) {
+        const int w = rb * KS + k;
         sg += red[((w * kMaxNG + G) * 8 + i) * 32 + lane];
         su += red[((w * kMaxNG + G) * 8 + 4 + i) * 32 + lane];
       }
       const int j = G * 8 + 2 * c + (i & 1);
-      if (j < n) h[size_t(q0 + j) * a.w + r0 + g + (i >= 2 ? 8 : 0)] = f2bf(silu(sg) * su);
+      if (j < n) {
+        const int row = r0 + rb * kRows + g + (i >= 2 ? 8 : 0);
+        if (lblk) {  // LoRA: + s B1 (A1 x), + s B3 (A3 x)
+          const LoraOffsets lo = lora_offsets(a.d, a.w, a.lrank);
+          const float* u = a.u13 + size_t(q0 + j) * 2 * a.lrank;
+          sg += lora_up<__nv_bfloat16>(lblk, lo.b1, row, u, a.lrank, a.lscale);
+          su += lora_up<__nv_bfloat16>(lblk, lo.b3, row, u + a.lrank, a.lrank, a.lscale);
+        }
+        h[size_t(q0 + j) * a.w + row] = f2bf(silu(sg) * su);
+      }
     }
   }
   __syncthreads();
 }
 
-// GEMM2 for 16 output rows (r0..r0+15 of W2), contraction part `kp` of `ks`, and n <= 32 tokens.
+// GEMM2 for RB blocks of 16 output rows of W2 starting at r0, contraction part kp of ks, and
+// n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part.
 // red: shared scratch [kWarps][kMaxNG][4][32] floats. Output plane kp of o.
 template <int NG>
-__device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, int r0, int q0, int n,
-                                          int kp, int ks, float* red) {
+__device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, const void* lblk,
+                                          int r0, int q0, int n, int kp, int ks, int RB, int KS,
+                                          float* red) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
+  const int rw = r0 + (warp / KS) * kRows;
   const size_t rowb = size_t(a.w) * 2;
   const char* w2 = blk + size_t(2) * a.w * a.d * 2;
-  const char* wg = w2 + size_t(r0 + g) * rowb + c * 16;
+  const char* wg = w2 + size_t(rw + g) * rowb + c * 16;
   const char* wh = wg + 8 * rowb;
   const char* hr[NG];
 #pragma unroll
@@ -198,7 +241,7 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, int
 
   int p0, p1, c0, c1;
   warp_slice(int(rowb / (kChunk * 2)), ks, kp, p0, p1);
-  warp_slice(p1 - p0, kWarps, warp, c0, c1);
+  warp_slice(p1 - p0, KS, warp % KS, c0, c1);
 #pragma unroll 2
   for (int ch = p0 + c0; ch < p0 + c1; ++ch) {
     const size_t k = size_t(ch) * kChunk * 2;
@@ -218,53 +261,64 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, int
 #pragma unroll
     for (int i = 0; i < 4; ++i) red[((warp * kMaxNG + G) * 4 + i) * 32 + lane] = acc[G][i];
   __syncthreads();
-  if (warp < NG) {
-    const int G = warp;
-    float* o = a.o + size_t(kp) * a.o_plane;
+  float* o = a.o + size_t(kp) * a.o_plane;
+  for (int p = warp; p < RB * NG; p += kWarps) {
+    const int rb = p / NG, G = p % NG;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       float sum = 0.f;
-#pragma unroll
-      for (int w = 0; w < kWarps; ++w) sum += red[((w * kMaxNG + G) * 4 + i) * 32 + lane];
+      for (int k = 0; k < KS; ++k) sum += red[(((rb * KS + k) * kMaxNG + G) * 4 + i) * 32 + lane];
       const int j = G * 8 + 2 * c + (i & 1);
-      if (j < n) o[size_t(q0 + j) * a.d + r0 + g + (i >= 2 ? 8 : 0)] = sum;
+      if (j < n) {
+        const int row = r0 + rb * kRows + g + (i >= 2 ? 8 : 0);
+        if (lblk && kp == 0)  // LoRA: + s B2 (A2 h), once (in the first partial plane)
+          sum += lora_up<__nv_bfloat16>(lblk, lora_offsets(a.d, a.w, a.lrank).b2, row,
+                                        a.u2 + size_t(q0 + j) * a.lrank, a.lrank, a.lscale);
+        o[size_t(q0 + j) * a.d + row] = sum;
+      }
     }
   }
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_constant__ FfnArgs a) {
+__global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_constant__ FfnArgs a,
+                                                               int RB) {
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  build_dec_items(it, a, a.w, 1);
+  const int KS = kWarps / RB;
+  build_dec_items(it, a, a.w / (kRows * RB), 1);
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
     const int s = dec_seg(it, item);
-    const int r0 = (item - it.first[s]) * kRows;
+    const int r0 = (item - it.first[s]) * kRows * RB;
     const char* blk = it.blk[s];
-    // passes of at most 32 tokens; a second pass re-reads the 16 rows from L2, not HBM
+    const void* lblk = a.lrank ? a.lblk[s] : nullptr;
+    // passes of at most 32 tokens; a second pass re-reads the rows from L2, not HBM
     for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
       const int n = min(kPassTokens, it.off[s + 1] - q0);
-      if (n <= 8) dec13_item<1>(a, blk, r0, q0, n, red);
-      else if (n <= 16) dec13_item<2>(a, blk, r0, q0, n, red);
-      else dec13_item<4>(a, blk, r0, q0, n, red);
+      if (n <= 8) dec13_item<1>(a, blk, lblk, r0, q0, n, RB, KS, red);
+      else if (n <= 16) dec13_item<2>(a, blk, lblk, r0, q0, n, RB, KS, red);
+      else dec13_item<4>(a, blk, lblk, r0, q0, n, RB, KS, red);
     }
   }
 }
 
-__global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_constant__ FfnArgs a) {
+__global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_constant__ FfnArgs a,
+                                                              int RB) {
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 4 * 32];
-  build_dec_items(it, a, a.d, a.ksplit);
+  const int KS = kWarps / RB;
+  build_dec_items(it, a, a.d / (kRows * RB), a.ksplit);
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
     const int s = dec_seg(it, item);
     const int local = item - it.first[s];
-    const int r0 = (local / it.ksplit) * kRows, kp = local % it.ksplit;
+    const int r0 = (local / it.ksplit) * kRows * RB, kp = local % it.ksplit;
     const char* blk = it.blk[s];
+    const void* lblk = a.lrank ? a.lblk[s] : nullptr;
     for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
       const int n = min(kPassTokens, it.off[s + 1] - q0);
-      if (n <= 8) dec2_item<1>(a, blk, r0, q0, n, kp, it.ksplit, red);
-      else if (n <= 16) dec2_item<2>(a, blk, r0, q0, n, kp, it.ksplit, red);
-      else dec2_item<4>(a, blk, r0, q0, n, kp, it.ksplit, red);
+      if (n <= 8) dec2_item<1>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+      else if (n <= 16) dec2_item<2>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+      else dec2_item<4>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
     }
   }
 }
@@ -280,16 +334,31 @@ int blocks_per_sm(const void* fn) {
 
 int decode_ksplit(int T) { return T <= 4 ? 4 : (T <= 16 ? 2 : 1); }
 
-cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s) {
+// Row blocks per CTA item: the smallest RB in {1, 2, 4, 8} whose 8 / RB contraction slices give
+// every warp at least 8 chunks of 64 (while the rows still split into whole items). More slices
+// mean finer items and better balance; fewer mean longer, better pipelined loops.
+int rows_per_item(int rows, int contraction) {
+  const int nch = contraction / kChunk;
+  int rb = 1;
+  while (rb < kWarps && nch / (kWarps / rb) < 8 && rows % (kRows * rb * 2) == 0) rb *= 2;
+  return rb;
+}
+
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
   static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel));
   static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel));
-  prof_begin(kProfDec13, s);
-  dec13_kernel<<<num_sms * nb13, kWarps * 32, 0, s>>>(a);
-  prof_end(kProfDec13, s);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  const int rb13 = rows_per_item(a.w, a.d);
+  const int rb2 = rows_per_item(a.d, a.w / a.ksplit);
+  cudaError_t e = cudaSuccess;
+  if (stages & 1) {
+    prof_begin(kProfDec13, s);
+    dec13_kernel<<<num_sms * nb13, kWarps * 32, 0, s>>>(a, rb13);
+    prof_end(kProfDec13, s);
+    e = cudaGetLastError();
+  }
+  if (e != cudaSuccess || !(stages & 2)) return e;
   prof_begin(kProfDec2, s);
-  dec2_kernel<<<num_sms * nb2, kWarps * 32, 0, s>>>(a);
+  dec2_kernel<<<num_sms * nb2, kWarps * 32, 0, s>>>(a, rb2);
   prof_end(kProfDec2, s);
   return cudaGetLastError();
 }

@@ -78,8 +78,8 @@ __device__ __forceinline__ int find_seg(const Items& it, int item) {
 
 // h[q, r] = silu(W1[r] . x_t) * (W3[r] . x_t) for rows r = r0, r0 + 1 and NT tokens of a segment.
 template <typename TW, int NT>
-__device__ __forceinline__ void ffn13_tile(const FfnArgs& a, const char* blk, int r0, int q0,
-                                           int nt, const int* tok, int lane) {
+__device__ __forceinline__ void ffn13_tile(const FfnArgs& a, const char* blk, const void* lblk,
+                                           int r0, int q0, int nt, const int* tok, int lane) {
   using C = W16<TW>;
   const size_t rowb = size_t(a.d) * sizeof(TW);
   const char* w1a = blk + size_t(r0) * rowb;
@@ -121,9 +121,17 @@ __device__ __forceinline__ void ffn13_tile(const FfnArgs& a, const char* blk, in
 #pragma unroll
   for (int j = 0; j < NT; ++j) {
     if (j < nt) {
-      const float ga = warp_sum(g0[j]), ua = warp_sum(u0[j]);
-      const float gb = warp_sum(g1[j]), ub = warp_sum(u1[j]);
+      float ga = warp_sum(g0[j]), ua = warp_sum(u0[j]);
+      float gb = warp_sum(g1[j]), ub = warp_sum(u1[j]);
       if (lane == j) {
+        if (lblk) {  // LoRA: + s B1 (A1 x), + s B3 (A3 x)
+          const LoraOffsets lo = lora_offsets(a.d, a.w, a.lrank);
+          const float* u = a.u13 + size_t(q0 + j) * 2 * a.lrank;
+          ga += lora_up<TW>(lblk, lo.b1, r0, u, a.lrank, a.lscale);
+          gb += lora_up<TW>(lblk, lo.b1, r0 + 1, u, a.lrank, a.lscale);
+          ua += lora_up<TW>(lblk, lo.b3, r0, u + a.lrank, a.lrank, a.lscale);
+          ub += lora_up<TW>(lblk, lo.b3, r0 + 1, u + a.lrank, a.lrank, a.lscale);
+        }
         float2 v = make_float2(silu(ga) * ua, silu(gb) * ub);
         *reinterpret_cast<float2*>(h + size_t(q0 + j) * a.w + r0) = v;
       }
@@ -133,8 +141,8 @@ __device__ __forceinline__ void ffn13_tile(const FfnArgs& a, const char* blk, in
 
 // o[q, j] = W2[j] . h_q for output rows j = r0, r0 + 1 and NT permuted rows q0.. of a segment.
 template <typename TW, int NT>
-__device__ __forceinline__ void ffn2_tile(const FfnArgs& a, const char* blk, int r0, int q0, int nt,
-                                          int lane) {
+__device__ __forceinline__ void ffn2_tile(const FfnArgs& a, const char* blk, const void* lblk,
+                                          int r0, int q0, int nt, int lane) {
   using C = W16<TW>;
   const size_t rowb = size_t(a.w) * sizeof(TW);
   const char* w2 = blk + size_t(2) * a.w * a.d * sizeof(TW);
@@ -171,8 +179,16 @@ __device__ __forceinline__ void ffn2_tile(const FfnArgs& a, const char* blk, int
 #pragma unroll
   for (int j = 0; j < NT; ++j) {
     if (j < nt) {
-      const float va = warp_sum(s0[j]), vb = warp_sum(s1[j]);
-      if (lane == j) *reinterpret_cast<float2*>(a.o + size_t(q0 + j) * a.d + r0) = make_float2(va, vb);
+      float va = warp_sum(s0[j]), vb = warp_sum(s1[j]);
+      if (lane == j) {
+        if (lblk) {  // LoRA: + s B2 (A2 h)
+          const size_t b2 = lora_offsets(a.d, a.w, a.lrank).b2;
+          const float* u = a.u2 + size_t(q0 + j) * a.lrank;
+          va += lora_up<TW>(lblk, b2, r0, u, a.lrank, a.lscale);
+          vb += lora_up<TW>(lblk, b2, r0 + 1, u, a.lrank, a.lscale);
+        }
+        *reinterpret_cast<float2*>(a.o + size_t(q0 + j) * a.d + r0) = make_float2(va, vb);
+      }
     }
   }
 }
@@ -186,16 +202,17 @@ __global__ void __launch_bounds__(kWarps * 32) ffn13_kernel(const __grid_constan
     const int s = find_seg(it, item);
     const int r0 = (item - it.first[s]) * kRowsPerItem + warp * kRowsPerWarp;
     const char* blk = it.blk[s];
+    const void* lblk = a.lrank ? a.lblk[s] : nullptr;
     const int q_begin = it.off[s], q_end = it.off[s + 1];
     for (int q0 = q_begin; q0 < q_end; q0 += kTokGroup) {
       const int nt = min(kTokGroup, q_end - q0);
       int tok[kTokGroup];
 #pragma unroll
       for (int j = 0; j < kTokGroup; ++j) tok[j] = j < nt ? a.perm[q0 + j] : 0;
-      if (nt == 1) ffn13_tile<TW, 1>(a, blk, r0, q0, nt, tok, lane);
-      else if (nt == 2) ffn13_tile<TW, 2>(a, blk, r0, q0, nt, tok, lane);
-      else if (nt <= 4) ffn13_tile<TW, 4>(a, blk, r0, q0, nt, tok, lane);
-      else ffn13_tile<TW, 8>(a, blk, r0, q0, nt, tok, lane);
+      if (nt == 1) ffn13_tile<TW, 1>(a, blk, lblk, r0, q0, nt, tok, lane);
+      else if (nt == 2) ffn13_tile<TW, 2>(a, blk, lblk, r0, q0, nt, tok, lane);
+      else if (nt <= 4) ffn13_tile<TW, 4>(a, blk, lblk, r0, q0, nt, tok, lane);
+      else ffn13_tile<TW, 8>(a, blk, lblk, r0, q0, nt, tok, lane);
     }
   }
 }
@@ -209,13 +226,14 @@ __global__ void __launch_bounds__(kWarps * 32) ffn2_kernel(const __grid_constant
     const int s = find_seg(it, item);
     const int r0 = (item - it.first[s]) * kRowsPerItem + warp * kRowsPerWarp;
     const char* blk = it.blk[s];
+    const void* lblk = a.lrank ? a.lblk[s] : nullptr;
     const int q_begin = it.off[s], q_end = it.off[s + 1];
     for (int q0 = q_begin; q0 < q_end; q0 += kTokGroup) {
       const int nt = min(kTokGroup, q_end - q0);
-      if (nt == 1) ffn2_tile<TW, 1>(a, blk, r0, q0, nt, lane);
-      else if (nt == 2) ffn2_tile<TW, 2>(a, blk, r0, q0, nt, lane);
-      else if (nt <= 4) ffn2_tile<TW, 4>(a, blk, r0, q0, nt, lane);
-      else ffn2_tile<TW, 8>(a, blk, r0, q0, nt, lane);
+      if (nt == 1) ffn2_tile<TW, 1>(a, blk, lblk, r0, q0, nt, lane);
+      else if (nt == 2) ffn2_tile<TW, 2>(a, blk, lblk, r0, q0, nt, lane);
+      else if (nt <= 4) ffn2_tile<TW, 4>(a, blk, lblk, r0, q0, nt, lane);
+      else ffn2_tile<TW, 8>(a, blk, lblk, r0, q0, nt, lane);
     }
   }
 }
@@ -265,14 +283,17 @@ int resident_blocks(const void* fn, int threads) {
 }
 
 template <typename TW>
-cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s) {
+cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
   static int nb13 = resident_blocks(reinterpret_cast<const void*>(ffn13_kernel<TW>), kWarps * 32);
   static int nb2 = resident_blocks(reinterpret_cast<const void*>(ffn2_kernel<TW>), kWarps * 32);
-  prof_begin(kProfFfn13, s);
-  ffn13_kernel<TW><<<num_sms * nb13, kWarps * 32, 0, s>>>(a);
-  prof_end(kProfFfn13, s);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  cudaError_t e = cudaSuccess;
+  if (stages & 1) {
+    prof_begin(kProfFfn13, s);
+    ffn13_kernel<TW><<<num_sms * nb13, kWarps * 32, 0, s>>>(a);
+    prof_end(kProfFfn13, s);
+    e = cudaGetLastError();
+  }
+  if (e != cudaSuccess || !(stages & 2)) return e;
   prof_begin(kProfFfn2, s);
   ffn2_kernel<TW><<<num_sms * nb2, kWarps * 32, 0, s>>>(a);
   prof_end(kProfFfn2, s);
@@ -281,9 +302,9 @@ cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s) 
 
 }  // namespace
 
-cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s) {
+cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s, int stages) {
   if (dtype != MCFT_F32) return cudaErrorInvalidValue;  // bf16 layers use the decode or TC path
-  return launch_rowwise_typed<float>(a, num_sms, s);
+  return launch_rowwise_typed<float>(a, num_sms, s, stages);
 }
 
 cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s) {

@@ -51,7 +51,30 @@ struct TcParams {
   unsigned* err;
   uint32_t wmask[3];  // segments that have weights
   int nseg, kblocks, ntiles_n, ldo, b_half, group_m;
+  // LoRA (Stage 2): adapter block per segment (NULL: none), down-projections u [rows, ustride],
+  // element offsets of the up matrices (B1, B3 for GEMM13; B2 for GEMM2), scale alpha / r.
+  const char* lblk[kMaxSeg];
+  const float* lu;
+  int lustride;
+  size_t lb0, lb1;
+  float lscale;
 };
+
+// s * <u, B[row]> for rank R (B rows of R bf16 values, u in registers).
+template <int R>
+__device__ __forceinline__ float lora_dot(const char* blk, size_t b_off, int row, const float* u,
+                                          float scale) {
+  const uint4* b = reinterpret_cast<const uint4*>(blk + (b_off + size_t(row) * R) * 2);
+  float acc = 0.f;
+#pragma unroll
+  for (int v = 0; v < R / 8; ++v) {
+    float w8[8];
+    unpack8(__ldg(b + v), w8);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc = fmaf(u[8 * v + i], w8[i], acc);
+  }
+  return scale * acc;
+}
 
 struct SmemCtl {
   uint64_t full[STAGES], empty[STAGES], tfull[2], tempty[2], drain;
@@ -186,7 +209,7 @@ __device__ __forceinline__ int seg_of_row(const SmemCtl* c, int row) {
   return s;
 }
 
-template <int EPI>
+template <int EPI, int LR>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -306,6 +329,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       tc_fence_after();
       const uint32_t taddr = tmem + b * BN + (uint32_t(q * 32) << 16);
       const size_t grow = size_t(mt) * BM + row;
+      // LoRA down-projections of this row (A1 x, A3 x) or (A2 h), kept in registers
+      constexpr int LRA = LR > 0 ? LR : 1;
+      float ua[LRA], ub[LRA];
+      const char* lb = nullptr;
+      if constexpr (LR > 0) {
+        lb = p.lblk[seg_of_row(ctl, mt * BM)];
+        if (lb) {
+          const float* uq = p.lu + grow * p.lustride;
+#pragma unroll
+          for (int j = 0; j < LR; ++j) {
+            ua[j] = uq[j];
+            ub[j] = EPI == EPI_SWIGLU ? uq[LR + j] : 0.f;
+          }
+        }
+      }
       if constexpr (EPI == EPI_SWIGLU) {
         uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo + size_t(nt) * (BN / 2);
 #pragma unroll 1
@@ -314,13 +352,26 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           tmem_ld16(taddr + c, g);
           tmem_ld16(taddr + BN / 2 + c, u);
           tmem_ld_wait();
+          float gf[16], uf[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            gf[i] = __uint_as_float(g[i]);
+            uf[i] = __uint_as_float(u[i]);
+          }
+          if constexpr (LR > 0) {
+            if (lb) {  // + s B1 (A1 x), + s B3 (A3 x)
+              const int n0 = nt * (BN / 2) + c;
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                gf[i] += lora_dot<LR>(lb, p.lb0, n0 + i, ua, p.lscale);
+                uf[i] += lora_dot<LR>(lb, p.lb1, n0 + i, ub, p.lscale);
+              }
+            }
+          }
           uint32_t pk[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const float h0 = silu(__uint_as_float(g[2 * i])) * __uint_as_float(u[2 * i]);
-            const float h1 = silu(__uint_as_float(g[2 * i + 1])) * __uint_as_float(u[2 * i + 1]);
-            pk[i] = pack2bf(h0, h1);
-          }
+          for (int i = 0; i < 8; ++i)
+            pk[i] = pack2bf(silu(gf[2 * i]) * uf[2 * i], silu(gf[2 * i + 1]) * uf[2 * i + 1]);
           uint4* dst = reinterpret_cast<uint4*>(out + c);
           dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
@@ -332,11 +383,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           uint32_t v[16];
           tmem_ld16(taddr + c, v);
           tmem_ld_wait();
+          float f[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[i]);
+          if constexpr (LR > 0) {
+            if (lb) {  // + s B2 (A2 h)
+#pragma unroll
+              for (int i = 0; i < 16; ++i) f[i] += lora_dot<LR>(lb, p.lb0, nt * BN + c + i, ua, p.lscale);
+            }
+          }
           float4* dst = reinterpret_cast<float4*>(out + c);
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
-                                 __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
+          for (int i = 0; i < 4; ++i) dst[i] = make_float4(f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
         }
       }
       tc_fence_before();
@@ -392,21 +450,32 @@ int group_for(size_t a_tile_bytes) {
   return g < 1 ? 1 : int(g > 4096 ? 4096 : g);
 }
 
-template <int EPI>
+template <int EPI, int LR>
 cudaError_t launch_one(const TcParams& p, int num_sms, cudaStream_t s) {
   static cudaError_t attr = cudaFuncSetAttribute(
-      gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+      gemm_tc_kernel<EPI, LR>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (attr != cudaSuccess) return attr;
   const int kid = EPI == EPI_SWIGLU ? kProfGemm13 : kProfGemm2;
   prof_begin(kid, s);
-  gemm_tc_kernel<EPI><<<num_sms, kThreads, kSmemBytes, s>>>(p);
+  gemm_tc_kernel<EPI, LR><<<num_sms, kThreads, kSmemBytes, s>>>(p);
   prof_end(kid, s);
   return cudaGetLastError();
 }
 
+template <int EPI>
+cudaError_t launch_rank(const TcParams& p, int rank, int num_sms, cudaStream_t s) {
+  switch (rank) {
+    case 0: return launch_one<EPI, 0>(p, num_sms, s);
+    case 8: return launch_one<EPI, 8>(p, num_sms, s);
+    case 16: return launch_one<EPI, 16>(p, num_sms, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 }  // namespace
 
-cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s) {
+cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
+                          int stages) {
   TcParams p13, p2;
   memset(&p13, 0, sizeof(p13));
   memset(&p2, 0, sizeof(p2));
@@ -441,9 +510,26 @@ cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sm
   p2.ldo = int(d);
   p2.b_half = 0;
   p2.group_m = group_for(size_t(BM) * w * 2);
-  cudaError_t e = launch_one<EPI_SWIGLU>(p13, num_sms, s);
-  if (e != cudaSuccess) return e;
-  return launch_one<EPI_F32>(p2, num_sms, s);
+  if (a.lrank > 0) {
+    const LoraOffsets lo = lora_offsets(a.d, a.w, a.lrank);
+    for (int sgi = 0; sgi < a.nseg; ++sgi) {
+      p13.lblk[sgi] = reinterpret_cast<const char*>(a.lblk[sgi]);
+      p2.lblk[sgi] = p13.lblk[sgi];
+    }
+    p13.lu = a.u13;
+    p13.lustride = 2 * a.lrank;
+    p13.lb0 = lo.b1;
+    p13.lb1 = lo.b3;
+    p13.lscale = a.lscale;
+    p2.lu = a.u2;
+    p2.lustride = a.lrank;
+    p2.lb0 = lo.b2;
+    p2.lscale = a.lscale;
+  }
+  cudaError_t e = cudaSuccess;
+  if (stages & 1) e = launch_rank<EPI_SWIGLU>(p13, a.lrank, num_sms, s);
+  if (e != cudaSuccess || !(stages & 2)) return e;
+  return launch_rank<EPI_F32>(p2, a.lrank, num_sms, s);
 }
 
 }  // namespace mcft

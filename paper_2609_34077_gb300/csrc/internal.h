@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include "../../include/mcft.h"
+#include "common.cuh"
 
 namespace mcft {
 
@@ -32,14 +33,49 @@ struct WsHeader {
 // Device workspace of one mcft_moe_forward call. Segments 0..E-1 are the routed experts,
 // E..E+S-1 the shared experts (every token). Offsets are in permuted rows.
 struct WsLayout {
+  int lrank;      // LoRA rank (0: no adapters)
   bool tc;        // tensor-core path (bf16, large T)
   bool decode;    // bf16 decode path (T <= 64)
   int pad;        // rows per segment are padded to a multiple of this (128 on the TC path)
   int mcap;       // capacity in permuted rows
   int ks;         // partial planes of o (contraction split of the decode GEMM2)
-  size_t hdr, cnt, off, pos, perm, xp, h, o, total;
+  size_t hdr, cnt, off, pos, perm, xp, h, o, u13, u2, total;
 };
-WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T);
+WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lrank = 0);
+
+// LoRA adapter block of one expert (layer dtype, row-major), element offsets for rank r:
+// [A1 (r x d) | B1 (w x r) | A3 (r x d) | B3 (w x r) | A2 (r x w) | B2 (d x r)].
+struct LoraOffsets {
+  size_t a1, b1, a3, b3, a2, b2, total;
+};
+__host__ __device__ inline LoraOffsets lora_offsets(int d, int w, int r) {
+  LoraOffsets o;
+  o.a1 = 0;
+  o.b1 = size_t(r) * d;
+  o.a3 = o.b1 + size_t(w) * r;
+  o.b3 = o.a3 + size_t(r) * d;
+  o.a2 = o.b3 + size_t(w) * r;
+  o.b2 = o.a2 + size_t(r) * w;
+  o.total = o.b2 + size_t(d) * r;
+  return o;
+}
+
+// LoRA down-projection u[q] = A v_q for the permuted rows (lora.cu).
+struct LoraDownArgs {
+  const void* in;        // input rows: x [T, K] (by token) or h [mcap, K] (by permuted row)
+  size_t in_stride;      // elements per input row
+  const int* row_tok;    // token of each permuted row, -1 for padding rows
+  int by_token;          // 1: input row = row_tok[q]; 0: input row = q
+  const int* off;
+  const WsHeader* hdr;
+  int nseg;
+  const void* lblk[72];  // adapter block of each segment (NULL: none)
+  size_t a_off0, a_off1; // element offsets of the A matrices used (second only at stage 13)
+  int r, K;              // rank, contraction length
+  float* u;              // output [mcap, ustride]
+  int ustride;
+};
+cudaError_t launch_lora_down(const LoraDownArgs& a, int dtype, int outs, int mcap, cudaStream_t s);
 
 struct PermuteArgs {
   const int32_t* idx;
@@ -79,7 +115,40 @@ struct FfnArgs {
   const unsigned long long* wtab;
   const unsigned long long* ready;
   int phase;
+  // LoRA (Stage 2): adapter block of each segment (NULL: none), rank, scale alpha / r, and the
+  // down-projections u13 [mcap, 2r] (A1 x, A3 x) and u2 [mcap, r] (A2 h) from lora_down.
+  const void* lblk[72];
+  int lrank;
+  float lscale;
+  const float* u13;
+  const float* u2;
 };
+
+// s * sum_j u[j] B[row][j] for a LoRA up-projection B [rows, r] (layer dtype TW).
+template <typename TW>
+__device__ __forceinline__ float lora_up(const void* blk, size_t b_off, int row, const float* u,
+                                         int r, float scale);
+template <>
+__device__ __forceinline__ float lora_up<__nv_bfloat16>(const void* blk, size_t b_off, int row,
+                                                        const float* u, int r, float scale) {
+  const char* b = reinterpret_cast<const char*>(blk) + (b_off + size_t(row) * r) * 2;
+  float acc = 0.f;
+  for (int j = 0; j < r; j += 8) {
+    float w8[8];
+    unpack8(__ldg(reinterpret_cast<const uint4*>(b + j * 2)), w8);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc = fmaf(u[j + i], w8[i], acc);
+  }
+  return scale * acc;
+}
+template <>
+__device__ __forceinline__ float lora_up<float>(const void* blk, size_t b_off, int row, const float* u,
+                                                int r, float scale) {
+  const float* b = reinterpret_cast<const float*>(blk) + b_off + size_t(row) * r;
+  float acc = 0.f;
+  for (int j = 0; j < r; ++j) acc = fmaf(u[j], __ldg(b + j), acc);
+  return scale * acc;
+}
 
 // Segment s of a forward: its block address and whether this launch computes it.
 __device__ __forceinline__ const void* seg_block(const FfnArgs& a, int s) {
@@ -90,10 +159,14 @@ __device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned l
   const bool hit = s >= a.E || ((hits >> s) & 1ull);
   return a.phase == 1 ? hit : !hit;
 }
-cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s);  // fp32
-cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s);  // bf16, T <= 64
+// stages: bit 0 = GEMM13 (+ SwiGLU), bit 1 = GEMM2
+cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s,
+                               int stages = 3);  // fp32
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s,
+                              int stages = 3);  // bf16, T <= 64
 int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
-cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s);
+cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
+                          int stages = 3);
 
 struct CombineArgs {
   const float* o;
@@ -144,7 +217,7 @@ mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_er
 
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
-       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfCount };
+       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

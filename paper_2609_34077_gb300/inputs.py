@@ -127,6 +127,30 @@ def expert_block(seed: int, shape: LayerShape, expert, layer: int = 0) -> torch.
     return as_dtype(a, shape.dtype)
 
 
+def lora_block(seed: int, shape: LayerShape, expert, rank: int = 8, layer: int = 0,
+               std_a: float = 0.02, std_b: float = 0.05) -> torch.Tensor:
+    """Packed LoRA adapter of one expert, [A1 (r x d) | B1 (w x r) | A3 (r x d) | B3 (w x r) |
+    A2 (r x w) | B2 (d x r)]; A ~ N(0, std_a^2), B ~ N(0, std_b^2) (trained adapters: B != 0)."""
+    d, w, r = shape.d, shape.w, rank
+    sizes = [r * d, w * r, r * d, w * r, r * w, d * r]
+    parts = []
+    for i, n in enumerate(sizes):
+        parts.append(normal_f32(seed, (shape.name, "lora", layer, expert, rank, i), n,
+                                std_a if i % 2 == 0 else std_b))
+    return as_dtype(np.concatenate(parts), shape.dtype)
+
+
+def split_lora(block: torch.Tensor, shape: LayerShape, rank: int = 8):
+    """View a packed LoRA block as (A1, B1, A3, B3, A2, B2)."""
+    d, w, r = shape.d, shape.w, rank
+    shapes = [(r, d), (w, r), (r, d), (w, r), (r, w), (d, r)]
+    out, o = [], 0
+    for rr, cc in shapes:
+        out.append(block[o:o + rr * cc].view(rr, cc))
+        o += rr * cc
+    return tuple(out)
+
+
 def split_expert(block: torch.Tensor, shape: LayerShape):
     """View a packed expert block as (W1 [w,d], W3 [w,d], W2 [d,w])."""
     w, d = shape.w, shape.d

@@ -27,6 +27,9 @@ SIGNATURES = {
     "mcft_moe_workspace_size": (_i, [_vp, _i, C.POINTER(_sz)]),
     "mcft_moe_forward": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "mcft_moe_forward_noalloc": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "mcft_moe_workspace_size_lora": (_i, [_vp, _i, _i, C.POINTER(_sz)]),
+    "mcft_moe_forward_lora": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _vp, _vp, _vp, _i, C.c_float, _vp, _vp,
+                                   _sz, _vp]),
     "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, _i, C.POINTER(_vp)]),
     "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
     "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
@@ -167,6 +170,33 @@ def mcft_moe_forward(desc: LayerDesc, x, idx, gate, experts, shared=(), y=None, 
     _check(lib().mcft_moe_forward(C.byref(desc), _ptr(x), T, _ptr(idx), _ptr(gate),
                                   C.cast(ex, C.c_void_p), C.cast(sh, C.c_void_p), _ptr(y),
                                   _ptr(workspace), workspace.numel(), _stream(stream)))
+    return y
+
+
+def mcft_moe_workspace_size_lora(desc: LayerDesc, rank: int, T_max: int) -> int:
+    n = C.c_size_t(0)
+    _check(lib().mcft_moe_workspace_size_lora(C.byref(desc), int(rank), int(T_max), C.byref(n)))
+    return n.value
+
+
+def mcft_moe_forward_lora(desc: LayerDesc, x, idx, gate, experts, shared=(), expert_lora=None,
+                          shared_lora=None, rank=8, scale=2.0, y=None, workspace=None, stream=None):
+    """Layer forward with LoRA adapters (packed blocks, see include/mcft.h) on the experts."""
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.empty(mcft_moe_workspace_size_lora(desc, rank, T), dtype=torch.uint8,
+                                device=x.device)
+    ex = _ptr_array(experts, desc.E)
+    sh = _ptr_array(shared, desc.n_shared)
+    el = _ptr_array(expert_lora, desc.E)
+    sl = _ptr_array(shared_lora, desc.n_shared)
+    _check(lib().mcft_moe_forward_lora(C.byref(desc), _ptr(x), T, _ptr(idx), _ptr(gate),
+                                       C.cast(ex, C.c_void_p), C.cast(sh, C.c_void_p),
+                                       C.cast(el, C.c_void_p), C.cast(sl, C.c_void_p), int(rank),
+                                       float(scale), _ptr(y), _ptr(workspace), workspace.numel(),
+                                       _stream(stream)))
     return y
 
 

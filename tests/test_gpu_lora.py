@@ -1,0 +1,65 @@
+"""Stage-2 forward with LoRA adapters on the experts (Section 3.2; rank 8 / alpha 16, Appendix B)
+against the oracle, through the C ABI, on the three FFN paths: fp32 (CUDA cores), bf16 decode
+(T <= 64, HBM-streaming GEMV) and bf16 prefill (T > 64, tcgen05 grouped GEMM)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_34077_gb300 import inputs as I
+from paper_2609_34077_gb300 import mcft as M
+from tests.gpu_helpers import TOL_BF16, TOL_F32, check_output, expert_triples, f64, shared_triples, weights
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+TINY_SH = I.LayerShape("lora-f32-shared", d=128, E=8, K=2, w=192, n_shared=1, gate=I.GATE_RENORM,
+                       dtype=I.F32, cache_slots=4, keep=4)
+BF_MIX = I.LayerShape("lora-bf16-mix", d=512, E=8, K=2, w=384, n_shared=0, gate=I.GATE_RENORM,
+                      dtype=I.BF16, cache_slots=4, keep=4)
+BF_DS = I.LayerShape("lora-bf16-ds", d=256, E=16, K=4, w=256, n_shared=2, gate=I.GATE_PLAIN,
+                     dtype=I.BF16, cache_slots=6, keep=8)
+
+
+def _case(shape, T, rank, seed, with_adapter):
+    lw = weights(shape, seed)
+    x = I.hidden_iid(seed + 1, shape, T)
+    ids = I.random_ids(seed + 2, 1, T, shape.K, shape.E, hot=range(shape.keep))[0]
+    gate = np.random.default_rng(seed + 3).uniform(0.05, 1.0, (T, shape.K)).astype(np.float32)
+    ad = [I.lora_block(seed, shape, e, rank) if with_adapter(e) else None for e in range(shape.E)]
+    sad = [I.lora_block(seed, shape, ("shared", s), rank) for s in range(shape.n_shared)]
+    desc = M.desc_of(shape)
+    y = M.mcft_moe_forward_lora(
+        desc, x.to(DEV), torch.from_numpy(ids).to(DEV), torch.from_numpy(gate).to(DEV),
+        [b.to(DEV) for b in lw.experts], [b.to(DEV) for b in lw.shared],
+        [None if b is None else b.to(DEV) for b in ad], [b.to(DEV) for b in sad], rank, 16.0 / rank)
+    M.mcft_device_error()
+    split = lambda b: None if b is None else tuple(f64(t) for t in I.split_lora(b, shape, rank))
+    ref = oracle.ffn.moe_layer(f64(x), ids, gate.astype(np.float64), expert_triples(lw, shape),
+                               shared_triples(lw, shape), lora=[split(b) for b in ad],
+                               shared_lora=[split(b) for b in sad], lora_scale=16.0 / rank)
+    base = oracle.ffn.moe_layer(f64(x), ids, gate.astype(np.float64), expert_triples(lw, shape),
+                                shared_triples(lw, shape))
+    return y, ref, base
+
+
+@pytest.mark.parametrize("shape,T", [(TINY_SH, 7), (TINY_SH, 100), (BF_MIX, 1), (BF_MIX, 16),
+                                     (BF_MIX, 300), (BF_DS, 8), (BF_DS, 64), (BF_DS, 257)],
+                         ids=["f32-T7", "f32-T100", "mix-T1", "mix-T16", "mix-T300", "ds-T8",
+                              "ds-T64", "ds-T257"])
+@pytest.mark.parametrize("rank", [8, 16])
+def test_lora_forward_parity(shape, T, rank):
+    tol = TOL_F32 if shape.dtype == I.F32 else TOL_BF16
+    y, ref, base = _case(shape, T, rank, 60 + T, lambda e: e % 3 != 1)  # some experts unadapted
+    check_output(y, ref, tol, f"{shape.name} T={T} r={rank}")
+    # the adapters change the output well beyond the tolerance (the test would see them missing)
+    row, _ = oracle.ffn.rel_err_rows(base, ref)
+    assert row.max() > 5 * tol
+
+
+def test_lora_rejects_bad_rank():
+    sh = BF_MIX
+    desc = M.desc_of(sh)
+    with pytest.raises(M.MCFTError) as ei:
+        M.mcft_moe_workspace_size_lora(desc, 4, 16)
+    assert ei.value.status == M.MCFT_ERR_UNSUPPORTED
