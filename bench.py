@@ -324,7 +324,11 @@ class DecodeStack:
     """L MoE layers decoding at batch 1, each with its own router, soft prior (random keep-k
     mask), AR(1) hidden-state stream and B cache slots; layers are not chained. The pinned host
     pool holds E distinct expert blocks that every layer aliases (a 32-layer Mixtral pool would be
-    90 GB): fetch counts and bytes are those of distinct per-layer experts."""
+    90 GB): fetch counts and bytes are those of distinct per-layer experts.
+
+    With the device-driven fetch a step has no host synchronisation, so `capture()` records one
+    step of all L layers as a CUDA graph; `step()` then copies the token's hidden states into the
+    graph's input buffer and replays it (one launch per token instead of ~10 per layer)."""
 
     def __init__(self, shape, L, steps, seed, dev, policy="LRU", path="device"):
         from paper_2609_34077_gb300 import mcft as M
@@ -334,11 +338,14 @@ class DecodeStack:
         pool = I.layer_weights(seed, shape, layer=0, pin=True)
         self.pool = pool
         self.shared = [b.to(dev) for b in pool.shared]
-        self.routers, self.priors, self.x = [], [], []
+        self.routers, self.priors = [], []
+        x = torch.empty((steps, L, shape.d), dtype=torch.bfloat16)
         for l in range(L):
             self.routers.append(I.router_weight(seed, shape, l).to(dev))
             self.priors.append(I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep, l)))
-            self.x.append(I.ar1_streams(seed, shape, steps, 1, l)[:, 0].contiguous().to(dev))
+            x[:, l] = I.ar1_streams(seed, shape, steps, 1, l)[:, 0]
+        self.x = x.to(dev)                      # [steps, L, d]
+        self.xin = torch.empty((L, shape.d), dtype=torch.bfloat16, device=dev)
         host = [pool.experts[e] for _ in range(L) for e in range(shape.E)]
         self.cache = M.mcft_cache_create(L, shape.E, shape.cache_slots, shape.expert_bytes, host,
                                          max_assign=shape.K, policy=policy)
@@ -346,13 +353,15 @@ class DecodeStack:
         self.idx = torch.empty((L, shape.K), dtype=torch.int32, device=dev)
         self.gate = torch.empty((L, shape.K), dtype=torch.float32, device=dev)
         self.y = torch.empty((L, shape.d), dtype=torch.bfloat16, device=dev)
-        self.compute = torch.cuda.current_stream(dev)
+        self.compute = torch.cuda.Stream(dev)
         self.copy = torch.cuda.Stream(dev)
+        self.graph = None
 
-    def step(self, s):
+    def layers(self):
+        """Enqueue one decode step of every layer on the compute stream (inputs in self.xin)."""
         M = self.M
         for l in range(self.L):
-            x = self.x[l][s:s + 1]
+            x = self.xin[l:l + 1]
             M.mcft_route(self.desc, x, self.routers[l], M.MCFT_ROUTE_SOFT_PRIOR, prior=self.priors[l],
                          idx=self.idx[l:l + 1], gate=self.gate[l:l + 1], stream=self.compute)
             M.mcft_cache_step(self.cache, l, self.idx[l:l + 1], stream=self.compute)
@@ -367,18 +376,40 @@ class DecodeStack:
                                    self.shared, y=self.y[l:l + 1], workspace=self.ws,
                                    stream=self.compute)
 
+    def capture(self):
+        assert self.path == "device"
+        self.graph = torch.cuda.CUDAGraph()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(self.graph, stream=self.compute):
+            self.layers()
+        torch.cuda.synchronize()
 
-def run_stack(shape, L, steps, warmup, seed, dev, policy="LRU", path="device"):
-    """Decode `warmup + steps` tokens through an L-layer stack; TPOT over the last `steps`."""
+    def step(self, s):
+        # input copy, then the step, in order on the compute stream (replay() launches the graph
+        # on the current stream)
+        with torch.cuda.stream(self.compute):
+            self.xin.copy_(self.x[s], non_blocking=True)
+            if self.graph is not None:
+                self.graph.replay()
+            else:
+                self.layers()
+
+
+def run_stack(shape, L, steps, warmup, seed, dev, policy="LRU", path="device", graph=False):
+    """Decode `warmup + steps` tokens through an L-layer stack; TPOT over the last `steps`.
+    With graph=True the step is captured after the warm-up and replayed (no per-kernel timing)."""
     from paper_2609_34077_gb300 import mcft as M
 
-    S = DecodeStack(shape, L, warmup + steps, seed, dev, policy, path)
+    S = DecodeStack(shape, L, warmup + steps + 1, seed, dev, policy, path)
     for s in range(warmup):
         S.step(s)
     torch.cuda.synchronize()
+    if graph:
+        # the capture records the step but also runs nothing; the cache is untouched by it
+        S.capture()
     h0, f0, b0 = M.mcft_cache_stats(S.cache, -1)
     M.mcft_profile_reset()
-    M.mcft_profile_enable(True)
+    M.mcft_profile_enable(not graph)
     elapsed = time_steps(S.step, warmup, steps, S.compute)
     M.mcft_profile_enable(False)
     prof = M.mcft_profile_read()
@@ -386,16 +417,18 @@ def run_stack(shape, L, steps, warmup, seed, dev, policy="LRU", path="device"):
     h1, f1, b1 = M.mcft_cache_stats(S.cache, -1)
     hits, fetches = h1 - h0, f1 - f0
     res = dict(workload=f"{shape.name} decode stack, {L} layers, batch 1, {policy}",
-               layers=L, policy=policy, fetch_path=path, steps=steps, warmup=warmup,
-               tpot_ms=elapsed * 1e3 / steps, tokens_per_s=steps / elapsed,
+               layers=L, policy=policy, fetch_path=path, cuda_graph=graph, steps=steps,
+               warmup=warmup, tpot_ms=elapsed * 1e3 / steps, tokens_per_s=steps / elapsed,
                fetches_per_token=fetches / steps, hit_rate=hits / max(1, hits + fetches),
                fetches_per_token_whole_stream=f1 / (warmup + steps),
                hit_rate_whole_stream=h1 / max(1, h1 + f1),
                fetch_gb_per_token=fetches * shape.expert_bytes / steps / 1e9,
-               kernel_ms_per_token=sum(v[1] for v in prof.values()) / steps,
-               gpu_launches=int(sum(v[0] for v in prof.values())),
-               kernels={k: dict(launches=v[0], ms=round(v[1], 3)) for k, v in prof.items() if v[0]},
+               link_bound_tpot_ms=fetches * shape.expert_bytes / steps / 210e9 * 1e3,
                host_pool="E distinct pinned blocks aliased by every layer")
+    if not graph:
+        res.update(kernel_ms_per_token=sum(v[1] for v in prof.values()) / steps,
+                   gpu_launches=int(sum(v[0] for v in prof.values())),
+                   kernels={k: dict(launches=v[0], ms=round(v[1], 3)) for k, v in prof.items() if v[0]})
     del S
     torch.cuda.empty_cache()
     return res
@@ -549,6 +582,7 @@ def main():
     ap.add_argument("--workload", default="layer", choices=["layer", "stack-mixtral", "stack-dsv2"],
                     help="layer: the single-layer decode line; stack-*: the full decode stack")
     ap.add_argument("--policy", default="LRU", choices=["LRU", "LFU", "FIFO"])
+    ap.add_argument("--graph", action="store_true", help="stack workloads: replay a captured step")
     args = ap.parse_args()
     if args.workload != "layer":
         import __graft_entry__
@@ -556,7 +590,8 @@ def main():
         __graft_entry__.build()
         torch.cuda.set_device(0)
         shape, L = (I.MIXTRAL, 32) if args.workload == "stack-mixtral" else (I.DSV2_LITE, 26)
-        res = run_stack(shape, L, args.steps, args.warmup, 60, torch.device("cuda", 0), args.policy)
+        res = run_stack(shape, L, args.steps, args.warmup, 60, torch.device("cuda", 0), args.policy,
+                        graph=args.graph)
         res.update(metric="masked MoE decode stack tokens/s", value=res["tokens_per_s"],
                    unit="tokens/s", higher_is_better=True, dtype="bf16", data="synthetic")
         print(json.dumps(res), flush=True)
