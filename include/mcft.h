@@ -222,6 +222,39 @@ mcft_status mcft_cache_step(mcft_cache* cache, int layer, const int32_t* idx, in
 mcft_status mcft_fetch_experts(mcft_cache* cache, int layer, mcft_stream_t compute_stream,
                                mcft_stream_t copy_stream, const void** expert_ptrs);
 
+/* ---------------------------------------------------------------------------------------------
+ * Stage-1 mask machinery (Section 3.2 "Stage 1" Eq. stage1 and "Mask optimization" Eq. ste).
+ *
+ * mcft_mask_sample: per layer l, pi_l = softmax(m~_l) and a binary mask with exactly e_keep ones:
+ * E' = e_keep experts drawn without replacement from pi_l (MultinomialSample), realised by the
+ * Gumbel-top-k rule with caller-drawn uniforms: key_e = log pi_e - log(-log u_e); the e_keep
+ * largest keys are drawn (ties to the lower index). This has the law of sequential draws without
+ * replacement. All pointers device: m_tilde, uniforms [L, E] fp32 (uniforms in (0, 1); one
+ * outside sets the device error word and that expert is never drawn), mask [L, E] bytes out,
+ * pi [L, E] fp32 out. 1 <= e_keep <= E <= 64. */
+mcft_status mcft_mask_sample(const float* m_tilde, const float* uniforms, int L, int E, int e_keep,
+                             uint8_t* mask, float* pi, mcft_stream_t stream);
+
+/* mcft_gate_grad: dL/dg_{t,k} = < dL/dy_t , F_{idx[t,k]}(x_t) > for the batch of the last
+ * mcft_moe_forward (or _lora, _cached) call that used `workspace` with this desc and T: the expert
+ * outputs are read from that workspace, which must be left untouched in between.
+ *   dy device [T, d] layer dtype (gradient of the loss with respect to y); dgate device [T, K]
+ *   fp32 out. */
+mcft_status mcft_gate_grad(const mcft_layer_desc* desc, const void* dy, int T, const void* workspace,
+                           size_t ws_bytes, float* dgate, mcft_stream_t stream);
+
+/* mcft_mask_grad: the straight-through mask gradient of one layer (Eq. ste). The loss reaches m
+ * through the gates of the active experts, computed from p * m with m = 1 on A: renormalised gates
+ * (Mixtral) give dL/dm_e = sum_{t: e in A_t} g_{t,e} (dL/dg_{t,e} - sum_i g_{t,i} dL/dg_{t,i}),
+ * plain gates (DeepSeek) dL/dm_e = sum_{t: e in A_t} g_{t,e} dL/dg_{t,e}; the sum runs over every
+ * token of the batch (deterministic order). Then dL/dm~ = (diag(pi) - pi pi^T) dL/dm.
+ *   idx, gate, dgate device [T, K]; pi device [E]; dm device [E] out; dm_tilde device [E] out,
+ *   or accumulated into when `accumulate` is non-zero (the paper accumulates the mask gradient
+ *   over several steps before one update). */
+mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, const float* gate,
+                           const float* dgate, int T, const float* pi, float* dm, float* dm_tilde,
+                           int accumulate, mcft_stream_t stream);
+
 /* mcft_moe_forward_cached: mcft_moe_forward for a decode step of `layer` whose experts come from
  * the cache, with the fetch driven by the device and overlapped with compute; no host round trip.
  * Call it after mcft_cache_step(cache, layer, idx, ...) on compute_stream, instead of

@@ -10,9 +10,12 @@ Everything is a plain, slow, readable restatement of the paper's definitions in 
 * ``routing``  - router logits, softmax, Top-K under a hard mask or a soft prior, gate weights
   (Section 3.1 Eq. topk; Section 3.2 Eq. stage1 and Eq. inference).
 * ``ffn``      - SwiGLU expert, gated combine, shared experts (Section 3.1 Eq. topk).
-* ``cache``    - per-layer expert cache with LRU replacement, fetch accounting and the hit-rate /
-  fetches-per-token metrics (Section 4.1 "Simulation", Eq. metrics), in two independent formulations.
+* ``cache``    - per-layer expert cache with LRU / LFU / FIFO replacement, fetch accounting and the
+  hit-rate / fetches-per-token metrics (Section 4.1 "Simulation", Eq. metrics), in two independent
+  formulations.
+* ``mask``     - Stage-1 mask sampling and the straight-through mask gradient (Section 3.2
+  Eq. stage1 and Eq. ste).
 
 Pins (tests marked ``not gpu``) tie each function to something other than itself; see the tests.
 """
-from . import cache, ffn, routing  # noqa: F401
+from . import cache, ffn, mask, routing  # noqa: F401

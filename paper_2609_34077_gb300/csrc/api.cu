@@ -598,6 +598,56 @@ mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_s
   return MCFT_OK;
 }
 
+mcft_status mcft_mask_sample(const float* m_tilde, const float* uniforms, int L, int E, int e_keep,
+                             uint8_t* mask, float* pi, mcft_stream_t stream) {
+  if (!m_tilde || !uniforms || !mask || !pi) return fail(MCFT_ERR_INVALID, "NULL pointer argument");
+  if (L < 0 || E < 1) return fail(MCFT_ERR_INVALID, "bad L = %d or E = %d", L, E);
+  if (E > kMaxE) return fail(MCFT_ERR_UNSUPPORTED, "E = %d > %d", E, kMaxE);
+  if (e_keep < 1 || e_keep > E)
+    return fail(MCFT_ERR_INVALID, "E' = %d must be in [1, E = %d]", e_keep, E);
+  if (L == 0) return MCFT_OK;
+  MaskSampleArgs a{m_tilde, uniforms, L, E, e_keep, mask, pi, device_error_word()};
+  cudaError_t e = launch_mask_sample(a, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "mask sampling kernel launch");
+  return MCFT_OK;
+}
+
+mcft_status mcft_gate_grad(const mcft_layer_desc* desc, const void* dy, int T, const void* workspace,
+                           size_t ws_bytes, float* dgate, mcft_stream_t stream) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
+  if (T == 0) return MCFT_OK;
+  if (!dy || !workspace || !dgate) return fail(MCFT_ERR_INVALID, "NULL pointer argument");
+  if (reinterpret_cast<uintptr_t>(dy) & 15u) return fail(MCFT_ERR_INVALID, "dy must be 16-byte aligned");
+  const WsLayout L =
+      ws_layout(desc->d, desc->E, desc->K, desc->w, desc->n_shared, desc->dtype, T);
+  if (ws_bytes < L.o + size_t(L.ks) * L.mcap * desc->d * 4)
+    return fail(MCFT_ERR_INVALID, "workspace of %zu bytes is not a forward workspace for T = %d",
+                ws_bytes, T);
+  const char* ws = static_cast<const char*>(workspace);
+  GateGradArgs a{dy, reinterpret_cast<const float*>(ws + L.o), reinterpret_cast<const int*>(ws + L.pos),
+                 reinterpret_cast<const WsHeader*>(ws + L.hdr), size_t(L.mcap) * desc->d, T, desc->K,
+                 desc->d, L.ks, dgate};
+  cudaError_t e = launch_gate_grad(a, desc->dtype, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gate gradient kernel launch");
+  return MCFT_OK;
+}
+
+mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, const float* gate,
+                           const float* dgate, int T, const float* pi, float* dm, float* dm_tilde,
+                           int accumulate, mcft_stream_t stream) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
+  if (!idx || !gate || !dgate || !pi || !dm || !dm_tilde)
+    return fail(MCFT_ERR_INVALID, "NULL pointer argument");
+  MaskGradArgs a{idx, gate, dgate, pi, T, desc->K, desc->E, desc->gate, accumulate ? 1 : 0, dm, dm_tilde};
+  cudaError_t e = launch_mask_grad(a, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "mask gradient kernel launch");
+  return MCFT_OK;
+}
+
 mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, int T,
                                     const int32_t* idx, const float* gate, mcft_cache* c, int layer,
                                     const void* const* shared, void* y, void* workspace,

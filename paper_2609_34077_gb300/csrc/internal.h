@@ -212,6 +212,39 @@ struct FetchArgs {
 };
 cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s);
 
+// Stage-1 mask machinery (mask.cu)
+struct MaskSampleArgs {
+  const float* m_tilde;   // [L, E]
+  const float* uniforms;  // [L, E] in (0, 1)
+  int L, E, e_keep;
+  uint8_t* mask;          // [L, E] out
+  float* pi;              // [L, E] out
+  unsigned* err;
+};
+cudaError_t launch_mask_sample(const MaskSampleArgs& a, cudaStream_t s);
+
+struct GateGradArgs {
+  const void* dy;      // [T, d] layer dtype
+  const float* o;      // forward workspace: expert output rows, ks planes o_plane apart
+  const int* pos;      // forward workspace: permuted row of each assignment
+  const WsHeader* hdr;
+  size_t o_plane;
+  int T, K, d, ks;
+  float* dgate;        // [T, K] out
+};
+cudaError_t launch_gate_grad(const GateGradArgs& a, int dtype, cudaStream_t s);
+
+struct MaskGradArgs {
+  const int32_t* idx;   // [T, K]
+  const float* gate;    // [T, K]
+  const float* dgate;   // [T, K]
+  const float* pi;      // [E]
+  int T, K, E, gate_mode, accumulate;
+  float* dm;            // [E] out: dL/dm
+  float* dm_tilde;      // [E] out (or accumulated): dL/dm~
+};
+cudaError_t launch_mask_grad(const MaskGradArgs& a, cudaStream_t s);
+
 unsigned* device_error_word();  // device address of the current device's error word
 mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_error() text
 

@@ -1,0 +1,186 @@
+// Stage-1 mask machinery (Section 3.2, Eq. stage1 and Eq. ste).
+//
+// mask_sample: pi = softmax(m~) per layer and E' experts drawn without replacement from pi, as the
+//   Gumbel-top-k rule with caller-provided uniforms: key_e = log pi_e - log(-log u_e), the E'
+//   largest keys (ties to the lower index) form the binary mask. One warp per layer, two experts
+//   per lane, E' rounds of a shuffle arg-max.
+// gate_grad: dL/dg_{t,k} = < dL/dy_t , F_{A_{t,k}}(x_t) >, the expert outputs F being the rows the
+//   forward left in its workspace (summed over its partial planes). One warp per assignment.
+// mask_grad: dL/dm_e = sum over tokens t with e in A_t of g_{t,e} (dg_{t,e} - sum_i g_{t,i} dg_{t,i})
+//   for renormalised gates, g_{t,e} dg_{t,e} for plain gates (the gates of the active experts are
+//   computed from p * m with m = 1 on A); one CTA per expert, every thread walking a fixed stride of
+//   the assignments and a fixed-order tree reduction, so the sum is deterministic. Then
+//   dL/dm~ = (diag(pi) - pi pi^T) dL/dm (straight-through estimator and softmax Jacobian),
+//   optionally accumulated over several steps (the paper accumulates T steps per update).
+#include "common.cuh"
+#include "internal.h"
+
+namespace mcft {
+namespace {
+
+__global__ void __launch_bounds__(32) mask_sample_kernel(const __grid_constant__ MaskSampleArgs a) {
+  const int l = blockIdx.x, lane = threadIdx.x, E = a.E;
+  const float* mt = a.m_tilde + size_t(l) * E;
+  const float* u = a.uniforms + size_t(l) * E;
+  float v[2], key[2];
+  bool ok[2];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int e = lane + 32 * j;
+    v[j] = e < E ? mt[e] : -INFINITY;
+    mx = fmaxf(mx, v[j]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float se = 0.f;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) se += lane + 32 * j < E ? expf(v[j] - mx) : 0.f;
+  se = warp_sum(se);
+  const float lse = logf(se);
+  bool bad = false;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int e = lane + 32 * j;
+    ok[j] = e < E;
+    key[j] = -INFINITY;
+    if (ok[j]) {
+      const float lp = v[j] - mx - lse;  // log pi_e
+      a.pi[size_t(l) * E + e] = expf(lp);
+      const float ue = u[e];
+      if (!(ue > 0.f && ue < 1.f)) {
+        bad = true;
+        ok[j] = false;
+      } else {
+        key[j] = lp - logf(-logf(ue));
+      }
+    }
+  }
+  if (__any_sync(0xffffffffu, bad) && lane == 0) set_error(a.err, kErrInvalid);
+  bool taken[2] = {false, false};
+  for (int r = 0; r < a.e_keep; ++r) {
+    float bv = -INFINITY;
+    int bi = 1 << 30;
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int e = lane + 32 * j;
+      if (ok[j] && !taken[j] && (key[j] > bv || (key[j] == bv && e < bi) || bi == (1 << 30))) {
+        bv = key[j];
+        bi = e;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float v2 = __shfl_xor_sync(0xffffffffu, bv, o);
+      const int i2 = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (v2 > bv || (v2 == bv && i2 < bi)) { bv = v2; bi = i2; }
+    }
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+      if (lane + 32 * j == bi) taken[j] = true;
+  }
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int e = lane + 32 * j;
+    if (e < E) a.mask[size_t(l) * E + e] = taken[j] ? 1 : 0;
+  }
+}
+
+template <typename TY>
+__global__ void __launch_bounds__(256) gate_grad_kernel(const __grid_constant__ GateGradArgs a) {
+  if (a.hdr->abort) return;
+  const int lane = threadIdx.x & 31;
+  const int n = a.T * a.K;
+  for (int i = blockIdx.x * 8 + (threadIdx.x >> 5); i < n; i += gridDim.x * 8) {
+    const int t = i / a.K;
+    const size_t row = size_t(a.pos[i]) * a.d;
+    float acc = 0.f;
+    for (int c = lane * 4; c < a.d; c += 128) {
+      float4 o = *reinterpret_cast<const float4*>(a.o + row + c);
+      for (int p = 1; p < a.ks; ++p) {
+        const float4 u = *reinterpret_cast<const float4*>(a.o + size_t(p) * a.o_plane + row + c);
+        o.x += u.x; o.y += u.y; o.z += u.z; o.w += u.w;
+      }
+      float dy[4];
+      if constexpr (sizeof(TY) == 2) {
+        const uint2 v = *reinterpret_cast<const uint2*>(
+            reinterpret_cast<const uint16_t*>(a.dy) + size_t(t) * a.d + c);
+        dy[0] = bf16lo(v.x); dy[1] = bf16hi(v.x); dy[2] = bf16lo(v.y); dy[3] = bf16hi(v.y);
+      } else {
+        const float4 v = *reinterpret_cast<const float4*>(
+            reinterpret_cast<const float*>(a.dy) + size_t(t) * a.d + c);
+        dy[0] = v.x; dy[1] = v.y; dy[2] = v.z; dy[3] = v.w;
+      }
+      acc = fmaf(dy[0], o.x, acc);
+      acc = fmaf(dy[1], o.y, acc);
+      acc = fmaf(dy[2], o.z, acc);
+      acc = fmaf(dy[3], o.w, acc);
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) a.dgate[i] = acc;
+  }
+}
+
+__global__ void __launch_bounds__(256) mask_grad_kernel(const __grid_constant__ MaskGradArgs a) {
+  __shared__ float part[256];
+  const int e = blockIdx.x, tid = threadIdx.x;
+  const int n = a.T * a.K;
+  float acc = 0.f;
+  for (int i = tid; i < n; i += blockDim.x) {
+    if (a.idx[i] != e) continue;
+    const int t = i / a.K;
+    const float g = a.gate[i], dg = a.dgate[i];
+    if (a.gate_mode == MCFT_GATE_RENORM) {
+      float inner = 0.f;  // sum_i g_{t,i} dL/dg_{t,i}
+      for (int k = 0; k < a.K; ++k)
+        inner = fmaf(a.gate[size_t(t) * a.K + k], a.dgate[size_t(t) * a.K + k], inner);
+      acc += g * (dg - inner);
+    } else {
+      acc += g * dg;
+    }
+  }
+  part[tid] = acc;
+  __syncthreads();
+  for (int s = 128; s > 0; s >>= 1) {
+    if (tid < s) part[tid] += part[tid + s];
+    __syncthreads();
+  }
+  if (tid == 0) a.dm[e] = part[0];
+}
+
+__global__ void __launch_bounds__(32) mask_tilde_kernel(const __grid_constant__ MaskGradArgs a) {
+  const int lane = threadIdx.x, E = a.E;
+  float s = 0.f;
+  for (int e = lane; e < E; e += 32) s += a.pi[e] * a.dm[e];
+  s = warp_sum(s);  // pi . dL/dm
+  for (int e = lane; e < E; e += 32) {
+    const float v = a.pi[e] * (a.dm[e] - s);
+    a.dm_tilde[e] = a.accumulate ? a.dm_tilde[e] + v : v;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_mask_sample(const MaskSampleArgs& a, cudaStream_t s) {
+  mask_sample_kernel<<<a.L, 32, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gate_grad(const GateGradArgs& a, int dtype, cudaStream_t s) {
+  const int n = a.T * a.K;
+  int blocks = (n + 7) / 8;
+  if (blocks > 4096) blocks = 4096;
+  if (dtype == MCFT_BF16) gate_grad_kernel<uint16_t><<<blocks, 256, 0, s>>>(a);
+  else gate_grad_kernel<float><<<blocks, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mask_grad(const MaskGradArgs& a, cudaStream_t s) {
+  mask_grad_kernel<<<a.E, 256, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  mask_tilde_kernel<<<1, 32, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace mcft

@@ -177,6 +177,13 @@ def prior_from_mask(mask: np.ndarray, gamma: float = 2.0) -> np.ndarray:
     return (e / e.sum()).astype(np.float32)
 
 
+def uniforms(seed: int, shape, tag="u") -> np.ndarray:
+    """fp32 uniforms strictly inside (0, 1) (for the mask sampler's Gumbel keys)."""
+    g = np.random.Generator(np.random.Philox(key=_key(seed, tag, tuple(np.atleast_1d(shape)))))
+    u = g.random(size=shape, dtype=np.float64)
+    return np.clip(u, 2.0 ** -24, 1 - 2.0 ** -24).astype(np.float32)
+
+
 def mask_from_ids(E: int, ids) -> np.ndarray:
     m = np.zeros(E, np.uint8)
     m[list(ids)] = 1

@@ -34,6 +34,9 @@ SIGNATURES = {
     "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
     "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
     "mcft_moe_forward_cached": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _sz, _vp, _vp]),
+    "mcft_mask_sample": (_i, [_vp, _vp, _i, _i, _i, _vp, _vp, _vp]),
+    "mcft_gate_grad": (_i, [_vp, _vp, _i, _vp, _sz, _vp, _vp]),
+    "mcft_mask_grad": (_i, [_vp, _vp, _vp, _vp, _i, _vp, _vp, _vp, _i, _vp]),
     "mcft_cache_last_misses": (_i, [_vp, _i, C.POINTER(_i), _vp, _vp]),
     "mcft_cache_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64),
                               C.POINTER(C.c_uint64), _vp]),
@@ -334,3 +337,36 @@ def mcft_profile_read():
     _check(lib().mcft_profile_read(n.value, C.cast(names, C.c_void_p), C.cast(launches, C.c_void_p),
                                    C.cast(ms, C.c_void_p), C.byref(n)))
     return {names[i].decode(): (launches[i], ms[i]) for i in range(n.value)}
+
+
+def mcft_mask_sample(m_tilde, uniforms, e_keep, stream=None):
+    """(mask [L, E] uint8, pi [L, E] fp32) from m~ and uniforms [L, E] (device tensors)."""
+    L, E = m_tilde.shape
+    mask = torch.empty((L, E), dtype=torch.uint8, device=m_tilde.device)
+    pi = torch.empty((L, E), dtype=torch.float32, device=m_tilde.device)
+    _check(lib().mcft_mask_sample(_ptr(m_tilde), _ptr(uniforms), L, E, int(e_keep), _ptr(mask),
+                                  _ptr(pi), _stream(stream)))
+    return mask, pi
+
+
+def mcft_gate_grad(desc: LayerDesc, dy, workspace, dgate=None, stream=None):
+    """dL/dg [T, K] from dL/dy and the workspace of the forward of the same batch."""
+    T = dy.shape[0]
+    if dgate is None:
+        dgate = torch.empty((T, desc.K), dtype=torch.float32, device=dy.device)
+    _check(lib().mcft_gate_grad(C.byref(desc), _ptr(dy), T, _ptr(workspace), workspace.numel(),
+                                _ptr(dgate), _stream(stream)))
+    return dgate
+
+
+def mcft_mask_grad(desc: LayerDesc, idx, gate, dgate, pi, dm=None, dm_tilde=None, accumulate=False,
+                   stream=None):
+    """(dL/dm [E], dL/dm~ [E]) of one layer (straight-through estimator, Eq. ste)."""
+    T = idx.shape[0]
+    if dm is None:
+        dm = torch.empty(desc.E, dtype=torch.float32, device=idx.device)
+    if dm_tilde is None:
+        dm_tilde = torch.zeros(desc.E, dtype=torch.float32, device=idx.device)
+    _check(lib().mcft_mask_grad(C.byref(desc), _ptr(idx), _ptr(gate), _ptr(dgate), T, _ptr(pi),
+                                _ptr(dm), _ptr(dm_tilde), 1 if accumulate else 0, _stream(stream)))
+    return dm, dm_tilde

@@ -18,12 +18,16 @@ STEPS = 1024
 POLICIES = ("LRU", "LFU", "FIFO")
 
 
-@pytest.mark.parametrize("shape,L", [(I.MIXTRAL, 32), (I.DSV2_LITE, 26)], ids=["mixtral-32", "dsv2-26"])
-def test_stack_fetch_counts_exact(shape, L):
+@pytest.mark.parametrize("shape,L,B", [(I.MIXTRAL, 32, 4), (I.DSV2_LITE, 26, 12),
+                                       (I.MIXTRAL, 32, 2), (I.MIXTRAL, 32, 6),
+                                       (I.DSV2_LITE, 26, 24), (I.DSV2_LITE, 26, 36)],
+                         ids=["mixtral-32-B4", "dsv2-26-B12", "mixtral-32-B2", "mixtral-32-B6",
+                              "dsv2-26-B24", "dsv2-26-B36"])
+def test_stack_fetch_counts_exact(shape, L, B):
+    """Also the cache-budget sweep of Fig. 3 (B in {2, 4, 6} Mixtral, {12, 24, 36} DeepSeek)."""
     seed = 50
     desc = M.desc_of(shape)
-    caches = {p: M.mcft_cache_create(L, shape.E, shape.cache_slots, max_assign=shape.K, policy=p)
-              for p in POLICIES}
+    caches = {p: M.mcft_cache_create(L, shape.E, B, max_assign=shape.K, policy=p) for p in POLICIES}
     ref_counts = {p: np.zeros((L, 2), np.int64) for p in POLICIES}  # oracle (hits, fetches)
     exact_layers = []
     for layer in range(L):
@@ -43,7 +47,7 @@ def test_stack_fetch_counts_exact(shape, L):
         for p in POLICIES:
             for s in range(STEPS):
                 M.mcft_cache_step(caches[p], layer, idx[s:s + 1])
-            oc = oracle.cache.SlotCache(shape.E, shape.cache_slots, p)
+            oc = oracle.cache.SlotCache(shape.E, B, p)
             for s in range(STEPS):
                 h, f, b, _ = oc.step(r["idx"][s])
                 ref_counts[p][layer] += (h, f)
@@ -59,4 +63,4 @@ def test_stack_fetch_counts_exact(shape, L):
         n = len(exact_layers)
         hr, fpt = oracle.cache.metrics(tot[0], tot[1], STEPS, n, shape.K)
         assert fpt == pytest.approx(n * shape.K * (1 - hr))  # Eq. metrics at batch 1
-        print(f"{shape.name} {p}: HR {100 * hr:.2f} %  Fetches/tok {fpt:.3f} over {n} layers")
+        print(f"{shape.name} B={B} {p}: HR {100 * hr:.2f} %  Fetches/tok {fpt:.3f} over {n} layers")
