@@ -44,10 +44,12 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f4a9f9398fa959c3", 1.0015,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "a9fca224659abaa5", 1.0017,
                      "profiles/ffn_decode_mixtral_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f4a9f9398fa959c3", 1.0042,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "a9fca224659abaa5", 1.0032,
                     "profiles/ffn_decode_mixtral_decode.md"),
+    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "31f4483ef0759b6d", 1.0002,
+              "profiles/fetch_kernel_mixtral_decode_b16.md"),
 }
 
 
@@ -538,13 +540,22 @@ def _config(batch):
 
 
 def profile_case(case: str, dev) -> int:
-    """A few forwards with every expert resident on the device (no cache, no fetch): the small
-    launch sequence that ncu captures. decode16: Mixtral-shaped decode, batch 16 (rowwise GEMV);
-    decode1: batch 1; prefill: T = 4096 tokens, hard mask keep 4 of 8 (tcgen05 GEMMs)."""
+    """A few forwards: the small launch sequences that ncu captures. decode16 / decode1:
+    Mixtral-shaped decode at batch 16 / 1 with every expert resident (decode FFN); prefill:
+    T = 4096 tokens, hard mask keep 4 of 8 (tcgen05 GEMMs); fetch16: three decode steps at batch
+    16 through the cache with the device-driven fetch (fetch kernel)."""
     from paper_2609_34077_gb300 import mcft as M
 
     sh = I.MIXTRAL
     desc = M.desc_of(sh)
+    if case == "fetch16":  # decode steps with the cache and the device-driven fetch
+        L = DecodeLayer(sh, 16, 7, dev)
+        for s in range(3):
+            L.step(s, path="device")
+        M.mcft_device_error()
+        torch.cuda.synchronize()
+        print(json.dumps({"case": case, "fetches": M.mcft_cache_stats(L.cache, 0)[1]}))
+        return 0
     if case == "prefill":
         T, mode = 4096, M.MCFT_ROUTE_HARD_MASK
         kw = dict(mask=I.keep_mask(7, sh.E, 4))
@@ -577,7 +588,7 @@ def main():
     ap.add_argument("--batch", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
-    ap.add_argument("--case", choices=["decode16", "decode1", "prefill"],
+    ap.add_argument("--case", choices=["decode16", "decode1", "prefill", "fetch16"],
                     help="run only a few resident-expert forwards (for profiler captures)")
     ap.add_argument("--workload", default="layer", choices=["layer", "stack-mixtral", "stack-dsv2"],
                     help="layer: the single-layer decode line; stack-*: the full decode stack")
@@ -652,7 +663,9 @@ def main():
     fetch_roof = dict(bound="host-link", kernel="fetch", unit="GB/s",
                       achieved=fetched / (msf / 1e3) / 1e9 if msf else None, peak=link,
                       peak_source="pinned host-to-device copy probe in this run (352 MB, best of 10)",
-                      traffic=None, alg_bytes_per_launch=fetched / max(1, nf), launches=nf)
+                      traffic=(traffic_ratio("fetch") * fetched / max(1, nf)
+                               if traffic_ratio("fetch") else None),
+                      alg_bytes_per_launch=fetched / max(1, nf), launches=nf)
     fetch_roof["frac"] = fetch_roof["achieved"] / link if msf else None
     line = dict(
         metric=METRIC, value=tokens / max_el, unit="tokens/s", n_gpus=world, steps=args.steps,
