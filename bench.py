@@ -487,9 +487,10 @@ def run_prefill(steps, warmup, seed, dev, peaks):
 # ------------------------------------------------------------------------------------------------
 # CPU oracle timing (the reported baseline, and the reference arm)
 
-def oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0, lw=None):
+def oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0, lw=None, warmup=0, max_steps=None):
     """The CPU oracle (routing + LRU accounting + fp64 SwiGLU combine) on decode steps of the same
-    stream until ~budget_s of work; returns (tokens/s, steps done)."""
+    stream: `warmup` untimed steps, then timed steps until `max_steps` or ~budget_s of work;
+    returns (tokens/s, timed steps)."""
     import oracle
 
     lw = lw or I.layer_weights(seed, shape)
@@ -498,34 +499,46 @@ def oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0, lw=None):
     wr = lw.router.double().numpy()
     ex = [tuple(t.double().numpy() for t in I.split_expert(b, shape)) for b in lw.experts]
     sh = [tuple(t.double().numpy() for t in I.split_expert(b, shape)) for b in lw.shared]
-    cache = oracle.cache.LRUStamps(shape.E, shape.cache_slots)
-    t0 = time.perf_counter()
-    n = 0
-    while True:
-        x = xs[n % STREAM_STEPS].double().numpy()
+    cache = oracle.cache.SlotCache(shape.E, shape.cache_slots, "LRU")
+
+    def step(i):
+        x = xs[i % STREAM_STEPS].double().numpy()
         r = oracle.routing.route(x, wr, shape.K, oracle.routing.MODE_SOFT_PRIOR, shape.gate, prior=prior)
         cache.step(r["idx"])
         oracle.ffn.moe_layer(x, r["idx"], r["gate"], ex, sh)
+
+    for i in range(warmup):
+        step(i)
+    limit = max_steps if max_steps else STREAM_STEPS
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        step(warmup + n)
         n += 1
         el = time.perf_counter() - t0
-        if el >= budget_s or n >= STREAM_STEPS:
+        if el >= budget_s or n >= limit:
             return batch * n / el, n
 
 
 def reference_arm(args, rank, world):
+    """The reference arm: there is no reference implementation to run (the paper ships no code),
+    so this times the CPU oracle as it stands on the host cores, on the same workload, metric and
+    unit: args.warmup untimed decode steps, then up to args.steps timed ones (each one decode step
+    of 16 rows), stopping after two minutes. Under torchrun only rank 0 runs it."""
     if rank != 0:
         return 0
     shape, batch = I.MIXTRAL, 16
     seed = replica_seed(0, 0)
     lw = I.layer_weights(seed, shape)
-    budget = max(2.0, min(20.0, 6.0 * args.steps / max(1, args.steps)))
-    tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=budget, lw=lw)
+    tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=120.0, lw=lw,
+                                        warmup=args.warmup, max_steps=args.steps)
     line = dict(impl="reference", metric=METRIC, value=tps, unit="tokens/s", n_gpus=args.gpus,
-                steps=n, warmup=0, ms_per_step=1e3 * batch / tps, higher_is_better=True,
+                steps=n, warmup=args.warmup, ms_per_step=1e3 * batch / tps, higher_is_better=True,
                 scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
                 config=_config(batch),
                 cpu_baseline=dict(value=tps, unit="tokens/s", cores=_CORES, kind="oracle",
-                                  sample=f"{n} decode steps x batch {batch} of the same stream"),
+                                  sample=f"{n} decode steps x batch {batch} of the same stream "
+                                         f"after {args.warmup} untimed (fp64 numpy)"),
                 e2e=dict(value=tps, unit="tokens/s", h2d_bytes_per_step=0, d2h_bytes_per_step=0))
     print(json.dumps(line), flush=True)
     return 0
