@@ -4,10 +4,11 @@
 // F(x) = W2 (silu(W1 x) * (W3 x)) for each expert segment (Section 3.1, SwiGLU experts). At
 // decode the selected experts' weights are the only large operand, so the kernels are built to
 // read every weight byte once, in whole lines, with many loads in flight:
-//  * a CTA item is RB blocks of 16 consecutive rows of W1 and W3 (GEMM13) or of W2 (GEMM2) of
-//    one segment; its 8 warps are RB x KS (KS = 8 / RB contraction slices per row block, chosen
-//    so every warp walks at least 8 chunks), each walking its slice 64 elements at a time; in
-//    each load instruction the 4 lanes of a quad read 64 contiguous bytes of one row;
+//  * a CTA item is RB blocks of 16 consecutive rows of W1 and W3 (GEMM13), or of 32 rows of W2
+//    (GEMM2, two MMA tiles sharing the activation fragments), of one segment; its 8 warps are
+//    RB x KS (KS = 8 / RB contraction slices per row block, chosen so every warp walks at least 8
+//    chunks), each walking its slice 64 elements at a time; in each load instruction the 4 lanes
+//    of a quad read 64 contiguous bytes of one row;
 //  * the 16 x 64 weight slab is the A operand of four m16n8k16 MMAs (the contraction order inside
 //    a 64-wide chunk is permuted identically for A and B, which leaves every dot product intact);
 //    the B operand is 8 tokens of the segment, so one A fragment serves up to 32 tokens per pass
@@ -24,7 +25,8 @@ namespace mcft {
 namespace {
 
 constexpr int kWarps = 8;
-constexpr int kRows = 16;        // weight rows per CTA item
+constexpr int kRows = 16;        // weight rows per warp (GEMM13: one MMA tile)
+constexpr int kRows2 = 32;       // weight rows per warp (GEMM2: two MMA tiles)
 constexpr int kChunk = 64;       // contraction elements per step (128 bytes of a row)
 constexpr int kPassTokens = 32;  // tokens per pass (4 MMA column groups of 8)
 constexpr int kMaxNG = kPassTokens / 8;
@@ -213,64 +215,73 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
   __syncthreads();
 }
 
-// GEMM2 for RB blocks of 16 output rows of W2 starting at r0, contraction part kp of ks, and
-// n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part.
-// red: shared scratch [kWarps][kMaxNG][4][32] floats. Output plane kp of o.
+// GEMM2 for RB blocks of 32 output rows of W2 starting at r0 (two 16-row MMA tiles per warp that
+// share the h fragments, so each lane keeps 8 weight loads in flight per chunk), contraction part
+// kp of ks, and n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part.
+// red: shared scratch [kWarps][kMaxNG][8][32] floats. Output plane kp of o.
 template <int NG>
 __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, const void* lblk,
                                           int r0, int q0, int n, int kp, int ks, int RB, int KS,
                                           float* red) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
-  const int rw = r0 + (warp / KS) * kRows;
+  const int rw = r0 + (warp / KS) * kRows2;
   const size_t rowb = size_t(a.w) * 2;
   const char* w2 = blk + size_t(2) * a.w * a.d * 2;
-  const char* wg = w2 + size_t(rw + g) * rowb + c * 16;
+  const char* wg = w2 + size_t(rw + g) * rowb + c * 16;  // tile 0: rows g, g + 8
   const char* wh = wg + 8 * rowb;
+  const char* vg = wg + 16 * rowb;                        // tile 1: rows 16 + g, 24 + g
+  const char* vh = wg + 24 * rowb;
   const char* hr[NG];
 #pragma unroll
   for (int G = 0; G < NG; ++G) {
     const int j = G * 8 + g;
     hr[G] = reinterpret_cast<const char*>(a.h) + size_t(q0 + (j < n ? j : 0)) * rowb + c * 16;
   }
-  float acc[NG][4];
+  float acc[NG][8];
 #pragma unroll
   for (int G = 0; G < NG; ++G)
 #pragma unroll
-    for (int i = 0; i < 4; ++i) acc[G][i] = 0.f;
+    for (int i = 0; i < 8; ++i) acc[G][i] = 0.f;
 
   int p0, p1, c0, c1;
   warp_slice(int(rowb / (kChunk * 2)), ks, kp, p0, p1);
   warp_slice(p1 - p0, KS, warp % KS, c0, c1);
-#pragma unroll 2
   for (int ch = p0 + c0; ch < p0 + c1; ++ch) {
     const size_t k = size_t(ch) * kChunk * 2;
     const uint4 ag0 = ld_stream16(wg + k), ag1 = ld_stream16(wg + k + 64);
     const uint4 ah0 = ld_stream16(wh + k), ah1 = ld_stream16(wh + k + 64);
+    const uint4 bg0 = ld_stream16(vg + k), bg1 = ld_stream16(vg + k + 64);
+    const uint4 bh0 = ld_stream16(vh + k), bh1 = ld_stream16(vh + k + 64);
 #pragma unroll
     for (int G = 0; G < NG; ++G) {
       const uint4 x0 = ldg16(hr[G] + k), x1 = ldg16(hr[G] + k + 64);
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t xb0 = word(x0, x1, 2 * j), xb1 = word(x0, x1, 2 * j + 1);
         mma16816(acc[G], word(ag0, ag1, 2 * j), word(ah0, ah1, 2 * j), word(ag0, ag1, 2 * j + 1),
-                 word(ah0, ah1, 2 * j + 1), word(x0, x1, 2 * j), word(x0, x1, 2 * j + 1));
+                 word(ah0, ah1, 2 * j + 1), xb0, xb1);
+        mma16816(acc[G] + 4, word(bg0, bg1, 2 * j), word(bh0, bh1, 2 * j),
+                 word(bg0, bg1, 2 * j + 1), word(bh0, bh1, 2 * j + 1), xb0, xb1);
+      }
     }
   }
 #pragma unroll
   for (int G = 0; G < NG; ++G)
 #pragma unroll
-    for (int i = 0; i < 4; ++i) red[((warp * kMaxNG + G) * 4 + i) * 32 + lane] = acc[G][i];
+    for (int i = 0; i < 8; ++i) red[((warp * kMaxNG + G) * 8 + i) * 32 + lane] = acc[G][i];
   __syncthreads();
+  // accumulator element i: tile i / 4, row g ((i & 3) < 2) or g + 8, token column 2c + (i & 1)
   float* o = a.o + size_t(kp) * a.o_plane;
   for (int p = warp; p < RB * NG; p += kWarps) {
     const int rb = p / NG, G = p % NG;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 8; ++i) {
       float sum = 0.f;
-      for (int k = 0; k < KS; ++k) sum += red[(((rb * KS + k) * kMaxNG + G) * 4 + i) * 32 + lane];
+      for (int k = 0; k < KS; ++k) sum += red[(((rb * KS + k) * kMaxNG + G) * 8 + i) * 32 + lane];
       const int j = G * 8 + 2 * c + (i & 1);
       if (j < n) {
-        const int row = r0 + rb * kRows + g + (i >= 2 ? 8 : 0);
+        const int row = r0 + rb * kRows2 + (i >> 2) * 16 + g + ((i & 3) >= 2 ? 8 : 0);
         if (lblk && kp == 0)  // LoRA: + s B2 (A2 h), once (in the first partial plane)
           sum += lora_up<__nv_bfloat16>(lblk, lora_offsets(a.d, a.w, a.lrank).b2, row,
                                         a.u2 + size_t(q0 + j) * a.lrank, a.lrank, a.lscale);
@@ -305,13 +316,13 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
 __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_constant__ FfnArgs a,
                                                               int RB) {
   __shared__ DecItems it;
-  __shared__ float red[kWarps * kMaxNG * 4 * 32];
+  __shared__ float red[kWarps * kMaxNG * 8 * 32];
   const int KS = kWarps / RB;
-  build_dec_items(it, a, a.d / (kRows * RB), a.ksplit);
+  build_dec_items(it, a, a.d / (kRows2 * RB), a.ksplit);
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
     const int s = dec_seg(it, item);
     const int local = item - it.first[s];
-    const int r0 = (local / it.ksplit) * kRows * RB, kp = local % it.ksplit;
+    const int r0 = (local / it.ksplit) * kRows2 * RB, kp = local % it.ksplit;
     const char* blk = it.blk[s];
     const void* lblk = a.lrank ? a.lblk[s] : nullptr;
     for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
@@ -337,18 +348,18 @@ int decode_ksplit(int T) { return T <= 4 ? 4 : (T <= 16 ? 2 : 1); }
 // Row blocks per CTA item: the smallest RB in {1, 2, 4, 8} whose 8 / RB contraction slices give
 // every warp at least 8 chunks of 64 (while the rows still split into whole items). More slices
 // mean finer items and better balance; fewer mean longer, better pipelined loops.
-int rows_per_item(int rows, int contraction) {
+int rows_per_item(int rows, int contraction, int rows_per_warp) {
   const int nch = contraction / kChunk;
   int rb = 1;
-  while (rb < kWarps && nch / (kWarps / rb) < 8 && rows % (kRows * rb * 2) == 0) rb *= 2;
+  while (rb < kWarps && nch / (kWarps / rb) < 8 && rows % (rows_per_warp * rb * 2) == 0) rb *= 2;
   return rb;
 }
 
 cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
   static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel));
   static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel));
-  const int rb13 = rows_per_item(a.w, a.d);
-  const int rb2 = rows_per_item(a.d, a.w / a.ksplit);
+  const int rb13 = rows_per_item(a.w, a.d, kRows);
+  const int rb2 = rows_per_item(a.d, a.w / a.ksplit, kRows2);
   cudaError_t e = cudaSuccess;
   if (stages & 1) {
     prof_begin(kProfDec13, s);
