@@ -15,7 +15,10 @@ Everything is a plain, slow, readable restatement of the paper's definitions in 
   formulations.
 * ``mask``     - Stage-1 mask sampling and the straight-through mask gradient (Section 3.2
   Eq. stage1 and Eq. ste).
+* ``stack``    - the chained decode stack (residual stream, RMSNorm, one masked MoE block per layer)
+  and the next-layer prediction that drives expert prefetch; the cache's prefetch event is in
+  ``cache``.
 
 Pins (tests marked ``not gpu``) tie each function to something other than itself; see the tests.
 """
-from . import cache, ffn, mask, routing  # noqa: F401
+from . import cache, ffn, mask, routing, stack  # noqa: F401

@@ -24,6 +24,15 @@ Readings: LFU counts persist across evictions (the paper evicts "the least frequ
 experts"); FIFO hits do not refresh the insertion order; ties always fall to the older use and
 then the lower expert id.
 
+Prefetch (offloading systems load experts ahead of need, Section 2; the paper gives no rule): a
+prefetch of a set P (at most B experts) is a cache event of its own between two steps, with its
+own time stamp. Experts of P already cached are touched (last use = the event; no access is
+counted, so LFU counts stay those of real steps). The others, in ascending id, take the lowest
+free slot or evict, among slots not touched at this event, the smallest policy key (an insertion
+stamps last use and insertion with the event); if no slot qualifies the expert is skipped. Each
+load is one prefetch fetch. A prefetched expert that the next step uses is a hit of that step and
+counts as a useful prefetch; the pending set is cleared at every step.
+
 Two independent formulations are given: ``SlotCache`` (per-slot arrays and an argmin of the policy
 key) and ``OrderedCache`` (an ordered list of cached experts kept in victim order). Tests require
 them to agree.
@@ -51,6 +60,9 @@ class SlotCache:
         self.ins = [-1] * B
         self.freq = [0] * E
         self.t = 0
+        self.pf = set()      # experts loaded by prefetch since the last step (still cached)
+        self.prefetched = 0  # prefetch loads so far
+        self.useful = 0      # prefetched experts used by the step that followed
 
     def _key(self, s):
         e = self.tag[s]
@@ -73,6 +85,8 @@ class SlotCache:
                 raise ValueError(f"expert id {e} out of range")
         for e in U:
             self.freq[e] += 1
+        self.useful += len(self.pf & set(U))
+        self.pf = set()
         hits = 0
         for s in range(self.B):
             if self.tag[s] in U:
@@ -82,22 +96,54 @@ class SlotCache:
         for e in U:
             if e in self.tag:
                 continue
-            free = [s for s in range(self.B) if self.tag[s] < 0]
-            if free:
-                slot = free[0]
-            else:
-                cand = [s for s in range(self.B) if self.last[s] < t]
-                if not cand:
-                    misses.append((e, -1))
-                    continue
-                slot = min(cand, key=self._key)
-            self.tag[slot] = e
-            self.last[slot] = t
-            self.ins[slot] = t
+            slot = self._claim(t)
+            if slot is None:
+                misses.append((e, -1))
+                continue
+            self._insert(slot, e, t)
             misses.append((e, slot))
         self.t += 1
         bypass = sum(1 for _, s in misses if s < 0)
         return hits, len(misses), bypass, misses
+
+    def _claim(self, t):
+        """Slot for an insertion at event t: the lowest free slot, else the smallest policy key
+        among slots not touched at t, else None."""
+        free = [s for s in range(self.B) if self.tag[s] < 0]
+        if free:
+            return free[0]
+        cand = [s for s in range(self.B) if self.last[s] < t]
+        return min(cand, key=self._key) if cand else None
+
+    def _insert(self, slot, e, t):
+        self.pf.discard(self.tag[slot])
+        self.tag[slot] = e
+        self.last[slot] = t
+        self.ins[slot] = t
+
+    def prefetch(self, experts):
+        """Prefetch event for the set `experts` (at most B distinct ids). Returns the (expert,
+        slot) loads in processing order."""
+        t = self.t
+        P = sorted(set(int(e) for e in experts))
+        if len(P) > self.B or any(not 0 <= e < self.E for e in P):
+            raise ValueError("a prefetch names at most B valid experts")
+        for s in range(self.B):
+            if self.tag[s] in P:
+                self.last[s] = t
+        loads = []
+        for e in P:
+            if e in self.tag:
+                continue
+            slot = self._claim(t)
+            if slot is None:
+                continue
+            self._insert(slot, e, t)
+            self.pf.add(e)
+            loads.append((e, slot))
+        self.t += 1
+        self.prefetched += len(loads)
+        return loads
 
 
 class LRUStamps(SlotCache):
@@ -127,6 +173,9 @@ class OrderedCache:
         self.free = list(range(B))
         self.count = [0] * E
         self.t = 0
+        self.pf = set()
+        self.prefetched = 0
+        self.useful = 0
 
     def _place(self, e):
         """(Re)insert e at its position in the victim order after it was touched at step t."""
@@ -157,40 +206,80 @@ class OrderedCache:
                 raise ValueError(f"expert id {e} out of range")
         for e in U:
             self.count[e] += 1
+        self.useful += sum(1 for e in U if e in self.pf)
+        self.pf = set()
         touched = set()
         hits = 0
         for e in U:
             if e in self.slot_of:
                 hits += 1
-                touched.add(e)
-                if self.policy != "FIFO":
-                    self._remove(e)
-                    self._place(e)
+                self._touch(e, touched)
         misses = []
         for e in U:
             if e in self.slot_of:
                 continue
-            if self.free:
-                slot = self.free.pop(0)
-            else:
-                victim = next((v for v in self.order if v not in touched), None)
-                if victim is None:
-                    misses.append((e, -1))
-                    continue
-                self._remove(victim)
-                slot = self.slot_of.pop(victim)
+            slot = self._take_slot(touched)
+            if slot is None:
+                misses.append((e, -1))
+                continue
             self.slot_of[e] = slot
             touched.add(e)
             self._place(e)
             misses.append((e, slot))
+        self._end_event(touched)
+        bypass = sum(1 for _, s in misses if s < 0)
+        return hits, len(misses), bypass, misses
+
+    def _touch(self, e, touched):
+        touched.add(e)
+        if self.policy != "FIFO":
+            self._remove(e)
+            self._place(e)
+
+    def _take_slot(self, touched):
+        """A free slot, else the slot of the first expert in victim order not touched at this
+        event (evicting it), else None."""
+        if self.free:
+            return self.free.pop(0)
+        victim = next((v for v in self.order if v not in touched), None)
+        if victim is None:
+            return None
+        self._remove(victim)
+        self.pf.discard(victim)
+        return self.slot_of.pop(victim)
+
+    def _end_event(self, touched):
         if self.policy == "LRU":
-            # experts touched in one step: lower id first (older) among equal last use
+            # experts touched at one event: lower id first (older) among equal last use
             tail = [v for v in self.order if v in touched]
             head = [v for v in self.order if v not in touched]
             self.order = head + sorted(tail)
         self.t += 1
-        bypass = sum(1 for _, s in misses if s < 0)
-        return hits, len(misses), bypass, misses
+
+    def prefetch(self, experts):
+        """Prefetch event (see the module header); returns the (expert, slot) loads."""
+        P = sorted(set(int(e) for e in experts))
+        if len(P) > self.B or any(not 0 <= e < self.E for e in P):
+            raise ValueError("a prefetch names at most B valid experts")
+        touched = set()
+        for e in P:
+            if e in self.slot_of:
+                self._touch(e, touched)
+        loads = []
+        for e in P:
+            if e in self.slot_of:
+                continue
+            slot = self._take_slot(touched)
+            if slot is None:
+                continue
+            self.slot_of[e] = slot
+            touched.add(e)
+            self._place(e)
+            self.pf.add(e)
+            loads.append((e, slot))
+        self._end_event(touched)
+        self.prefetched += len(loads)
+        return loads
 
     def state(self):
         """(tag per slot) for comparison with SlotCache."""
@@ -207,14 +296,17 @@ class LRUList(OrderedCache):
         super().__init__(E, B, "LRU")
 
 
-def simulate(steps_ids, E: int, B: int, cls=SlotCache, policy: str = "LRU"):
-    """Run one layer's cache over a stream of steps; steps_ids[t] holds the ids chosen at step t.
+def simulate(steps_ids, E: int, B: int, cls=SlotCache, policy: str = "LRU", prefetch=None):
+    """Run one layer's cache over a stream of steps; steps_ids[t] holds the ids chosen at step t
+    and, when given, prefetch[t] the set prefetched just before step t (None: no prefetch event).
 
     Returns per-step arrays hits, fetches, bypass and the list of per-step miss lists.
     """
     c = cls(E, B, policy)
     h, f, b, ml = [], [], [], []
-    for ids in steps_ids:
+    for t, ids in enumerate(steps_ids):
+        if prefetch is not None and prefetch[t] is not None:
+            c.prefetch(prefetch[t])
         hi, fi, bi, mi = c.step(ids)
         h.append(hi)
         f.append(fi)

@@ -29,9 +29,15 @@ def _load_traces():
             ids, hits, misses = [p.strip() for p in line[4:].split("|")]
             ml = [tuple(int(v) for v in m.split(":")) for m in misses.split()[1:]]
             cur["steps"].append(([int(v) for v in ids.split(",")], int(hits.split()[1]), ml))
+        elif line.startswith("prefetch"):
+            ids, loads = [p.strip() for p in line[8:].split("|")]
+            ll = [tuple(int(v) for v in m.split(":")) for m in loads.split()[1:]]
+            cur["steps"].append(([int(v) for v in ids.split(",")], None, ll))
         elif line.startswith("total"):
             f = line.split()
             cur["total"] = dict(hits=int(f[2]), fetches=int(f[4]), bypass=int(f[6]))
+            if len(f) > 8:
+                cur["total"].update(prefetched=int(f[8]), useful=int(f[10]))
     return traces
 
 
@@ -44,11 +50,16 @@ def test_hand_traces(cls, tr):
     c = cls(tr["E"], tr["B"], tr["policy"])
     th = tf = tb = 0
     for ids, hits, misses in tr["steps"]:
+        if hits is None:  # prefetch event
+            assert c.prefetch(ids) == misses
+            continue
         h, f, b, ml = c.step(ids)
         assert h == hits
         assert ml == misses
         th, tf, tb = th + h, tf + f, tb + b
     assert (th, tf, tb) == (tr["total"]["hits"], tr["total"]["fetches"], tr["total"]["bypass"])
+    if "prefetched" in tr["total"]:
+        assert (c.prefetched, c.useful) == (tr["total"]["prefetched"], tr["total"]["useful"])
 
 
 def test_table2_metric_identity():
@@ -85,6 +96,74 @@ def test_two_formulations_agree(T, K, E, B, policy):
         ra, rb = a.step(ids[s]), b.step(ids[s])
         assert ra == rb
         assert a.tag == b.state()
+
+
+def _random_prefetches(seed, steps, E, B, n_max, p=0.7):
+    g = np.random.default_rng(seed)
+    out = []
+    for _ in range(steps):
+        if g.random() < p:
+            out.append(sorted(g.choice(E, size=int(g.integers(1, n_max + 1)), replace=False).tolist()))
+        else:
+            out.append(None)
+    return out
+
+
+@pytest.mark.parametrize("policy", C.POLICIES)
+@pytest.mark.parametrize("T,K,E,B,n_max", [(1, 2, 8, 4, 2), (4, 2, 8, 4, 4), (1, 6, 64, 12, 6),
+                                           (8, 6, 64, 12, 12), (2, 1, 5, 2, 1)])
+def test_two_formulations_agree_with_prefetch(T, K, E, B, n_max, policy):
+    ids = inputs.random_ids(16, 300, T, K, E, hot=range(min(E, B + 2)), p_hot=0.7)
+    pfs = _random_prefetches(17, ids.shape[0], E, B, n_max)
+    a, b = C.SlotCache(E, B, policy), C.OrderedCache(E, B, policy)
+    for s in range(ids.shape[0]):
+        if pfs[s] is not None:
+            assert a.prefetch(pfs[s]) == b.prefetch(pfs[s])
+            assert a.tag == b.state()
+        assert a.step(ids[s]) == b.step(ids[s])
+        assert a.tag == b.state()
+    assert (a.prefetched, a.useful) == (b.prefetched, b.useful)
+    assert a.prefetched > 0
+
+
+@pytest.mark.parametrize("policy", C.POLICIES)
+def test_prefetch_invariants(policy):
+    """After a prefetch of P (|P| <= B) every expert of P is cached; a step using exactly P then
+    has no miss and counts every loaded expert as useful; prefetching a cached set loads nothing."""
+    E, B = 16, 6
+    g = np.random.default_rng(18)
+    c = C.SlotCache(E, B, policy)
+    for s in range(200):
+        P = sorted(g.choice(E, size=int(g.integers(1, B + 1)), replace=False).tolist())
+        before = c.useful
+        loads = c.prefetch(P)
+        assert set(P) <= set(c.tag)
+        assert c.prefetch(P) == []
+        h, f, b, _ = c.step(P)
+        assert (h, f, b) == (len(P), 0, 0)
+        assert c.useful - before == len(loads)
+        c.step(g.choice(E, size=3, replace=False))
+
+
+@pytest.mark.parametrize("policy", C.POLICIES)
+def test_perfect_prefetch_moves_every_fetch_to_the_prefetch(policy):
+    """Prefetching exactly the next step's experts (a perfect predictor, |U| <= B): demand
+    fetches vanish after the first step, and prefetch loads plus the first step's fetches equal the
+    plain cache's fetches (the prefetch makes the step's decisions one event early, with the same
+    victims: the same slots are excluded and the keys keep their order)."""
+    E, K, B = 8, 2, 4
+    ids = inputs.random_ids(19, 200, 1, K, E, hot=range(5), p_hot=0.8)
+    plain = C.simulate(ids, E, B, policy=policy)
+    pf = [None] + [sorted(set(ids[t].reshape(-1).tolist())) for t in range(1, len(ids))]
+    c = C.SlotCache(E, B, policy)
+    f0 = c.step(ids[0])[1]
+    demand = 0
+    for t in range(1, len(ids)):
+        c.prefetch(pf[t])
+        demand += c.step(ids[t])[1]
+    assert demand == 0
+    assert c.prefetched == c.useful
+    assert c.prefetched + f0 == plain[1].sum()
 
 
 @pytest.mark.parametrize("policy", C.POLICIES)
@@ -146,3 +225,7 @@ def test_invalid():
     c = C.LRUStamps(4, 2)
     with pytest.raises(ValueError):
         c.step([5])
+    with pytest.raises(ValueError):
+        c.prefetch([0, 1, 2])
+    with pytest.raises(ValueError):
+        c.prefetch([4])
