@@ -436,6 +436,87 @@ def run_stack(shape, L, steps, warmup, seed, dev, policy="LRU", path="device", g
     return res
 
 
+class ChainStack:
+    """L chained MoE layers (mcft_stack: residual stream, per-layer RMSNorm, soft-prior routing,
+    device cache with device-driven fetch, optional prefetch of each next layer's predicted
+    experts) decoding at batch 1. Each layer has its own router, RMSNorm scale and random soft-prior
+    mask; the pinned host pool holds E distinct expert blocks that every layer aliases (as in
+    DecodeStack). The stream entering layer 0 is the AR(1) recipe in fp32, one row per token."""
+
+    def __init__(self, shape, L, steps, seed, dev, policy="LRU", n_prefetch=0):
+        from paper_2609_34077_gb300 import mcft as M
+
+        self.M, self.shape, self.L, self.dev = M, shape, L, dev
+        desc = M.desc_of(shape)
+        pool = I.layer_weights(seed, shape, layer=0, pin=True)
+        self.pool = pool
+        shared = [b.to(dev) for b in pool.shared]
+        routers = [I.router_weight(seed, shape, l).to(dev) for l in range(L)]
+        gammas = [I.norm_weight(seed, shape, l).to(dev) for l in range(L)]
+        priors = np.stack([I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep, l))
+                           for l in range(L)])
+        host = [pool.experts[e] for _ in range(L) for e in range(shape.E)]
+        self.cache = M.mcft_cache_create(L, shape.E, shape.cache_slots, shape.expert_bytes, host,
+                                         max_assign=shape.K, policy=policy)
+        self.stack = M.mcft_stack_create(desc, routers, priors, gammas,
+                                         [shared] * L if shape.n_shared else None, shape.norm_eps,
+                                         self.cache, n_prefetch=n_prefetch, T_max=1)
+        self.x0 = I.residual_stream(seed, shape, steps, 1).to(dev)  # [steps, 1, d]
+        self.x = torch.empty((1, shape.d), dtype=torch.float32, device=dev)
+        self.compute = torch.cuda.Stream(dev)
+        self.copy = torch.cuda.Stream(dev)
+        self.graph = None
+
+    def capture(self):
+        self.graph = torch.cuda.CUDAGraph()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(self.graph, stream=self.compute):
+            self.M.mcft_stack_step(self.stack, self.x, self.compute, self.copy)
+        torch.cuda.synchronize()
+
+    def step(self, s):
+        with torch.cuda.stream(self.compute):
+            self.x.copy_(self.x0[s], non_blocking=True)
+            if self.graph is not None:
+                self.graph.replay()
+            else:
+                self.M.mcft_stack_step(self.stack, self.x, self.compute, self.copy)
+
+
+def run_chain(shape, L, steps, warmup, seed, dev, policy="LRU", n_prefetch=0, graph=True):
+    """Decode `warmup + steps` tokens through a chained L-layer stack; TPOT over the last `steps`."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    S = ChainStack(shape, L, warmup + steps + 1, seed, dev, policy, n_prefetch)
+    torch.cuda.synchronize()
+    for s in range(warmup):
+        S.step(s)
+    torch.cuda.synchronize()
+    if graph:
+        S.capture()  # records one step; runs nothing
+    h0, f0, _ = M.mcft_cache_stats(S.cache, -1)
+    p0, u0 = M.mcft_cache_prefetch_stats(S.cache, -1)
+    elapsed = time_steps(S.step, warmup, steps, S.compute)
+    M.mcft_device_error()
+    h1, f1, _ = M.mcft_cache_stats(S.cache, -1)
+    p1, u1 = M.mcft_cache_prefetch_stats(S.cache, -1)
+    fetches, pref, useful = f1 - f0, p1 - p0, u1 - u0
+    moved = (fetches + pref) * shape.expert_bytes / steps
+    res = dict(workload=f"{shape.name} chained decode stack, {L} layers, batch 1, {policy}, "
+                        f"prefetch {n_prefetch or 'off'}",
+               layers=L, policy=policy, n_prefetch=n_prefetch, cuda_graph=graph, steps=steps,
+               warmup=warmup, tpot_ms=elapsed * 1e3 / steps, tokens_per_s=steps / elapsed,
+               demand_fetches_per_token=fetches / steps, prefetches_per_token=pref / steps,
+               useful_prefetches_per_token=useful / steps,
+               prefetch_accuracy=useful / pref if pref else None,
+               hit_rate=(h1 - h0) / max(1, h1 - h0 + fetches),
+               link_gb_per_token=moved / 1e9, link_bound_tpot_ms=moved / 210e9 * 1e3,
+               host_pool="E distinct pinned blocks aliased by every layer")
+    del S
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_prefill(steps, warmup, seed, dev, peaks):
     from paper_2609_34077_gb300 import mcft as M
 
@@ -603,8 +684,12 @@ def main():
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
     ap.add_argument("--case", choices=["decode16", "decode1", "prefill", "fetch16"],
                     help="run only a few resident-expert forwards (for profiler captures)")
-    ap.add_argument("--workload", default="layer", choices=["layer", "stack-mixtral", "stack-dsv2"],
-                    help="layer: the single-layer decode line; stack-*: the full decode stack")
+    ap.add_argument("--workload", default="layer",
+                    choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2"],
+                    help="layer: the single-layer decode line; stack-*: the full decode stack "
+                         "(layers on independent streams); chain-*: the chained stack")
+    ap.add_argument("--prefetch", type=int, default=0,
+                    help="chain workloads: experts prefetched per layer (0 = off)")
     ap.add_argument("--policy", default="LRU", choices=["LRU", "LFU", "FIFO"])
     ap.add_argument("--graph", action="store_true", help="stack workloads: replay a captured step")
     args = ap.parse_args()
@@ -613,9 +698,13 @@ def main():
 
         __graft_entry__.build()
         torch.cuda.set_device(0)
-        shape, L = (I.MIXTRAL, 32) if args.workload == "stack-mixtral" else (I.DSV2_LITE, 26)
-        res = run_stack(shape, L, args.steps, args.warmup, 60, torch.device("cuda", 0), args.policy,
-                        graph=args.graph)
+        shape, L = (I.MIXTRAL, 32) if args.workload.endswith("mixtral") else (I.DSV2_LITE, 26)
+        if args.workload.startswith("chain"):
+            res = run_chain(shape, L, args.steps, args.warmup, 60, torch.device("cuda", 0),
+                            args.policy, args.prefetch, graph=args.graph)
+        else:
+            res = run_stack(shape, L, args.steps, args.warmup, 60, torch.device("cuda", 0),
+                            args.policy, graph=args.graph)
         res.update(metric="masked MoE decode stack tokens/s", value=res["tokens_per_s"],
                    unit="tokens/s", higher_is_better=True, dtype="bf16", data="synthetic")
         print(json.dumps(res), flush=True)

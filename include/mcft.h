@@ -264,7 +264,8 @@ mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, cons
  * permutation and the FFN of the experts that were hits (and of the shared experts) run at the
  * same time; then compute_stream waits for the copies and computes the fetched experts and the
  * combine. Results equal mcft_moe_forward's with the same experts.
- * Section 3.1 Eq. topk (the layer) and Section 4.1 / P:L53, P:L106 (fetch on a miss).
+ * Section 3.1 Eq. topk (the layer); Section 1 and Section 3.1 "Preliminaries" (every miss is a fetch
+ * from host memory).
  *   cache  created with host blocks (not accounting-only); its E and expert size match desc
  *   other arguments as for mcft_moe_forward (the routed expert addresses come from the cache)
  * Supports the decode path (bf16 with T <= 64, or fp32); larger bf16 calls return
@@ -274,6 +275,32 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
                                     int layer, const void* const* shared, void* y, void* workspace,
                                     size_t ws_bytes, mcft_stream_t compute_stream,
                                     mcft_stream_t copy_stream);
+
+/* mcft_cache_prefetch: a prefetch event of `layer` (no counterpart rule in the paper; offloading
+ * systems load experts ahead of need, Section 2 "Offloading systems for MoE inference"). From the
+ * predicted routing idx_pred (device [T, K] int32, e.g. mcft_route of the layer's router on a
+ * speculative input) the set P = the n_max experts named most often (ties to the lower id) is
+ * formed; members of P already cached are touched (last use = this event, which has a time stamp
+ * of its own between two steps; no LFU access is counted); the others, in ascending id, take the
+ * lowest free slot or evict, among slots not touched at this event, the smallest policy key.
+ * Each load counts as one prefetched expert; a prefetched expert that the layer's next
+ * mcft_cache_step uses counts as useful. Decided on the device on `stream`.
+ * The loads are fetched (device-driven, host link) on the copy stream of the next
+ * mcft_moe_forward_cached or mcft_fetch_experts call on this cache, behind that call's own misses
+ * (or, for this layer, before them); the compute stream of the layer's next forward waits for
+ * them before computing any expert. All calls on one cache must use one copy stream.
+ *   1 <= n_max <= B; T*K <= max_assign.
+ * Errors: MCFT_ERR_INVALID (bad arguments; a previous prefetch of the layer not yet fetched);
+ * MCFT_ERR_UNSUPPORTED (host blocks without device-visible addresses); an id out of range sets the
+ * device error word and changes no state. Accounting-only caches record the decision only. */
+mcft_status mcft_cache_prefetch(mcft_cache* cache, int layer, const int32_t* idx_pred, int T, int K,
+                                int n_max, mcft_stream_t stream);
+
+/* mcft_cache_prefetch_stats: cumulative prefetched experts and useful prefetches (prefetched
+ * experts used by the next step) of one layer, or summed when layer = -1. Prefetched experts are
+ * link traffic on top of mcft_cache_stats's fetches. Synchronises `stream` first. */
+mcft_status mcft_cache_prefetch_stats(const mcft_cache* cache, int layer, uint64_t* prefetched,
+                                      uint64_t* useful, mcft_stream_t stream);
 
 /* mcft_cache_last_misses: the miss list of the last mcft_cache_step of `layer`, after
  * mcft_fetch_experts (or a synchronisation of its stream): n_out = number of fetches;
@@ -293,7 +320,8 @@ mcft_status mcft_cache_stats(const mcft_cache* cache, int layer, uint64_t* hits,
 mcft_status mcft_cache_tags(const mcft_cache* cache, int layer, int32_t* tags, mcft_stream_t stream);
 
 /* mcft_cache_export / mcft_cache_import: checkpoint of the whole cache state (tags, last-use and
- * insertion steps, access counts, step counters, counters); import into a cache created with the
+ * insertion steps, access counts, step counters, counters, pending prefetch set); call them with no
+ * prefetch awaiting its fetch. Import into a cache created with the
  * same L, E, B and policy resumes a stream
  * with identical decisions. Slot contents are not part of the state: after an import, the slots
  * the tags name must be refilled by the caller (or the cache used in accounting mode).
@@ -303,6 +331,64 @@ mcft_status mcft_cache_import(mcft_cache* cache, const void* buf, size_t bytes, 
 
 /* mcft_cache_destroy: free everything mcft_cache_create allocated (synchronises the device). */
 void mcft_cache_destroy(mcft_cache* cache);
+
+/* ---------------------------------------------------------------------------------------------
+ * Chained decode stack: the residual stream between MoE blocks.
+ *
+ * mcft_residual_rmsnorm: for each of the T rows, x <- x + y (when y is not NULL), then
+ * u = gamma * x / sqrt(mean_j x[j]^2 + eps) (when gamma is not NULL): the block-input RMSNorm of the
+ * paper's models (Mixtral-8x7B, DeepSeek-V2-Lite; Section 4, Table 4), which the paper uses but
+ * does not restate; eps is 1e-5 for Mixtral, 1e-6 for DeepSeek-V2-Lite. Without attention blocks a
+ * decode step of an L-layer stack is u_0 = RMSNorm_0(x_0); for each layer l: route u_l, run the
+ * layer on u_l into y_l, then x_{l+1} = x_l + y_l and u_{l+1} = RMSNorm_{l+1}(x_{l+1}) (one call).
+ *   x      device [T, d] fp32 residual stream, updated in place when y is given
+ *   y      device [T, d] layer dtype, or NULL
+ *   gamma  device [d] layer dtype, or NULL (then u is not written)
+ *   u      device [T, d] layer dtype out (bf16: rounded to nearest even)
+ * All pointers 16-byte aligned; 0 <= eps <= 1. One CTA per row; the sum of squares is reduced in a
+ * fixed order (deterministic). Asynchronous on `stream`. */
+mcft_status mcft_residual_rmsnorm(const mcft_layer_desc* desc, float* x, const void* y, int T,
+                                  const void* gamma, float eps, void* u, mcft_stream_t stream);
+
+/* mcft_stack_create: an L-layer chained decode stack on the residual stream (no counterpart API in
+ * the paper; its models are such stacks with attention blocks in between, which this library does
+ * not have). Each step runs, per layer l: RMSNorm_l, soft-prior routing (Section 3.2 Eq. inference)
+ * by layer l's router, the cache step of layer l, optionally the prefetch event of layer l+1 from
+ * the routing of RMSNorm_{l+1}(x_l) by layer l+1 (the stream before layer l's output is added),
+ * mcft_moe_forward_cached of layer l, and x <- x + y. No host synchronisation: a step can be
+ * captured in a CUDA graph.
+ *   routers    host [L] device pointers to router weights [E, d] (layer dtype)
+ *   priors     host [L*E] fp32 soft priors, every entry > 0 and finite (copied)
+ *   gammas     host [L] device pointers to RMSNorm scales [d] (layer dtype)
+ *   shared     host [L*S] device pointers to shared expert blocks (NULL when S = 0)
+ *   eps        RMSNorm epsilon in [0, 1]
+ *   cache      created with L layers, desc's E and expert size, host blocks with device-visible
+ *              addresses; used by this stack's steps only while they run
+ *   n_prefetch 0 = no prefetch, else the n_max of mcft_cache_prefetch (1 <= n_prefetch <= B)
+ *   T_max      largest batch of a step (at most 64 for bf16)
+ * The pointed-to weights stay owned by the caller and must outlive the stack. Allocates the
+ * stack's activations, routing buffers and one workspace. Synchronous. */
+typedef struct mcft_stack mcft_stack;
+mcft_status mcft_stack_create(const mcft_layer_desc* desc, int L, const void* const* routers,
+                              const float* priors, const void* const* gammas,
+                              const void* const* shared, float eps, mcft_cache* cache,
+                              int n_prefetch, int T_max, mcft_stack** out);
+
+/* mcft_stack_step: one decode step of all L layers for T tokens (1 <= T <= T_max).
+ *   x  device [T, d] fp32: the stream entering layer 0 on input, leaving layer L-1 on output.
+ * Kernels on compute_stream, expert fetches on copy_stream. Asynchronous. */
+mcft_status mcft_stack_step(mcft_stack* stack, float* x, int T, mcft_stream_t compute_stream,
+                            mcft_stream_t copy_stream);
+
+/* mcft_stack_routing: host copies of layer `layer`'s routing in the last step: idx and gate
+ * [T, K], and idx_pred [T, K], the prediction made for this layer during the previous layer
+ * (valid for layer >= 1 with prefetch on; -1 otherwise). Any pointer may be NULL. Synchronises
+ * `stream` after the copies. */
+mcft_status mcft_stack_routing(const mcft_stack* stack, int layer, int32_t* idx, float* gate,
+                               int32_t* idx_pred, mcft_stream_t stream);
+
+/* mcft_stack_destroy: synchronise the device and free what mcft_stack_create allocated. */
+void mcft_stack_destroy(mcft_stack* stack);
 
 /* ---------------------------------------------------------------------------------------------
  * mcft_device_error: synchronise `stream`, return and clear the device error word of the current

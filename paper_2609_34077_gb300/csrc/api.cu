@@ -144,9 +144,16 @@ struct mcft_cache {
   unsigned long long* d_ptr_tab = nullptr;  // [L*E] block address of each selected expert
   unsigned long long* d_ready = nullptr;    // [L] hit mask of the last step
   unsigned long long* d_host_src = nullptr; // [L*E] device-visible addresses of the host blocks
+  unsigned long long* d_pfmask = nullptr;   // [L] experts loaded by a prefetch since the last step
+  int32_t* d_pf_list = nullptr;             // [L][1 + E] fetch list of the last prefetch
+  unsigned long long* d_pf_tab = nullptr;   // [L*E] destinations of the last prefetch's loads
   char* d_slots = nullptr;    // [L*B] expert blocks
   char* d_staging = nullptr;  // [n_staging] expert blocks
   std::vector<cudaEvent_t> ev_step;  // per layer: recorded after its cache step
+  std::vector<cudaEvent_t> ev_pf_step, ev_pf_done;  // per layer: after a prefetch decision / fetch
+  // per layer: 0 no prefetch outstanding, 1 decided (fetch not yet enqueued), 2 fetch enqueued and
+  // not yet waited for by a compute stream
+  std::vector<int> pf_state;
   cudaEvent_t ev_copy = nullptr;
   bool device_fetch = false;  // every host block has a device-visible address
 };
@@ -168,8 +175,12 @@ void cache_free(mcft_cache* c) {
   cudaFree(c->d_ptr_tab);
   cudaFree(c->d_ready);
   cudaFree(c->d_host_src);
-  for (cudaEvent_t e : c->ev_step)
-    if (e) cudaEventDestroy(e);
+  cudaFree(c->d_pfmask);
+  cudaFree(c->d_pf_list);
+  cudaFree(c->d_pf_tab);
+  for (const auto* v : {&c->ev_step, &c->ev_pf_step, &c->ev_pf_done})
+    for (cudaEvent_t e : *v)
+      if (e) cudaEventDestroy(e);
   if (c->ev_copy) cudaEventDestroy(c->ev_copy);
   delete c;
 }
@@ -183,20 +194,36 @@ const char* loc_ptr(const mcft_cache* c, int layer, int loc) {
 struct CacheStateHeader {
   uint32_t magic, L, E, B, policy, pad;
 };
-constexpr uint32_t kStateMagic = 0x4d434655u;
+constexpr uint32_t kStateMagic = 0x4d434656u;
 
 // Bytes of the exported state: header, tag [L*B] i32, last and ins [L*B] i64, freq [L*E] i64,
-// step [L] i64, counters [L*3] u64.
+// step [L] i64, counters [L*5] u64, prefetch mask [L] u64.
 size_t state_bytes(const mcft_cache* c) {
   const size_t LB = size_t(c->L) * c->B, LE = size_t(c->L) * c->E;
-  return sizeof(CacheStateHeader) + LB * 4 + LB * 8 * 2 + LE * 8 + size_t(c->L) * 8 + size_t(c->L) * 24;
+  return sizeof(CacheStateHeader) + LB * 4 + LB * 8 * 2 + LE * 8 + size_t(c->L) * 8 +
+         size_t(c->L) * 8 * kCacheCounters + size_t(c->L) * 8;
+}
+
+// Enqueue on `copy` the fetch of every prefetch decided but not yet fetched (in layer order).
+mcft_status enqueue_prefetch_fetches(mcft_cache* c, cudaStream_t copy) {
+  for (int l = 0; l < c->L; ++l) {
+    if (c->pf_state[l] != 1) continue;
+    MCFT_CUDA(cudaStreamWaitEvent(copy, c->ev_pf_step[l], 0));
+    FetchArgs fe{c->d_pf_list + size_t(l) * (1 + c->E), c->d_host_src + size_t(l) * c->E,
+                 c->d_pf_tab + size_t(l) * c->E, c->expert_bytes};
+    cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy, true);
+    if (e != cudaSuccess) return cuda_fail(e, "prefetch fetch kernel launch");
+    MCFT_CUDA(cudaEventRecord(c->ev_pf_done[l], copy));
+    c->pf_state[l] = 2;
+  }
+  return MCFT_OK;
 }
 
 }  // namespace
 
 extern "C" {
 
-int mcft_version(void) { return 100; }
+int mcft_version(void) { return 200; }
 
 const char* mcft_last_error(void) { return g_last_error.c_str(); }
 
@@ -505,13 +532,19 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_ins, sizeof(int64_t) * L * B));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_freq, sizeof(int64_t) * L * E));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_step, sizeof(int64_t) * L));
-  MCFT_CACHE_CUDA(cudaMalloc(&c->d_cnt, sizeof(unsigned long long) * L * 3));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_cnt, sizeof(unsigned long long) * L * kCacheCounters));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_pfmask, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_pfmask, 0, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_pf_list, sizeof(int32_t) * L * (1 + E)));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_pf_list, 0, sizeof(int32_t) * L * (1 + E)));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_pf_tab, sizeof(unsigned long long) * L * E));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_pf_tab, 0, sizeof(unsigned long long) * L * E));
   MCFT_CACHE_CUDA(cudaMemset(c->d_tag, 0xff, sizeof(int32_t) * L * B));  // -1 = empty
   MCFT_CACHE_CUDA(cudaMemset(c->d_last, 0xff, sizeof(int64_t) * L * B));
   MCFT_CACHE_CUDA(cudaMemset(c->d_ins, 0xff, sizeof(int64_t) * L * B));
   MCFT_CACHE_CUDA(cudaMemset(c->d_freq, 0, sizeof(int64_t) * L * E));
   MCFT_CACHE_CUDA(cudaMemset(c->d_step, 0, sizeof(int64_t) * L));
-  MCFT_CACHE_CUDA(cudaMemset(c->d_cnt, 0, sizeof(unsigned long long) * L * 3));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_cnt, 0, sizeof(unsigned long long) * L * kCacheCounters));
   MCFT_CACHE_CUDA(cudaHostAlloc(&c->h_miss, sizeof(int32_t) * L * c->miss_stride, cudaHostAllocMapped));
   memset(c->h_miss, 0, sizeof(int32_t) * L * c->miss_stride);
   MCFT_CACHE_CUDA(cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->d_miss), c->h_miss, 0));
@@ -543,8 +576,14 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
     for (auto v : src) c->device_fetch = c->device_fetch && v != 0;
   }
   c->ev_step.assign(L, nullptr);
-  for (int l = 0; l < L; ++l)
+  c->ev_pf_step.assign(L, nullptr);
+  c->ev_pf_done.assign(L, nullptr);
+  c->pf_state.assign(L, 0);
+  for (int l = 0; l < L; ++l) {
     MCFT_CACHE_CUDA(cudaEventCreateWithFlags(&c->ev_step[l], cudaEventDisableTiming));
+    MCFT_CACHE_CUDA(cudaEventCreateWithFlags(&c->ev_pf_step[l], cudaEventDisableTiming));
+    MCFT_CACHE_CUDA(cudaEventCreateWithFlags(&c->ev_pf_done[l], cudaEventDisableTiming));
+  }
   MCFT_CACHE_CUDA(cudaEventCreateWithFlags(&c->ev_copy, cudaEventDisableTiming));
   MCFT_CACHE_CUDA(cudaDeviceSynchronize());
 #undef MCFT_CACHE_CUDA
@@ -560,7 +599,8 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
   if (T * K > c->max_assign)
     return fail(MCFT_ERR_INVALID, "T*K = %d exceeds max_assign = %d", T * K, c->max_assign);
   CacheStepArgs a{idx, T * K, c->E, c->B, layer, c->policy, c->d_tag, c->d_last, c->d_ins,
-                  c->d_freq, c->d_step, c->d_cnt, c->d_miss + size_t(layer) * c->miss_stride,
+                  c->d_freq, c->d_step, c->d_cnt, c->d_pfmask,
+                  c->d_miss + size_t(layer) * c->miss_stride,
                   c->d_miss_dev + size_t(layer) * c->miss_stride,
                   c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer,
                   c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
@@ -583,6 +623,15 @@ mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_s
   const int32_t* m_exp = m + 1;
   const int32_t* loc_of = m + 1 + 2 * E;
   for (int e = 0; e < E; ++e) expert_ptrs[e] = loc_ptr(c, layer, loc_of[e]);
+  // a prefetch of this layer decided before the step lands before the step's own copies
+  if (c->pf_state[layer] == 1) {
+    mcft_status st = enqueue_prefetch_fetches(c, copy_stream);
+    if (st != MCFT_OK) return st;
+  }
+  if (c->pf_state[layer] == 2) {
+    MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_pf_done[layer], 0));
+    c->pf_state[layer] = 0;
+  }
   if (c->d_slots && nm > 0) {
     // Every earlier use of these slots finished before the cache step's event (same stream).
     for (int i = 0; i < nm; ++i) {
@@ -595,6 +644,76 @@ mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_s
     MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
     MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
   }
+  // prefetches of later layers stream in behind this layer's copies
+  return enqueue_prefetch_fetches(c, copy_stream);
+}
+
+mcft_status mcft_cache_prefetch(mcft_cache* c, int layer, const int32_t* idx_pred, int T, int K,
+                                int n_max, mcft_stream_t stream) {
+  if (!c || !idx_pred) return fail(MCFT_ERR_INVALID, "NULL cache or idx_pred");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  if (T < 1 || K < 1 || K > c->E) return fail(MCFT_ERR_INVALID, "bad T = %d or K = %d", T, K);
+  if (T * K > c->max_assign)
+    return fail(MCFT_ERR_INVALID, "T*K = %d exceeds max_assign = %d", T * K, c->max_assign);
+  if (n_max < 1 || n_max > c->B)
+    return fail(MCFT_ERR_INVALID, "n_max = %d must be in [1, B = %d]", n_max, c->B);
+  if (c->d_slots && !c->device_fetch)
+    return fail(MCFT_ERR_UNSUPPORTED, "prefetch needs host blocks with device-visible addresses");
+  if (c->pf_state[layer] == 1)
+    return fail(MCFT_ERR_INVALID, "the previous prefetch of layer %d was never fetched (run a "
+                "forward or mcft_fetch_experts first)", layer);
+  // the previous prefetch's list is rewritten and its slots may be chosen again
+  if (c->pf_state[layer] == 2) {
+    MCFT_CUDA(cudaStreamWaitEvent(stream, c->ev_pf_done[layer], 0));
+    c->pf_state[layer] = 0;
+  }
+  PrefetchArgs a{idx_pred, T * K, n_max, c->E, c->B, layer, c->policy, c->d_tag, c->d_last,
+                 c->d_ins, c->d_freq, c->d_step, c->d_cnt, c->d_pfmask,
+                 c->d_pf_list + size_t(layer) * (1 + c->E), c->d_pf_tab + size_t(layer) * c->E,
+                 c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
+                 c->expert_bytes, device_error_word()};
+  cudaError_t e = launch_prefetch(a, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "prefetch kernel launch");
+  if (c->d_slots) {
+    MCFT_CUDA(cudaEventRecord(c->ev_pf_step[layer], stream));
+    c->pf_state[layer] = 1;
+  }
+  return MCFT_OK;
+}
+
+mcft_status mcft_cache_prefetch_stats(const mcft_cache* c, int layer, uint64_t* prefetched,
+                                      uint64_t* useful, mcft_stream_t stream) {
+  if (!c || !prefetched || !useful) return fail(MCFT_ERR_INVALID, "NULL argument");
+  if (layer < -1 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  std::vector<unsigned long long> h(size_t(c->L) * kCacheCounters);
+  MCFT_CUDA(cudaMemcpyAsync(h.data(), c->d_cnt, h.size() * sizeof(h[0]), cudaMemcpyDeviceToHost, stream));
+  MCFT_CUDA(cudaStreamSynchronize(stream));
+  uint64_t p = 0, u = 0;
+  for (int l = 0; l < c->L; ++l) {
+    if (layer >= 0 && l != layer) continue;
+    p += h[size_t(l) * kCacheCounters + 3];
+    u += h[size_t(l) * kCacheCounters + 4];
+  }
+  *prefetched = p;
+  *useful = u;
+  return MCFT_OK;
+}
+
+mcft_status mcft_residual_rmsnorm(const mcft_layer_desc* desc, float* x, const void* y, int T,
+                                  const void* gamma, float eps, void* u, mcft_stream_t stream) {
+  mcft_status st = check_desc(desc);
+  if (st != MCFT_OK) return st;
+  if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
+  if (T == 0) return MCFT_OK;
+  if (!x) return fail(MCFT_ERR_INVALID, "x is NULL");
+  if (gamma && !u) return fail(MCFT_ERR_INVALID, "u is NULL while gamma is given");
+  if (!(eps >= 0.f) || eps > 1.f) return fail(MCFT_ERR_INVALID, "eps = %g must be in [0, 1]", eps);
+  if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y) |
+       reinterpret_cast<uintptr_t>(gamma) | reinterpret_cast<uintptr_t>(u)) & 15u)
+    return fail(MCFT_ERR_INVALID, "x, y, gamma and u must be 16-byte aligned");
+  NormArgs a{x, y, gamma, u, T, desc->d, eps};
+  cudaError_t e = launch_resid_norm(a, desc->dtype, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "residual/RMSNorm kernel launch");
   return MCFT_OK;
 }
 
@@ -688,6 +807,12 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
   int* pos = reinterpret_cast<int*>(ws + L.pos);
   int* perm = reinterpret_cast<int*>(ws + L.perm);
   unsigned* err = device_error_word();
+  // 0. a prefetch of this layer decided before the step lands first (it may target the slots the
+  //    step's misses overwrite)
+  if (c->pf_state[layer] == 1) {
+    st = enqueue_prefetch_fetches(c, copy_stream);
+    if (st != MCFT_OK) return st;
+  }
   // 1. the missed experts stream in on the copy stream, after this layer's cache step
   MCFT_CUDA(cudaStreamWaitEvent(copy_stream, c->ev_step[layer], 0));
   FetchArgs fe{c->d_miss_dev + size_t(layer) * c->miss_stride, c->d_host_src + size_t(layer) * E,
@@ -695,6 +820,14 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
   cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy_stream);
   if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
+  // 1b. prefetches decided for later layers stream in behind this layer's misses
+  st = enqueue_prefetch_fetches(c, copy_stream);
+  if (st != MCFT_OK) return st;
+  // hits may be experts a prefetch is still bringing in
+  if (c->pf_state[layer] == 2) {
+    MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_pf_done[layer], 0));
+    c->pf_state[layer] = 0;
+  }
   // 2. meanwhile: permutation and the experts that were hits (and the shared experts)
   PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
   e = launch_permute(pa, compute_stream);
@@ -749,15 +882,15 @@ mcft_status mcft_cache_stats(const mcft_cache* c, int layer, uint64_t* hits, uin
                              uint64_t* bypass, mcft_stream_t stream) {
   if (!c || !hits || !fetches || !bypass) return fail(MCFT_ERR_INVALID, "NULL argument");
   if (layer < -1 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
-  std::vector<unsigned long long> h(size_t(c->L) * 3);
+  std::vector<unsigned long long> h(size_t(c->L) * kCacheCounters);
   MCFT_CUDA(cudaMemcpyAsync(h.data(), c->d_cnt, h.size() * sizeof(h[0]), cudaMemcpyDeviceToHost, stream));
   MCFT_CUDA(cudaStreamSynchronize(stream));
   uint64_t a = 0, b = 0, d = 0;
   for (int l = 0; l < c->L; ++l) {
     if (layer >= 0 && l != layer) continue;
-    a += h[size_t(l) * 3];
-    b += h[size_t(l) * 3 + 1];
-    d += h[size_t(l) * 3 + 2];
+    a += h[size_t(l) * kCacheCounters];
+    b += h[size_t(l) * kCacheCounters + 1];
+    d += h[size_t(l) * kCacheCounters + 2];
   }
   *hits = a;
   *fetches = b;
@@ -789,7 +922,8 @@ mcft_status mcft_cache_export(const mcft_cache* c, void* buf, size_t* bytes, mcf
   p += sizeof(h);
   const struct { const void* src; size_t n; } parts[] = {
       {c->d_tag, LB * 4}, {c->d_last, LB * 8}, {c->d_ins, LB * 8}, {c->d_freq, LE * 8},
-      {c->d_step, size_t(c->L) * 8}, {c->d_cnt, size_t(c->L) * 24}};
+      {c->d_step, size_t(c->L) * 8}, {c->d_cnt, size_t(c->L) * 8 * kCacheCounters},
+      {c->d_pfmask, size_t(c->L) * 8}};
   for (const auto& part : parts) {
     MCFT_CUDA(cudaMemcpyAsync(p, part.src, part.n, cudaMemcpyDeviceToHost, stream));
     p += part.n;
@@ -816,7 +950,8 @@ mcft_status mcft_cache_import(mcft_cache* c, const void* buf, size_t bytes, mcft
     if (tags[i] < -1 || tags[i] >= c->E) return fail(MCFT_ERR_INVALID, "corrupt tag in state");
   const struct { void* dst; size_t n; } parts[] = {
       {c->d_tag, LB * 4}, {c->d_last, LB * 8}, {c->d_ins, LB * 8}, {c->d_freq, LE * 8},
-      {c->d_step, size_t(c->L) * 8}, {c->d_cnt, size_t(c->L) * 24}};
+      {c->d_step, size_t(c->L) * 8}, {c->d_cnt, size_t(c->L) * 8 * kCacheCounters},
+      {c->d_pfmask, size_t(c->L) * 8}};
   for (const auto& part : parts) {
     MCFT_CUDA(cudaMemcpyAsync(part.dst, p, part.n, cudaMemcpyHostToDevice, stream));
     p += part.n;

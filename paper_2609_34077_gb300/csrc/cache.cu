@@ -9,6 +9,14 @@
 // this step only (bypass). The miss list and the expert -> location map are written straight
 // into host-mapped pinned memory, so the host can issue the fetches as soon as the step's event
 // completes.
+//
+// Prefetch (offloading systems load experts ahead of need, Section 2; the rule is this library's):
+// a prefetch is a cache event of its own, one time stamp between two steps. Its set is the n_max
+// experts named most often by a predicted routing (ties to the lower id); members already cached
+// are touched (last use = the event, no access counted), the others, in ascending id, take the
+// lowest free slot or evict, among slots not touched at the event, the smallest policy key. The
+// loads form a separate fetch list, so a prefetch never disturbs the miss list of a step whose
+// fetch may still be in flight. The next step counts hits on prefetched experts as useful.
 #include "common.cuh"
 #include "internal.h"
 
@@ -89,6 +97,8 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
         ++hits;
       }
     }
+    const unsigned long long pf = a.pfmask[a.layer];
+    const int useful = __popcll(pf & mine & cached);
     unsigned long long miss = mine & ~cached;
     while (miss) {
       const int e = __ffsll(static_cast<long long>(miss)) - 1;  // ascending expert id
@@ -118,10 +128,12 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
     }
     s_out[0] = nm;
     a.step[a.layer] = t + 1;
-    unsigned long long* c = a.counters + size_t(a.layer) * 3;
+    unsigned long long* c = a.counters + size_t(a.layer) * kCacheCounters;
     c[0] += hits;
     c[1] += nm;
     c[2] += nbyp;
+    c[4] += useful;
+    a.pfmask[a.layer] = 0;
   }
   cached = __shfl_sync(0xffffffffu, cached, 0);
   __syncwarp();
@@ -152,6 +164,107 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
   __threadfence_system();
 }
 
+// Prefetch decision (one warp). The lanes count how many predicted (token, k) entries name each
+// expert; lane 0 ranks, touches, claims slots and writes the fetch list.
+__global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ PrefetchArgs a) {
+  __shared__ int cnt[kMaxE];
+  __shared__ int32_t s_tag[kMaxE];
+  __shared__ int64_t s_last[kMaxE], s_ins[kMaxE], s_freq[kMaxE];
+  __shared__ int32_t s_list[1 + kMaxE];
+  const int lane = threadIdx.x, B = a.B, E = a.E;
+  for (int e = lane; e < E; e += 32) cnt[e] = 0;
+  __syncwarp();
+  int bad = 0;
+  for (int i = lane; i < a.n; i += 32) {
+    const int e = a.idx[i];
+    if (e < 0 || e >= E) bad = 1;
+    else atomicAdd(&cnt[e], 1);
+  }
+  bad = __any_sync(0xffffffffu, bad);
+  if (bad) {  // no state change on bad input
+    if (lane == 0) {
+      set_error(a.err, kErrInvalid);
+      a.list[0] = 0;
+    }
+    return;
+  }
+  int32_t* tag = a.tag + size_t(a.layer) * B;
+  int64_t* last = a.last + size_t(a.layer) * B;
+  int64_t* ins = a.ins + size_t(a.layer) * B;
+  for (int i = lane; i < B; i += 32) {
+    s_tag[i] = tag[i];
+    s_last[i] = last[i];
+    s_ins[i] = ins[i];
+  }
+  for (int e = lane; e < E; e += 32) s_freq[e] = a.freq[size_t(a.layer) * E + e];
+  __syncwarp();
+  if (lane == 0) {
+    const int64_t t = a.step[a.layer];
+    // the set: n_max experts by (count descending, id ascending)
+    unsigned long long P = 0;
+    for (int j = 0; j < a.n_max; ++j) {
+      int best = -1;
+      for (int e = 0; e < E; ++e)
+        if (cnt[e] > 0 && !((P >> e) & 1ull) && (best < 0 || cnt[e] > cnt[best])) best = e;
+      if (best < 0) break;
+      P |= 1ull << best;
+    }
+    unsigned long long cached = 0;
+    for (int sl = 0; sl < B; ++sl) {
+      const int e = s_tag[sl];
+      if (e < 0) continue;
+      cached |= 1ull << e;
+      if ((P >> e) & 1ull) s_last[sl] = t;
+    }
+    unsigned long long pf = a.pfmask[a.layer];
+    unsigned long long load = P & ~cached;
+    int nl = 0;
+    while (load) {
+      const int e = __ffsll(static_cast<long long>(load)) - 1;
+      load &= load - 1;
+      int slot = -1;
+      for (int sl = 0; sl < B; ++sl)
+        if (s_tag[sl] < 0) { slot = sl; break; }
+      if (slot < 0) {
+        for (int sl = 0; sl < B; ++sl) {
+          if (s_last[sl] >= t) continue;  // touched at this event: never a victim
+          if (slot < 0 || victim_before(a.policy, sl, slot, s_tag, s_last, s_ins, s_freq)) slot = sl;
+        }
+      }
+      if (slot < 0) continue;  // unreachable with n_max <= B; kept for safety
+      if (s_tag[slot] >= 0) pf &= ~(1ull << s_tag[slot]);
+      s_tag[slot] = e;
+      s_last[slot] = t;
+      s_ins[slot] = t;
+      pf |= 1ull << e;
+      s_list[1 + nl] = e;
+      ++nl;
+    }
+    s_list[0] = nl;
+    a.pfmask[a.layer] = pf;
+    a.step[a.layer] = t + 1;
+    a.counters[size_t(a.layer) * kCacheCounters + 3] += nl;
+  }
+  __syncwarp();
+  for (int i = lane; i < B; i += 32) {
+    tag[i] = s_tag[i];
+    last[i] = s_last[i];
+    ins[i] = s_ins[i];
+  }
+  const int nl = s_list[0];
+  for (int i = lane; i <= nl; i += 32) a.list[i] = s_list[i];
+  for (int e = lane; e < E; e += 32) a.ptr_tab[e] = 0;
+  __syncwarp();
+  for (int i = lane; i < nl; i += 32) {
+    const int e = s_list[1 + i];
+    int slot = 0;
+    for (int sl = 0; sl < B; ++sl)
+      if (s_tag[sl] == e) slot = sl;
+    a.ptr_tab[e] = a.slots ? reinterpret_cast<unsigned long long>(a.slots + size_t(slot) * a.expert_bytes)
+                           : 0ull;
+  }
+}
+
 // Copy the missed experts' blocks host -> device with 16-byte loads over the host link. Work
 // units are 64 KB pieces of the missed blocks, spread over the grid.
 __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ FetchArgs a) {
@@ -180,10 +293,18 @@ __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ Fetc
 
 }  // namespace
 
-cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s) {
-  prof_begin(kProfFetch, s);
+cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch) {
+  const int kid = prefetch ? kProfPfFetch : kProfFetch;
+  prof_begin(kid, s);
   fetch_kernel<<<blocks, 256, 0, s>>>(a);
-  prof_end(kProfFetch, s);
+  prof_end(kid, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prefetch(const PrefetchArgs& a, cudaStream_t s) {
+  prof_begin(kProfPrefetch, s);
+  prefetch_kernel<<<1, 32, 0, s>>>(a);
+  prof_end(kProfPrefetch, s);
   return cudaGetLastError();
 }
 

@@ -190,7 +190,8 @@ struct CacheStepArgs {
   int64_t* ins;       // [L*B] step of insertion (FIFO)
   int64_t* freq;      // [L*E] accesses per expert since the stream began (LFU)
   int64_t* step;      // [L]
-  unsigned long long* counters;  // [L*3] hits, fetches, bypass
+  unsigned long long* counters;  // [L*kCacheCounters] hits, fetches, bypass, prefetched, useful
+  unsigned long long* pfmask;    // [L] experts loaded by a prefetch since the layer's last step
   int32_t* miss_out;  // host-mapped, per layer: [n_miss, expert[E], loc[E], loc_of[E]]
   int32_t* miss_dev;  // device copy of the same list (read by the fetch kernel)
   unsigned long long* ptr_tab;  // device [E]: block address of each selected expert, else 0
@@ -202,6 +203,29 @@ struct CacheStepArgs {
 };
 cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s);
 
+constexpr int kCacheCounters = 5;  // per layer: hits, fetches, bypass, prefetched, useful
+
+// Prefetch decision of one layer: the n_max experts named most often by the predicted routing
+// (ties to the lower id) are touched or loaded into the layer's slots (cache.cu).
+struct PrefetchArgs {
+  const int32_t* idx;  // predicted routing [n]
+  int n, n_max;
+  int E, B, layer, policy;
+  int32_t* tag;
+  int64_t* last;
+  int64_t* ins;
+  const int64_t* freq;
+  int64_t* step;
+  unsigned long long* counters;
+  unsigned long long* pfmask;
+  int32_t* list;                  // device, this layer: [n_load, expert[E]] (fetch list)
+  unsigned long long* ptr_tab;    // device [E]: destination of each loaded expert, else 0
+  const char* slots;              // this layer's first slot block (NULL in accounting mode)
+  size_t expert_bytes;
+  unsigned* err;
+};
+cudaError_t launch_prefetch(const PrefetchArgs& a, cudaStream_t s);
+
 // Device-driven fetch: copy the blocks of a layer's missed experts from pinned host memory
 // (device-visible addresses host_src[E]) into the addresses ptr_tab[E] chosen by the cache step.
 struct FetchArgs {
@@ -210,7 +234,19 @@ struct FetchArgs {
   const unsigned long long* ptr_tab;  // [E]
   size_t bytes;                       // per expert block, multiple of 16
 };
-cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s);
+cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch = false);
+
+// Residual update and RMSNorm of the stream entering a MoE block (norm.cu): x += y (when y is
+// given), then u = gamma * x / sqrt(mean(x^2) + eps) (when gamma is given). One CTA per row.
+struct NormArgs {
+  float* x;            // [T, d] fp32 residual stream
+  const void* y;       // [T, d] layer dtype or NULL
+  const void* gamma;   // [d] layer dtype or NULL
+  void* u;             // [T, d] layer dtype (written when gamma is given)
+  int T, d;
+  float eps;
+};
+cudaError_t launch_resid_norm(const NormArgs& a, int dtype, cudaStream_t s);
 
 // Stage-1 mask machinery (mask.cu)
 struct MaskSampleArgs {
@@ -250,7 +286,8 @@ mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_er
 
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
-       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfCount };
+       kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfNorm,
+       kProfPrefetch, kProfPfFetch, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

@@ -14,7 +14,8 @@ namespace {
 
 const char* const kNames[kProfCount] = {
     "route",     "cache_step", "permute", "gather",       "ffn13_rowwise", "ffn2_rowwise",
-    "gemm13_tc", "gemm2_tc",   "combine", "ffn13_decode", "ffn2_decode", "fetch", "lora_down"};
+    "gemm13_tc", "gemm2_tc",   "combine", "ffn13_decode", "ffn2_decode", "fetch", "lora_down",
+    "rmsnorm",   "prefetch",   "fetch_prefetch"};
 
 struct Pending {
   int kid;

@@ -14,7 +14,9 @@ Recipe (all draws are Philox4x32-10 counter-based streams from numpy, keyed by
   rho = 0.8, generated in fp32 then rounded to bf16;
 * keep-k masks: a seeded Fisher-Yates shuffle of the E expert ids, first k ids kept;
 * soft-prior stand-in for the learned mask: ``m~ = gamma * m`` with gamma = 2, and
-  ``pi = softmax(m~)`` (the map the paper's Stage 1 uses to turn m~ into pi).
+  ``pi = softmax(m~)`` (the map the paper's Stage 1 uses to turn m~ into pi);
+* RMSNorm scales of a chained stack: ``1 + N(0, 0.1^2)`` per hidden unit, per layer; the stream
+  entering the stack: the AR(1) recipe above, kept in fp32 (the residual stream's precision).
 """
 from __future__ import annotations
 
@@ -47,6 +49,7 @@ class LayerShape:
     dtype: int
     cache_slots: int
     keep: int  # experts kept by the stand-in mask
+    norm_eps: float = 1e-5  # RMSNorm epsilon of the model's block inputs
 
     @property
     def expert_elems(self) -> int:
@@ -63,7 +66,7 @@ TINY = LayerShape("tiny-fp32", d=256, E=8, K=2, w=512, n_shared=0, gate=GATE_REN
 MIXTRAL = LayerShape("mixtral-8x7b", d=4096, E=8, K=2, w=14336, n_shared=0, gate=GATE_RENORM,
                      dtype=BF16, cache_slots=4, keep=4)
 DSV2_LITE = LayerShape("deepseek-v2-lite", d=2048, E=64, K=6, w=1408, n_shared=2, gate=GATE_PLAIN,
-                       dtype=BF16, cache_slots=12, keep=16)
+                       dtype=BF16, cache_slots=12, keep=16, norm_eps=1e-6)
 
 
 def _key(seed: int, *ids) -> int:
@@ -116,6 +119,18 @@ def router_weight(seed: int, shape: LayerShape, layer: int = 0) -> torch.Tensor:
     """Router weight W [E, d] ~ N(0, 0.02^2)."""
     a = normal_f32(seed, (shape.name, "router", layer), shape.E * shape.d, 0.02)
     return as_dtype(a.reshape(shape.E, shape.d), shape.dtype)
+
+
+def norm_weight(seed: int, shape: LayerShape, layer: int = 0) -> torch.Tensor:
+    """RMSNorm scale gamma [d] ~ 1 + N(0, 0.1^2) in the layer dtype."""
+    a = normal_f32(seed, (shape.name, "norm", layer), shape.d, 0.1) + np.float32(1.0)
+    return as_dtype(a, shape.dtype)
+
+
+def residual_stream(seed: int, shape: LayerShape, steps: int, rows: int) -> torch.Tensor:
+    """Stream entering the first block of a chained stack, [steps, rows, d] fp32: the AR(1)
+    decode recipe (rounded to the layer dtype, as token embeddings are stored), widened to fp32."""
+    return ar1_streams(seed, shape, steps, rows, layer=-1).float()
 
 
 def expert_block(seed: int, shape: LayerShape, expert, layer: int = 0) -> torch.Tensor:

@@ -41,6 +41,13 @@ SIGNATURES = {
     "mcft_cache_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64),
                               C.POINTER(C.c_uint64), _vp]),
     "mcft_cache_tags": (_i, [_vp, _i, _vp, _vp]),
+    "mcft_cache_prefetch": (_i, [_vp, _i, _vp, _i, _i, _i, _vp]),
+    "mcft_cache_prefetch_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64), _vp]),
+    "mcft_residual_rmsnorm": (_i, [_vp, _vp, _vp, _i, _vp, C.c_float, _vp, _vp]),
+    "mcft_stack_create": (_i, [_vp, _i, _vp, _vp, _vp, _vp, C.c_float, _vp, _i, _i, C.POINTER(_vp)]),
+    "mcft_stack_step": (_i, [_vp, _vp, _i, _vp, _vp]),
+    "mcft_stack_routing": (_i, [_vp, _i, _vp, _vp, _vp, _vp]),
+    "mcft_stack_destroy": (None, [_vp]),
     "mcft_cache_export": (_i, [_vp, _vp, C.POINTER(_sz), _vp]),
     "mcft_cache_import": (_i, [_vp, _vp, _sz, _vp]),
     "mcft_cache_destroy": (None, [_vp]),
@@ -295,6 +302,95 @@ def mcft_cache_stats(cache: Cache, layer=-1, stream=None):
     _check(lib().mcft_cache_stats(C.c_void_p(cache.handle), layer, C.byref(h), C.byref(f),
                                   C.byref(b), _stream(stream)))
     return h.value, f.value, b.value
+
+
+def mcft_cache_prefetch(cache: Cache, layer, idx_pred, n_max, stream=None):
+    """Prefetch event of `layer` from the predicted routing idx_pred [T, K] int32 (device)."""
+    T, K = idx_pred.shape
+    _check(lib().mcft_cache_prefetch(C.c_void_p(cache.handle), layer, _ptr(idx_pred), T, K,
+                                     int(n_max), _stream(stream)))
+
+
+def mcft_cache_prefetch_stats(cache: Cache, layer=-1, stream=None):
+    """(prefetched, useful) cumulative counts of one layer or of all layers (layer = -1)."""
+    p, u = C.c_uint64(), C.c_uint64()
+    _check(lib().mcft_cache_prefetch_stats(C.c_void_p(cache.handle), layer, C.byref(p), C.byref(u),
+                                           _stream(stream)))
+    return p.value, u.value
+
+
+def mcft_residual_rmsnorm(desc: LayerDesc, x, y=None, gamma=None, eps=1e-5, u=None, stream=None):
+    """x [T, d] fp32 (updated in place when y is given); returns u [T, d] in the layer dtype
+    (allocated on x's device if not given) when gamma is given, else None."""
+    T = x.shape[0]
+    if gamma is not None and u is None:
+        u = torch.empty((T, desc.d), dtype=torch.bfloat16 if desc.dtype == MCFT_BF16 else torch.float32,
+                        device=x.device)
+    _check(lib().mcft_residual_rmsnorm(C.byref(desc), _ptr(x), _ptr(y) if y is not None else None, T,
+                                       _ptr(gamma) if gamma is not None else None, C.c_float(eps),
+                                       _ptr(u) if gamma is not None else None, _stream(stream)))
+    return u
+
+
+class Stack:
+    """Handle of an mcft_stack (chained decode stack over a cache)."""
+
+    def __init__(self, handle, L, K, keep):
+        self.handle, self.L, self.K, self._keep = handle, L, K, keep
+        self.last_T = 0
+
+    def __del__(self):
+        if getattr(self, "handle", None):
+            try:
+                mcft_stack_destroy(self)
+            except Exception:
+                pass
+
+
+def mcft_stack_create(desc: LayerDesc, routers, priors, gammas, shared, eps, cache: Cache,
+                      n_prefetch=0, T_max=1) -> Stack:
+    """routers, gammas: L device tensors; priors: [L, E] array-like (fp32 > 0); shared: L lists of
+    S device blocks (or None when S = 0)."""
+    L = len(routers)
+    import numpy as _np
+    pri = _np.ascontiguousarray(_np.asarray(priors, _np.float32).reshape(-1))
+    rp = _ptr_array(routers, L)
+    gp = _ptr_array(gammas, L)
+    flat = [b for row in shared for b in row] if shared else []
+    sp = _ptr_array(flat, len(flat))
+    h = C.c_void_p()
+    _check(lib().mcft_stack_create(C.byref(desc), L, C.cast(rp, C.c_void_p), pri.ctypes.data,
+                                   C.cast(gp, C.c_void_p), C.cast(sp, C.c_void_p) if flat else None,
+                                   C.c_float(eps), C.c_void_p(cache.handle), int(n_prefetch),
+                                   int(T_max), C.byref(h)))
+    # keep everything the stack points to alive with it
+    return Stack(h.value, L, desc.K, (list(routers), list(gammas), flat, cache))
+
+
+def mcft_stack_step(stack: Stack, x, compute_stream=None, copy_stream=None):
+    """x [T, d] fp32 device tensor, updated in place (x_0 in, x_L out)."""
+    T = x.shape[0]
+    _check(lib().mcft_stack_step(C.c_void_p(stack.handle), _ptr(x), T, _stream(compute_stream),
+                                 _stream(copy_stream)))
+    stack.last_T = T
+
+
+def mcft_stack_routing(stack: Stack, layer, stream=None):
+    """(idx [T, K] int32, gate [T, K] fp32, idx_pred [T, K] int32) numpy copies of the last step."""
+    import numpy as _np
+    T, K = stack.last_T, stack.K
+    idx = _np.empty((T, K), _np.int32)
+    gate = _np.empty((T, K), _np.float32)
+    pred = _np.empty((T, K), _np.int32)
+    _check(lib().mcft_stack_routing(C.c_void_p(stack.handle), layer, idx.ctypes.data,
+                                    gate.ctypes.data, pred.ctypes.data, _stream(stream)))
+    return idx, gate, pred
+
+
+def mcft_stack_destroy(stack: Stack):
+    if stack.handle:
+        lib().mcft_stack_destroy(C.c_void_p(stack.handle))
+        stack.handle = None
 
 
 def mcft_cache_tags(cache: Cache, layer, stream=None):

@@ -1,0 +1,213 @@
+"""Chained decode stack (mcft_stack_step) against the oracle's chain (oracle.stack.chain).
+
+Every layer reads RMSNorm of the residual stream, routes it under its soft prior, runs through the
+device cache (device-driven fetch) and adds its output to the stream; with prefetch on, each next
+layer's experts are predicted and loaded while the current layer runs. Per step, layer and token:
+* the routing (and, with prefetch, the prediction) equals the oracle's as a set; the order may
+  differ only where adjacent selected scores are within the band, the set only where the K-th and
+  (K+1)-th are; after a set change the token's later layers are valid alternatives and are not
+  compared further;
+* gates of the experts the GPU chose are within gate_atol of the oracle's p-derived gates;
+* the stream leaving the stack equals the oracle's within tol, row-wise;
+* until the first step with a set change, the slot tags of every layer after the step and the five
+  cache counters equal those of per-layer oracle caches fed the oracle's routing and predictions.
+
+Tolerances. In fp32 the stream's error stays near 1e-6, so the paper-level near-tie rule applies
+(relative score gap 1e-4; gates 1e-5; stream 1e-4). In bf16 the stream carries the rounding of u,
+h and every layer output (unit roundoff 2^-9) and each block amplifies what it receives, so the
+drift from the fp64 chain grows with depth. A numpy emulation of those rounding points against the
+fp64 chain, on these shapes and inputs, measured: Mixtral widths, logit error 5e-3 at layer 0,
+4e-2 by layer 8, 8e-2 by layer 31; gate error 1.1e-2 (8 layers) and 2.3e-2 (32 layers) absolute;
+stream row error 1.0e-2 (8 layers) and 2.5e-2 (32 layers). DeepSeek-V2-Lite widths over 26 layers:
+logit error 1.1e-2, gates 8e-4, stream 4.6e-3. The bands and bounds below are about twice those.
+"""
+import functools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_34077_gb300 import inputs as I
+from paper_2609_34077_gb300 import mcft as M
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@functools.lru_cache(maxsize=2)
+def _pool(shape, seed, L, distinct):
+    """Host blocks (pinned) and fp64 oracle triples. distinct=False: every layer aliases layer
+    0's experts (the full-size stacks; fetch traffic is unchanged)."""
+    lws = [I.layer_weights(seed, shape, layer=l if distinct else 0, pin=True)
+           for l in (range(L) if distinct else range(1))]
+    trip = [[tuple(t.double().numpy() for t in I.split_expert(b, shape)) for b in lw.experts]
+            for lw in lws]
+    shared = [[tuple(t.double().numpy() for t in I.split_expert(b, shape)) for b in lw.shared]
+              for lw in lws]
+    return lws, trip, shared
+
+
+def _stack(shape, L, seed, distinct):
+    lws, trip, shared_t = _pool(shape, seed, L, distinct)
+    pick = (lambda l: l) if distinct else (lambda l: 0)
+    routers = [I.router_weight(seed, shape, l) for l in range(L)]
+    gammas = [I.norm_weight(seed, shape, l) for l in range(L)]
+    priors = np.stack([I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep, l)) for l in range(L)])
+    layers = [dict(router=routers[l].double().numpy(), prior=priors[l].astype(np.float64),
+                   gamma=gammas[l].double().numpy(), experts=trip[pick(l)], shared=shared_t[pick(l)])
+              for l in range(L)]
+    host = [lws[pick(l)].experts[e] for l in range(L) for e in range(shape.E)]
+    shared_dev = [[b.to(DEV) for b in lws[pick(l)].shared] for l in range(L)]
+    return dict(layers=layers, host=host, routers=[r.to(DEV) for r in routers],
+                gammas=[g.to(DEV) for g in gammas], priors=priors, shared=shared_dev)
+
+
+def _oracle_caches(shape, L, B, policy):
+    return [oracle.cache.SlotCache(shape.E, B, policy) for _ in range(L)]
+
+
+def _compare(got, ref, t, band, what):
+    """'same', 'order' (same set, order differs inside a near tie) or 'set' (set differs inside
+    a near tie); anything else fails."""
+    want = ref["idx"][t]
+    if np.array_equal(got, want):
+        return "same"
+    if set(got.tolist()) == set(want.tolist()):
+        assert ref["gap_in"][t] < band, f"{what}: order {got} != {want} outside a near tie"
+        return "order"
+    assert ref["gap_k"][t] < band, f"{what}: set {got} != {want} outside a near tie"
+    assert len(set(got.tolist())) == len(got)
+    return "set"
+
+
+def run_and_compare(shape, L, T, steps, B, policy, n_prefetch, distinct, seed, band, gate_atol, tol,
+                    min_cache_steps=None):
+    st = _stack(shape, L, seed, distinct)
+    desc = M.desc_of(shape)
+    cache = M.mcft_cache_create(L, shape.E, B, shape.expert_bytes, st["host"], max_assign=T * shape.K,
+                                policy=policy)
+    stack = M.mcft_stack_create(desc, st["routers"], st["priors"], st["gammas"],
+                                st["shared"] if shape.n_shared else None, shape.norm_eps, cache,
+                                n_prefetch=n_prefetch, T_max=T)
+    x0 = I.residual_stream(seed, shape, steps, T)
+    x_dev = x0.to(DEV)
+    torch.cuda.synchronize()
+    compute, copy = torch.cuda.Stream(), torch.cuda.Stream()
+    ref_caches = _oracle_caches(shape, L, B, policy)
+    ref_tot = np.zeros(3, np.int64)
+    cache_ok_until = steps  # first step with any divergence
+    diverged_tokens = 0
+    compared_rows = 0
+    for s in range(steps):
+        x = x_dev[s]
+        M.mcft_stack_step(stack, x, compute, copy)
+        compute.synchronize()
+        M.mcft_device_error()
+        xL_ref, recs = oracle.stack.chain(x0[s].double().numpy(), st["layers"], shape.K, shape.gate,
+                                          shape.norm_eps, predict=n_prefetch > 0)
+        alive = np.ones(T, bool)  # tokens not yet past a divergence in this step
+        step_diverged = False
+        for l in range(L):
+            idx, gate, pred = M.mcft_stack_routing(stack, l)
+            r = recs[l]["r"]
+            for t in range(T):
+                if not alive[t]:
+                    continue
+                if _compare(idx[t], r, t, band, f"step {s} layer {l} token {t}") == "set":
+                    alive[t] = False
+                    step_diverged = True
+                    continue
+                pa = r["p"][t, idx[t]]
+                g_ref = pa / pa.sum() if shape.gate == I.GATE_RENORM else pa
+                np.testing.assert_allclose(gate[t], g_ref, rtol=0, atol=gate_atol,
+                                           err_msg=f"gates, step {s} layer {l} token {t}")
+                if n_prefetch and l >= 1:
+                    q = recs[l - 1]["pred"]
+                    what = f"step {s} prediction for layer {l} token {t}"
+                    if _compare(pred[t], q, t, band, what) == "set":
+                        step_diverged = True
+        if step_diverged and cache_ok_until == steps:
+            cache_ok_until = s
+        diverged_tokens += int((~alive).sum())
+        got = x.cpu().double().numpy()
+        for t in np.nonzero(alive)[0]:
+            err = np.abs(got[t] - xL_ref[t]).max() / np.abs(xL_ref[t]).max()
+            assert err <= tol, f"step {s} token {t}: stream error {err:.3e}"
+            compared_rows += 1
+        if cache_ok_until == steps:
+            for l in range(L):
+                if n_prefetch and l >= 1:
+                    ref_caches[l].prefetch(oracle.stack.prefetch_set(recs[l - 1]["pred"]["idx"],
+                                                                     n_prefetch))
+                h, f, b, _ = ref_caches[l].step(recs[l]["r"]["idx"])
+                ref_tot += (h, f, b)
+                assert M.mcft_cache_tags(cache, l) == ref_caches[l].tag, f"step {s} layer {l}"
+            assert M.mcft_cache_stats(cache, -1) == tuple(int(v) for v in ref_tot)
+            assert M.mcft_cache_prefetch_stats(cache, -1) == (
+                sum(c.prefetched for c in ref_caches), sum(c.useful for c in ref_caches))
+    assert compared_rows >= steps * T // 2, (compared_rows, diverged_tokens)
+    if min_cache_steps is not None:
+        assert cache_ok_until >= min_cache_steps, cache_ok_until
+    if n_prefetch:
+        p, u = M.mcft_cache_prefetch_stats(cache, -1)
+        assert p > 0
+    del stack
+    return M.mcft_cache_stats(cache, -1), M.mcft_cache_prefetch_stats(cache, -1)
+
+
+@pytest.mark.parametrize("policy", ["LRU", "LFU", "FIFO"])
+@pytest.mark.parametrize("n_prefetch", [0, 2])
+def test_chain_fp32_tiny_exact(policy, n_prefetch):
+    run_and_compare(I.TINY, L=8, T=4, steps=12, B=4, policy=policy, n_prefetch=n_prefetch,
+                    distinct=True, seed=60, band=1e-4, gate_atol=1e-5, tol=1e-4, min_cache_steps=6)
+
+
+@pytest.mark.parametrize("n_prefetch", [0, 2])
+def test_chain_mixtral_8_layers_bf16(n_prefetch):
+    run_and_compare(I.MIXTRAL, L=8, T=2, steps=4, B=4, policy="LRU", n_prefetch=n_prefetch,
+                    distinct=False, seed=61, band=0.1, gate_atol=0.025, tol=2.5e-2)
+
+
+def test_chain_mixtral_32_layers_bf16():
+    run_and_compare(I.MIXTRAL, L=32, T=2, steps=3, B=4, policy="LFU", n_prefetch=2,
+                    distinct=False, seed=61, band=0.15, gate_atol=0.05, tol=5e-2)
+
+
+@pytest.mark.parametrize("n_prefetch", [0, 6])
+def test_chain_deepseek_26_layers_bf16(n_prefetch):
+    run_and_compare(I.DSV2_LITE, L=26, T=2, steps=4, B=12, policy="LFU", n_prefetch=n_prefetch,
+                    distinct=False, seed=62, band=0.03, gate_atol=2e-3, tol=1e-2)
+
+
+def test_prefetch_does_not_change_the_stream():
+    """The stack's output does not depend on prefetching (only where the bytes come from)."""
+    shape, L, T = I.TINY, 4, 3
+    outs = []
+    for n_prefetch in (0, 2):
+        st = _stack(shape, L, 63, True)
+        cache = M.mcft_cache_create(L, shape.E, 4, shape.expert_bytes, st["host"],
+                                    max_assign=T * shape.K)
+        stack = M.mcft_stack_create(M.desc_of(shape), st["routers"], st["priors"], st["gammas"],
+                                    None, shape.norm_eps, cache, n_prefetch=n_prefetch, T_max=T)
+        x = I.residual_stream(63, shape, 5, T).to(DEV)
+        torch.cuda.synchronize()
+        for s in range(5):
+            M.mcft_stack_step(stack, x[s])
+        torch.cuda.synchronize()
+        outs.append(x.cpu())
+    assert torch.equal(outs[0], outs[1])
+
+
+def test_stack_invalid():
+    shape = I.TINY
+    st = _stack(shape, 2, 64, True)
+    cache = M.mcft_cache_create(2, shape.E, 4, shape.expert_bytes, st["host"], max_assign=2)
+    desc = M.desc_of(shape)
+    with pytest.raises(M.MCFTError):  # prior entry <= 0
+        M.mcft_stack_create(desc, st["routers"], np.zeros_like(st["priors"]), st["gammas"], None,
+                            1e-5, cache, T_max=1)
+    stack = M.mcft_stack_create(desc, st["routers"], st["priors"], st["gammas"], None, 1e-5, cache,
+                                T_max=1)
+    with pytest.raises(M.MCFTError):  # T > T_max
+        M.mcft_stack_step(stack, torch.zeros((2, shape.d), device=DEV))
