@@ -278,17 +278,21 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
 
 /* mcft_cache_prefetch: a prefetch event of `layer` (no counterpart rule in the paper; offloading
  * systems load experts ahead of need, Section 2 "Offloading systems for MoE inference"). From the
- * predicted routing idx_pred (device [T, K] int32, e.g. mcft_route of the layer's router on a
- * speculative input) the set P = the n_max experts named most often (ties to the lower id) is
- * formed; members of P already cached are touched (last use = this event, which has a time stamp
- * of its own between two steps; no LFU access is counted); the others, in ascending id, take the
- * lowest free slot or evict, among slots not touched at this event, the smallest policy key.
+ * predicted routing idx_pred (device [T, K] int32, each row in descending score, e.g. mcft_route
+ * of the layer's router on a speculative input) the candidates are the experts it names, ranked by
+ * how many predictions name them, then the best rank k at which a token predicts them, then the
+ * lower id. Every cached candidate is touched (last use = this event, which has a time stamp of
+ * its own between two steps; no LFU access is counted), so this event evicts none of them; the
+ * n_max best-ranked uncached candidates, in ascending id, take the lowest free slot or evict,
+ * among slots not touched at this event, the smallest policy key (skipped if none qualifies).
  * Each load counts as one prefetched expert; a prefetched expert that the layer's next
  * mcft_cache_step uses counts as useful. Decided on the device on `stream`.
  * The loads are fetched (device-driven, host link) on the copy stream of the next
  * mcft_moe_forward_cached or mcft_fetch_experts call on this cache, behind that call's own misses
- * (or, for this layer, before them); the compute stream of the layer's next forward waits for
- * them before computing any expert. All calls on one cache must use one copy stream.
+ * (or, for this layer, before them). The layer's next step treats experts still arriving from
+ * the prefetch like its misses: mcft_moe_forward_cached computes them after its copies,
+ * mcft_fetch_experts makes compute_stream wait for them. All calls on one cache must use one copy
+ * stream.
  *   1 <= n_max <= B; T*K <= max_assign.
  * Errors: MCFT_ERR_INVALID (bad arguments; a previous prefetch of the layer not yet fetched);
  * MCFT_ERR_UNSUPPORTED (host blocks without device-visible addresses); an id out of range sets the

@@ -25,13 +25,15 @@ experts"); FIFO hits do not refresh the insertion order; ties always fall to the
 then the lower expert id.
 
 Prefetch (offloading systems load experts ahead of need, Section 2; the paper gives no rule): a
-prefetch of a set P (at most B experts) is a cache event of its own between two steps, with its
-own time stamp. Experts of P already cached are touched (last use = the event; no access is
-counted, so LFU counts stay those of real steps). The others, in ascending id, take the lowest
-free slot or evict, among slots not touched at this event, the smallest policy key (an insertion
-stamps last use and insertion with the event); if no slot qualifies the expert is skipped. Each
-load is one prefetch fetch. A prefetched expert that the next step uses is a hit of that step and
-counts as a useful prefetch; the pending set is cleared at every step.
+prefetch is a cache event of its own between two steps, with its own time stamp, given a ranked
+list of candidate experts (the predicted ones, most likely first) and a cap n_max <= B on loads.
+Every candidate already cached is touched (last use = the event; no access is counted, so LFU
+counts stay those of real steps), so no load of this event evicts it. The first n_max candidates
+not cached are loaded, in ascending id: each takes the lowest free slot or evicts, among slots not
+touched at this event, the smallest policy key (an insertion stamps last use and insertion with
+the event); if no slot qualifies the expert is skipped. Each load is one prefetch fetch. A
+prefetched expert that the next step uses is a hit of that step and counts as a useful prefetch;
+the pending set is cleared at every step.
 
 Two independent formulations are given: ``SlotCache`` (per-slot arrays and an argmin of the policy
 key) and ``OrderedCache`` (an ordered list of cached experts kept in victim order). Tests require
@@ -121,20 +123,20 @@ class SlotCache:
         self.last[slot] = t
         self.ins[slot] = t
 
-    def prefetch(self, experts):
-        """Prefetch event for the set `experts` (at most B distinct ids). Returns the (expert,
-        slot) loads in processing order."""
+    def prefetch(self, candidates, n_max=None):
+        """Prefetch event for the ranked candidate list (distinct ids, most likely first), loading
+        at most n_max (default B) of them. Returns the (expert, slot) loads in processing order."""
         t = self.t
-        P = sorted(set(int(e) for e in experts))
-        if len(P) > self.B or any(not 0 <= e < self.E for e in P):
-            raise ValueError("a prefetch names at most B valid experts")
+        cand = _check_candidates(candidates, self.E)
+        n_max = self.B if n_max is None else n_max
+        if not 1 <= n_max <= self.B:
+            raise ValueError("a prefetch loads between 1 and B experts")
         for s in range(self.B):
-            if self.tag[s] in P:
+            if self.tag[s] in cand:
                 self.last[s] = t
+        P = sorted([e for e in cand if e not in self.tag][:n_max])
         loads = []
         for e in P:
-            if e in self.tag:
-                continue
             slot = self._claim(t)
             if slot is None:
                 continue
@@ -144,6 +146,13 @@ class SlotCache:
         self.t += 1
         self.prefetched += len(loads)
         return loads
+
+
+def _check_candidates(candidates, E):
+    cand = [int(e) for e in candidates]
+    if len(set(cand)) != len(cand) or any(not 0 <= e < E for e in cand):
+        raise ValueError("prefetch candidates must be distinct valid expert ids")
+    return cand
 
 
 class LRUStamps(SlotCache):
@@ -256,19 +265,19 @@ class OrderedCache:
             self.order = head + sorted(tail)
         self.t += 1
 
-    def prefetch(self, experts):
+    def prefetch(self, candidates, n_max=None):
         """Prefetch event (see the module header); returns the (expert, slot) loads."""
-        P = sorted(set(int(e) for e in experts))
-        if len(P) > self.B or any(not 0 <= e < self.E for e in P):
-            raise ValueError("a prefetch names at most B valid experts")
+        cand = _check_candidates(candidates, self.E)
+        n_max = self.B if n_max is None else n_max
+        if not 1 <= n_max <= self.B:
+            raise ValueError("a prefetch loads between 1 and B experts")
         touched = set()
-        for e in P:
+        for e in sorted(cand):
             if e in self.slot_of:
                 self._touch(e, touched)
+        P = sorted([e for e in cand if e not in self.slot_of][:n_max])
         loads = []
         for e in P:
-            if e in self.slot_of:
-                continue
             slot = self._take_slot(touched)
             if slot is None:
                 continue
@@ -298,7 +307,8 @@ class LRUList(OrderedCache):
 
 def simulate(steps_ids, E: int, B: int, cls=SlotCache, policy: str = "LRU", prefetch=None):
     """Run one layer's cache over a stream of steps; steps_ids[t] holds the ids chosen at step t
-    and, when given, prefetch[t] the set prefetched just before step t (None: no prefetch event).
+    and, when given, prefetch[t] = (ranked candidates, n_max) of a prefetch just before step t
+    (None: no prefetch event).
 
     Returns per-step arrays hits, fetches, bypass and the list of per-step miss lists.
     """
@@ -306,7 +316,7 @@ def simulate(steps_ids, E: int, B: int, cls=SlotCache, policy: str = "LRU", pref
     h, f, b, ml = [], [], [], []
     for t, ids in enumerate(steps_ids):
         if prefetch is not None and prefetch[t] is not None:
-            c.prefetch(prefetch[t])
+            c.prefetch(*prefetch[t])
         hi, fi, bi, mi = c.step(ids)
         h.append(hi)
         f.append(fi)

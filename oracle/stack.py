@@ -17,9 +17,10 @@ Readings (the paper states none of this):
 * Prefetch prediction (offloading systems load experts ahead of need, Section 2 "Offloading
   systems for MoE inference"; the paper gives no rule of its own): while layer l runs, layer
   l+1's experts are predicted by routing RMSNorm_{l+1}(x_l), i.e. layer l+1's norm,
-  router and prior applied to the stream before layer l adds its output. The prefetch set of a step
-  is the distinct predicted experts ranked by how many (token, k) predictions name them, ties to the
-  lower id, cut at n_max.
+  router and prior applied to the stream before layer l adds its output. The prefetch candidates
+  of a step are the distinct predicted experts ranked by how many (token, k) predictions name them,
+  then by the best rank k at which any token predicts them (the K predictions of a token are in
+  descending score), then by id; the cache loads at most n_max of them (oracle.cache).
 """
 from __future__ import annotations
 
@@ -64,9 +65,15 @@ def chain(x0, layers, K, gate_mode, eps, predict=False):
     return x, recs
 
 
-def prefetch_set(idx_pred, n_max):
-    """Experts to prefetch from predicted routing idx_pred [T, K]: distinct ids ranked by the
-    number of predictions naming them (descending), ties to the lower id, first n_max."""
-    ids, counts = np.unique(np.asarray(idx_pred).reshape(-1), return_counts=True)
-    order = np.lexsort((ids, -counts))
-    return [int(e) for e in ids[order][:n_max]]
+def prefetch_candidates(idx_pred):
+    """Prefetch candidates from predicted routing idx_pred [T, K] (each row in descending score):
+    distinct ids ranked by the number of predictions naming them (descending), then the best rank
+    k at which they are predicted (ascending), then id (ascending)."""
+    idx_pred = np.asarray(idx_pred)
+    count, best = {}, {}
+    for row in idx_pred:
+        for k, e in enumerate(row.tolist()):
+            count[e] = count.get(e, 0) + 1
+            best[e] = min(best.get(e, k), k)
+    ranked = sorted(count, key=lambda e: (-count[e], best[e], e))
+    return [int(e) for e in ranked]

@@ -667,7 +667,7 @@ mcft_status mcft_cache_prefetch(mcft_cache* c, int layer, const int32_t* idx_pre
     MCFT_CUDA(cudaStreamWaitEvent(stream, c->ev_pf_done[layer], 0));
     c->pf_state[layer] = 0;
   }
-  PrefetchArgs a{idx_pred, T * K, n_max, c->E, c->B, layer, c->policy, c->d_tag, c->d_last,
+  PrefetchArgs a{idx_pred, T * K, K, n_max, c->E, c->B, layer, c->policy, c->d_tag, c->d_last,
                  c->d_ins, c->d_freq, c->d_step, c->d_cnt, c->d_pfmask,
                  c->d_pf_list + size_t(layer) * (1 + c->E), c->d_pf_tab + size_t(layer) * c->E,
                  c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
@@ -820,14 +820,13 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
   cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy_stream);
   if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
+  // Experts a prefetch of this layer is still bringing in are not in the step's ready mask: the
+  // FFN computes them in phase 2, after compute_stream waits for ev_copy, which follows their
+  // fetch on this copy stream.
+  if (c->pf_state[layer] == 2) c->pf_state[layer] = 0;
   // 1b. prefetches decided for later layers stream in behind this layer's misses
   st = enqueue_prefetch_fetches(c, copy_stream);
   if (st != MCFT_OK) return st;
-  // hits may be experts a prefetch is still bringing in
-  if (c->pf_state[layer] == 2) {
-    MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_pf_done[layer], 0));
-    c->pf_state[layer] = 0;
-  }
   // 2. meanwhile: permutation and the experts that were hits (and the shared experts)
   PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
   e = launch_permute(pa, compute_stream);

@@ -11,12 +11,16 @@
 // completes.
 //
 // Prefetch (offloading systems load experts ahead of need, Section 2; the rule is this library's):
-// a prefetch is a cache event of its own, one time stamp between two steps. Its set is the n_max
-// experts named most often by a predicted routing (ties to the lower id); members already cached
-// are touched (last use = the event, no access counted), the others, in ascending id, take the
-// lowest free slot or evict, among slots not touched at the event, the smallest policy key. The
+// a prefetch is a cache event of its own, one time stamp between two steps. Its candidates are
+// the experts of a predicted routing, ranked by how many predictions name them, then the best
+// rank k at which a token predicts them, then the lower id. Every cached candidate is touched
+// (last use = the event, no access counted); the n_max best-ranked uncached candidates, in
+// ascending id, take the lowest free slot or evict, among slots not touched at the event, the
+// smallest policy key. The
 // loads form a separate fetch list, so a prefetch never disturbs the miss list of a step whose
-// fetch may still be in flight. The next step counts hits on prefetched experts as useful.
+// fetch may still be in flight. The next step counts hits on prefetched experts as useful, and
+// leaves them out of its ready mask: their bytes arrive on the copy stream, so the FFN computes
+// them with the step's misses, after the copies.
 #include "common.cuh"
 #include "internal.h"
 
@@ -79,7 +83,7 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
   }
   for (int e = lane; e < E; e += 32) s_freq[e] = freq[e] + ((mine >> e) & 1ull);
   __syncwarp();
-  unsigned long long cached = 0;
+  unsigned long long cached = 0, pf = 0;
   int hits = 0, nm = 0, nbyp = 0;
   const int64_t t = a.step[a.layer];
   if (lane == 0) {
@@ -97,7 +101,7 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
         ++hits;
       }
     }
-    const unsigned long long pf = a.pfmask[a.layer];
+    pf = a.pfmask[a.layer];
     const int useful = __popcll(pf & mine & cached);
     unsigned long long miss = mine & ~cached;
     while (miss) {
@@ -136,6 +140,7 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
     a.pfmask[a.layer] = 0;
   }
   cached = __shfl_sync(0xffffffffu, cached, 0);
+  pf = __shfl_sync(0xffffffffu, pf, 0);
   __syncwarp();
   // write back the state and publish the step's miss list and expert table (all lanes)
   for (int i = lane; i < B; i += 32) {
@@ -156,7 +161,8 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
       p = reinterpret_cast<unsigned long long>(loc < B ? a.slots + size_t(loc) * a.expert_bytes
                                                        : a.staging + size_t(loc - B) * a.expert_bytes);
     a.ptr_tab[e] = p;
-    if (loc >= 0 && loc < B && ((cached >> e) & 1ull)) hitbits |= 1ull << e;
+    // ready now: hits whose bytes are not still coming from a prefetch
+    if (loc >= 0 && loc < B && ((cached & ~pf) >> e) & 1ull) hitbits |= 1ull << e;
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) hitbits |= __shfl_xor_sync(0xffffffffu, hitbits, o);
@@ -167,18 +173,25 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
 // Prefetch decision (one warp). The lanes count how many predicted (token, k) entries name each
 // expert; lane 0 ranks, touches, claims slots and writes the fetch list.
 __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ PrefetchArgs a) {
-  __shared__ int cnt[kMaxE];
+  __shared__ int cnt[kMaxE], rank[kMaxE];
   __shared__ int32_t s_tag[kMaxE];
   __shared__ int64_t s_last[kMaxE], s_ins[kMaxE], s_freq[kMaxE];
   __shared__ int32_t s_list[1 + kMaxE];
   const int lane = threadIdx.x, B = a.B, E = a.E;
-  for (int e = lane; e < E; e += 32) cnt[e] = 0;
+  for (int e = lane; e < E; e += 32) {
+    cnt[e] = 0;
+    rank[e] = 1 << 30;
+  }
   __syncwarp();
   int bad = 0;
   for (int i = lane; i < a.n; i += 32) {
     const int e = a.idx[i];
-    if (e < 0 || e >= E) bad = 1;
-    else atomicAdd(&cnt[e], 1);
+    if (e < 0 || e >= E) {
+      bad = 1;
+    } else {
+      atomicAdd(&cnt[e], 1);
+      atomicMin(&rank[e], i % a.K);
+    }
   }
   bad = __any_sync(0xffffffffu, bad);
   if (bad) {  // no state change on bad input
@@ -200,24 +213,28 @@ __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ Pr
   __syncwarp();
   if (lane == 0) {
     const int64_t t = a.step[a.layer];
-    // the set: n_max experts by (count descending, id ascending)
-    unsigned long long P = 0;
-    for (int j = 0; j < a.n_max; ++j) {
-      int best = -1;
-      for (int e = 0; e < E; ++e)
-        if (cnt[e] > 0 && !((P >> e) & 1ull) && (best < 0 || cnt[e] > cnt[best])) best = e;
-      if (best < 0) break;
-      P |= 1ull << best;
-    }
-    unsigned long long cached = 0;
+    // every cached candidate is touched; the loads are the n_max best-ranked uncached candidates
+    // by (count descending, best rank ascending, id ascending)
+    unsigned long long cand = 0, cached = 0;
+    for (int e = 0; e < E; ++e)
+      if (cnt[e] > 0) cand |= 1ull << e;
     for (int sl = 0; sl < B; ++sl) {
       const int e = s_tag[sl];
       if (e < 0) continue;
       cached |= 1ull << e;
-      if ((P >> e) & 1ull) s_last[sl] = t;
+      if ((cand >> e) & 1ull) s_last[sl] = t;
+    }
+    unsigned long long load = 0;
+    for (int j = 0; j < a.n_max; ++j) {
+      int best = -1;
+      for (int e = 0; e < E; ++e) {
+        if (!(((cand & ~cached & ~load) >> e) & 1ull)) continue;
+        if (best < 0 || cnt[e] > cnt[best] || (cnt[e] == cnt[best] && rank[e] < rank[best])) best = e;
+      }
+      if (best < 0) break;
+      load |= 1ull << best;
     }
     unsigned long long pf = a.pfmask[a.layer];
-    unsigned long long load = P & ~cached;
     int nl = 0;
     while (load) {
       const int e = __ffsll(static_cast<long long>(load)) - 1;

@@ -205,11 +205,12 @@ cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s);
 
 constexpr int kCacheCounters = 5;  // per layer: hits, fetches, bypass, prefetched, useful
 
-// Prefetch decision of one layer: the n_max experts named most often by the predicted routing
-// (ties to the lower id) are touched or loaded into the layer's slots (cache.cu).
+// Prefetch decision of one layer: the experts of the predicted routing that are cached are
+// touched, and the n_max best-ranked uncached ones (by count, then best predicted rank, then id)
+// are loaded into the layer's slots (cache.cu).
 struct PrefetchArgs {
-  const int32_t* idx;  // predicted routing [n]
-  int n, n_max;
+  const int32_t* idx;  // predicted routing [n / K][K], each row in descending score
+  int n, K, n_max;
   int E, B, layer, policy;
   int32_t* tag;
   int64_t* last;

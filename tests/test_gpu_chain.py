@@ -138,8 +138,8 @@ def run_and_compare(shape, L, T, steps, B, policy, n_prefetch, distinct, seed, b
         if cache_ok_until == steps:
             for l in range(L):
                 if n_prefetch and l >= 1:
-                    ref_caches[l].prefetch(oracle.stack.prefetch_set(recs[l - 1]["pred"]["idx"],
-                                                                     n_prefetch))
+                    ref_caches[l].prefetch(
+                        oracle.stack.prefetch_candidates(recs[l - 1]["pred"]["idx"]), n_prefetch)
                 h, f, b, _ = ref_caches[l].step(recs[l]["r"]["idx"])
                 ref_tot += (h, f, b)
                 assert M.mcft_cache_tags(cache, l) == ref_caches[l].tag, f"step {s} layer {l}"

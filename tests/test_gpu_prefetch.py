@@ -1,7 +1,7 @@
 """Prefetch events of the device cache (mcft_cache_prefetch) against the oracle, bit-exact.
 
 Decisions: random predicted routings and step routings through the device cache in accounting mode
-and through oracle.cache.SlotCache with oracle.stack.prefetch_set; slot tags after every event and
+and through oracle.cache.SlotCache with oracle.stack.prefetch_candidates; slot tags after every event and
 all five counters must be equal. Data: with slots and pinned host blocks, every expert a step
 selects must hold its host block's bytes, whether it came from the step's own fetch, from a
 prefetch streamed in behind an earlier layer's misses, or from an earlier step."""
@@ -32,7 +32,7 @@ def test_prefetch_decisions_exact(policy, E, B, K, T, n_max):
     for s in range(steps):
         if s % 3 != 2:
             M.mcft_cache_prefetch(c, 0, torch.from_numpy(preds[s]).to(DEV), n_max)
-            ref.prefetch(oracle.stack.prefetch_set(preds[s], n_max))
+            ref.prefetch(oracle.stack.prefetch_candidates(preds[s]), n_max)
             assert M.mcft_cache_tags(c, 0) == ref.tag, f"after the prefetch before step {s}"
         M.mcft_cache_step(c, 0, torch.from_numpy(ids[s]).to(DEV))
         h, f, b, _ = ref.step(ids[s])

@@ -30,9 +30,11 @@ def _load_traces():
             ml = [tuple(int(v) for v in m.split(":")) for m in misses.split()[1:]]
             cur["steps"].append(([int(v) for v in ids.split(",")], int(hits.split()[1]), ml))
         elif line.startswith("prefetch"):
-            ids, loads = [p.strip() for p in line[8:].split("|")]
+            head, loads = [p.strip() for p in line[8:].split("|")]
+            f = head.split()
+            n_max = int(f[2]) if len(f) > 2 else None
             ll = [tuple(int(v) for v in m.split(":")) for m in loads.split()[1:]]
-            cur["steps"].append(([int(v) for v in ids.split(",")], None, ll))
+            cur["steps"].append((([int(v) for v in f[0].split(",")], n_max), None, ll))
         elif line.startswith("total"):
             f = line.split()
             cur["total"] = dict(hits=int(f[2]), fetches=int(f[4]), bypass=int(f[6]))
@@ -50,8 +52,8 @@ def test_hand_traces(cls, tr):
     c = cls(tr["E"], tr["B"], tr["policy"])
     th = tf = tb = 0
     for ids, hits, misses in tr["steps"]:
-        if hits is None:  # prefetch event
-            assert c.prefetch(ids) == misses
+        if hits is None:  # prefetch event: (ranked candidates, n_max)
+            assert c.prefetch(*ids) == misses
             continue
         h, f, b, ml = c.step(ids)
         assert h == hits
@@ -99,11 +101,13 @@ def test_two_formulations_agree(T, K, E, B, policy):
 
 
 def _random_prefetches(seed, steps, E, B, n_max, p=0.7):
+    """Random (ranked candidates, cap) pairs; candidate lists may be longer than the cap and B."""
     g = np.random.default_rng(seed)
     out = []
     for _ in range(steps):
         if g.random() < p:
-            out.append(sorted(g.choice(E, size=int(g.integers(1, n_max + 1)), replace=False).tolist()))
+            cand = g.choice(E, size=int(g.integers(1, min(E, 2 * B) + 1)), replace=False).tolist()
+            out.append((cand, int(g.integers(1, n_max + 1))))
         else:
             out.append(None)
     return out
@@ -118,7 +122,7 @@ def test_two_formulations_agree_with_prefetch(T, K, E, B, n_max, policy):
     a, b = C.SlotCache(E, B, policy), C.OrderedCache(E, B, policy)
     for s in range(ids.shape[0]):
         if pfs[s] is not None:
-            assert a.prefetch(pfs[s]) == b.prefetch(pfs[s])
+            assert a.prefetch(*pfs[s]) == b.prefetch(*pfs[s])
             assert a.tag == b.state()
         assert a.step(ids[s]) == b.step(ids[s])
         assert a.tag == b.state()
@@ -164,6 +168,26 @@ def test_perfect_prefetch_moves_every_fetch_to_the_prefetch(policy):
     assert demand == 0
     assert c.prefetched == c.useful
     assert c.prefetched + f0 == plain[1].sum()
+
+
+@pytest.mark.parametrize("policy", C.POLICIES)
+def test_capped_prefetch_never_evicts_a_candidate(policy):
+    """Every cached candidate is touched, so a capped prefetch loads only into slots of
+    non-candidates: the cached candidates are all still cached after it."""
+    E, B = 12, 5
+    g = np.random.default_rng(20)
+    c = C.SlotCache(E, B, policy)
+    for s in range(300):
+        c.step(g.choice(E, size=2, replace=False))
+        cand = g.choice(E, size=int(g.integers(1, E)), replace=False).tolist()
+        before = set(c.tag) & set(cand)
+        n_max = int(g.integers(1, B + 1))
+        loads = c.prefetch(cand, n_max)
+        assert before <= set(c.tag)
+        # loads come from the n_max best-ranked uncached candidates, as many as untouched slots allow
+        unc = [e for e in cand if e not in before]
+        assert {e for e, _ in loads} <= set(unc[:n_max])
+        assert len(loads) == min(n_max, len(unc), B - len(before))
 
 
 @pytest.mark.parametrize("policy", C.POLICIES)
@@ -226,6 +250,9 @@ def test_invalid():
     with pytest.raises(ValueError):
         c.step([5])
     with pytest.raises(ValueError):
-        c.prefetch([0, 1, 2])
+        c.prefetch([0, 0])
     with pytest.raises(ValueError):
         c.prefetch([4])
+    for n_max in (0, 3):
+        with pytest.raises(ValueError):
+            c.prefetch([0, 1, 2], n_max)

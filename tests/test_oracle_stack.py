@@ -101,9 +101,10 @@ def test_identity_experts_closed_form():
             assert x1[t, j] == pytest.approx(x0[t, j] + v / (1.0 + math.exp(-v)) * v, rel=1e-12, abs=1e-14)
 
 
-def test_prefetch_set_ranking():
-    assert S.prefetch_set(np.array([[3, 1], [1, 2], [2, 1]]), 2) == [1, 2]
-    assert S.prefetch_set(np.array([[3, 1], [1, 2], [2, 1]]), 5) == [1, 2, 3]
-    assert S.prefetch_set(np.array([[5, 0], [0, 5]]), 2) == [0, 5]
-    assert S.prefetch_set(np.array([[5, 0], [0, 5]]), 1) == [0]
-    assert S.prefetch_set(np.array([[7, 2, 4]]), 3) == [2, 4, 7]
+def test_prefetch_candidate_ranking():
+    """Hand-worked: counts first, then the best predicted rank, then the id."""
+    assert S.prefetch_candidates(np.array([[3, 1], [1, 2], [2, 1]])) == [1, 2, 3]
+    assert S.prefetch_candidates(np.array([[5, 0], [0, 5]])) == [0, 5]   # same count, both rank 0
+    assert S.prefetch_candidates(np.array([[7, 2, 4]])) == [7, 2, 4]     # one token: its own order
+    assert S.prefetch_candidates(np.array([[4, 1], [1, 3]])) == [1, 4, 3]  # 4 at rank 0, 3 at 1
+    assert S.prefetch_candidates(np.array([[6, 3], [2, 6]])) == [6, 2, 3]  # 2 at rank 0 beats 3
