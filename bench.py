@@ -495,13 +495,15 @@ def run_chain(shape, L, steps, warmup, seed, dev, policy="LRU", n_prefetch=0, gr
     if graph:
         S.capture()  # records one step; runs nothing
     h0, f0, _ = M.mcft_cache_stats(S.cache, -1)
-    p0, u0 = M.mcft_cache_prefetch_stats(S.cache, -1)
+    p0, u0, m0 = M.mcft_cache_prefetch_stats(S.cache, -1)
     elapsed = time_steps(S.step, warmup, steps, S.compute)
     M.mcft_device_error()
     h1, f1, _ = M.mcft_cache_stats(S.cache, -1)
-    p1, u1 = M.mcft_cache_prefetch_stats(S.cache, -1)
+    p1, u1, m1 = M.mcft_cache_prefetch_stats(S.cache, -1)
     fetches, pref, useful = f1 - f0, p1 - p0, u1 - u0
-    moved = (fetches + pref) * shape.expert_bytes / steps
+    # bytes on the host link: every demand fetch in full, prefetches as far as they ran (a
+    # prefetch the next step dropped stops early)
+    moved = (fetches * shape.expert_bytes + (m1 - m0)) / steps
     res = dict(workload=f"{shape.name} chained decode stack, {L} layers, batch 1, {policy}, "
                         f"prefetch {n_prefetch or 'off'}",
                layers=L, policy=policy, n_prefetch=n_prefetch, cuda_graph=graph, steps=steps,
@@ -509,6 +511,7 @@ def run_chain(shape, L, steps, warmup, seed, dev, policy="LRU", n_prefetch=0, gr
                demand_fetches_per_token=fetches / steps, prefetches_per_token=pref / steps,
                useful_prefetches_per_token=useful / steps,
                prefetch_accuracy=useful / pref if pref else None,
+               prefetch_gb_moved_per_token=(m1 - m0) / steps / 1e9,
                hit_rate=(h1 - h0) / max(1, h1 - h0 + fetches),
                link_gb_per_token=moved / 1e9, link_bound_tpot_ms=moved / 210e9 * 1e3,
                host_pool="E distinct pinned blocks aliased by every layer")

@@ -204,9 +204,10 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
                               const void* const* host_experts, int max_assign, int policy,
                               mcft_cache** out);
 
-/* mcft_cache_step: one decode step of one layer. Reads idx (device [T, K] int32), decides hits,
- * misses, evictions and bypasses on the device, updates the counters and writes the step's miss
- * list to host-mapped memory for mcft_fetch_experts. Asynchronous on `stream`.
+/* mcft_cache_step: one decode step of one layer. Reads idx (device [T, K] int32), drops the
+ * experts the layer's last prefetch loaded that this step does not use (mcft_cache_prefetch),
+ * decides hits, misses, evictions and bypasses on the device, updates the counters and writes the
+ * step's miss list to host-mapped memory for mcft_fetch_experts. Asynchronous on `stream`.
  * Errors: MCFT_ERR_INVALID (layer out of range, T*K > max_assign, NULL idx); an id out of range
  * sets the device error word and the step changes no state. */
 mcft_status mcft_cache_step(mcft_cache* cache, int layer, const int32_t* idx, int T, int K,
@@ -286,7 +287,9 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
  * n_max best-ranked uncached candidates, in ascending id, take the lowest free slot or evict,
  * among slots not touched at this event, the smallest policy key (skipped if none qualifies).
  * Each load counts as one prefetched expert; a prefetched expert that the layer's next
- * mcft_cache_step uses counts as useful. Decided on the device on `stream`.
+ * mcft_cache_step uses counts as useful, one it does not use is dropped by that step (its slot
+ * becomes free before the step's hits and misses) and the prefetch's fetch stops copying it.
+ * Decided on the device on `stream`.
  * The loads are fetched (device-driven, host link) on the copy stream of the next
  * mcft_moe_forward_cached or mcft_fetch_experts call on this cache, behind that call's own misses
  * (or, for this layer, before them). The layer's next step treats experts still arriving from
@@ -300,11 +303,12 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
 mcft_status mcft_cache_prefetch(mcft_cache* cache, int layer, const int32_t* idx_pred, int T, int K,
                                 int n_max, mcft_stream_t stream);
 
-/* mcft_cache_prefetch_stats: cumulative prefetched experts and useful prefetches (prefetched
- * experts used by the next step) of one layer, or summed when layer = -1. Prefetched experts are
- * link traffic on top of mcft_cache_stats's fetches. Synchronises `stream` first. */
+/* mcft_cache_prefetch_stats: cumulative prefetched experts, useful prefetches (prefetched
+ * experts used by the next step) and bytes the prefetch fetches actually copied (a dropped
+ * prefetch stops early) of one layer, or summed when layer = -1. The counts are decisions and
+ * exact; bytes_moved depends on timing. Synchronises `stream` first. */
 mcft_status mcft_cache_prefetch_stats(const mcft_cache* cache, int layer, uint64_t* prefetched,
-                                      uint64_t* useful, mcft_stream_t stream);
+                                      uint64_t* useful, uint64_t* bytes_moved, mcft_stream_t stream);
 
 /* mcft_cache_last_misses: the miss list of the last mcft_cache_step of `layer`, after
  * mcft_fetch_experts (or a synchronisation of its stream): n_out = number of fetches;

@@ -32,8 +32,10 @@ counts stay those of real steps), so no load of this event evicts it. The first 
 not cached are loaded, in ascending id: each takes the lowest free slot or evicts, among slots not
 touched at this event, the smallest policy key (an insertion stamps last use and insertion with
 the event); if no slot qualifies the expert is skipped. Each load is one prefetch fetch. A
-prefetched expert that the next step uses is a hit of that step and counts as a useful prefetch;
-the pending set is cleared at every step.
+prefetched expert that the next step uses is a hit of that step and counts as a useful prefetch.
+Prefetched experts the next step does not use are dropped when it begins (their slots become
+free before its hits and misses are processed), so a wrong prediction can be cancelled while its
+bytes are still in flight; the pending set is cleared at every step.
 
 Two independent formulations are given: ``SlotCache`` (per-slot arrays and an argmin of the policy
 key) and ``OrderedCache`` (an ordered list of cached experts kept in victim order). Tests require
@@ -88,6 +90,9 @@ class SlotCache:
         for e in U:
             self.freq[e] += 1
         self.useful += len(self.pf & set(U))
+        for s in range(self.B):  # unused prefetched experts are dropped
+            if self.tag[s] in self.pf and self.tag[s] not in U:
+                self.tag[s], self.last[s], self.ins[s] = -1, -1, -1
         self.pf = set()
         hits = 0
         for s in range(self.B):
@@ -216,6 +221,10 @@ class OrderedCache:
         for e in U:
             self.count[e] += 1
         self.useful += sum(1 for e in U if e in self.pf)
+        for e in sorted(self.pf - set(U)):  # unused prefetched experts are dropped
+            self._remove(e)
+            self.free.append(self.slot_of.pop(e))
+        self.free.sort()
         self.pf = set()
         touched = set()
         hits = 0

@@ -145,6 +145,8 @@ struct mcft_cache {
   unsigned long long* d_ready = nullptr;    // [L] hit mask of the last step
   unsigned long long* d_host_src = nullptr; // [L*E] device-visible addresses of the host blocks
   unsigned long long* d_pfmask = nullptr;   // [L] experts loaded by a prefetch since the last step
+  unsigned long long* d_pf_cancel = nullptr;  // [L] prefetched experts the next step dropped
+  unsigned long long* d_pf_moved = nullptr;   // [L] bytes the prefetch fetches copied
   int32_t* d_pf_list = nullptr;             // [L][1 + E] fetch list of the last prefetch
   unsigned long long* d_pf_tab = nullptr;   // [L*E] destinations of the last prefetch's loads
   char* d_slots = nullptr;    // [L*B] expert blocks
@@ -176,6 +178,8 @@ void cache_free(mcft_cache* c) {
   cudaFree(c->d_ready);
   cudaFree(c->d_host_src);
   cudaFree(c->d_pfmask);
+  cudaFree(c->d_pf_cancel);
+  cudaFree(c->d_pf_moved);
   cudaFree(c->d_pf_list);
   cudaFree(c->d_pf_tab);
   for (const auto* v : {&c->ev_step, &c->ev_pf_step, &c->ev_pf_done})
@@ -210,7 +214,8 @@ mcft_status enqueue_prefetch_fetches(mcft_cache* c, cudaStream_t copy) {
     if (c->pf_state[l] != 1) continue;
     MCFT_CUDA(cudaStreamWaitEvent(copy, c->ev_pf_step[l], 0));
     FetchArgs fe{c->d_pf_list + size_t(l) * (1 + c->E), c->d_host_src + size_t(l) * c->E,
-                 c->d_pf_tab + size_t(l) * c->E, c->expert_bytes};
+                 c->d_pf_tab + size_t(l) * c->E, c->expert_bytes, c->d_pf_cancel + l,
+                 c->d_pf_moved + l};
     cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy, true);
     if (e != cudaSuccess) return cuda_fail(e, "prefetch fetch kernel launch");
     MCFT_CUDA(cudaEventRecord(c->ev_pf_done[l], copy));
@@ -535,6 +540,10 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_cnt, sizeof(unsigned long long) * L * kCacheCounters));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_pfmask, sizeof(unsigned long long) * L));
   MCFT_CACHE_CUDA(cudaMemset(c->d_pfmask, 0, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_pf_cancel, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_pf_cancel, 0, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_pf_moved, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_pf_moved, 0, sizeof(unsigned long long) * L));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_pf_list, sizeof(int32_t) * L * (1 + E)));
   MCFT_CACHE_CUDA(cudaMemset(c->d_pf_list, 0, sizeof(int32_t) * L * (1 + E)));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_pf_tab, sizeof(unsigned long long) * L * E));
@@ -599,7 +608,7 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
   if (T * K > c->max_assign)
     return fail(MCFT_ERR_INVALID, "T*K = %d exceeds max_assign = %d", T * K, c->max_assign);
   CacheStepArgs a{idx, T * K, c->E, c->B, layer, c->policy, c->d_tag, c->d_last, c->d_ins,
-                  c->d_freq, c->d_step, c->d_cnt, c->d_pfmask,
+                  c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
                   c->d_miss + size_t(layer) * c->miss_stride,
                   c->d_miss_dev + size_t(layer) * c->miss_stride,
                   c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer,
@@ -668,7 +677,7 @@ mcft_status mcft_cache_prefetch(mcft_cache* c, int layer, const int32_t* idx_pre
     c->pf_state[layer] = 0;
   }
   PrefetchArgs a{idx_pred, T * K, K, n_max, c->E, c->B, layer, c->policy, c->d_tag, c->d_last,
-                 c->d_ins, c->d_freq, c->d_step, c->d_cnt, c->d_pfmask,
+                 c->d_ins, c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
                  c->d_pf_list + size_t(layer) * (1 + c->E), c->d_pf_tab + size_t(layer) * c->E,
                  c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                  c->expert_bytes, device_error_word()};
@@ -682,20 +691,25 @@ mcft_status mcft_cache_prefetch(mcft_cache* c, int layer, const int32_t* idx_pre
 }
 
 mcft_status mcft_cache_prefetch_stats(const mcft_cache* c, int layer, uint64_t* prefetched,
-                                      uint64_t* useful, mcft_stream_t stream) {
-  if (!c || !prefetched || !useful) return fail(MCFT_ERR_INVALID, "NULL argument");
+                                      uint64_t* useful, uint64_t* bytes_moved,
+                                      mcft_stream_t stream) {
+  if (!c || !prefetched || !useful || !bytes_moved) return fail(MCFT_ERR_INVALID, "NULL argument");
   if (layer < -1 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
-  std::vector<unsigned long long> h(size_t(c->L) * kCacheCounters);
+  std::vector<unsigned long long> h(size_t(c->L) * kCacheCounters), m(c->L);
   MCFT_CUDA(cudaMemcpyAsync(h.data(), c->d_cnt, h.size() * sizeof(h[0]), cudaMemcpyDeviceToHost, stream));
+  MCFT_CUDA(cudaMemcpyAsync(m.data(), c->d_pf_moved, m.size() * sizeof(m[0]), cudaMemcpyDeviceToHost,
+                            stream));
   MCFT_CUDA(cudaStreamSynchronize(stream));
-  uint64_t p = 0, u = 0;
+  uint64_t p = 0, u = 0, b = 0;
   for (int l = 0; l < c->L; ++l) {
     if (layer >= 0 && l != layer) continue;
     p += h[size_t(l) * kCacheCounters + 3];
     u += h[size_t(l) * kCacheCounters + 4];
+    b += m[l];
   }
   *prefetched = p;
   *useful = u;
+  *bytes_moved = b;
   return MCFT_OK;
 }
 
@@ -816,7 +830,7 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
   // 1. the missed experts stream in on the copy stream, after this layer's cache step
   MCFT_CUDA(cudaStreamWaitEvent(copy_stream, c->ev_step[layer], 0));
   FetchArgs fe{c->d_miss_dev + size_t(layer) * c->miss_stride, c->d_host_src + size_t(layer) * E,
-               c->d_ptr_tab + size_t(layer) * E, c->expert_bytes};
+               c->d_ptr_tab + size_t(layer) * E, c->expert_bytes, nullptr, nullptr};
   cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy_stream);
   if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));

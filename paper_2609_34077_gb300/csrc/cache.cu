@@ -20,7 +20,10 @@
 // loads form a separate fetch list, so a prefetch never disturbs the miss list of a step whose
 // fetch may still be in flight. The next step counts hits on prefetched experts as useful, and
 // leaves them out of its ready mask: their bytes arrive on the copy stream, so the FFN computes
-// them with the step's misses, after the copies.
+// them with the step's misses, after the copies. Prefetched experts the step does not use are
+// dropped first (slots freed) and flagged in the layer's cancel mask, which the prefetch's fetch
+// kernel reads before each piece: a wrong prediction stops using the host link as soon as the
+// step's routing is known.
 #include "common.cuh"
 #include "internal.h"
 
@@ -91,6 +94,17 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
     int32_t* m_loc = s_out + 1 + E;
     int32_t* loc_of = s_out + 1 + 2 * E;
     for (int e = 0; e < E; ++e) loc_of[e] = -1;
+    pf = a.pfmask[a.layer];
+    const unsigned long long drop = pf & ~mine;  // prefetched experts this step does not use
+    for (int sl = 0; sl < B; ++sl) {
+      const int e = s_tag[sl];
+      if (e >= 0 && ((drop >> e) & 1ull)) {
+        s_tag[sl] = -1;
+        s_last[sl] = -1;
+        s_ins[sl] = -1;
+      }
+    }
+    a.cancel[a.layer] = drop;
     for (int sl = 0; sl < B; ++sl) {
       const int e = s_tag[sl];
       if (e < 0) continue;
@@ -101,7 +115,6 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
         ++hits;
       }
     }
-    pf = a.pfmask[a.layer];
     const int useful = __popcll(pf & mine & cached);
     unsigned long long miss = mine & ~cached;
     while (miss) {
@@ -259,6 +272,7 @@ __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ Pr
     }
     s_list[0] = nl;
     a.pfmask[a.layer] = pf;
+    a.cancel[a.layer] = 0;
     a.step[a.layer] = t + 1;
     a.counters[size_t(a.layer) * kCacheCounters + 3] += nl;
   }
@@ -291,10 +305,18 @@ __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ Fetc
   const size_t units = size_t(n) * per;
   for (size_t u = blockIdx.x; u < units; u += gridDim.x) {
     const int e = a.miss[1 + int(u / per)];
+    if (a.cancel) {  // a step dropped this prefetched expert: stop moving it (block-uniform read)
+      __shared__ unsigned long long c;
+      __syncthreads();
+      if (threadIdx.x == 0) c = *reinterpret_cast<const volatile unsigned long long*>(a.cancel);
+      __syncthreads();
+      if ((c >> e) & 1ull) continue;
+    }
     const uint4* src = reinterpret_cast<const uint4*>(a.host_src[e]);
     uint4* dst = reinterpret_cast<uint4*>(a.ptr_tab[e]);
     const size_t w0 = (u % per) * piece;
     const size_t w1 = w0 + piece < words ? w0 + piece : words;
+    if (a.moved && threadIdx.x == 0) atomicAdd(a.moved, (unsigned long long)(w1 - w0) * 16ull);
     const size_t stride = blockDim.x;
     for (size_t w = w0 + threadIdx.x; w < w1; w += 4 * stride) {
       uint4 v[4];

@@ -192,6 +192,7 @@ struct CacheStepArgs {
   int64_t* step;      // [L]
   unsigned long long* counters;  // [L*kCacheCounters] hits, fetches, bypass, prefetched, useful
   unsigned long long* pfmask;    // [L] experts loaded by a prefetch since the layer's last step
+  unsigned long long* cancel;    // [L] prefetched experts this step dropped (read by the fetch)
   int32_t* miss_out;  // host-mapped, per layer: [n_miss, expert[E], loc[E], loc_of[E]]
   int32_t* miss_dev;  // device copy of the same list (read by the fetch kernel)
   unsigned long long* ptr_tab;  // device [E]: block address of each selected expert, else 0
@@ -219,6 +220,7 @@ struct PrefetchArgs {
   int64_t* step;
   unsigned long long* counters;
   unsigned long long* pfmask;
+  unsigned long long* cancel;     // [L]: cleared for the layer by a new prefetch
   int32_t* list;                  // device, this layer: [n_load, expert[E]] (fetch list)
   unsigned long long* ptr_tab;    // device [E]: destination of each loaded expert, else 0
   const char* slots;              // this layer's first slot block (NULL in accounting mode)
@@ -234,6 +236,8 @@ struct FetchArgs {
   const unsigned long long* host_src; // [E]
   const unsigned long long* ptr_tab;  // [E]
   size_t bytes;                       // per expert block, multiple of 16
+  const unsigned long long* cancel;   // prefetch fetches: experts to stop copying, else NULL
+  unsigned long long* moved;          // prefetch fetches: bytes copied (accumulated), else NULL
 };
 cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch = false);
 

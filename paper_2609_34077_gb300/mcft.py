@@ -42,7 +42,8 @@ SIGNATURES = {
                               C.POINTER(C.c_uint64), _vp]),
     "mcft_cache_tags": (_i, [_vp, _i, _vp, _vp]),
     "mcft_cache_prefetch": (_i, [_vp, _i, _vp, _i, _i, _i, _vp]),
-    "mcft_cache_prefetch_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64), _vp]),
+    "mcft_cache_prefetch_stats": (_i, [_vp, _i, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64),
+                                       C.POINTER(C.c_uint64), _vp]),
     "mcft_residual_rmsnorm": (_i, [_vp, _vp, _vp, _i, _vp, C.c_float, _vp, _vp]),
     "mcft_stack_create": (_i, [_vp, _i, _vp, _vp, _vp, _vp, C.c_float, _vp, _i, _i, C.POINTER(_vp)]),
     "mcft_stack_step": (_i, [_vp, _vp, _i, _vp, _vp]),
@@ -312,11 +313,11 @@ def mcft_cache_prefetch(cache: Cache, layer, idx_pred, n_max, stream=None):
 
 
 def mcft_cache_prefetch_stats(cache: Cache, layer=-1, stream=None):
-    """(prefetched, useful) cumulative counts of one layer or of all layers (layer = -1)."""
-    p, u = C.c_uint64(), C.c_uint64()
+    """(prefetched, useful, bytes_moved) cumulative for one layer or all layers (layer = -1)."""
+    p, u, b = C.c_uint64(), C.c_uint64(), C.c_uint64()
     _check(lib().mcft_cache_prefetch_stats(C.c_void_p(cache.handle), layer, C.byref(p), C.byref(u),
-                                           _stream(stream)))
-    return p.value, u.value
+                                           C.byref(b), _stream(stream)))
+    return p.value, u.value, b.value
 
 
 def mcft_residual_rmsnorm(desc: LayerDesc, x, y=None, gamma=None, eps=1e-5, u=None, stream=None):

@@ -144,16 +144,16 @@ def run_and_compare(shape, L, T, steps, B, policy, n_prefetch, distinct, seed, b
                 ref_tot += (h, f, b)
                 assert M.mcft_cache_tags(cache, l) == ref_caches[l].tag, f"step {s} layer {l}"
             assert M.mcft_cache_stats(cache, -1) == tuple(int(v) for v in ref_tot)
-            assert M.mcft_cache_prefetch_stats(cache, -1) == (
+            assert M.mcft_cache_prefetch_stats(cache, -1)[:2] == (
                 sum(c.prefetched for c in ref_caches), sum(c.useful for c in ref_caches))
     assert compared_rows >= steps * T // 2, (compared_rows, diverged_tokens)
     if min_cache_steps is not None:
         assert cache_ok_until >= min_cache_steps, cache_ok_until
     if n_prefetch:
-        p, u = M.mcft_cache_prefetch_stats(cache, -1)
+        p, u, _ = M.mcft_cache_prefetch_stats(cache, -1)
         assert p > 0
     del stack
-    return M.mcft_cache_stats(cache, -1), M.mcft_cache_prefetch_stats(cache, -1)
+    return M.mcft_cache_stats(cache, -1), M.mcft_cache_prefetch_stats(cache, -1)[:2]
 
 
 @pytest.mark.parametrize("policy", ["LRU", "LFU", "FIFO"])

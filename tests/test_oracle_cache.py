@@ -191,6 +191,24 @@ def test_capped_prefetch_never_evicts_a_candidate(policy):
 
 
 @pytest.mark.parametrize("policy", C.POLICIES)
+def test_unused_prefetches_are_dropped(policy):
+    """After a step, none of the experts the preceding prefetch loaded and the step did not use is
+    cached, and the step's fetches are exactly its experts not cached after the drop."""
+    E, B = 10, 4
+    g = np.random.default_rng(21)
+    c = C.SlotCache(E, B, policy)
+    for s in range(300):
+        loads = c.prefetch(g.choice(E, size=int(g.integers(1, 6)), replace=False).tolist(),
+                           int(g.integers(1, B + 1)))
+        U = set(g.choice(E, size=2, replace=False).tolist())
+        unused = {e for e, _ in loads} - U
+        cached_after_drop = set(c.tag) - unused
+        h, f, b, _ = c.step(sorted(U))
+        assert not unused & set(c.tag)
+        assert h == len(U & cached_after_drop) and f == len(U - cached_after_drop)
+
+
+@pytest.mark.parametrize("policy", C.POLICIES)
 def test_batch1_fetch_identity(policy):
     """At batch 1 with K distinct experts per step: f = K - h every step, and over the stream
     Fetches/tok = L K (1 - HR) (Eq. metrics)."""
