@@ -496,7 +496,11 @@ def run_chain(shape, L, steps, warmup, seed, dev, policy="LRU", n_prefetch=0, gr
         S.capture()  # records one step; runs nothing
     h0, f0, _ = M.mcft_cache_stats(S.cache, -1)
     p0, u0, m0 = M.mcft_cache_prefetch_stats(S.cache, -1)
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(not graph)
     elapsed = time_steps(S.step, warmup, steps, S.compute)
+    M.mcft_profile_enable(False)
+    prof = M.mcft_profile_read()
     M.mcft_device_error()
     h1, f1, _ = M.mcft_cache_stats(S.cache, -1)
     p1, u1, m1 = M.mcft_cache_prefetch_stats(S.cache, -1)
@@ -515,6 +519,9 @@ def run_chain(shape, L, steps, warmup, seed, dev, policy="LRU", n_prefetch=0, gr
                hit_rate=(h1 - h0) / max(1, h1 - h0 + fetches),
                link_gb_per_token=moved / 1e9, link_bound_tpot_ms=moved / 210e9 * 1e3,
                host_pool="E distinct pinned blocks aliased by every layer")
+    if not graph:
+        res.update(kernel_ms_per_token={k: round(v[1] / steps, 4) for k, v in prof.items() if v[0]},
+                   launches_per_token={k: v[0] / steps for k, v in prof.items() if v[0]})
     del S
     torch.cuda.empty_cache()
     return res

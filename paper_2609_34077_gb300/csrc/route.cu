@@ -6,28 +6,33 @@
 // scores to the lower expert index. Gates come from p = softmax(z): renormalised over the active
 // set (Mixtral) or p_i itself (DeepSeek).
 //
-// Layout: 8 warps split d; each lane keeps one fp32 partial sum per expert; warps combine through
-// shared memory; warp 0 ranks (two experts per lane, shuffle arg-max) and writes idx / gate.
+// Layout: one CTA of 16 warps per token. The E x d router is split into tasks (expert, contraction
+// part): with E >= 16 each warp owns whole experts; with fewer experts each expert is split into up
+// to 16 / E parts so every warp has work. A lane loads its part's chunks of x and of the expert
+// row together, up to 8 chunks of 16 bytes in flight per lane and pass (one pass for d <= 4096 at
+// these expert counts), so a decode token's router (64 KB Mixtral, 256 KB DeepSeek) is read in
+// about one memory round trip instead of one per expert. Partial sums are reduced with shuffles
+// and added in shared memory in a fixed order; warp 0 ranks (two experts per lane, shuffle
+// arg-max) and writes idx / gate.
 #include "common.cuh"
 #include "internal.h"
 
 namespace mcft {
 namespace {
 
-constexpr int kWarps = 8;
+constexpr int kWarps = 16;
 
 template <typename TX>
 struct Chunk;  // 16 bytes of a row: 8 bf16 or 4 fp32
 template <>
 struct Chunk<__nv_bfloat16> {
   static constexpr int n = 8;
-  __device__ static void load(const void* p, float* f) { unpack8(ldg16(p), f); }
+  __device__ static void unpack(uint4 v, float* f) { unpack8(v, f); }
 };
 template <>
 struct Chunk<float> {
   static constexpr int n = 4;
-  __device__ static void load(const void* p, float* f) {
-    uint4 v = ldg16(p);
+  __device__ static void unpack(uint4 v, float* f) {
     f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
     f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
   }
@@ -43,49 +48,64 @@ __device__ __forceinline__ void warp_argmax(float& v, int& i) {
   }
 }
 
-template <typename TX, int MAXE>
+// Contraction parts per expert: the largest power of two p with E * p <= kWarps that divides the
+// row's chunk count (the same on host and device).
+__host__ __device__ inline int route_parts(int E, int nchunk) {
+  int p = 1;
+  while (2 * p * E <= kWarps && nchunk % (2 * p) == 0) p *= 2;
+  return p;
+}
+
+// NCH = 16-byte chunks a lane keeps in flight per task and pass (2, 4 or 8).
+template <typename TX, int NCH>
 __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constant__ RouteArgs a) {
-  __shared__ float part[kWarps][MAXE];
-  __shared__ float zs[MAXE];
+  __shared__ float part[kMaxE][kWarps];
+  __shared__ float zs[kMaxE];
   const int t = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E, d = a.d;
   using C = Chunk<TX>;
   const int nchunk = d / C::n;
-
-  float acc[MAXE];
-#pragma unroll
-  for (int e = 0; e < MAXE; ++e) acc[e] = 0.f;
+  const int parts = route_parts(E, nchunk);
+  const int per_part = nchunk / parts;
 
   const char* xrow = reinterpret_cast<const char*>(a.x) + size_t(t) * d * sizeof(TX);
   const char* wr = reinterpret_cast<const char*>(a.w_router);
   const size_t wrow = size_t(d) * sizeof(TX);
-  for (int c = warp * 32 + lane; c < nchunk; c += kWarps * 32) {
-    float xv[C::n];
-    C::load(xrow + size_t(c) * 16, xv);
+  for (int task = warp; task < E * parts; task += kWarps) {
+    const int e = task / parts, pt = task % parts;
+    const char* xp = xrow + size_t(pt) * per_part * 16;
+    const char* wp = wr + e * wrow + size_t(pt) * per_part * 16;
+    float acc = 0.f;
+    for (int base = 0; base < per_part; base += 32 * NCH) {
+      uint4 xv[NCH], wv[NCH];
 #pragma unroll
-    for (int e = 0; e < MAXE; ++e) {
-      if (e < E) {
-        float wv[C::n];
-        C::load(wr + e * wrow + size_t(c) * 16, wv);
+      for (int i = 0; i < NCH; ++i) {
+        const int c = base + i * 32 + lane;
+        if (c < per_part) {
+          xv[i] = ldg16(xp + size_t(c) * 16);
+          wv[i] = ldg16(wp + size_t(c) * 16);
+        }
+      }
 #pragma unroll
-        for (int j = 0; j < C::n; ++j) acc[e] = fmaf(xv[j], wv[j], acc[e]);
+      for (int i = 0; i < NCH; ++i) {
+        if (base + i * 32 + lane < per_part) {
+          float xf[C::n], wf[C::n];
+          C::unpack(xv[i], xf);
+          C::unpack(wv[i], wf);
+#pragma unroll
+          for (int j = 0; j < C::n; ++j) acc = fmaf(xf[j], wf[j], acc);
+        }
       }
     }
-  }
-#pragma unroll
-  for (int e = 0; e < MAXE; ++e) {
-    if (e < E) {
-      float v = warp_sum(acc[e]);
-      if (lane == 0) part[warp][e] = v;
-    }
+    acc = warp_sum(acc);
+    if (lane == 0) part[e][pt] = acc;
   }
   __syncthreads();
   if (warp != 0) return;
   for (int e = lane; e < E; e += 32) {
     float v = 0.f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) v += part[w][e];
+    for (int p = 0; p < parts; ++p) v += part[e][p];
     zs[e] = v;
   }
   __syncwarp();
@@ -161,12 +181,13 @@ __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constan
 
 template <typename TX>
 cudaError_t launch_typed(const RouteArgs& a, cudaStream_t s) {
+  const int nchunk = a.d / Chunk<TX>::n;
+  const int per_lane = (nchunk / route_parts(a.E, nchunk) + 31) / 32;  // chunks per lane and task
   dim3 grid(a.T), block(kWarps * 32);
   prof_begin(kProfRoute, s);
-  if (a.E <= 8) route_kernel<TX, 8><<<grid, block, 0, s>>>(a);
-  else if (a.E <= 16) route_kernel<TX, 16><<<grid, block, 0, s>>>(a);
-  else if (a.E <= 32) route_kernel<TX, 32><<<grid, block, 0, s>>>(a);
-  else route_kernel<TX, 64><<<grid, block, 0, s>>>(a);
+  if (per_lane <= 2) route_kernel<TX, 2><<<grid, block, 0, s>>>(a);
+  else if (per_lane <= 4) route_kernel<TX, 4><<<grid, block, 0, s>>>(a);
+  else route_kernel<TX, 8><<<grid, block, 0, s>>>(a);  // longer rows take several passes
   prof_end(kProfRoute, s);
   return cudaGetLastError();
 }
