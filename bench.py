@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "a9fca224659abaa5", 1.0017,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c22f1524ed6121c4", 1.0023,
                      "profiles/ffn_decode_mixtral_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "a9fca224659abaa5", 1.0032,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c22f1524ed6121c4", 1.0047,
                     "profiles/ffn_decode_mixtral_decode.md"),
-    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "31f4483ef0759b6d", 1.0002,
+    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "5dbac2ee4a52025b", 0.9558,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
 }
 
@@ -654,11 +654,15 @@ def profile_case(case: str, dev) -> int:
     desc = M.desc_of(sh)
     if case == "fetch16":  # decode steps with the cache and the device-driven fetch
         L = DecodeLayer(sh, 16, 7, dev)
+        per_step = []
         for s in range(3):
+            before = M.mcft_cache_stats(L.cache, 0)[1]
             L.step(s, path="device")
+            torch.cuda.synchronize()
+            per_step.append(M.mcft_cache_stats(L.cache, 0)[1] - before)
         M.mcft_device_error()
-        torch.cuda.synchronize()
-        print(json.dumps({"case": case, "fetches": M.mcft_cache_stats(L.cache, 0)[1]}))
+        print(json.dumps({"case": case, "fetches_per_step": per_step,
+                          "fetch_bytes_per_step": [n * sh.expert_bytes for n in per_step]}))
         return 0
     if case == "prefill":
         T, mode = 4096, M.MCFT_ROUTE_HARD_MASK

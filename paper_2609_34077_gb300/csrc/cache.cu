@@ -46,6 +46,7 @@ __device__ __forceinline__ bool victim_before(int policy, int s, int v, const in
 }
 
 __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ CacheStepArgs a) {
+  pdl_wait();
   __shared__ int32_t s_tag[kMaxE];
   __shared__ int64_t s_last[kMaxE], s_ins[kMaxE], s_freq[kMaxE];
   __shared__ int32_t s_out[1 + 3 * kMaxE];  // n_miss, miss experts, miss locations, loc_of
@@ -186,6 +187,7 @@ __global__ void __launch_bounds__(32) cache_step_kernel(const __grid_constant__ 
 // Prefetch decision (one warp). The lanes count how many predicted (token, k) entries name each
 // expert; lane 0 ranks, touches, claims slots and writes the fetch list.
 __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ PrefetchArgs a) {
+  pdl_wait();
   __shared__ int cnt[kMaxE], rank[kMaxE];
   __shared__ int32_t s_tag[kMaxE];
   __shared__ int64_t s_last[kMaxE], s_ins[kMaxE], s_freq[kMaxE];
@@ -299,6 +301,7 @@ __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ Pr
 // Copy the missed experts' blocks host -> device with 16-byte loads over the host link. Work
 // units are 64 KB pieces of the missed blocks, spread over the grid.
 __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ FetchArgs a) {
+  pdl_wait();
   const int n = a.miss[0];
   const size_t words = a.bytes / 16, piece = 4096;
   const size_t per = (words + piece - 1) / piece;
@@ -342,16 +345,16 @@ cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool pr
 
 cudaError_t launch_prefetch(const PrefetchArgs& a, cudaStream_t s) {
   prof_begin(kProfPrefetch, s);
-  prefetch_kernel<<<1, 32, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(prefetch_kernel, dim3(1), dim3(32), 0, s, a);
   prof_end(kProfPrefetch, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_cache_step(const CacheStepArgs& a, cudaStream_t s) {
   prof_begin(kProfCache, s);
-  cache_step_kernel<<<1, 32, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(cache_step_kernel, dim3(1), dim3(32), 0, s, a);
   prof_end(kProfCache, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace mcft

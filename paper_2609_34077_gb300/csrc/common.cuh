@@ -26,6 +26,12 @@ struct alignas(16) V16 {
   uint4 u;
 };
 
+// Programmatic dependent launch: a kernel launched with programmatic stream serialization may
+// start while the previous kernel of its stream is still finishing; this wait returns once that
+// kernel has completed and its memory operations are visible. Every kernel of the library calls
+// it before its first global memory access (a no-op for kernels launched without the attribute).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ uint4 ldg16(const void* p) {
   return __ldg(reinterpret_cast<const uint4*>(p));
 }

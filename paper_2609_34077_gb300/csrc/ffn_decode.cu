@@ -294,6 +294,7 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
 
 __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_constant__ FfnArgs a,
                                                                int RB) {
+  pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
   const int KS = kWarps / RB;
@@ -315,6 +316,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
 
 __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_constant__ FfnArgs a,
                                                               int RB) {
+  pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
   const int KS = kWarps / RB;
@@ -363,15 +365,15 @@ cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int
   cudaError_t e = cudaSuccess;
   if (stages & 1) {
     prof_begin(kProfDec13, s);
-    dec13_kernel<<<num_sms * nb13, kWarps * 32, 0, s>>>(a, rb13);
+    e = launch_pdl(dec13_kernel, dim3(num_sms * nb13), dim3(kWarps * 32), 0, s, a, rb13);
     prof_end(kProfDec13, s);
-    e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaGetLastError();
   }
   if (e != cudaSuccess || !(stages & 2)) return e;
   prof_begin(kProfDec2, s);
-  dec2_kernel<<<num_sms * nb2, kWarps * 32, 0, s>>>(a, rb2);
+  e = launch_pdl(dec2_kernel, dim3(num_sms * nb2), dim3(kWarps * 32), 0, s, a, rb2);
   prof_end(kProfDec2, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace mcft

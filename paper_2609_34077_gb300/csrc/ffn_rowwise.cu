@@ -195,6 +195,7 @@ __device__ __forceinline__ void ffn2_tile(const FfnArgs& a, const char* blk, con
 
 template <typename TW>
 __global__ void __launch_bounds__(kWarps * 32) ffn13_kernel(const __grid_constant__ FfnArgs a) {
+  pdl_wait();
   __shared__ Items it;
   build_items(it, a, a.w);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -219,6 +220,7 @@ __global__ void __launch_bounds__(kWarps * 32) ffn13_kernel(const __grid_constan
 
 template <typename TW>
 __global__ void __launch_bounds__(kWarps * 32) ffn2_kernel(const __grid_constant__ FfnArgs a) {
+  pdl_wait();
   __shared__ Items it;
   build_items(it, a, a.d);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -250,6 +252,7 @@ __device__ __forceinline__ float4 row_sum(const CombineArgs& a, size_t at) {
 
 template <typename TY>
 __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineArgs a) {
+  pdl_wait();
   if (a.hdr->abort) return;
   const int nq = a.d / 4;  // float4 columns per row
   const size_t total = size_t(a.T) * nq;
@@ -289,15 +292,15 @@ cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s, 
   cudaError_t e = cudaSuccess;
   if (stages & 1) {
     prof_begin(kProfFfn13, s);
-    ffn13_kernel<TW><<<num_sms * nb13, kWarps * 32, 0, s>>>(a);
+    e = launch_pdl(ffn13_kernel<TW>, dim3(num_sms * nb13), dim3(kWarps * 32), 0, s, a);
     prof_end(kProfFfn13, s);
-    e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaGetLastError();
   }
   if (e != cudaSuccess || !(stages & 2)) return e;
   prof_begin(kProfFfn2, s);
-  ffn2_kernel<TW><<<num_sms * nb2, kWarps * 32, 0, s>>>(a);
+  e = launch_pdl(ffn2_kernel<TW>, dim3(num_sms * nb2), dim3(kWarps * 32), 0, s, a);
   prof_end(kProfFfn2, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace
@@ -313,10 +316,11 @@ cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s) {
   size_t blocks = (total + 255) / 256;
   if (blocks > 4096) blocks = 4096;
   prof_begin(kProfCombine, s);
-  if (dtype == MCFT_BF16) combine_kernel<uint16_t><<<unsigned(blocks), 256, 0, s>>>(a);
-  else combine_kernel<float><<<unsigned(blocks), 256, 0, s>>>(a);
+  const cudaError_t e = dtype == MCFT_BF16
+      ? launch_pdl(combine_kernel<uint16_t>, dim3(unsigned(blocks)), dim3(256), 0, s, a)
+      : launch_pdl(combine_kernel<float>, dim3(unsigned(blocks)), dim3(256), 0, s, a);
   prof_end(kProfCombine, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace mcft

@@ -211,6 +211,7 @@ __device__ __forceinline__ int seg_of_row(const SmemCtl* c, int row) {
 
 template <int EPI, int LR>
 __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;

@@ -38,6 +38,7 @@ struct In16<float> {
 // T: dtype of the input rows and of the adapter (the layer dtype); R: outputs per row (2r or r).
 template <typename T, int R>
 __global__ void __launch_bounds__(kWarps * 32) lora_down_kernel(const __grid_constant__ LoraDownArgs a) {
+  pdl_wait();
   __shared__ int s_off[kMaxSeg + 1];
   __shared__ int s_nseg;
   if (threadIdx.x == 0) s_nseg = a.hdr->abort == 0 ? a.nseg : 0;

@@ -19,6 +19,7 @@ namespace mcft {
 namespace {
 
 __global__ void __launch_bounds__(32) mask_sample_kernel(const __grid_constant__ MaskSampleArgs a) {
+  pdl_wait();
   const int l = blockIdx.x, lane = threadIdx.x, E = a.E;
   const float* mt = a.m_tilde + size_t(l) * E;
   const float* u = a.uniforms + size_t(l) * E;
@@ -88,6 +89,7 @@ __global__ void __launch_bounds__(32) mask_sample_kernel(const __grid_constant__
 
 template <typename TY>
 __global__ void __launch_bounds__(256) gate_grad_kernel(const __grid_constant__ GateGradArgs a) {
+  pdl_wait();
   if (a.hdr->abort) return;
   const int lane = threadIdx.x & 31;
   const int n = a.T * a.K;
@@ -122,6 +124,7 @@ __global__ void __launch_bounds__(256) gate_grad_kernel(const __grid_constant__ 
 }
 
 __global__ void __launch_bounds__(256) mask_grad_kernel(const __grid_constant__ MaskGradArgs a) {
+  pdl_wait();
   __shared__ float part[256];
   const int e = blockIdx.x, tid = threadIdx.x;
   const int n = a.T * a.K;
@@ -149,6 +152,7 @@ __global__ void __launch_bounds__(256) mask_grad_kernel(const __grid_constant__ 
 }
 
 __global__ void __launch_bounds__(32) mask_tilde_kernel(const __grid_constant__ MaskGradArgs a) {
+  pdl_wait();
   const int lane = threadIdx.x, E = a.E;
   float s = 0.f;
   for (int e = lane; e < E; e += 32) s += a.pi[e] * a.dm[e];

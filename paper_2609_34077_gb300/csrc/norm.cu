@@ -34,6 +34,7 @@ __device__ __forceinline__ void store4(void* p, size_t i, float4 v) {
 
 template <typename T>
 __global__ void __launch_bounds__(256) resid_norm_kernel(const __grid_constant__ NormArgs a) {
+  pdl_wait();
   __shared__ float part[8];
   const size_t row = size_t(blockIdx.x) * a.d;
   float* x = a.x + row;
@@ -69,10 +70,11 @@ __global__ void __launch_bounds__(256) resid_norm_kernel(const __grid_constant__
 
 cudaError_t launch_resid_norm(const NormArgs& a, int dtype, cudaStream_t s) {
   prof_begin(kProfNorm, s);
-  if (dtype == MCFT_BF16) resid_norm_kernel<uint16_t><<<a.T, 256, 0, s>>>(a);
-  else resid_norm_kernel<float><<<a.T, 256, 0, s>>>(a);
+  const cudaError_t e = dtype == MCFT_BF16
+      ? launch_pdl(resid_norm_kernel<uint16_t>, dim3(a.T), dim3(256), 0, s, a)
+      : launch_pdl(resid_norm_kernel<float>, dim3(a.T), dim3(256), 0, s, a);
   prof_end(kProfNorm, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace mcft

@@ -11,6 +11,7 @@ namespace {
 constexpr int kThreads = 1024;
 
 __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant__ PermuteArgs a) {
+  pdl_wait();
   __shared__ int hist[kMaxSeg];
   __shared__ int run[kMaxE];
   __shared__ int offs[kMaxSeg + 1];
@@ -89,6 +90,7 @@ __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant
 
 // xp[r, :] = x[perm[r], :] (bf16), zero rows for padding.
 __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ GatherArgs a) {
+  pdl_wait();
   if (a.hdr->abort) return;
   const int mrows = a.hdr->mrows;
   const int nch = a.d / 8;  // 16-byte chunks per row
@@ -109,17 +111,17 @@ __global__ void __launch_bounds__(256) gather_kernel(const __grid_constant__ Gat
 
 cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s) {
   prof_begin(kProfPermute, s);
-  permute_kernel<<<1, kThreads, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(permute_kernel, dim3(1), dim3(kThreads), 0, s, a);
   prof_end(kProfPermute, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t launch_gather(const GatherArgs& a, cudaStream_t s) {
   const int grid = a.mcap < 4096 ? (a.mcap > 0 ? a.mcap : 1) : 4096;
   prof_begin(kProfGather, s);
-  gather_kernel<<<grid, 256, 0, s>>>(a);
+  const cudaError_t e = launch_pdl(gather_kernel, dim3(grid), dim3(256), 0, s, a);
   prof_end(kProfGather, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace mcft

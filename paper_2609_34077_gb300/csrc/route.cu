@@ -59,6 +59,7 @@ __host__ __device__ inline int route_parts(int E, int nchunk) {
 // NCH = 16-byte chunks a lane keeps in flight per task and pass (2, 4 or 8).
 template <typename TX, int NCH>
 __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constant__ RouteArgs a) {
+  pdl_wait();
   __shared__ float part[kMaxE][kWarps];
   __shared__ float zs[kMaxE];
   const int t = blockIdx.x;
@@ -185,11 +186,12 @@ cudaError_t launch_typed(const RouteArgs& a, cudaStream_t s) {
   const int per_lane = (nchunk / route_parts(a.E, nchunk) + 31) / 32;  // chunks per lane and task
   dim3 grid(a.T), block(kWarps * 32);
   prof_begin(kProfRoute, s);
-  if (per_lane <= 2) route_kernel<TX, 2><<<grid, block, 0, s>>>(a);
-  else if (per_lane <= 4) route_kernel<TX, 4><<<grid, block, 0, s>>>(a);
-  else route_kernel<TX, 8><<<grid, block, 0, s>>>(a);  // longer rows take several passes
+  const cudaError_t e =
+      per_lane <= 2   ? launch_pdl(route_kernel<TX, 2>, grid, block, 0, s, a)
+      : per_lane <= 4 ? launch_pdl(route_kernel<TX, 4>, grid, block, 0, s, a)
+                      : launch_pdl(route_kernel<TX, 8>, grid, block, 0, s, a);  // long rows: passes
   prof_end(kProfRoute, s);
-  return cudaGetLastError();
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace
