@@ -786,6 +786,19 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
                                     const void* const* shared, void* y, void* workspace,
                                     size_t ws_bytes, mcft_stream_t compute_stream,
                                     mcft_stream_t copy_stream) {
+  return mcft::forward_cached_impl(desc, x, T, idx, gate, c, layer, shared, y, workspace, ws_bytes,
+                                   compute_stream, copy_stream, false);
+}
+
+}  // extern "C"
+
+namespace mcft {
+
+mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int T,
+                                const int32_t* idx, const float* gate, mcft_cache* c, int layer,
+                                const void* const* shared, void* y, void* workspace,
+                                size_t ws_bytes, cudaStream_t compute_stream,
+                                cudaStream_t copy_stream, bool permuted) {
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (!c) return fail(MCFT_ERR_INVALID, "cache is NULL");
@@ -841,10 +854,13 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
   // 1b. prefetches decided for later layers stream in behind this layer's misses
   st = enqueue_prefetch_fetches(c, copy_stream);
   if (st != MCFT_OK) return st;
-  // 2. meanwhile: permutation and the experts that were hits (and the shared experts)
-  PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
-  e = launch_permute(pa, compute_stream);
-  if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
+  // 2. meanwhile: permutation (unless the fused prologue wrote it into this workspace) and the
+  //    experts that were hits (and the shared experts)
+  if (!permuted) {
+    PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
+    e = launch_permute(pa, compute_stream);
+    if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
+  }
   FfnArgs fa{};
   fa.x = x;
   fa.off = off;
@@ -875,6 +891,89 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
   if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
   return MCFT_OK;
 }
+
+mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y, const void* gamma,
+                           const void* gamma_next, float eps, void* u, const void* w_router,
+                           const float* prior, int32_t* idx, float* gate, const void* w_router_next,
+                           const float* prior_next, int32_t* pred, float* gate_pred,
+                           mcft_cache* c, int layer, int n_prefetch, void* workspace,
+                           size_t ws_bytes, cudaStream_t stream) {
+  const int E = desc->E, K = desc->K, S = desc->n_shared;
+  if (!prologue_supported(desc->d, E, 1) || K > kMaxK)
+    return fail(MCFT_ERR_UNSUPPORTED, "the fused prologue serves one token with d <= 4096, K <= 8");
+  if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
+  const bool do_pred = gamma_next != nullptr;
+  const bool do_pf = do_pred && n_prefetch > 0 && layer + 1 < c->L;
+  if (do_pf && (n_prefetch > c->B || (c->d_slots && !c->device_fetch)))
+    return fail(MCFT_ERR_INVALID, "bad prefetch settings");
+  const WsLayout L = ws_layout(desc->d, E, K, desc->w, S, desc->dtype, 1);
+  if (ws_bytes < L.total) return fail(MCFT_ERR_INVALID, "workspace too small");
+  if (do_pf) {
+    if (c->pf_state[layer + 1] == 1)
+      return fail(MCFT_ERR_INVALID, "the previous prefetch of layer %d was never fetched", layer + 1);
+    if (c->pf_state[layer + 1] == 2) {
+      MCFT_CUDA(cudaStreamWaitEvent(stream, c->ev_pf_done[layer + 1], 0));
+      c->pf_state[layer + 1] = 0;
+    }
+  }
+  unsigned* err = device_error_word();
+  PrologueArgs a{};
+  a.x = x;
+  a.y = y;
+  a.gamma = gamma;
+  a.gamma_next = gamma_next;
+  a.u = u;
+  a.eps = eps;
+  a.d = desc->d;
+  auto route_args = [&](RouteArgs& r, const void* w, const float* pri, int32_t* out, float* g) {
+    r.x = u;
+    r.w_router = w;
+    r.T = 1;
+    r.d = desc->d;
+    r.E = E;
+    r.K = K;
+    r.mode = MCFT_ROUTE_SOFT_PRIOR;
+    r.gate_mode = desc->gate;
+    for (int e = 0; e < E; ++e) r.prior[e] = pri[e];
+    r.idx = out;
+    r.gate = g;
+    r.err = err;
+  };
+  route_args(a.route, w_router, prior, idx, gate);
+  if (do_pred) route_args(a.pred, w_router_next, prior_next, pred, gate_pred);
+  a.cache = CacheStepArgs{idx, K, E, c->B, layer, c->policy, c->d_tag, c->d_last, c->d_ins,
+                          c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
+                          c->d_miss + size_t(layer) * c->miss_stride,
+                          c->d_miss_dev + size_t(layer) * c->miss_stride,
+                          c->d_ptr_tab + size_t(layer) * E, c->d_ready + layer,
+                          c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
+                          c->d_staging, c->expert_bytes, err};
+  a.do_prefetch = do_pf ? 1 : 0;
+  if (do_pf) {
+    const int l1 = layer + 1;
+    a.prefetch = PrefetchArgs{pred, K, K, n_prefetch, E, c->B, l1, c->policy, c->d_tag, c->d_last,
+                              c->d_ins, c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
+                              c->d_pf_list + size_t(l1) * (1 + E), c->d_pf_tab + size_t(l1) * E,
+                              c->d_slots ? c->d_slots + size_t(l1) * c->B * c->expert_bytes : nullptr,
+                              c->expert_bytes, err};
+  }
+  char* ws = static_cast<char*>(workspace);
+  a.perm = PermuteArgs{idx, 1, K, E, S, L.pad, L.mcap, reinterpret_cast<WsHeader*>(ws + L.hdr),
+                       reinterpret_cast<int*>(ws + L.cnt), reinterpret_cast<int*>(ws + L.off),
+                       reinterpret_cast<int*>(ws + L.pos), reinterpret_cast<int*>(ws + L.perm), err};
+  cudaError_t e = launch_prologue(a, desc->dtype, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "prologue kernel launch");
+  MCFT_CUDA(cudaEventRecord(c->ev_step[layer], stream));
+  if (do_pf && c->d_slots) {
+    MCFT_CUDA(cudaEventRecord(c->ev_pf_step[layer + 1], stream));
+    c->pf_state[layer + 1] = 1;
+  }
+  return MCFT_OK;
+}
+
+}  // namespace mcft
+
+extern "C" {
 
 mcft_status mcft_cache_last_misses(const mcft_cache* c, int layer, int* n_out, int32_t* experts,
                                    int32_t* slots) {

@@ -263,6 +263,27 @@ struct FetchArgs {
 };
 cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch = false);
 
+// Fused decode prologue of one chained-stack layer at batch 1 (prologue.cu): residual update and
+// RMSNorm, routing of layer l, cache step of layer l, prediction and prefetch event of layer l+1,
+// permutation, in one launch of an 8-CTA cluster.
+struct PrologueArgs {
+  float* x;                // [1, d] fp32 stream (updated when y is given)
+  const void* y;           // [1, d] previous layer's output (layer dtype) or NULL
+  const void* gamma;       // [d] this layer's RMSNorm scale
+  const void* gamma_next;  // [d] the next layer's (prediction), NULL: no prediction
+  void* u;                 // [1, d] out: this layer's normalised input
+  float eps;
+  int d;
+  RouteArgs route;         // this layer (route.x unused)
+  RouteArgs pred;          // the next layer's prediction (when gamma_next is given)
+  CacheStepArgs cache;     // this layer's step (cache.idx = route.idx)
+  int do_prefetch;
+  PrefetchArgs prefetch;   // the next layer's prefetch event (prefetch.idx = pred.idx)
+  PermuteArgs perm;        // this layer's permutation (perm.idx = route.idx, T = 1)
+};
+bool prologue_supported(int d, int E, int T);
+cudaError_t launch_prologue(const PrologueArgs& a, int dtype, cudaStream_t s);
+
 // Residual update and RMSNorm of the stream entering a MoE block (norm.cu): x += y (when y is
 // given), then u = gamma * x / sqrt(mean(x^2) + eps) (when gamma is given). One CTA per row.
 struct NormArgs {
@@ -311,10 +332,29 @@ cudaError_t launch_mask_grad(const MaskGradArgs& a, cudaStream_t s);
 unsigned* device_error_word();  // device address of the current device's error word
 mcft_status set_error_message(mcft_status st, const char* msg);  // mcft_last_error() text
 
+// The device-driven cached forward (mcft_moe_forward_cached); permuted = the workspace already
+// holds this call's permutation (written by the fused prologue), so it is not recomputed.
+mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int T,
+                                const int32_t* idx, const float* gate, mcft_cache* c, int layer,
+                                const void* const* shared, void* y, void* workspace,
+                                size_t ws_bytes, cudaStream_t compute_stream,
+                                cudaStream_t copy_stream, bool permuted);
+
+// One fused prologue launch for layer `layer` of a chained stack at batch 1 (prologue.cu): the
+// stream update and norm, routing, the cache step, the next layer's prediction and prefetch event
+// (when gamma_next is given and n_prefetch > 0), the permutation into `workspace`. Records the
+// cache step's (and the prefetch's) events as mcft_cache_step / mcft_cache_prefetch do.
+mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y, const void* gamma,
+                           const void* gamma_next, float eps, void* u, const void* w_router,
+                           const float* prior, int32_t* idx, float* gate, const void* w_router_next,
+                           const float* prior_next, int32_t* pred, float* gate_pred,
+                           mcft_cache* c, int layer, int n_prefetch, void* workspace,
+                           size_t ws_bytes, cudaStream_t stream);
+
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
        kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfNorm,
-       kProfPrefetch, kProfPfFetch, kProfCount };
+       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

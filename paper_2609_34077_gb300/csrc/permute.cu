@@ -37,17 +37,40 @@ __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant
     }
     return;
   }
-  if (tid == 0) {
-    offs[0] = 0;
-    for (int s = 0; s < nseg; ++s) {
-      const int len = s < a.E ? hist[s] : a.T;
-      a.cnt[s] = len;
-      offs[s + 1] = offs[s] + (len + a.pad - 1) / a.pad * a.pad;
+  // padded exclusive scan of the segment sizes: warp 0, three segments per lane (kMaxSeg <= 96)
+  if (warp == 0) {
+    int len[3], padded[3], sum = 0;
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+      const int sg = lane * 3 + j;
+      len[j] = sg < nseg ? (sg < a.E ? hist[sg] : a.T) : 0;
+      padded[j] = (len[j] + a.pad - 1) / a.pad * a.pad;
+      sum += padded[j];
     }
-    for (int s = 0; s <= nseg; ++s) a.off[s] = offs[s];
-    a.hdr->abort = 0;
-    a.hdr->nseg = nseg;
-    a.hdr->mrows = offs[nseg];
+    int incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    int excl = incl - sum;
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+      const int sg = lane * 3 + j;
+      if (sg < nseg) {
+        offs[sg] = excl;
+        a.off[sg] = excl;
+        a.cnt[sg] = len[j];
+      }
+      excl += padded[j];
+    }
+    if (lane == 31) {
+      offs[nseg] = incl;
+      a.off[nseg] = incl;
+      a.hdr->abort = 0;
+      a.hdr->nseg = nseg;
+      a.hdr->mrows = incl;
+    }
   }
   __syncthreads();
 
@@ -77,14 +100,20 @@ __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant
     }
     __syncthreads();
   }
-  // padding rows of routed segments; shared segments list every token in order
-  for (int s = 0; s < nseg; ++s) {
-    const int len = s < a.E ? hist[s] : a.T;
-    const int r0 = offs[s];
-    for (int r = tid; r < offs[s + 1] - r0; r += kThreads) {
-      if (s >= a.E && r < len) a.perm[r0 + r] = r;
-      else if (r >= len) a.perm[r0 + r] = -1;
+  // padding rows of routed segments; shared segments list every token in order. One thread per
+  // row; its segment is found by binary search on the offsets.
+  const int mrows = offs[nseg];
+  for (int r = tid; r < mrows; r += kThreads) {
+    int lo = 0, hi = nseg;  // largest segment with offs[seg] <= r
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (offs[mid] <= r) lo = mid;
+      else hi = mid;
     }
+    const int len = lo < a.E ? hist[lo] : a.T;
+    const int local = r - offs[lo];
+    if (lo >= a.E && local < len) a.perm[r] = local;
+    else if (local >= len) a.perm[r] = -1;
   }
 }
 

@@ -12,6 +12,9 @@
 //     prefetch event of layer l+1 (its loads stream in behind layer l's misses)
 //   y_l = layer l on u_l with its cached experts (fetch overlapped with the hits' compute)
 //   x_{l+1} = x_l + y_l;  u_{l+1} = RMSNorm_{l+1}(x_{l+1})
+// At batch 1 each layer's steps before its expert FFN run as one fused prologue launch (an 8-CTA
+// cluster, prologue.cu) and the forward skips its permutation; larger batches use the separate
+// kernels above. Both make the same decisions.
 #include <cuda_runtime.h>
 #include <string.h>
 
@@ -125,7 +128,34 @@ mcft_status mcft_stack_step(mcft_stack* s, float* x, int T, mcft_stream_t comput
   const mcft_layer_desc* desc = &s->desc;
   const int L = s->L, E = desc->E, S = desc->n_shared, K = desc->K;
   const size_t plane = size_t(s->T_max) * K;
-  mcft_status st = mcft_residual_rmsnorm(desc, x, nullptr, T, s->gammas[0], s->eps, s->u, compute);
+  mcft_status st;
+  if (T == 1 && K <= mcft::kMaxK && mcft::prologue_supported(desc->d, E, T)) {
+    // batch 1: one fused prologue launch per layer (stream update, norm, routing, cache step,
+    // prediction and prefetch of the next layer, permutation), then the forward without its
+    // permutation; the last layer's output is added by a final residual update
+    for (int l = 0; l < L; ++l) {
+      int32_t* idx = s->idx + l * plane;
+      float* gate = s->gate + l * plane;
+      const bool pf = s->n_prefetch > 0 && l + 1 < L;
+      st = mcft::stack_prologue(desc, x, l == 0 ? nullptr : s->y, s->gammas[l],
+                                pf ? s->gammas[l + 1] : nullptr, s->eps, s->u, s->routers[l],
+                                s->priors.data() + size_t(l) * E, idx, gate,
+                                pf ? s->routers[l + 1] : nullptr,
+                                pf ? s->priors.data() + size_t(l + 1) * E : nullptr,
+                                pf ? s->pred + (l + 1) * plane : nullptr, s->gate_pred, s->cache, l,
+                                s->n_prefetch, s->ws, s->ws_bytes, compute);
+      if (st != MCFT_OK) return st;
+      st = mcft::forward_cached_impl(desc, s->u, T, idx, gate, s->cache, l,
+                                     S > 0 ? s->shared.data() + size_t(l) * S : nullptr, s->y,
+                                     s->ws, s->ws_bytes, compute, copy, true);
+      if (st != MCFT_OK) return st;
+    }
+    st = mcft_residual_rmsnorm(desc, x, s->y, T, nullptr, s->eps, nullptr, compute);
+    if (st != MCFT_OK) return st;
+    s->last_T = T;
+    return MCFT_OK;
+  }
+  st = mcft_residual_rmsnorm(desc, x, nullptr, T, s->gammas[0], s->eps, s->u, compute);
   if (st != MCFT_OK) return st;
   for (int l = 0; l < L; ++l) {
     int32_t* idx = s->idx + l * plane;

@@ -156,33 +156,40 @@ def run_and_compare(shape, L, T, steps, B, policy, n_prefetch, distinct, seed, b
     return M.mcft_cache_stats(cache, -1), M.mcft_cache_prefetch_stats(cache, -1)[:2]
 
 
+# T = 1 runs the fused per-layer prologue (one cluster launch: norm, routing, cache step,
+# prediction and prefetch, permutation); T > 1 the separate kernels.
+@pytest.mark.parametrize("T", [1, 4])
 @pytest.mark.parametrize("policy", ["LRU", "LFU", "FIFO"])
 @pytest.mark.parametrize("n_prefetch", [0, 2])
-def test_chain_fp32_tiny_exact(policy, n_prefetch):
-    run_and_compare(I.TINY, L=8, T=4, steps=12, B=4, policy=policy, n_prefetch=n_prefetch,
+def test_chain_fp32_tiny_exact(policy, n_prefetch, T):
+    run_and_compare(I.TINY, L=8, T=T, steps=12, B=4, policy=policy, n_prefetch=n_prefetch,
                     distinct=True, seed=60, band=1e-4, gate_atol=1e-5, tol=1e-4, min_cache_steps=6)
 
 
+@pytest.mark.parametrize("T", [1, 2])
 @pytest.mark.parametrize("n_prefetch", [0, 2])
-def test_chain_mixtral_8_layers_bf16(n_prefetch):
-    run_and_compare(I.MIXTRAL, L=8, T=2, steps=4, B=4, policy="LRU", n_prefetch=n_prefetch,
+def test_chain_mixtral_8_layers_bf16(n_prefetch, T):
+    run_and_compare(I.MIXTRAL, L=8, T=T, steps=4, B=4, policy="LRU", n_prefetch=n_prefetch,
                     distinct=False, seed=61, band=0.1, gate_atol=0.025, tol=2.5e-2)
 
 
-def test_chain_mixtral_32_layers_bf16():
-    run_and_compare(I.MIXTRAL, L=32, T=2, steps=3, B=4, policy="LFU", n_prefetch=2,
+@pytest.mark.parametrize("T", [1, 2])
+def test_chain_mixtral_32_layers_bf16(T):
+    run_and_compare(I.MIXTRAL, L=32, T=T, steps=3, B=4, policy="LFU", n_prefetch=2,
                     distinct=False, seed=61, band=0.15, gate_atol=0.05, tol=5e-2)
 
 
+@pytest.mark.parametrize("T", [1, 2])
 @pytest.mark.parametrize("n_prefetch", [0, 6])
-def test_chain_deepseek_26_layers_bf16(n_prefetch):
-    run_and_compare(I.DSV2_LITE, L=26, T=2, steps=4, B=12, policy="LFU", n_prefetch=n_prefetch,
+def test_chain_deepseek_26_layers_bf16(n_prefetch, T):
+    run_and_compare(I.DSV2_LITE, L=26, T=T, steps=4, B=12, policy="LFU", n_prefetch=n_prefetch,
                     distinct=False, seed=62, band=0.03, gate_atol=2e-3, tol=1e-2)
 
 
-def test_prefetch_does_not_change_the_stream():
+@pytest.mark.parametrize("T", [1, 3])
+def test_prefetch_does_not_change_the_stream(T):
     """The stack's output does not depend on prefetching (only where the bytes come from)."""
-    shape, L, T = I.TINY, 4, 3
+    shape, L = I.TINY, 4
     outs = []
     for n_prefetch in (0, 2):
         st = _stack(shape, L, 63, True)
