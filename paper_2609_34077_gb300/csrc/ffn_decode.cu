@@ -123,6 +123,33 @@ __device__ __forceinline__ uint32_t word(const uint4& lo, const uint4& hi, int i
   }
 }
 
+// Walk chunks [c0, c1): load(buf, ch) issues a chunk's weight loads, compute(buf, ch) consumes
+// them. With DB the next chunk's loads are issued before the current chunk's MMAs (two register
+// buffers, unrolled by two so nothing is copied), so a warp keeps one chunk in flight while it
+// computes; without DB each chunk is loaded, then consumed (token groups of more than 8, and any
+// group in the kernel compiled for 32-token passes, whose accumulators need the registers).
+template <bool DB, typename Load, typename Compute>
+__device__ __forceinline__ void stream_chunks(int c0, int c1, Load&& load, Compute&& compute) {
+  uint4 va[8];
+  if constexpr (DB) {
+    uint4 vb[8];
+    if (c0 < c1) load(va, c0);
+    int ch = c0;
+    for (; ch + 1 < c1; ch += 2) {
+      load(vb, ch + 1);
+      compute(va, ch);
+      if (ch + 2 < c1) load(va, ch + 2);
+      compute(vb, ch + 1);
+    }
+    if (ch < c1) compute(va, ch);
+  } else {
+    for (int ch = c0; ch < c1; ++ch) {
+      load(va, ch);
+      compute(va, ch);
+    }
+  }
+}
+
 // Chunks [c0, c1) of this warp's slice of a contraction of nch chunks.
 __device__ __forceinline__ void warp_slice(int nch, int parts, int part, int& c0, int& c1) {
   const int per = (nch + parts - 1) / parts;
@@ -133,7 +160,7 @@ __device__ __forceinline__ void warp_slice(int nch, int parts, int part, int& c0
 // GEMM13 + SwiGLU for RB blocks of 16 rows starting at r0 and n <= 32 tokens of one segment
 // starting at permuted row q0; warp w owns row block w / KS and contraction slice w % KS.
 // red: shared scratch [kWarps][kMaxNG][8][32] floats.
-template <int NG>
+template <int NG, bool DB>
 __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, const void* lblk,
                                            int r0, int q0, int n, int RB, int KS, float* red) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -159,25 +186,30 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
 
   int c0, c1;
   warp_slice(int(rowb / (kChunk * 2)), KS, warp % KS, c0, c1);
-  for (int ch = c0; ch < c1; ++ch) {
+  // one chunk's weights: W1 rows g / g+8 (lo, hi halves), then W3's
+  auto load = [&](uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
-    const uint4 ag0 = ld_stream16(w1g + k), ag1 = ld_stream16(w1g + k + 64);
-    const uint4 ah0 = ld_stream16(w1h + k), ah1 = ld_stream16(w1h + k + 64);
-    const uint4 bg0 = ld_stream16(w3g + k), bg1 = ld_stream16(w3g + k + 64);
-    const uint4 bh0 = ld_stream16(w3h + k), bh1 = ld_stream16(w3h + k + 64);
+    v[0] = ld_stream16(w1g + k); v[1] = ld_stream16(w1g + k + 64);
+    v[2] = ld_stream16(w1h + k); v[3] = ld_stream16(w1h + k + 64);
+    v[4] = ld_stream16(w3g + k); v[5] = ld_stream16(w3g + k + 64);
+    v[6] = ld_stream16(w3h + k); v[7] = ld_stream16(w3h + k + 64);
+  };
+  auto compute = [&](const uint4* v, int ch) {
+    const size_t k = size_t(ch) * kChunk * 2;
 #pragma unroll
     for (int G = 0; G < NG; ++G) {
       const uint4 x0 = ldg16(xr[G] + k), x1 = ldg16(xr[G] + k + 64);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint32_t xb0 = word(x0, x1, 2 * j), xb1 = word(x0, x1, 2 * j + 1);
-        mma16816(accg[G], word(ag0, ag1, 2 * j), word(ah0, ah1, 2 * j), word(ag0, ag1, 2 * j + 1),
-                 word(ah0, ah1, 2 * j + 1), xb0, xb1);
-        mma16816(accu[G], word(bg0, bg1, 2 * j), word(bh0, bh1, 2 * j), word(bg0, bg1, 2 * j + 1),
-                 word(bh0, bh1, 2 * j + 1), xb0, xb1);
+        mma16816(accg[G], word(v[0], v[1], 2 * j), word(v[2], v[3], 2 * j),
+                 word(v[0], v[1], 2 * j + 1), word(v[2], v[3], 2 * j + 1), xb0, xb1);
+        mma16816(accu[G], word(v[4], v[5], 2 * j), word(v[6], v[7], 2 * j),
+                 word(v[4], v[5], 2 * j + 1), word(v[6], v[7], 2 * j + 1), xb0, xb1);
       }
     }
-  }
+  };
+  stream_chunks<DB>(c0, c1, load, compute);
 #pragma unroll
   for (int G = 0; G < NG; ++G)
 #pragma unroll
@@ -219,7 +251,7 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
 // share the h fragments, so each lane keeps 8 weight loads in flight per chunk), contraction part
 // kp of ks, and n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part.
 // red: shared scratch [kWarps][kMaxNG][8][32] floats. Output plane kp of o.
-template <int NG>
+template <int NG, bool DB>
 __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, const void* lblk,
                                           int r0, int q0, int n, int kp, int ks, int RB, int KS,
                                           float* red) {
@@ -247,25 +279,30 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
   int p0, p1, c0, c1;
   warp_slice(int(rowb / (kChunk * 2)), ks, kp, p0, p1);
   warp_slice(p1 - p0, KS, warp % KS, c0, c1);
-  for (int ch = p0 + c0; ch < p0 + c1; ++ch) {
+  // one chunk's weights: tile 0 rows g / g+8 (lo, hi halves), then tile 1's
+  auto load = [&](uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
-    const uint4 ag0 = ld_stream16(wg + k), ag1 = ld_stream16(wg + k + 64);
-    const uint4 ah0 = ld_stream16(wh + k), ah1 = ld_stream16(wh + k + 64);
-    const uint4 bg0 = ld_stream16(vg + k), bg1 = ld_stream16(vg + k + 64);
-    const uint4 bh0 = ld_stream16(vh + k), bh1 = ld_stream16(vh + k + 64);
+    v[0] = ld_stream16(wg + k); v[1] = ld_stream16(wg + k + 64);
+    v[2] = ld_stream16(wh + k); v[3] = ld_stream16(wh + k + 64);
+    v[4] = ld_stream16(vg + k); v[5] = ld_stream16(vg + k + 64);
+    v[6] = ld_stream16(vh + k); v[7] = ld_stream16(vh + k + 64);
+  };
+  auto compute = [&](const uint4* v, int ch) {
+    const size_t k = size_t(ch) * kChunk * 2;
 #pragma unroll
     for (int G = 0; G < NG; ++G) {
       const uint4 x0 = ldg16(hr[G] + k), x1 = ldg16(hr[G] + k + 64);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint32_t xb0 = word(x0, x1, 2 * j), xb1 = word(x0, x1, 2 * j + 1);
-        mma16816(acc[G], word(ag0, ag1, 2 * j), word(ah0, ah1, 2 * j), word(ag0, ag1, 2 * j + 1),
-                 word(ah0, ah1, 2 * j + 1), xb0, xb1);
-        mma16816(acc[G] + 4, word(bg0, bg1, 2 * j), word(bh0, bh1, 2 * j),
-                 word(bg0, bg1, 2 * j + 1), word(bh0, bh1, 2 * j + 1), xb0, xb1);
+        mma16816(acc[G], word(v[0], v[1], 2 * j), word(v[2], v[3], 2 * j),
+                 word(v[0], v[1], 2 * j + 1), word(v[2], v[3], 2 * j + 1), xb0, xb1);
+        mma16816(acc[G] + 4, word(v[4], v[5], 2 * j), word(v[6], v[7], 2 * j),
+                 word(v[4], v[5], 2 * j + 1), word(v[6], v[7], 2 * j + 1), xb0, xb1);
       }
     }
-  }
+  };
+  stream_chunks<DB>(p0 + c0, p0 + c1, load, compute);
 #pragma unroll
   for (int G = 0; G < NG; ++G)
 #pragma unroll
@@ -292,6 +329,10 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
   __syncthreads();
 }
 
+// MAXNG: the largest token group (8 tokens each) this launch needs, from its batch size; a pass
+// takes at most 8 * MAXNG tokens, and only the item variants up to MAXNG are compiled into the
+// kernel, so the small-batch kernels keep the registers for double-buffered loads.
+template <int MAXNG>
 __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_constant__ FfnArgs a,
                                                                int RB) {
   pdl_wait();
@@ -304,16 +345,18 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
     const int r0 = (item - it.first[s]) * kRows * RB;
     const char* blk = it.blk[s];
     const void* lblk = a.lrank ? a.lblk[s] : nullptr;
-    // passes of at most 32 tokens; a second pass re-reads the rows from L2, not HBM
-    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
-      const int n = min(kPassTokens, it.off[s + 1] - q0);
-      if (n <= 8) dec13_item<1>(a, blk, lblk, r0, q0, n, RB, KS, red);
-      else if (n <= 16) dec13_item<2>(a, blk, lblk, r0, q0, n, RB, KS, red);
-      else dec13_item<4>(a, blk, lblk, r0, q0, n, RB, KS, red);
+    // passes of at most 8 * MAXNG tokens; a later pass re-reads the rows from L2, not HBM
+    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
+      const int n = min(8 * MAXNG, it.off[s + 1] - q0);
+      if (n <= 8) dec13_item<1, MAXNG <= 2>(a, blk, lblk, r0, q0, n, RB, KS, red);
+      else if (MAXNG == 2 || n <= 16)
+        dec13_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, RB, KS, red);
+      else dec13_item<MAXNG, false>(a, blk, lblk, r0, q0, n, RB, KS, red);
     }
   }
 }
 
+template <int MAXNG>
 __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_constant__ FfnArgs a,
                                                               int RB) {
   pdl_wait();
@@ -327,11 +370,12 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
     const int r0 = (local / it.ksplit) * kRows2 * RB, kp = local % it.ksplit;
     const char* blk = it.blk[s];
     const void* lblk = a.lrank ? a.lblk[s] : nullptr;
-    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += kPassTokens) {
-      const int n = min(kPassTokens, it.off[s + 1] - q0);
-      if (n <= 8) dec2_item<1>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
-      else if (n <= 16) dec2_item<2>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
-      else dec2_item<4>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
+      const int n = min(8 * MAXNG, it.off[s + 1] - q0);
+      if (n <= 8) dec2_item<1, MAXNG <= 2>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+      else if (MAXNG == 2 || n <= 16)
+        dec2_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+      else dec2_item<MAXNG, false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
     }
   }
 }
@@ -357,23 +401,31 @@ int rows_per_item(int rows, int contraction, int rows_per_warp) {
   return rb;
 }
 
-cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
-  static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel));
-  static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel));
+template <int MAXNG>
+cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
+  static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel<MAXNG>));
+  static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel<MAXNG>));
   const int rb13 = rows_per_item(a.w, a.d, kRows);
   const int rb2 = rows_per_item(a.d, a.w / a.ksplit, kRows2);
   cudaError_t e = cudaSuccess;
   if (stages & 1) {
     prof_begin(kProfDec13, s);
-    e = launch_pdl(dec13_kernel, dim3(num_sms * nb13), dim3(kWarps * 32), 0, s, a, rb13);
+    e = launch_pdl(dec13_kernel<MAXNG>, dim3(num_sms * nb13), dim3(kWarps * 32), 0, s, a, rb13);
     prof_end(kProfDec13, s);
     if (e == cudaSuccess) e = cudaGetLastError();
   }
   if (e != cudaSuccess || !(stages & 2)) return e;
   prof_begin(kProfDec2, s);
-  e = launch_pdl(dec2_kernel, dim3(num_sms * nb2), dim3(kWarps * 32), 0, s, a, rb2);
+  e = launch_pdl(dec2_kernel<MAXNG>, dim3(num_sms * nb2), dim3(kWarps * 32), 0, s, a, rb2);
   prof_end(kProfDec2, s);
   return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
+  // a segment holds at most T tokens (routed experts: distinct per token; shared: all T)
+  if (a.T <= 8) return launch_decode_ng<1>(a, num_sms, s, stages);
+  if (a.T <= 16) return launch_decode_ng<2>(a, num_sms, s, stages);
+  return launch_decode_ng<4>(a, num_sms, s, stages);
 }
 
 }  // namespace mcft
