@@ -186,6 +186,16 @@ def test_chain_deepseek_26_layers_bf16(n_prefetch, T):
                     distinct=False, seed=62, band=0.03, gate_atol=2e-3, tol=1e-2)
 
 
+@pytest.mark.parametrize("shape,T,L", [(I.DSV2_LITE, 64, 3), (I.MIXTRAL, 16, 4)],
+                         ids=["dsv2-64-tokens", "mixtral-16-tokens"])
+def test_chain_large_batch_bf16(shape, T, L):
+    """The largest decode batches of the stack (bypass fetches into staging buffers when a step
+    needs more experts than the layer has slots)."""
+    run_and_compare(shape, L=L, T=T, steps=2, B=shape.cache_slots, policy="LFU",
+                    n_prefetch=shape.K, distinct=False, seed=65, band=0.03 if shape.E == 64 else 0.1,
+                    gate_atol=2e-3 if shape.E == 64 else 0.025, tol=1e-2 if shape.E == 64 else 2.5e-2)
+
+
 @pytest.mark.parametrize("T", [1, 3])
 def test_prefetch_does_not_change_the_stream(T):
     """The stack's output does not depend on prefetching (only where the bytes come from)."""
