@@ -247,6 +247,7 @@ mcft_status mcft_device_error(mcft_stream_t stream) {
 mcft_status mcft_route(const mcft_layer_desc* desc, const void* x, int T, const void* w_router,
                        int mode, const uint8_t* mask, const float* prior, int32_t* idx, float* gate,
                        mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_route");
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
@@ -478,6 +479,7 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
                              const float* gate, const void* const* experts,
                              const void* const* shared, void* y, void* workspace, size_t ws_bytes,
                              mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_moe_forward");
   return forward_impl(desc, x, T, idx, gate, experts, shared, nullptr, y, workspace, ws_bytes,
                       stream);
 }
@@ -488,6 +490,7 @@ mcft_status mcft_moe_forward_lora(const mcft_layer_desc* desc, const void* x, in
                                   const void* const* expert_lora, const void* const* shared_lora,
                                   int lora_rank, float lora_scale, void* y, void* workspace,
                                   size_t ws_bytes, mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_moe_forward_lora");
   mcft_status st = check_lora(lora_rank, lora_scale);
   if (st != MCFT_OK) return st;
   const LoraArgs la{expert_lora, shared_lora, lora_rank, lora_scale};
@@ -602,6 +605,7 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
 
 mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T, int K,
                             mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_cache_step");
   if (!c || !idx) return fail(MCFT_ERR_INVALID, "NULL cache or idx");
   if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
   if (T < 1 || K < 1 || K > c->E) return fail(MCFT_ERR_INVALID, "bad T = %d or K = %d", T, K);
@@ -622,6 +626,7 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
 
 mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_stream,
                                mcft_stream_t copy_stream, const void** expert_ptrs) {
+  mcft::NvtxRange nvtx_range("mcft_fetch_experts");
   if (!c || !expert_ptrs) return fail(MCFT_ERR_INVALID, "NULL cache or expert_ptrs");
   if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
   // The miss list is known only once routing and the cache decision have run.
@@ -659,6 +664,7 @@ mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_s
 
 mcft_status mcft_cache_prefetch(mcft_cache* c, int layer, const int32_t* idx_pred, int T, int K,
                                 int n_max, mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_cache_prefetch");
   if (!c || !idx_pred) return fail(MCFT_ERR_INVALID, "NULL cache or idx_pred");
   if (layer < 0 || layer >= c->L) return fail(MCFT_ERR_INVALID, "layer %d out of range", layer);
   if (T < 1 || K < 1 || K > c->E) return fail(MCFT_ERR_INVALID, "bad T = %d or K = %d", T, K);
@@ -715,6 +721,7 @@ mcft_status mcft_cache_prefetch_stats(const mcft_cache* c, int layer, uint64_t* 
 
 mcft_status mcft_residual_rmsnorm(const mcft_layer_desc* desc, float* x, const void* y, int T,
                                   const void* gamma, float eps, void* u, mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_residual_rmsnorm");
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
@@ -733,6 +740,7 @@ mcft_status mcft_residual_rmsnorm(const mcft_layer_desc* desc, float* x, const v
 
 mcft_status mcft_mask_sample(const float* m_tilde, const float* uniforms, int L, int E, int e_keep,
                              uint8_t* mask, float* pi, mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_mask_sample");
   if (!m_tilde || !uniforms || !mask || !pi) return fail(MCFT_ERR_INVALID, "NULL pointer argument");
   if (L < 0 || E < 1) return fail(MCFT_ERR_INVALID, "bad L = %d or E = %d", L, E);
   if (E > kMaxE) return fail(MCFT_ERR_UNSUPPORTED, "E = %d > %d", E, kMaxE);
@@ -747,6 +755,7 @@ mcft_status mcft_mask_sample(const float* m_tilde, const float* uniforms, int L,
 
 mcft_status mcft_gate_grad(const mcft_layer_desc* desc, const void* dy, int T, const void* workspace,
                            size_t ws_bytes, float* dgate, mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_gate_grad");
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
@@ -770,6 +779,7 @@ mcft_status mcft_gate_grad(const mcft_layer_desc* desc, const void* dy, int T, c
 mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, const float* gate,
                            const float* dgate, int T, const float* pi, float* dm, float* dm_tilde,
                            int accumulate, mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_mask_grad");
   mcft_status st = check_desc(desc);
   if (st != MCFT_OK) return st;
   if (T < 0) return fail(MCFT_ERR_INVALID, "T = %d < 0", T);
@@ -786,6 +796,7 @@ mcft_status mcft_moe_forward_cached(const mcft_layer_desc* desc, const void* x, 
                                     const void* const* shared, void* y, void* workspace,
                                     size_t ws_bytes, mcft_stream_t compute_stream,
                                     mcft_stream_t copy_stream) {
+  mcft::NvtxRange nvtx_range("mcft_moe_forward_cached");
   return mcft::forward_cached_impl(desc, x, T, idx, gate, c, layer, shared, y, workspace, ws_bytes,
                                    compute_stream, copy_stream, false);
 }

@@ -7,10 +7,21 @@
 
 #include <utility>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/mcft.h"
 #include "common.cuh"
 
 namespace mcft {
+
+// NVTX range around a C-ABI call, so timeline profilers show route / cache step / fetch / forward /
+// stack step by name (header-only NVTX: nothing happens unless a profiler is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 // Launch `kernel` with programmatic stream serialization (programmatic dependent launch): its CTAs
 // may be scheduled while the previous kernel in `s` drains, and the kernel's pdl_wait() holds its

@@ -67,6 +67,7 @@ extern "C" mcft_status mcft_moe_forward_noalloc(const mcft_layer_desc* desc, con
                                                 const void* const* experts,
                                                 const void* const* shared, void* y,
                                                 mcft_stream_t stream) {
+  mcft::NvtxRange nvtx_range("mcft_moe_forward_noalloc");
   size_t need = 0;
   mcft_status st = mcft_moe_workspace_size(desc, T, &need);
   if (st != MCFT_OK) return st;

@@ -123,6 +123,7 @@ mcft_status mcft_stack_create(const mcft_layer_desc* desc, int L, const void* co
 
 mcft_status mcft_stack_step(mcft_stack* s, float* x, int T, mcft_stream_t compute,
                             mcft_stream_t copy) {
+  mcft::NvtxRange nvtx_range("mcft_stack_step");
   if (!s || !x) return stack_fail(MCFT_ERR_INVALID, "NULL stack or x");
   if (T < 1 || T > s->T_max) return stack_fail(MCFT_ERR_INVALID, "T must be in [1, T_max]");
   const mcft_layer_desc* desc = &s->desc;
