@@ -63,6 +63,10 @@ int num_sms() {
 
 size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
 
+// CTAs of the device-driven fetch kernel: a quarter of the SMs (the host link is the bound, and
+// the rest of the GPU stays with the FFN of the experts that were hits).
+int fetch_blocks() { return num_sms() / 4 > 0 ? num_sms() / 4 : 1; }
+
 mcft_status check_desc(const mcft_layer_desc* d) {
   if (!d) return fail(MCFT_ERR_INVALID, "desc is NULL");
   if (d->d <= 0 || d->d % 64) return fail(MCFT_ERR_INVALID, "d = %d must be a positive multiple of 64", d->d);
@@ -216,7 +220,7 @@ mcft_status enqueue_prefetch_fetches(mcft_cache* c, cudaStream_t copy) {
     FetchArgs fe{c->d_pf_list + size_t(l) * (1 + c->E), c->d_host_src + size_t(l) * c->E,
                  c->d_pf_tab + size_t(l) * c->E, c->expert_bytes, c->d_pf_cancel + l,
                  c->d_pf_moved + l};
-    cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy, true);
+    cudaError_t e = launch_fetch(fe, fetch_blocks(), copy, true);
     if (e != cudaSuccess) return cuda_fail(e, "prefetch fetch kernel launch");
     MCFT_CUDA(cudaEventRecord(c->ev_pf_done[l], copy));
     c->pf_state[l] = 2;
@@ -855,7 +859,7 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   MCFT_CUDA(cudaStreamWaitEvent(copy_stream, c->ev_step[layer], 0));
   FetchArgs fe{c->d_miss_dev + size_t(layer) * c->miss_stride, c->d_host_src + size_t(layer) * E,
                c->d_ptr_tab + size_t(layer) * E, c->expert_bytes, nullptr, nullptr};
-  cudaError_t e = launch_fetch(fe, num_sms() / 4 > 0 ? num_sms() / 4 : 1, copy_stream);
+  cudaError_t e = launch_fetch(fe, fetch_blocks(), copy_stream);
   if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
   // Experts a prefetch of this layer is still bringing in are not in the step's ready mask: the
@@ -890,10 +894,13 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   fa.err = err;
   fa.wtab = c->d_ptr_tab + size_t(layer) * E;
   fa.ready = c->d_ready + layer;
+  // an expert fetch (this layer's misses, or a later layer's prefetch) may run alongside either
+  // phase: each of its CTAs takes one FFN CTA's slot on its SM
+  const int displaced = fetch_blocks();
   for (int phase = 1; phase <= 2; ++phase) {
     fa.phase = phase;
     if (phase == 2) MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
-    e = L.decode ? launch_ffn_decode(fa, num_sms(), compute_stream)
+    e = L.decode ? launch_ffn_decode(fa, num_sms(), compute_stream, 3, displaced)
                  : launch_ffn_rowwise(fa, desc->dtype, num_sms(), compute_stream);
     if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
   }

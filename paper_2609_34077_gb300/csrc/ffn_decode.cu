@@ -17,7 +17,9 @@
 //    applies silu(gate) * up and stores h in bf16; GEMM2 stores fp32 outputs. At small batches
 //    GEMM2 also splits the contraction across `ksplit` CTAs (partial planes of o, summed in the
 //    combine kernel) so that few selected experts still give every SM work.
-// Items are spread over a persistent grid.
+// Items are spread over a persistent grid (static striding). When an expert fetch kernel runs at the
+// same time, the caller sizes the grid to the CTAs that can be resident next to it, so no CTA of
+// the grid starts late with items of its own.
 #include "common.cuh"
 #include "internal.h"
 
@@ -402,30 +404,35 @@ int rows_per_item(int rows, int contraction, int rows_per_warp) {
 }
 
 template <int MAXNG>
-cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
+cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int stages,
+                             int displaced) {
   static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel<MAXNG>));
   static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel<MAXNG>));
+  // one CTA per SM slot, less the slots that concurrently running CTAs of another kernel take
+  const int g13 = max(num_sms, num_sms * nb13 - displaced);
+  const int g2 = max(num_sms, num_sms * nb2 - displaced);
   const int rb13 = rows_per_item(a.w, a.d, kRows);
   const int rb2 = rows_per_item(a.d, a.w / a.ksplit, kRows2);
   cudaError_t e = cudaSuccess;
   if (stages & 1) {
     prof_begin(kProfDec13, s);
-    e = launch_pdl(dec13_kernel<MAXNG>, dim3(num_sms * nb13), dim3(kWarps * 32), 0, s, a, rb13);
+    e = launch_pdl(dec13_kernel<MAXNG>, dim3(g13), dim3(kWarps * 32), 0, s, a, rb13);
     prof_end(kProfDec13, s);
     if (e == cudaSuccess) e = cudaGetLastError();
   }
   if (e != cudaSuccess || !(stages & 2)) return e;
   prof_begin(kProfDec2, s);
-  e = launch_pdl(dec2_kernel<MAXNG>, dim3(num_sms * nb2), dim3(kWarps * 32), 0, s, a, rb2);
+  e = launch_pdl(dec2_kernel<MAXNG>, dim3(g2), dim3(kWarps * 32), 0, s, a, rb2);
   prof_end(kProfDec2, s);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages) {
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages,
+                              int displaced) {
   // a segment holds at most T tokens (routed experts: distinct per token; shared: all T)
-  if (a.T <= 8) return launch_decode_ng<1>(a, num_sms, s, stages);
-  if (a.T <= 16) return launch_decode_ng<2>(a, num_sms, s, stages);
-  return launch_decode_ng<4>(a, num_sms, s, stages);
+  if (a.T <= 8) return launch_decode_ng<1>(a, num_sms, s, stages, displaced);
+  if (a.T <= 16) return launch_decode_ng<2>(a, num_sms, s, stages, displaced);
+  return launch_decode_ng<4>(a, num_sms, s, stages, displaced);
 }
 
 }  // namespace mcft

@@ -195,8 +195,10 @@ __device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned l
 // stages: bit 0 = GEMM13 (+ SwiGLU), bit 1 = GEMM2
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s,
                                int stages = 3);  // fp32
-cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s,
-                              int stages = 3);  // bf16, T <= 64
+// displaced: CTA slots taken by another kernel running at the same time (the expert fetch); the
+// persistent grid is that much smaller, so every CTA is resident from the start.
+cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages = 3,
+                              int displaced = 0);  // bf16, T <= 64
 int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
 cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
                           int stages = 3);
