@@ -48,6 +48,8 @@ TRAFFIC = {
                      "profiles/ffn_decode_mixtral_decode.md"),
     "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "238714c66b89d496", 1.0047,
                     "profiles/ffn_decode_mixtral_decode.md"),
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "", None,
+                   "profiles/ffn_decode_mixtral_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "71e2bb67dbc90a66", 0.9566,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
 }
@@ -236,11 +238,13 @@ def unique_per_step(idx_steps):
 def decode_roofline(prof, U, steps, batch, shape, peaks):
     """HBM roofline of the decode FFN kernels. Algorithmic bytes per launch: the W1 and W3 rows
     (GEMM13) or W2 rows (GEMM2) of every expert the step selected, read once, plus the token
-    activations in and out. Returns (dominant kernel's roofline dict, {kernel: GB/s})."""
+    activations in and out; the fused kernel (both GEMMs in one launch) reads all three. Returns
+    (dominant kernel's roofline dict, {kernel: GB/s})."""
     sel = sum(U)
     T, K, d, w = batch, shape.K, shape.d, shape.w
-    alg = {"ffn13_decode": sel * 2 * w * d * 2 + steps * (T * d * 2 + T * K * w * 2),
-           "ffn2_decode": sel * w * d * 2 + steps * T * K * (w * 2 + d * 4)}
+    b13 = sel * 2 * w * d * 2 + steps * (T * d * 2 + T * K * w * 2)
+    b2 = sel * w * d * 2 + steps * T * K * (w * 2 + d * 4)
+    alg = {"ffn13_decode": b13, "ffn2_decode": b2, "ffn_decode": b13 + b2}
     rates, best = {}, None
     for k, b in alg.items():
         n, ms = prof.get(k, (0, 0.0))

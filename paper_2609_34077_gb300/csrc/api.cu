@@ -115,6 +115,7 @@ WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lran
   L.off = o;  o = align256(o + sizeof(int) * (nseg + 1));
   L.pos = o;  o = align256(o + sizeof(int) * size_t(T) * K);
   L.perm = o; o = align256(o + sizeof(int) * size_t(L.mcap));
+  L.done = o; o = align256(o + sizeof(int) * nseg);
   L.xp = o;   o = align256(o + (L.tc ? size_t(L.mcap) * d * 2 : 0));
   L.h = o;    o = align256(o + size_t(L.mcap) * w * (dtype == MCFT_BF16 ? 2 : 4));
   L.o = o;    o = align256(o + size_t(L.ks) * L.mcap * d * 4);
@@ -374,7 +375,8 @@ mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, cons
   int* perm = reinterpret_cast<int*>(ws + L.perm);
   unsigned* err = device_error_word();
 
-  PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
+  int* done = reinterpret_cast<int*>(ws + L.done);
+  PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err, done};
   cudaError_t e = launch_permute(pa, stream);
   if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
 
@@ -383,6 +385,7 @@ mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, cons
   fa.off = off;
   fa.perm = perm;
   fa.hdr = hdr;
+  fa.done = done;
   for (int i = 0; i < E; ++i) fa.wblk[i] = experts[i];
   for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
   fa.h = ws + L.h;
@@ -848,6 +851,7 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   int* off = reinterpret_cast<int*>(ws + L.off);
   int* pos = reinterpret_cast<int*>(ws + L.pos);
   int* perm = reinterpret_cast<int*>(ws + L.perm);
+  int* done = reinterpret_cast<int*>(ws + L.done);
   unsigned* err = device_error_word();
   // 0. a prefetch of this layer decided before the step lands first (it may target the slots the
   //    step's misses overwrite)
@@ -872,7 +876,7 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   // 2. meanwhile: permutation (unless the fused prologue wrote it into this workspace) and the
   //    experts that were hits (and the shared experts)
   if (!permuted) {
-    PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err};
+    PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err, done};
     e = launch_permute(pa, compute_stream);
     if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
   }
@@ -881,6 +885,9 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   fa.off = off;
   fa.perm = perm;
   fa.hdr = hdr;
+  // no fused (cooperative) FFN here: a cooperative grid waits until all of its CTAs can be
+  // resident at once, which would hold it behind the concurrently running fetch kernel
+  fa.done = nullptr;
   for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
   fa.h = ws + L.h;
   fa.o = reinterpret_cast<float*>(ws + L.o);
@@ -978,7 +985,8 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
   char* ws = static_cast<char*>(workspace);
   a.perm = PermuteArgs{idx, 1, K, E, S, L.pad, L.mcap, reinterpret_cast<WsHeader*>(ws + L.hdr),
                        reinterpret_cast<int*>(ws + L.cnt), reinterpret_cast<int*>(ws + L.off),
-                       reinterpret_cast<int*>(ws + L.pos), reinterpret_cast<int*>(ws + L.perm), err};
+                       reinterpret_cast<int*>(ws + L.pos), reinterpret_cast<int*>(ws + L.perm), err,
+                       reinterpret_cast<int*>(ws + L.done)};
   cudaError_t e = launch_prologue(a, desc->dtype, stream);
   if (e != cudaSuccess) return cuda_fail(e, "prologue kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_step[layer], stream));

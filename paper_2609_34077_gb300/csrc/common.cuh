@@ -36,6 +36,16 @@ __device__ __forceinline__ uint4 ldg16(const void* p) {
   return __ldg(reinterpret_cast<const uint4*>(p));
 }
 
+// 16-byte load through L2 only (coherent with stores of other CTAs of the same kernel that were
+// published with a fence: no stale L1 line can be returned).
+__device__ __forceinline__ uint4 ldcg16(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
 // Streaming (read-once) 16-byte load: do not keep in L1.
 __device__ __forceinline__ uint4 ld_stream16(const void* p) {
   uint4 r;

@@ -293,7 +293,8 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
     const size_t k = size_t(ch) * kChunk * 2;
 #pragma unroll
     for (int G = 0; G < NG; ++G) {
-      const uint4 x0 = ldg16(hr[G] + k), x1 = ldg16(hr[G] + k + 64);
+      // h through L2 only: in the fused kernel other CTAs wrote it during this launch
+      const uint4 x0 = ldcg16(hr[G] + k), x1 = ldcg16(hr[G] + k + 64);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint32_t xb0 = word(x0, x1, 2 * j), xb1 = word(x0, x1, 2 * j + 1);
@@ -334,28 +335,54 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
 // MAXNG: the largest token group (8 tokens each) this launch needs, from its batch size; a pass
 // takes at most 8 * MAXNG tokens, and only the item variants up to MAXNG are compiled into the
 // kernel, so the small-batch kernels keep the registers for double-buffered loads.
+// One GEMM13 work item (RB blocks of 16 rows of one segment, all its tokens in passes of at most
+// 8 * MAXNG); returns the segment.
+template <int MAXNG, bool DBOK = true>
+__device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, int item, int RB,
+                                          float* red) {
+  const int KS = kWarps / RB;
+  const int s = dec_seg(it, item);
+  const int r0 = (item - it.first[s]) * kRows * RB;
+  const char* blk = it.blk[s];
+  const void* lblk = a.lrank ? a.lblk[s] : nullptr;
+  // passes of at most 8 * MAXNG tokens; a later pass re-reads the rows from L2, not HBM
+  for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
+    const int n = min(8 * MAXNG, it.off[s + 1] - q0);
+    if (n <= 8) dec13_item<1, DBOK && MAXNG <= 2>(a, blk, lblk, r0, q0, n, RB, KS, red);
+    else if (MAXNG == 2 || n <= 16)
+      dec13_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, RB, KS, red);
+    else dec13_item<MAXNG, false>(a, blk, lblk, r0, q0, n, RB, KS, red);
+  }
+  return s;
+}
+
+// One GEMM2 work item (RB blocks of 32 rows of W2 of one segment, one contraction part).
+template <int MAXNG, bool DBOK = true>
+__device__ __forceinline__ void run2_item(const FfnArgs& a, const DecItems& it, int item, int RB,
+                                          float* red) {
+  const int KS = kWarps / RB;
+  const int s = dec_seg(it, item);
+  const int local = item - it.first[s];
+  const int r0 = (local / it.ksplit) * kRows2 * RB, kp = local % it.ksplit;
+  const char* blk = it.blk[s];
+  const void* lblk = a.lrank ? a.lblk[s] : nullptr;
+  for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
+    const int n = min(8 * MAXNG, it.off[s + 1] - q0);
+    if (n <= 8) dec2_item<1, DBOK && MAXNG <= 2>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+    else if (MAXNG == 2 || n <= 16)
+      dec2_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+    else dec2_item<MAXNG, false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+  }
+}
+
 template <int MAXNG>
 __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_constant__ FfnArgs a,
                                                                int RB) {
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  const int KS = kWarps / RB;
   build_dec_items(it, a, a.w / (kRows * RB), 1);
-  for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
-    const int s = dec_seg(it, item);
-    const int r0 = (item - it.first[s]) * kRows * RB;
-    const char* blk = it.blk[s];
-    const void* lblk = a.lrank ? a.lblk[s] : nullptr;
-    // passes of at most 8 * MAXNG tokens; a later pass re-reads the rows from L2, not HBM
-    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
-      const int n = min(8 * MAXNG, it.off[s + 1] - q0);
-      if (n <= 8) dec13_item<1, MAXNG <= 2>(a, blk, lblk, r0, q0, n, RB, KS, red);
-      else if (MAXNG == 2 || n <= 16)
-        dec13_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, RB, KS, red);
-      else dec13_item<MAXNG, false>(a, blk, lblk, r0, q0, n, RB, KS, red);
-    }
-  }
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) run13_item<MAXNG>(a, it, item, RB, red);
 }
 
 template <int MAXNG>
@@ -364,20 +391,69 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  const int KS = kWarps / RB;
   build_dec_items(it, a, a.d / (kRows2 * RB), a.ksplit);
-  for (int item = blockIdx.x; item < it.total; item += gridDim.x) {
-    const int s = dec_seg(it, item);
-    const int local = item - it.first[s];
-    const int r0 = (local / it.ksplit) * kRows2 * RB, kp = local % it.ksplit;
-    const char* blk = it.blk[s];
-    const void* lblk = a.lrank ? a.lblk[s] : nullptr;
-    for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
-      const int n = min(8 * MAXNG, it.off[s + 1] - q0);
-      if (n <= 8) dec2_item<1, MAXNG <= 2>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
-      else if (MAXNG == 2 || n <= 16)
-        dec2_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
-      else dec2_item<MAXNG, false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) run2_item<MAXNG>(a, it, item, RB, red);
+}
+
+constexpr uint64_t kSegWaitNs = 2000000000ull;
+// the fused kernel holds both GEMMs' code, so it keeps double-buffered loads only where both fit
+// the register budget without spills (see -Xptxas -v)
+constexpr bool kFusedDB = false;
+
+// Bounded wait (one thread) until segment s has `need` finished GEMM13 items; false (and the call
+// aborted, so later waits return at once) if 2 s pass or the call is already aborting.
+__device__ bool wait_segment(const FfnArgs& a, int s, int need) {
+  const volatile int* p = a.done + s;
+  const volatile int* abort = &a.hdr->abort;
+  if (*p < need) {
+    const uint64_t t0 = globaltimer_ns();
+    while (*p < need) {
+      if (*abort) return false;
+      if (globaltimer_ns() - t0 > kSegWaitNs) {
+        set_error(a.err, kErrTimeout);
+        const_cast<WsHeader*>(a.hdr)->abort = 1;
+        return false;
+      }
+      __nanosleep(256);
+    }
+  }
+  __threadfence();
+  return true;
+}
+
+// GEMM13 and GEMM2 of a decode call in one cooperative launch: the work list is every GEMM13 item,
+// then every GEMM2 item, walked with static striding by a grid that is entirely resident (the
+// cooperative launch guarantees it). A GEMM13 item publishes its segment's progress after its h
+// rows are written and fenced; a GEMM2 item first waits (bounded) until its segment's GEMM13 items
+// are all done, then reads h through L2. Every wait is on items with lower indices, which CTAs
+// that are already running process before any item of their own that could wait, so the waits
+// always end. One launch instead of two, and a segment's GEMM2 overlaps other segments' GEMM13.
+// Used when nothing of ours runs alongside (mcft_moe_forward): a cooperative grid only starts
+// once all of its CTAs fit, so next to the expert fetch kernel it would wait for the fetch.
+template <int MAXNG>
+__global__ void __launch_bounds__(kWarps * 32, 2)
+    dec_fused_kernel(const __grid_constant__ FfnArgs a, int RB13, int RB2) {
+  pdl_wait();
+  __shared__ DecItems it13, it2;
+  __shared__ float red[kWarps * kMaxNG * 8 * 32];
+  __shared__ int s_ok;
+  build_dec_items(it13, a, a.w / (kRows * RB13), 1);
+  build_dec_items(it2, a, a.d / (kRows2 * RB2), a.ksplit);
+  const int n13 = it13.total, total = n13 + it2.total;
+  const int per13 = a.w / (kRows * RB13);  // GEMM13 items of every segment that has work
+  for (int item = blockIdx.x; item < total; item += gridDim.x) {
+    if (item < n13) {
+      const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, RB13, red);
+      __threadfence();  // this CTA's h rows, before the segment's count moves
+      __syncthreads();
+      if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
+    } else {
+      const int i2 = item - n13;
+      if (threadIdx.x == 0) s_ok = wait_segment(a, dec_seg(it2, i2), per13) ? 1 : 0;
+      __syncthreads();
+      const int ok = s_ok;
+      __syncthreads();
+      if (ok) run2_item<MAXNG, kFusedDB>(a, it2, i2, RB2, red);
     }
   }
 }
@@ -414,6 +490,24 @@ cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int 
   const int rb13 = rows_per_item(a.w, a.d, kRows);
   const int rb2 = rows_per_item(a.d, a.w / a.ksplit, kRows2);
   cudaError_t e = cudaSuccess;
+  if (stages == 3 && a.done && a.lrank == 0) {
+    // both GEMMs in one cooperative launch (every CTA resident: its waits always end)
+    static const int nbf = blocks_per_sm(reinterpret_cast<const void*>(dec_fused_kernel<MAXNG>));
+    const int gf = max(num_sms, num_sms * nbf - displaced);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(gf);
+    cfg.blockDim = dim3(kWarps * 32);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    prof_begin(kProfDecFused, s);
+    e = cudaLaunchKernelEx(&cfg, dec_fused_kernel<MAXNG>, a, rb13, rb2);
+    prof_end(kProfDecFused, s);
+    return e != cudaSuccess ? e : cudaGetLastError();
+  }
   if (stages & 1) {
     prof_begin(kProfDec13, s);
     e = launch_pdl(dec13_kernel<MAXNG>, dim3(g13), dim3(kWarps * 32), 0, s, a, rb13);

@@ -72,7 +72,7 @@ struct WsLayout {
   int pad;        // rows per segment are padded to a multiple of this (128 on the TC path)
   int mcap;       // capacity in permuted rows
   int ks;         // partial planes of o (contraction split of the decode GEMM2)
-  size_t hdr, cnt, off, pos, perm, xp, h, o, u13, u2, total;
+  size_t hdr, cnt, off, pos, perm, done, xp, h, o, u13, u2, total;
 };
 WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lrank = 0);
 
@@ -119,6 +119,7 @@ struct PermuteArgs {
   int* pos;    // [T*K] permuted row of assignment (t, k)
   int* perm;   // [mcap] token of each permuted row, -1 for padding
   unsigned* err;
+  int* done;   // [E+S] completed GEMM13 work items per segment (fused decode FFN), zeroed here
 };
 cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s);
 
@@ -155,6 +156,9 @@ struct FfnArgs {
   float lscale;
   const float* u13;
   const float* u2;
+  // [E+S] completed GEMM13 items per segment (zeroed by the permutation of the call): lets one
+  // fused decode launch start a segment's GEMM2 as soon as that segment's h is written
+  int* done;
 };
 
 // s * sum_j u[j] B[row][j] for a LoRA up-projection B [rows, r] (layer dtype TW).
@@ -367,7 +371,7 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
        kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfNorm,
-       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfCount };
+       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfDecFused, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 
