@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "238714c66b89d496", 1.0022,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "dc1fee43f4e052a7", 1.0020,
                      "profiles/ffn_decode_mixtral_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "238714c66b89d496", 1.0047,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "dc1fee43f4e052a7", 1.0048,
                     "profiles/ffn_decode_mixtral_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "", None,
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "dc1fee43f4e052a7", 1.0016,
                    "profiles/ffn_decode_mixtral_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "71e2bb67dbc90a66", 0.9566,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
