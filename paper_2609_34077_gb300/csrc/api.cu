@@ -115,7 +115,7 @@ WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lran
   L.off = o;  o = align256(o + sizeof(int) * (nseg + 1));
   L.pos = o;  o = align256(o + sizeof(int) * size_t(T) * K);
   L.perm = o; o = align256(o + sizeof(int) * size_t(L.mcap));
-  L.done = o; o = align256(o + sizeof(int) * nseg);
+  L.done = o; o = align256(o + sizeof(int) * (nseg + kClaimSlots));
   L.xp = o;   o = align256(o + (L.tc ? size_t(L.mcap) * d * 2 : 0));
   L.h = o;    o = align256(o + size_t(L.mcap) * w * (dtype == MCFT_BF16 ? 2 : 4));
   L.o = o;    o = align256(o + size_t(L.ks) * L.mcap * d * 4);
@@ -871,6 +871,8 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   // fetch on this copy stream.
   if (c->pf_state[layer] == 2) c->pf_state[layer] = 0;
   // 1b. prefetches decided for later layers stream in behind this layer's misses
+  int queued = 0;
+  for (int l = 0; l < c->L; ++l) queued += c->pf_state[l] == 1 ? 1 : 0;
   st = enqueue_prefetch_fetches(c, copy_stream);
   if (st != MCFT_OK) return st;
   // 2. meanwhile: permutation (unless the fused prologue wrote it into this workspace) and the
@@ -885,9 +887,7 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   fa.off = off;
   fa.perm = perm;
   fa.hdr = hdr;
-  // no fused (cooperative) FFN here: a cooperative grid waits until all of its CTAs can be
-  // resident at once, which would hold it behind the concurrently running fetch kernel
-  fa.done = nullptr;
+  fa.done = done;  // fused decode FFN (claimed items)
   for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
   fa.h = ws + L.h;
   fa.o = reinterpret_cast<float*>(ws + L.o);
@@ -901,13 +901,14 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   fa.err = err;
   fa.wtab = c->d_ptr_tab + size_t(layer) * E;
   fa.ready = c->d_ready + layer;
-  // an expert fetch (this layer's misses, or a later layer's prefetch) may run alongside either
-  // phase: each of its CTAs takes one FFN CTA's slot on its SM
-  const int displaced = fetch_blocks();
+  // A fetch kernel running alongside keeps its SM slots: this layer's misses (or an earlier
+  // prefetch still on the copy stream) during phase 1; during phase 2, which starts after the
+  // misses have landed, only prefetches queued behind them at 1b.
   for (int phase = 1; phase <= 2; ++phase) {
     fa.phase = phase;
     if (phase == 2) MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
-    e = L.decode ? launch_ffn_decode(fa, num_sms(), compute_stream, 3, displaced)
+    const int reserved = phase == 1 || queued > 0 ? fetch_blocks() : 0;
+    e = L.decode ? launch_ffn_decode(fa, num_sms(), compute_stream, 3, reserved)
                  : launch_ffn_rowwise(fa, desc->dtype, num_sms(), compute_stream);
     if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
   }

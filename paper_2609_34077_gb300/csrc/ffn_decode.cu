@@ -17,9 +17,12 @@
 //    applies silu(gate) * up and stores h in bf16; GEMM2 stores fp32 outputs. At small batches
 //    GEMM2 also splits the contraction across `ksplit` CTAs (partial planes of o, summed in the
 //    combine kernel) so that few selected experts still give every SM work.
-// Items are spread over a persistent grid (static striding). When an expert fetch kernel runs at the
-// same time, the caller sizes the grid to the CTAs that can be resident next to it, so no CTA of
-// the grid starts late with items of its own.
+// Items are spread over a persistent grid: claimed from a counter by the fused kernel (both GEMMs
+// in one launch, the path of every forward without LoRA adapters), with static striding by the
+// separate GEMM13 and GEMM2 kernels (the LoRA forward, whose down projection of h sits between).
+// Two CTAs of these kernels take all of an SM's registers, so when an expert fetch kernel may run
+// at the same time the caller reserves its slots: a grid that took them would keep the fetch from
+// starting until the FFN's CTAs exit.
 #include "common.cuh"
 #include "internal.h"
 
@@ -34,70 +37,99 @@ constexpr int kPassTokens = 32;  // tokens per pass (4 MMA column groups of 8)
 constexpr int kMaxNG = kPassTokens / 8;
 
 struct DecItems {
-  int nseg, total, ksplit;
-  int off[kMaxSeg + 1];
-  int first[kMaxSeg + 1];
+  int npos, total, ksplit;
+  int off[kMaxSeg + 1];    // by segment: permuted-row offsets
   const char* blk[kMaxSeg];
+  int seg[kMaxSeg];        // by position in the work list: segment
+  int first[kMaxSeg + 1];  // by position: first item
 };
 
-// Work list of this launch: items_per_seg items for every non-empty segment of the phase. Warp 0
-// builds it with one lane per segment (segments s = lane, lane + 32, lane + 64) and a shuffle
-// prefix sum, so the setup costs a few loads of latency, not one per segment.
+// Work list of a launch, built by one warp (the calling one) with one lane per segment (segments
+// s = lane, lane + 32, lane + 64): items_per_seg items for every non-empty segment of the phase,
+// segments in decreasing order of their token counts (ties by index), so that the items that take
+// longest (segments that need a second pass or more MMA columns) are handed out first and the
+// last ones are short. Only segments with work get a position. The caller synchronises the block
+// before reading it.
 __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int items_per_seg, int ksplit) {
-  if (threadIdx.x < 32) {
-    const int lane = threadIdx.x;
-    const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
-    const unsigned long long hits = a.ready ? *a.ready : 0ull;
-    int offs[3], cnt[3];
-    for (int j = 0; j < 3; ++j) {
-      const int s = lane + 32 * j;
-      offs[j] = s <= nseg ? a.off[s] : 0;
-      if (s <= nseg) it.off[s] = offs[j];
-    }
-    __syncwarp();
-    bool bad = false;
-    for (int j = 0; j < 3; ++j) {
-      const int s = lane + 32 * j;
-      cnt[j] = 0;
-      if (s < nseg) {
-        const char* b = reinterpret_cast<const char*>(seg_block(a, s));
-        it.blk[s] = b;
-        if (it.off[s + 1] > offs[j] && seg_in_phase(a, s, hits)) {
-          if (b == nullptr) bad = true;  // a selected expert without weights
-          else cnt[j] = items_per_seg * ksplit;
-        }
-      }
-    }
-    int base = 0;
-    for (int j = 0; j < 3; ++j) {
-      int v = cnt[j];
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int u = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= o) v += u;
-      }
-      const int s = lane + 32 * j;
-      if (s <= nseg) it.first[s] = base + v - cnt[j];
-      base += __shfl_sync(0xffffffffu, v, 31);
-    }
-    const bool any_bad = __any_sync(0xffffffffu, bad);
-    if (lane == 0) {
-      if (any_bad) {  // the other segments still run; later kernels of the call skip their work
-        set_error(a.err, kErrInvalid);
-        const_cast<WsHeader*>(a.hdr)->abort = 1;
-      }
-      it.nseg = nseg;
-      it.ksplit = ksplit;
-      it.total = base;
-    }
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
+  const unsigned long long hits = a.ready ? *a.ready : 0ull;
+  for (int j = 0; j < 3; ++j) {
+    const int s = lane + 32 * j;
+    if (s <= nseg) it.off[s] = a.off[s];
   }
-  __syncthreads();
+  __syncwarp();
+  bool bad = false;
+  int key[3];  // token count of a segment with work, else -1
+  unsigned work[3];
+  for (int j = 0; j < 3; ++j) {
+    const int s = lane + 32 * j;
+    key[j] = -1;
+    if (s < nseg) {
+      const char* b = reinterpret_cast<const char*>(seg_block(a, s));
+      it.blk[s] = b;
+      const int n = it.off[s + 1] - it.off[s];
+      if (n > 0 && seg_in_phase(a, s, hits)) {
+        if (b == nullptr) bad = true;  // a selected expert without weights
+        else key[j] = n;
+      }
+    }
+    work[j] = __ballot_sync(full, key[j] >= 0);
+  }
+  const int npos = __popc(work[0]) + __popc(work[1]) + __popc(work[2]);
+  // position of each segment with work: those before it have more tokens, or as many and a lower
+  // index (a strict total order, so the positions are 0 .. npos - 1, each taken once)
+  int rank[3] = {0, 0, 0};
+  for (int j2 = 0; j2 < 3; ++j2)
+    for (unsigned m = work[j2]; m != 0u; m &= m - 1u) {
+      const int src = __ffs(m) - 1, t = src + 32 * j2;
+      const int kt = __shfl_sync(full, key[j2], src);
+#pragma unroll
+      for (int j = 0; j < 3; ++j)
+        rank[j] += (kt > key[j] || (kt == key[j] && t < lane + 32 * j)) ? 1 : 0;
+    }
+  for (int j = 0; j < 3; ++j)
+    if (key[j] >= 0) {
+      it.seg[rank[j]] = lane + 32 * j;
+      it.first[rank[j]] = items_per_seg * ksplit;  // the item count, until the scan below
+    }
+  __syncwarp();
+  int base = 0;
+  for (int j = 0; j < 3; ++j) {
+    const int p = lane + 32 * j;
+    const int c = p < npos ? it.first[p] : 0;
+    int v = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int u = __shfl_up_sync(full, v, o);
+      if (lane >= o) v += u;
+    }
+    if (p <= npos) it.first[p] = base + v - c;
+    base += __shfl_sync(full, v, 31);
+  }
+  const bool any_bad = __any_sync(full, bad);
+  if (lane == 0) {
+    if (any_bad) {  // the other segments still run; later kernels of the call skip their work
+      set_error(a.err, kErrInvalid);
+      const_cast<WsHeader*>(a.hdr)->abort = 1;
+    }
+    it.npos = npos;
+    it.ksplit = ksplit;
+    it.total = base;
+  }
 }
 
-__device__ __forceinline__ int dec_seg(const DecItems& it, int item) {
-  int s = 0;
-  while (s + 1 < it.nseg && it.first[s + 1] <= item) ++s;
-  return s;
+// Position in the work list of an item (< it.total): the last position whose first item is at or
+// before it.
+__device__ __forceinline__ int dec_pos(const DecItems& it, int item) {
+  int lo = 0, hi = it.npos - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (it.first[mid] <= item) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
 }
 
 __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
@@ -341,8 +373,8 @@ template <int MAXNG, bool DBOK = true>
 __device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, int item, int RB,
                                           float* red) {
   const int KS = kWarps / RB;
-  const int s = dec_seg(it, item);
-  const int r0 = (item - it.first[s]) * kRows * RB;
+  const int p = dec_pos(it, item), s = it.seg[p];
+  const int r0 = (item - it.first[p]) * kRows * RB;
   const char* blk = it.blk[s];
   const void* lblk = a.lrank ? a.lblk[s] : nullptr;
   // passes of at most 8 * MAXNG tokens; a later pass re-reads the rows from L2, not HBM
@@ -361,8 +393,8 @@ template <int MAXNG, bool DBOK = true>
 __device__ __forceinline__ void run2_item(const FfnArgs& a, const DecItems& it, int item, int RB,
                                           float* red) {
   const int KS = kWarps / RB;
-  const int s = dec_seg(it, item);
-  const int local = item - it.first[s];
+  const int p = dec_pos(it, item), s = it.seg[p];
+  const int local = item - it.first[p];
   const int r0 = (local / it.ksplit) * kRows2 * RB, kp = local % it.ksplit;
   const char* blk = it.blk[s];
   const void* lblk = a.lrank ? a.lblk[s] : nullptr;
@@ -381,7 +413,8 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  build_dec_items(it, a, a.w / (kRows * RB), 1);
+  if (threadIdx.x < 32) build_dec_items(it, a, a.w / (kRows * RB), 1);
+  __syncthreads();
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) run13_item<MAXNG>(a, it, item, RB, red);
 }
 
@@ -391,7 +424,8 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  build_dec_items(it, a, a.d / (kRows2 * RB), a.ksplit);
+  if (threadIdx.x < 32) build_dec_items(it, a, a.d / (kRows2 * RB), a.ksplit);
+  __syncthreads();
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) run2_item<MAXNG>(a, it, item, RB, red);
 }
 
@@ -421,40 +455,52 @@ __device__ bool wait_segment(const FfnArgs& a, int s, int need) {
   return true;
 }
 
-// GEMM13 and GEMM2 of a decode call in one cooperative launch: the work list is every GEMM13 item,
-// then every GEMM2 item, walked with static striding by a grid that is entirely resident (the
-// cooperative launch guarantees it). A GEMM13 item publishes its segment's progress after its h
-// rows are written and fenced; a GEMM2 item first waits (bounded) until its segment's GEMM13 items
-// are all done, then reads h through L2. Every wait is on items with lower indices, which CTAs
-// that are already running process before any item of their own that could wait, so the waits
-// always end. One launch instead of two, and a segment's GEMM2 overlaps other segments' GEMM13.
-// Used when nothing of ours runs alongside (mcft_moe_forward): a cooperative grid only starts
-// once all of its CTAs fit, so next to the expert fetch kernel it would wait for the fetch.
+// GEMM13 and GEMM2 of a decode call in one launch. The work list is every GEMM13 item, then every
+// GEMM2 item; CTAs claim items from a counter in the workspace (one atomic per item, issued for the
+// next item while the current one runs), so CTAs that finish early take more and the launch ends
+// when the work does, and CTAs that start late (an expert fetch kernel holding part of the SMs)
+// only take what is left. A GEMM13 item publishes its segment's progress after its h rows are
+// written and fenced; a GEMM2 item first waits (bounded) until its segment's GEMM13 items are all
+// done, then reads h through L2. The waits always end: every GEMM13 item precedes every GEMM2 item
+// in the claim order, so when a GEMM2 item is claimed its segment's GEMM13 items have all been
+// claimed, each by a CTA that is running and finishes it without waiting on anything.
 template <int MAXNG>
 __global__ void __launch_bounds__(kWarps * 32, 2)
     dec_fused_kernel(const __grid_constant__ FfnArgs a, int RB13, int RB2) {
   pdl_wait();
   __shared__ DecItems it13, it2;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  __shared__ int s_ok;
-  build_dec_items(it13, a, a.w / (kRows * RB13), 1);
-  build_dec_items(it2, a, a.d / (kRows2 * RB2), a.ksplit);
-  const int n13 = it13.total, total = n13 + it2.total;
-  const int per13 = a.w / (kRows * RB13);  // GEMM13 items of every segment that has work
-  for (int item = blockIdx.x; item < total; item += gridDim.x) {
-    if (item < n13) {
+  __shared__ int s_next, s_ok;
+  const int warp = threadIdx.x >> 5;
+  if (warp == 0) build_dec_items(it13, a, a.w / (kRows * RB13), 1);
+  else if (warp == 1) build_dec_items(it2, a, a.d / (kRows2 * RB2), a.ksplit);
+  else if (threadIdx.x == 64) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
+  __syncthreads();
+  // Only the next claim stays live across an item body (the item index is consumed at its start;
+  // the bounds are re-read from shared memory). Thread 0 issues the claim before the body and
+  // publishes it after, so the atomic's round trip overlaps warp 0's weight loads.
+  for (;;) {
+    const int item = s_next;
+    __syncthreads();  // every thread has read it before thread 0 publishes the next
+    if (item < 0 || item >= it13.total + it2.total) break;
+    int next = 0;
+    if (threadIdx.x == 0) next = atomicAdd(a.done + a.nseg + a.phase, 1);
+    if (item < it13.total) {
       const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, RB13, red);
       __threadfence();  // this CTA's h rows, before the segment's count moves
       __syncthreads();
       if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
     } else {
-      const int i2 = item - n13;
-      if (threadIdx.x == 0) s_ok = wait_segment(a, dec_seg(it2, i2), per13) ? 1 : 0;
+      const int i2 = item - it13.total;
+      // every segment with work has w / (16 RB13) GEMM13 items
+      if (threadIdx.x == 0)
+        s_ok = wait_segment(a, it2.seg[dec_pos(it2, i2)], a.w / (kRows * RB13)) ? 1 : 0;
       __syncthreads();
       const int ok = s_ok;
-      __syncthreads();
       if (ok) run2_item<MAXNG, kFusedDB>(a, it2, i2, RB2, red);
     }
+    if (threadIdx.x == 0) s_next = next;
+    __syncthreads();
   }
 }
 
@@ -467,44 +513,37 @@ int blocks_per_sm(const void* fn) {
 
 }  // namespace
 
-int decode_ksplit(int T) { return T <= 4 ? 4 : (T <= 16 ? 2 : 1); }
+int decode_ksplit(int T) { return T <= 4 ? 8 : (T <= 16 ? 2 : 1); }
 
 // Row blocks per CTA item: the smallest RB in {1, 2, 4, 8} whose 8 / RB contraction slices give
-// every warp at least 8 chunks of 64 (while the rows still split into whole items). More slices
-// mean finer items and better balance; fewer mean longer, better pipelined loops.
-int rows_per_item(int rows, int contraction, int rows_per_warp) {
+// every warp at least min_chunks chunks of 64 (while the rows still split into whole items). More
+// slices mean finer items and better balance; fewer mean longer, better pipelined loops.
+constexpr int kMinChunks = 8;
+int rows_per_item(int rows, int contraction, int rows_per_warp, int min_chunks = kMinChunks) {
   const int nch = contraction / kChunk;
   int rb = 1;
-  while (rb < kWarps && nch / (kWarps / rb) < 8 && rows % (rows_per_warp * rb * 2) == 0) rb *= 2;
+  while (rb < kWarps && nch / (kWarps / rb) < min_chunks && rows % (rows_per_warp * rb * 2) == 0)
+    rb *= 2;
   return rb;
 }
 
 template <int MAXNG>
 cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int stages,
-                             int displaced) {
+                             int reserved) {
   static const int nb13 = blocks_per_sm(reinterpret_cast<const void*>(dec13_kernel<MAXNG>));
   static const int nb2 = blocks_per_sm(reinterpret_cast<const void*>(dec2_kernel<MAXNG>));
-  // one CTA per SM slot, less the slots that concurrently running CTAs of another kernel take
-  const int g13 = max(num_sms, num_sms * nb13 - displaced);
-  const int g2 = max(num_sms, num_sms * nb2 - displaced);
+  // one CTA per SM slot, less the slots left to another kernel
+  const int g13 = max(num_sms, num_sms * nb13 - reserved);
+  const int g2 = max(num_sms, num_sms * nb2 - reserved);
   const int rb13 = rows_per_item(a.w, a.d, kRows);
   const int rb2 = rows_per_item(a.d, a.w / a.ksplit, kRows2);
   cudaError_t e = cudaSuccess;
   if (stages == 3 && a.done && a.lrank == 0) {
-    // both GEMMs in one cooperative launch (every CTA resident: its waits always end)
+    // both GEMMs in one launch with claimed items
     static const int nbf = blocks_per_sm(reinterpret_cast<const void*>(dec_fused_kernel<MAXNG>));
-    const int gf = max(num_sms, num_sms * nbf - displaced);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(gf);
-    cfg.blockDim = dim3(kWarps * 32);
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    const int gf = max(num_sms, num_sms * nbf - reserved);
     prof_begin(kProfDecFused, s);
-    e = cudaLaunchKernelEx(&cfg, dec_fused_kernel<MAXNG>, a, rb13, rb2);
+    e = launch_pdl(dec_fused_kernel<MAXNG>, dim3(gf), dim3(kWarps * 32), 0, s, a, rb13, rb2);
     prof_end(kProfDecFused, s);
     return e != cudaSuccess ? e : cudaGetLastError();
   }
@@ -522,11 +561,11 @@ cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int 
 }
 
 cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages,
-                              int displaced) {
+                              int reserved) {
   // a segment holds at most T tokens (routed experts: distinct per token; shared: all T)
-  if (a.T <= 8) return launch_decode_ng<1>(a, num_sms, s, stages, displaced);
-  if (a.T <= 16) return launch_decode_ng<2>(a, num_sms, s, stages, displaced);
-  return launch_decode_ng<4>(a, num_sms, s, stages, displaced);
+  if (a.T <= 8) return launch_decode_ng<1>(a, num_sms, s, stages, reserved);
+  if (a.T <= 16) return launch_decode_ng<2>(a, num_sms, s, stages, reserved);
+  return launch_decode_ng<4>(a, num_sms, s, stages, reserved);
 }
 
 }  // namespace mcft

@@ -56,6 +56,10 @@ struct RouteArgs {
 cudaError_t launch_route(const RouteArgs& a, int dtype, cudaStream_t s);
 
 // Header at the start of the forward workspace.
+// Work-claim counters of the fused decode FFN that follow the per-segment progress counters in
+// the workspace: one per FFN phase (0 all segments, 1 hits, 2 misses).
+constexpr int kClaimSlots = 4;
+
 struct WsHeader {
   int abort;     // set when a kernel of this call found bad data; later kernels skip their work
   int nseg;      // E + n_shared
@@ -119,7 +123,7 @@ struct PermuteArgs {
   int* pos;    // [T*K] permuted row of assignment (t, k)
   int* perm;   // [mcap] token of each permuted row, -1 for padding
   unsigned* err;
-  int* done;   // [E+S] completed GEMM13 work items per segment (fused decode FFN), zeroed here
+  int* done;   // [E+S + kClaimSlots] progress and claim counters of the fused decode FFN, zeroed here
 };
 cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s);
 
@@ -156,8 +160,9 @@ struct FfnArgs {
   float lscale;
   const float* u13;
   const float* u2;
-  // [E+S] completed GEMM13 items per segment (zeroed by the permutation of the call): lets one
-  // fused decode launch start a segment's GEMM2 as soon as that segment's h is written
+  // [E+S] completed GEMM13 items per segment, then kClaimSlots work-claim counters (one per
+  // phase), all zeroed by the permutation of the call: they let one fused decode launch hand out
+  // its items dynamically and start a segment's GEMM2 as soon as that segment's h is written
   int* done;
 };
 
@@ -199,10 +204,10 @@ __device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned l
 // stages: bit 0 = GEMM13 (+ SwiGLU), bit 1 = GEMM2
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s,
                                int stages = 3);  // fp32
-// displaced: CTA slots taken by another kernel running at the same time (the expert fetch); the
-// persistent grid is that much smaller, so every CTA is resident from the start.
+// reserved: CTA slots left free for another kernel that may run at the same time (the expert
+// fetch, which otherwise could not start until the FFN's CTAs exit).
 cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages = 3,
-                              int displaced = 0);  // bf16, T <= 64
+                              int reserved = 0);  // bf16, T <= 64
 int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
 cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
                           int stages = 3);

@@ -29,7 +29,8 @@ __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant
     else atomicAdd(&hist[e], 1);
   }
   __syncthreads();
-  if (a.done && tid < nseg) a.done[tid] = 0;  // on every path, the abort path included
+  // progress and claim counters: on every path, the abort path included
+  if (a.done && tid < nseg + kClaimSlots) a.done[tid] = 0;
   if (bad) {
     if (tid == 0) {
       a.hdr->abort = 1;

@@ -73,8 +73,8 @@ __device__ inline void permute_one_warp(const PermuteArgs& a) {
   const int n = a.K, nseg = a.E + a.S;
   const int e = lane < n ? a.idx[lane] : -1;
   const bool bad = __any_sync(0xffffffffu, lane < n && (e < 0 || e >= a.E));
-  if (a.done)  // on every path, the abort path included
-    for (int sg = lane; sg < nseg; sg += 32) a.done[sg] = 0;
+  if (a.done)  // progress and claim counters: on every path, the abort path included
+    for (int sg = lane; sg < nseg + kClaimSlots; sg += 32) a.done[sg] = 0;
   const unsigned peers = __match_any_sync(0xffffffffu, e);
   int vals[kMaxK];  // every lane sees the token's K expert ids
 #pragma unroll
