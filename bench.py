@@ -44,12 +44,12 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "dc1fee43f4e052a7", 1.0020,
-                     "profiles/ffn_decode_mixtral_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "dc1fee43f4e052a7", 1.0048,
-                    "profiles/ffn_decode_mixtral_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "dc1fee43f4e052a7", 1.0016,
-                   "profiles/ffn_decode_mixtral_decode.md"),
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f87e9b340d17c731", None,
+                     "profiles/dec_fused_kernel_decode.md"),
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f87e9b340d17c731", None,
+                    "profiles/dec_fused_kernel_decode.md"),
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f87e9b340d17c731", 1.0018,
+                   "profiles/dec_fused_kernel_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "71e2bb67dbc90a66", 0.9566,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
 }
@@ -649,12 +649,13 @@ def _config(batch):
 
 def profile_case(case: str, dev) -> int:
     """A few forwards: the small launch sequences that ncu captures. decode16 / decode1:
-    Mixtral-shaped decode at batch 16 / 1 with every expert resident (decode FFN); prefill:
-    T = 4096 tokens, hard mask keep 4 of 8 (tcgen05 GEMMs); fetch16: three decode steps at batch
-    16 through the cache with the device-driven fetch (fetch kernel)."""
+    Mixtral-shaped decode at batch 16 / 1 with every expert resident (decode FFN); ds_decode1 /
+    ds_decode64: the same for the DeepSeek-V2-Lite shape at batch 1 / 64; prefill: T = 4096
+    tokens, hard mask keep 4 of 8 (tcgen05 GEMMs); fetch16: three decode steps at batch 16 through
+    the cache with the device-driven fetch (fetch kernel)."""
     from paper_2609_34077_gb300 import mcft as M
 
-    sh = I.MIXTRAL
+    sh = I.DSV2_LITE if case.startswith("ds_") else I.MIXTRAL
     desc = M.desc_of(sh)
     if case == "fetch16":  # decode steps with the cache and the device-driven fetch
         L = DecodeLayer(sh, 16, 7, dev)
@@ -674,17 +675,19 @@ def profile_case(case: str, dev) -> int:
         keep = [int(e) for e in np.nonzero(kw["mask"])[0]]
         x = I.hidden_iid(7, sh, T).to(dev)
     else:
-        T, mode = (16 if case == "decode16" else 1), M.MCFT_ROUTE_SOFT_PRIOR
+        T = {"decode16": 16, "decode1": 1, "ds_decode1": 1, "ds_decode64": 64}[case]
+        mode = M.MCFT_ROUTE_SOFT_PRIOR
         kw = dict(prior=I.prior_from_mask(I.keep_mask(7, sh.E, sh.keep)))
         keep = list(range(sh.E))
         x = I.ar1_streams(7, sh, 1, T)[0].to(dev)
     lw = I.layer_weights(7, sh, experts=keep)
     experts = [None if b is None else b.to(dev) for b in lw.experts]
+    shared = [b.to(dev) for b in lw.shared]
     wr = lw.router.to(dev)
     ws = torch.empty(M.mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=dev)
     for _ in range(3):
         idx, gate = M.mcft_route(desc, x, wr, mode, **kw)
-        y = M.mcft_moe_forward(desc, x, idx, gate, experts, workspace=ws)
+        y = M.mcft_moe_forward(desc, x, idx, gate, experts, shared, workspace=ws)
     M.mcft_device_error()
     torch.cuda.synchronize()
     print(json.dumps({"case": case, "T": T, "y_abs_mean": float(y.float().abs().mean())}))
@@ -700,7 +703,8 @@ def main():
     ap.add_argument("--batch", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
-    ap.add_argument("--case", choices=["decode16", "decode1", "prefill", "fetch16"],
+    ap.add_argument("--case", choices=["decode16", "decode1", "ds_decode1", "ds_decode64", "prefill",
+                                       "fetch16"],
                     help="run only a few resident-expert forwards (for profiler captures)")
     ap.add_argument("--workload", default="layer",
                     choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2"],
