@@ -37,7 +37,7 @@ constexpr int kPassTokens = 32;  // tokens per pass (4 MMA column groups of 8)
 constexpr int kMaxNG = kPassTokens / 8;
 
 struct DecItems {
-  int npos, total, ksplit;
+  int npos, total, ksplit, rb;  // rb: row blocks per item
   int off[kMaxSeg + 1];    // by segment: permuted-row offsets
   const char* blk[kMaxSeg];
   int seg[kMaxSeg];        // by position in the work list: segment
@@ -45,12 +45,15 @@ struct DecItems {
 };
 
 // Work list of a launch, built by one warp (the calling one) with one lane per segment (segments
-// s = lane, lane + 32, lane + 64): items_per_seg items for every non-empty segment of the phase,
-// segments in decreasing order of their token counts (ties by index), so that the items that take
-// longest (segments that need a second pass or more MMA columns) are handed out first and the
-// last ones are short. Only segments with work get a position. The caller synchronises the block
-// before reading it.
-__device__ void build_dec_items(DecItems& it, const FfnArgs& a, int items_per_seg, int ksplit) {
+// s = lane, lane + 32, lane + 64): for every non-empty segment of the phase, its rows in items of
+// rb blocks of rows_per_block rows, times ksplit contraction parts; segments in decreasing order
+// of their token counts (ties by index), so that the items that take longest (segments that need
+// a second pass or more MMA columns) are handed out first and the last ones are short. Only
+// segments with work get a position. rb starts at the caller's value and is halved while the list
+// would hold fewer than min_items items (few selected experts: finer items spread them over more
+// CTAs and shorten the launch's critical path). The caller synchronises the block before reading.
+__device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int rows_per_block,
+                                int rb, int ksplit, int min_items) {
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
@@ -78,6 +81,8 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int items_per_se
     work[j] = __ballot_sync(full, key[j] >= 0);
   }
   const int npos = __popc(work[0]) + __popc(work[1]) + __popc(work[2]);
+  while (rb > 1 && npos * ksplit * (rows / (rows_per_block * rb)) < min_items) rb >>= 1;
+  const int items_per_seg = rows / (rows_per_block * rb);
   // position of each segment with work: those before it have more tokens, or as many and a lower
   // index (a strict total order, so the positions are 0 .. npos - 1, each taken once)
   int rank[3] = {0, 0, 0};
@@ -116,6 +121,7 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int items_per_se
     }
     it.npos = npos;
     it.ksplit = ksplit;
+    it.rb = rb;
     it.total = base;
   }
 }
@@ -370,9 +376,9 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
 // One GEMM13 work item (RB blocks of 16 rows of one segment, all its tokens in passes of at most
 // 8 * MAXNG); returns the segment.
 template <int MAXNG, bool DBOK = true>
-__device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, int item, int RB,
+__device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, int item,
                                           float* red) {
-  const int KS = kWarps / RB;
+  const int RB = it.rb, KS = kWarps / RB;
   const int p = dec_pos(it, item), s = it.seg[p];
   const int r0 = (item - it.first[p]) * kRows * RB;
   const char* blk = it.blk[s];
@@ -390,9 +396,9 @@ __device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, 
 
 // One GEMM2 work item (RB blocks of 32 rows of W2 of one segment, one contraction part).
 template <int MAXNG, bool DBOK = true>
-__device__ __forceinline__ void run2_item(const FfnArgs& a, const DecItems& it, int item, int RB,
+__device__ __forceinline__ void run2_item(const FfnArgs& a, const DecItems& it, int item,
                                           float* red) {
-  const int KS = kWarps / RB;
+  const int RB = it.rb, KS = kWarps / RB;
   const int p = dec_pos(it, item), s = it.seg[p];
   const int local = item - it.first[p];
   const int r0 = (local / it.ksplit) * kRows2 * RB, kp = local % it.ksplit;
@@ -413,9 +419,9 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  if (threadIdx.x < 32) build_dec_items(it, a, a.w / (kRows * RB), 1);
+  if (threadIdx.x < 32) build_dec_items(it, a, a.w, kRows, RB, 1, 0);
   __syncthreads();
-  for (int item = blockIdx.x; item < it.total; item += gridDim.x) run13_item<MAXNG>(a, it, item, RB, red);
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) run13_item<MAXNG>(a, it, item, red);
 }
 
 template <int MAXNG>
@@ -424,9 +430,9 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  if (threadIdx.x < 32) build_dec_items(it, a, a.d / (kRows2 * RB), a.ksplit);
+  if (threadIdx.x < 32) build_dec_items(it, a, a.d, kRows2, RB, a.ksplit, 0);
   __syncthreads();
-  for (int item = blockIdx.x; item < it.total; item += gridDim.x) run2_item<MAXNG>(a, it, item, RB, red);
+  for (int item = blockIdx.x; item < it.total; item += gridDim.x) run2_item<MAXNG>(a, it, item, red);
 }
 
 constexpr uint64_t kSegWaitNs = 2000000000ull;
@@ -472,8 +478,9 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
   __shared__ int s_next, s_ok;
   const int warp = threadIdx.x >> 5;
-  if (warp == 0) build_dec_items(it13, a, a.w / (kRows * RB13), 1);
-  else if (warp == 1) build_dec_items(it2, a, a.d / (kRows2 * RB2), a.ksplit);
+  // GEMM13 items finer than RB13 when the launch has too few for its grid
+  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1, gridDim.x);
+  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit, 0);
   else if (threadIdx.x == 64) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
   __syncthreads();
   // Only the next claim stays live across an item body (the item index is consumed at its start;
@@ -486,18 +493,18 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
     int next = 0;
     if (threadIdx.x == 0) next = atomicAdd(a.done + a.nseg + a.phase, 1);
     if (item < it13.total) {
-      const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, RB13, red);
+      const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, red);
       __threadfence();  // this CTA's h rows, before the segment's count moves
       __syncthreads();
       if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
     } else {
       const int i2 = item - it13.total;
-      // every segment with work has w / (16 RB13) GEMM13 items
+      // every segment with work has w / (16 rb) GEMM13 items
       if (threadIdx.x == 0)
-        s_ok = wait_segment(a, it2.seg[dec_pos(it2, i2)], a.w / (kRows * RB13)) ? 1 : 0;
+        s_ok = wait_segment(a, it2.seg[dec_pos(it2, i2)], a.w / (kRows * it13.rb)) ? 1 : 0;
       __syncthreads();
       const int ok = s_ok;
-      if (ok) run2_item<MAXNG, kFusedDB>(a, it2, i2, RB2, red);
+      if (ok) run2_item<MAXNG, kFusedDB>(a, it2, i2, red);
     }
     if (threadIdx.x == 0) s_next = next;
     __syncthreads();

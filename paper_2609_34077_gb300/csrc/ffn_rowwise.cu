@@ -8,6 +8,8 @@
 //
 // combine: y[t] = sum_k gate[t,k] o[pos(t,k)] + sum_s o[shared row of t in segment E+s], summed in
 // k order then shared-expert order (deterministic).
+#include <type_traits>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -240,41 +242,75 @@ __global__ void __launch_bounds__(kWarps * 32) ffn2_kernel(const __grid_constant
   }
 }
 
-// Four consecutive outputs of one permuted row, summed over the partial planes in plane order.
-__device__ __forceinline__ float4 row_sum(const CombineArgs& a, size_t at) {
-  float4 v = *reinterpret_cast<const float4*>(a.o + at);
-  for (int p = 1; p < a.ks; ++p) {
-    const float4 u = *reinterpret_cast<const float4*>(a.o + size_t(p) * a.o_plane + at);
-    v.x += u.x; v.y += u.y; v.z += u.z; v.w += u.w;
-  }
-  return v;
-}
-
-template <typename TY>
+// y[t] = sum_k g[t,k] o[pos(t,k)] + sum_s o[shared row s of t] (Section 3.1), every o row first
+// summed over its partial planes in plane order, the rows in k order then shared order (a shared
+// row enters as fma(1, v, acc), which is exactly acc + v). The loads are what take time: each
+// thread takes its token's rows four at a time and issues the four index loads, then all 4 x KS
+// plane loads, before adding anything, so a row group costs two round trips to L2 instead of one
+// per row and plane. VEC outputs per thread: 4 (float4) while the planes are few, else 1 (more
+// threads for the same outputs, and registers for 4 rows x KS planes).
+template <typename TY, int KS, int VEC>
 __global__ void __launch_bounds__(256) combine_kernel(const __grid_constant__ CombineArgs a) {
+  using V = typename std::conditional<VEC == 4, float4, float>::type;
   pdl_wait();
   if (a.hdr->abort) return;
-  const int nq = a.d / 4;  // float4 columns per row
+  const int nq = a.d / VEC;  // vectors per output row
+  const int nr = a.K + a.S;
   const size_t total = size_t(a.T) * nq;
   for (size_t i = size_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
        i += size_t(gridDim.x) * blockDim.x) {
-    const int t = int(i / nq), c = int(i % nq) * 4;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int k = 0; k < a.K; ++k) {
-      const float g = a.gate[size_t(t) * a.K + k];
-      const float4 v = row_sum(a, size_t(a.pos[size_t(t) * a.K + k]) * a.d + c);
-      acc.x = fmaf(g, v.x, acc.x); acc.y = fmaf(g, v.y, acc.y);
-      acc.z = fmaf(g, v.z, acc.z); acc.w = fmaf(g, v.w, acc.w);
-    }
-    for (int s = 0; s < a.S; ++s) {
-      const float4 v = row_sum(a, size_t(a.off[a.E + s] + t) * a.d + c);
-      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    const int t = int(i / nq), c = int(i % nq) * VEC;
+    float acc[VEC];
+#pragma unroll
+    for (int e = 0; e < VEC; ++e) acc[e] = 0.f;
+    for (int r0 = 0; r0 < nr; r0 += 4) {
+      size_t row[4];
+      float g[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int r = r0 + j;
+        row[j] = 0;
+        g[j] = 1.f;
+        if (r < a.K) {
+          row[j] = size_t(a.pos[size_t(t) * a.K + r]);
+          g[j] = a.gate[size_t(t) * a.K + r];
+        } else if (r < nr) {
+          row[j] = size_t(a.off[a.E + r - a.K] + t);
+        }
+      }
+      V v[4][KS];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (r0 + j < nr)
+#pragma unroll
+          for (int p = 0; p < KS; ++p)
+            v[j][p] = *reinterpret_cast<const V*>(a.o + size_t(p) * a.o_plane + row[j] * a.d + c);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (r0 + j < nr) {
+          const float* f0 = reinterpret_cast<const float*>(&v[j][0]);
+          float sum[VEC];
+#pragma unroll
+          for (int e = 0; e < VEC; ++e) sum[e] = f0[e];
+#pragma unroll
+          for (int p = 1; p < KS; ++p) {
+            const float* f = reinterpret_cast<const float*>(&v[j][p]);
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) sum[e] += f[e];
+          }
+#pragma unroll
+          for (int e = 0; e < VEC; ++e) acc[e] = fmaf(g[j], sum[e], acc[e]);
+        }
     }
     if constexpr (sizeof(TY) == 4) {
-      *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.y) + size_t(t) * a.d + c) = acc;
+      float* y = reinterpret_cast<float*>(a.y) + size_t(t) * a.d + c;
+#pragma unroll
+      for (int e = 0; e < VEC; ++e) y[e] = acc[e];
+    } else if constexpr (VEC == 4) {
+      uint2 pk = make_uint2(pack2bf(acc[0], acc[1]), pack2bf(acc[2], acc[3]));
+      *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(a.y) + size_t(t) * a.d + c) = pk;
     } else {
-      uint2 p = make_uint2(pack2bf(acc.x, acc.y), pack2bf(acc.z, acc.w));
-      *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(a.y) + size_t(t) * a.d + c) = p;
+      reinterpret_cast<uint16_t*>(a.y)[size_t(t) * a.d + c] = f2bf(acc[0]);
     }
   }
 }
@@ -303,6 +339,25 @@ cudaError_t launch_rowwise_typed(const FfnArgs& a, int num_sms, cudaStream_t s, 
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+template <typename TY, int KS, int VEC>
+cudaError_t launch_combine_ks(const CombineArgs& a, cudaStream_t s) {
+  const size_t total = size_t(a.T) * (a.d / VEC);
+  size_t blocks = (total + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  return launch_pdl(combine_kernel<TY, KS, VEC>, dim3(unsigned(blocks)), dim3(256), 0, s, a);
+}
+
+template <typename TY>
+cudaError_t launch_combine_typed(const CombineArgs& a, cudaStream_t s) {
+  switch (a.ks) {  // the contraction splits of the decode GEMM2 (decode_ksplit) and 1
+    case 1: return launch_combine_ks<TY, 1, 4>(a, s);
+    case 2: return launch_combine_ks<TY, 2, 4>(a, s);
+    case 4: return launch_combine_ks<TY, 4, 1>(a, s);
+    case 8: return launch_combine_ks<TY, 8, 1>(a, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s, int stages) {
@@ -312,13 +367,9 @@ cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStr
 
 cudaError_t launch_combine(const CombineArgs& a, int dtype, cudaStream_t s) {
   if (a.T == 0) return cudaSuccess;
-  const size_t total = size_t(a.T) * (a.d / 4);
-  size_t blocks = (total + 255) / 256;
-  if (blocks > 4096) blocks = 4096;
   prof_begin(kProfCombine, s);
-  const cudaError_t e = dtype == MCFT_BF16
-      ? launch_pdl(combine_kernel<uint16_t>, dim3(unsigned(blocks)), dim3(256), 0, s, a)
-      : launch_pdl(combine_kernel<float>, dim3(unsigned(blocks)), dim3(256), 0, s, a);
+  const cudaError_t e = dtype == MCFT_BF16 ? launch_combine_typed<uint16_t>(a, s)
+                                           : launch_combine_typed<float>(a, s);
   prof_end(kProfCombine, s);
   return e != cudaSuccess ? e : cudaGetLastError();
 }
