@@ -30,6 +30,10 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
   __shared__ int32_t s_out[1 + 3 * kMaxE];  // n_miss, miss experts, miss locations, loc_of
   const int lane = threadIdx.x & 31;
   const int B = a.B, E = a.E;
+  // every global load of the step is issued up front (the layer's step and prefetch mask, then
+  // its slot state below), so the warp pays about one round trip for them, not one each
+  const int64_t t = a.step[a.layer];
+  const unsigned long long pf_in = a.pfmask[a.layer];
   unsigned long long mine = 0;
   int bad = 0;
   for (int i = lane; i < a.n; i += 32) {
@@ -67,13 +71,12 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
   __syncwarp();
   unsigned long long cached = 0, pf = 0;
   int hits = 0, nm = 0, nbyp = 0;
-  const int64_t t = a.step[a.layer];
   if (lane == 0) {
     int32_t* m_exp = s_out + 1;
     int32_t* m_loc = s_out + 1 + E;
     int32_t* loc_of = s_out + 1 + 2 * E;
     for (int e = 0; e < E; ++e) loc_of[e] = -1;
-    pf = a.pfmask[a.layer];
+    pf = pf_in;
     const unsigned long long drop = pf & ~mine;  // prefetched experts this step does not use
     for (int sl = 0; sl < B; ++sl) {
       const int e = s_tag[sl];
@@ -125,10 +128,10 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
     s_out[0] = nm;
     a.step[a.layer] = t + 1;
     unsigned long long* c = a.counters + size_t(a.layer) * kCacheCounters;
-    c[0] += hits;
-    c[1] += nm;
-    c[2] += nbyp;
-    c[4] += useful;
+    atomicAdd(c + 0, static_cast<unsigned long long>(hits));  // no value returned: no round trip
+    atomicAdd(c + 1, static_cast<unsigned long long>(nm));
+    atomicAdd(c + 2, static_cast<unsigned long long>(nbyp));
+    atomicAdd(c + 4, static_cast<unsigned long long>(useful));
     a.pfmask[a.layer] = 0;
   }
   cached = __shfl_sync(0xffffffffu, cached, 0);
@@ -159,7 +162,9 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) hitbits |= __shfl_xor_sync(0xffffffffu, hitbits, o);
   if (lane == 0) *a.ready = hitbits;
-  __threadfence_system();
+  // No fence: the FFN and fetch kernels read these after a kernel boundary (or an event), the host
+  // after synchronising on one; the running fetch kernel that polls the cancel mask only needs the
+  // write to arrive, in any order.
 }
 
 // Prefetch decision (one warp). The lanes count how many predicted (token, k) entries name each
@@ -171,6 +176,9 @@ __device__ inline void prefetch_warp(const PrefetchArgs& a) {
   __shared__ int64_t s_last[kMaxE], s_ins[kMaxE], s_freq[kMaxE];
   __shared__ int32_t s_list[1 + kMaxE];
   const int lane = threadIdx.x & 31, B = a.B, E = a.E;
+  // the layer's step and prefetch mask are loaded up front, beside the slot state below
+  const int64_t t = a.step[a.layer];
+  const unsigned long long pf_in = a.pfmask[a.layer];
   for (int e = lane; e < E; e += 32) {
     cnt[e] = 0;
     rank[e] = 1 << 30;
@@ -204,7 +212,6 @@ __device__ inline void prefetch_warp(const PrefetchArgs& a) {
   }
   for (int e = lane; e < E; e += 32) s_freq[e] = a.freq[size_t(a.layer) * E + e];
   __syncwarp();
-  const int64_t t = a.step[a.layer];
   // every cached candidate is touched; the loads are the n_max best-ranked uncached candidates by
   // (count descending, best rank ascending, id ascending): warp-parallel sets and a warp max over
   // one packed key per expert
@@ -234,7 +241,7 @@ __device__ inline void prefetch_warp(const PrefetchArgs& a) {
   }
   __syncwarp();
   if (lane == 0) {
-    unsigned long long pf = a.pfmask[a.layer];
+    unsigned long long pf = pf_in;
     int nl = 0;
     while (load) {
       const int e = __ffsll(static_cast<long long>(load)) - 1;
@@ -261,7 +268,7 @@ __device__ inline void prefetch_warp(const PrefetchArgs& a) {
     a.pfmask[a.layer] = pf;
     a.cancel[a.layer] = 0;
     a.step[a.layer] = t + 1;
-    a.counters[size_t(a.layer) * kCacheCounters + 3] += nl;
+    atomicAdd(a.counters + size_t(a.layer) * kCacheCounters + 3, static_cast<unsigned long long>(nl));
   }
   __syncwarp();
   for (int i = lane; i < B; i += 32) {

@@ -155,14 +155,17 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
   const int d = a.d, E = a.route.E;
   const int nr = a.gamma_next ? 2 : 1;
 
-  // 1. the stream row and its norm(s), in registers of the first 256 threads
-  float4 v[kRowVec];
+  // 1. the stream row and its norm(s), in registers of the first 256 threads; the scales are
+  //    loaded with the row (one round trip for all of it)
+  float4 v[kRowVec], gm[2][kRowVec];
   if (tid < kNormThreads) {
     float ss = 0.f;
 #pragma unroll
     for (int i = 0; i < kRowVec; ++i) {
       const int c = tid * 4 + i * 4 * kNormThreads;
       if (c < d) {
+        for (int q = 0; q < nr; ++q)
+          gm[q][i] = S::get4(reinterpret_cast<const ST*>(q ? a.gamma_next : a.gamma) + c);
         v[i] = *reinterpret_cast<const float4*>(a.x + c);
         if (a.y) {
           const float4 y = S::get4(reinterpret_cast<const ST*>(a.y) + c);
@@ -188,7 +191,7 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kThreads)
       const int c = tid * 4 + i * 4 * kNormThreads;
       if (c < d) {
         for (int q = 0; q < nr; ++q) {
-          const float4 g = S::get4(reinterpret_cast<const ST*>(q ? a.gamma_next : a.gamma) + c);
+          const float4 g = gm[q][i];
           S::put4(&us[q][c], make_float4(v[i].x * r * g.x, v[i].y * r * g.y, v[i].z * r * g.z,
                                         v[i].w * r * g.w));
         }
