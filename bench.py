@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f87e9b340d17c731", None,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "7948a218279da733", None,
                      "profiles/dec_fused_kernel_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f87e9b340d17c731", None,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "7948a218279da733", None,
                     "profiles/dec_fused_kernel_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "f87e9b340d17c731", 1.0018,
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "7948a218279da733", 1.0017,
                    "profiles/dec_fused_kernel_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "71e2bb67dbc90a66", 0.9566,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
@@ -307,6 +307,22 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, path="device", clo
         kernel_ms_per_step=sum(v[1] for k, v in prof.items() if k != "fetch") / steps,
     )
     return L, out, elapsed
+
+
+def alone_roofline(L, shape, batch, steps, first, peaks):
+    """The same decode steps with the host-driven fetch (the host reads the miss list, the copy
+    engine moves the experts): the expert FFN then runs alone on the GPU. Returns its roofline."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(True)
+    time_steps(lambda s: L.step(s, path="host"), first, steps, L.compute)
+    M.mcft_profile_enable(False)
+    prof = M.mcft_profile_read()
+    pos = [s % STREAM_STEPS for s in range(first, first + steps)]
+    roof, _ = decode_roofline(prof, unique_per_step([L.idx[p] for p in pos]), steps, batch, shape,
+                              peaks)
+    return dict(roof or {}, note="same FFN kernel in the host-driven step, where it runs alone")
 
 
 def run_decode_e2e(L, steps, first):
@@ -817,14 +833,21 @@ def main():
     del L
     torch.cuda.empty_cache()
     if not args.no_extra:
-        _, b1, _ = run_decode(shape, 1, min(args.steps, 256), args.warmup, seed + 1, dev, peaks)
+        nb1 = min(args.steps, 256)
+        Lb, b1, _ = run_decode(shape, 1, nb1, args.warmup, seed + 1, dev, peaks)
         b1.pop("kernels", None)
+        b1["roofline_alone"] = alone_roofline(Lb, shape, 1, nb1, args.warmup + nb1, peaks)
         line["batch1"] = b1
+        del Lb
         for bsz in (1, 64):
-            _, ds, _ = run_decode(I.DSV2_LITE, bsz, min(args.steps, 128), args.warmup, seed + 3,
-                                  dev, peaks)
+            nds = min(args.steps, 128)
+            Ld, ds, _ = run_decode(I.DSV2_LITE, bsz, nds, args.warmup, seed + 3, dev, peaks)
             ds.pop("kernels", None)
+            ds["roofline_alone"] = alone_roofline(Ld, I.DSV2_LITE, bsz, nds, args.warmup + nds,
+                                                  peaks)
             line[f"dsv2_b{bsz}"] = ds
+            del Ld
+            torch.cuda.empty_cache()
         line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)
     if rank == 0 and not args.no_cpu_baseline:
         tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0)
