@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "7948a218279da733", None,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", None,
                      "profiles/dec_fused_kernel_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "7948a218279da733", None,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", None,
                     "profiles/dec_fused_kernel_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "7948a218279da733", 1.0017,
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", 1.0016,
                    "profiles/dec_fused_kernel_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "71e2bb67dbc90a66", 0.9566,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),

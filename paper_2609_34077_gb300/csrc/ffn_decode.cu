@@ -49,11 +49,11 @@ struct DecItems {
 // rb blocks of rows_per_block rows, times ksplit contraction parts; segments in decreasing order
 // of their token counts (ties by index), so that the items that take longest (segments that need
 // a second pass or more MMA columns) are handed out first and the last ones are short. Only
-// segments with work get a position. rb starts at the caller's value and is halved while the list
-// would hold fewer than min_items items (few selected experts: finer items spread them over more
-// CTAs and shorten the launch's critical path). The caller synchronises the block before reading.
+// segments with work get a position. The item shape depends on the layer and the batch only, not
+// on which segments a launch computes, so an output is bit-identical whichever phase of a cached
+// forward computes it. The caller synchronises the block before reading the list.
 __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int rows_per_block,
-                                int rb, int ksplit, int min_items) {
+                                int rb, int ksplit) {
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
@@ -81,7 +81,6 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
     work[j] = __ballot_sync(full, key[j] >= 0);
   }
   const int npos = __popc(work[0]) + __popc(work[1]) + __popc(work[2]);
-  while (rb > 1 && npos * ksplit * (rows / (rows_per_block * rb)) < min_items) rb >>= 1;
   const int items_per_seg = rows / (rows_per_block * rb);
   // position of each segment with work: those before it have more tokens, or as many and a lower
   // index (a strict total order, so the positions are 0 .. npos - 1, each taken once)
@@ -419,7 +418,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec13_kernel(const __grid_cons
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  if (threadIdx.x < 32) build_dec_items(it, a, a.w, kRows, RB, 1, 0);
+  if (threadIdx.x < 32) build_dec_items(it, a, a.w, kRows, RB, 1);
   __syncthreads();
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) run13_item<MAXNG>(a, it, item, red);
 }
@@ -430,7 +429,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
   pdl_wait();
   __shared__ DecItems it;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  if (threadIdx.x < 32) build_dec_items(it, a, a.d, kRows2, RB, a.ksplit, 0);
+  if (threadIdx.x < 32) build_dec_items(it, a, a.d, kRows2, RB, a.ksplit);
   __syncthreads();
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) run2_item<MAXNG>(a, it, item, red);
 }
@@ -478,9 +477,8 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
   __shared__ int s_next, s_ok;
   const int warp = threadIdx.x >> 5;
-  // GEMM13 items finer than RB13 when the launch has too few for its grid
-  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1, gridDim.x);
-  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit, 0);
+  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1);
+  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit);
   else if (threadIdx.x == 64) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
   __syncthreads();
   // Only the next claim stays live across an item body (the item index is consumed at its start;

@@ -139,8 +139,9 @@ def test_ffn_empty_and_bad_ids():
     M.mcft_moe_forward(desc, x[:0], torch.empty((0, 2), dtype=torch.int32, device=DEV),
                        torch.empty((0, 2), device=DEV), ex, y=y0)
     M.mcft_device_error()
-    # an id out of range: the device error word is set and y is left untouched
-    for T in (16, 100):
+    # an id out of range: the device error word is set and y is left untouched (every decode
+    # kernel variant: 1, 16 and 64 tokens; and the tensor-core path)
+    for T in (1, 16, 64, 100):
         idx = torch.zeros((T, 2), dtype=torch.int32, device=DEV)
         idx[:, 1] = 1
         idx[T // 2, 1] = sh.E
@@ -151,7 +152,7 @@ def test_ffn_empty_and_bad_ids():
         assert ei.value.status == M.MCFT_ERR_INVALID
         assert torch.all(y == 7.0)
     # a selected expert with no weights
-    for T in (16, 100):
+    for T in (1, 16, 64, 100):
         idx = torch.zeros((T, 2), dtype=torch.int32, device=DEV)
         idx[:, 1] = 2
         missing = list(ex)

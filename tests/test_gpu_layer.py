@@ -102,3 +102,42 @@ def test_forward_cached_rejects_prefill_and_accounting_caches():
     g = torch.ones((1, 2), device=DEV)
     with pytest.raises(M.MCFTError):
         M.mcft_moe_forward_cached(desc, x, idx, g, acc, 0)
+
+
+@pytest.mark.parametrize("shape,T", [(SMALL_DS, 1), (SMALL_DS, 5), (SMALL_DS, 40), (SMALL_MIX, 16)],
+                         ids=["ds-b1", "ds-b5", "ds-b40", "mix-b16"])
+def test_cached_forward_equals_plain_forward_bitwise(shape, T):
+    """Where an expert's bytes come from does not change the bf16 decode output: a hit (first FFN
+    phase), a demand fetch or bypass (second phase), a prefetch still landing (second phase) and a
+    resident expert of the plain forward give the same bits, because the decode work items have
+    the same shape and summation order in every launch of a layer and batch size."""
+    desc = M.desc_of(shape)
+    lw = I.layer_weights(80, shape, pin=True)
+    cache = M.mcft_cache_create(1, shape.E, shape.cache_slots, shape.expert_bytes, lw.experts,
+                                max_assign=T * shape.K)
+    experts = [b.to(DEV) for b in lw.experts]
+    shared = [b.to(DEV) for b in lw.shared]
+    compute, copy = torch.cuda.Stream(), torch.cuda.Stream()
+    steps = 8
+    ids = I.random_ids(80, steps, T, shape.K, shape.E, hot=range(shape.keep), p_hot=0.8)
+    gates = np.random.default_rng(80).uniform(0.05, 1.0, (steps, T, shape.K)).astype(np.float32)
+    xs = [I.hidden_iid(81 + s, shape, T).to(DEV) for s in range(steps)]
+    idxs = [torch.from_numpy(ids[s]).to(DEV) for s in range(steps)]
+    gts = [torch.from_numpy(gates[s]).to(DEV) for s in range(steps)]
+    wsz = M.mcft_moe_workspace_size(desc, T)
+    ws_c, ws_p = (torch.empty(wsz, dtype=torch.uint8, device=DEV) for _ in range(2))
+    y_c, y_p = (torch.empty((T, shape.d), dtype=torch.bfloat16, device=DEV) for _ in range(2))
+    torch.cuda.synchronize()
+    for s in range(steps):
+        M.mcft_cache_step(cache, 0, idxs[s], stream=compute)
+        M.mcft_moe_forward_cached(desc, xs[s], idxs[s], gts[s], cache, 0, shared, y=y_c,
+                                  workspace=ws_c, compute_stream=compute, copy_stream=copy)
+        if s % 2 == 0 and s + 1 < steps:  # the next step then finds some experts still landing
+            M.mcft_cache_prefetch(cache, 0, idxs[s + 1], min(2, shape.cache_slots), stream=compute)
+        M.mcft_moe_forward(desc, xs[s], idxs[s], gts[s], experts, shared, y=y_p, workspace=ws_p,
+                           stream=compute)
+        compute.synchronize()
+        copy.synchronize()
+        assert torch.equal(y_c, y_p), f"step {s}"
+    M.mcft_device_error()
+    assert M.mcft_cache_stats(cache, 0)[1] > 0  # the stream did fetch
