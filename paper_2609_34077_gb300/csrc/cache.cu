@@ -1,7 +1,8 @@
 // Per-layer expert cache decision kernel (Section 4.1 "Simulation", Eq. metrics).
 //
 // One warp per call: the lanes gather the distinct experts of the step (a 64-bit set) from the
-// routing output, then lane 0 applies the replacement rule on the layer's device-resident tag,
+// routing output, then apply the replacement rule (each slot choice a warp-wide reduction, the
+// misses one at a time) on the layer's device-resident tag,
 // last-use, insertion and access-count arrays: every expert of the step counts one access, hits
 // refresh their last use, misses in ascending expert id take the lowest free slot or evict, among
 // slots not used this step, the smallest key of the policy (LRU: last use, expert id; LFU: access

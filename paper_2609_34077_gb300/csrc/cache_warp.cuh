@@ -9,19 +9,49 @@
 
 namespace mcft {
 
-// True when slot s precedes slot v in eviction order under the policy's key.
-__device__ __forceinline__ bool victim_before(int policy, int s, int v, const int32_t* tag,
+// Slot for an expert that enters at time stamp t, chosen by the whole warp (every lane returns the
+// same slot): the lowest free slot, else the victim among the slots not used at t, else -1. The
+// victim has the smallest key of the policy: (access count of its expert, last use, expert id) for
+// LFU, (last use, expert id) for LRU, (insertion, expert id) for FIFO, found by a warp arg-min over
+// one key per slot. Stamps of occupied slots are >= 0 and ids < 64, so a stamp and an id pack into
+// one 64-bit word; ids are distinct, so the minimum is unique.
+__device__ __forceinline__ int warp_pick_slot(int policy, int B, int64_t t, const int32_t* tag,
                                               const int64_t* last, const int64_t* ins,
                                               const int64_t* freq) {
-  if (policy == MCFT_CACHE_LFU) {
-    const int64_t fs = freq[tag[s]], fv = freq[tag[v]];
-    if (fs != fv) return fs < fv;
-  } else if (policy == MCFT_CACHE_FIFO) {
-    if (ins[s] != ins[v]) return ins[s] < ins[v];
-    return tag[s] < tag[v];
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const unsigned f0 = __ballot_sync(full, lane < B && tag[lane] < 0);
+  const unsigned f1 = __ballot_sync(full, lane + 32 < B && tag[lane + 32] < 0);
+  if (f0) return __ffs(f0) - 1;
+  if (f1) return 32 + __ffs(f1) - 1;
+  unsigned long long hi = ~0ull, lo = ~0ull;
+  int slot = -1;
+  for (int j = 0; j < 2; ++j) {
+    const int sl = lane + 32 * j;
+    if (sl < B && last[sl] < t) {  // no free slot: tag[sl] >= 0
+      const unsigned long long e = static_cast<unsigned long long>(tag[sl]);
+      const unsigned long long h =
+          policy == MCFT_CACHE_LFU ? static_cast<unsigned long long>(freq[e]) : 0ull;
+      const unsigned long long l =
+          (static_cast<unsigned long long>(policy == MCFT_CACHE_FIFO ? ins[sl] : last[sl]) << 8) | e;
+      if (h < hi || (h == hi && l < lo)) {
+        hi = h;
+        lo = l;
+        slot = sl;
+      }
+    }
   }
-  if (last[s] != last[v]) return last[s] < last[v];
-  return tag[s] < tag[v];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long h2 = __shfl_xor_sync(full, hi, o), l2 = __shfl_xor_sync(full, lo, o);
+    const int s2 = __shfl_xor_sync(full, slot, o);
+    if (h2 < hi || (h2 == hi && l2 < lo)) {
+      hi = h2;
+      lo = l2;
+      slot = s2;
+    }
+  }
+  return slot;
 }
 
 __device__ inline void cache_step_warp(const CacheStepArgs& a) {
@@ -69,53 +99,54 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
   }
   for (int e = lane; e < E; e += 32) s_freq[e] = freq[e] + ((mine >> e) & 1ull);
   __syncwarp();
-  unsigned long long cached = 0, pf = 0;
-  int hits = 0, nm = 0, nbyp = 0;
-  if (lane == 0) {
-    int32_t* m_exp = s_out + 1;
-    int32_t* m_loc = s_out + 1 + E;
-    int32_t* loc_of = s_out + 1 + 2 * E;
-    for (int e = 0; e < E; ++e) loc_of[e] = -1;
-    pf = pf_in;
-    const unsigned long long drop = pf & ~mine;  // prefetched experts this step does not use
-    for (int sl = 0; sl < B; ++sl) {
-      const int e = s_tag[sl];
-      if (e >= 0 && ((drop >> e) & 1ull)) {
-        s_tag[sl] = -1;
-        s_last[sl] = -1;
-        s_ins[sl] = -1;
-      }
+  // the replacement rule, warp-parallel over slots; misses one at a time in ascending id
+  int32_t* m_exp = s_out + 1;
+  int32_t* m_loc = s_out + 1 + E;
+  int32_t* loc_of = s_out + 1 + 2 * E;
+  const unsigned long long pf = pf_in;
+  const unsigned long long drop = pf & ~mine;  // prefetched experts this step does not use
+  for (int e = lane; e < E; e += 32) loc_of[e] = -1;
+  for (int sl = lane; sl < B; sl += 32) {
+    const int e = s_tag[sl];
+    if (e >= 0 && ((drop >> e) & 1ull)) {
+      s_tag[sl] = -1;
+      s_last[sl] = -1;
+      s_ins[sl] = -1;
     }
-    a.cancel[a.layer] = drop;
-    for (int sl = 0; sl < B; ++sl) {
-      const int e = s_tag[sl];
-      if (e < 0) continue;
-      cached |= 1ull << e;
-      if ((mine >> e) & 1ull) {
-        s_last[sl] = t;
-        loc_of[e] = sl;
-        ++hits;
-      }
+  }
+  if (lane == 0) a.cancel[a.layer] = drop;
+  __syncwarp();
+  unsigned long long cached = 0;
+  int hits = 0;
+  for (int sl = lane; sl < B; sl += 32) {
+    const int e = s_tag[sl];
+    if (e < 0) continue;
+    cached |= 1ull << e;
+    if ((mine >> e) & 1ull) {
+      s_last[sl] = t;
+      loc_of[e] = sl;
+      ++hits;
     }
-    const int useful = __popcll(pf & mine & cached);
-    unsigned long long miss = mine & ~cached;
-    while (miss) {
-      const int e = __ffsll(static_cast<long long>(miss)) - 1;  // ascending expert id
-      miss &= miss - 1;
-      int slot = -1;
-      for (int sl = 0; sl < B; ++sl)
-        if (s_tag[sl] < 0) { slot = sl; break; }
-      if (slot < 0) {
-        for (int sl = 0; sl < B; ++sl) {
-          if (s_last[sl] >= t) continue;  // used at this step: never a victim
-          if (slot < 0 || victim_before(a.policy, sl, slot, s_tag, s_last, s_ins, s_freq)) slot = sl;
-        }
-      }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    cached |= __shfl_xor_sync(0xffffffffu, cached, o);
+    hits += __shfl_xor_sync(0xffffffffu, hits, o);
+  }
+  __syncwarp();
+  const int useful = __popcll(pf & mine & cached);
+  unsigned long long miss = mine & ~cached;
+  int nm = 0, nbyp = 0;
+  while (miss) {
+    const int e = __ffsll(static_cast<long long>(miss)) - 1;  // ascending expert id
+    miss &= miss - 1;
+    const int slot = warp_pick_slot(a.policy, B, t, s_tag, s_last, s_ins, s_freq);
+    __syncwarp();
+    if (lane == 0) {
       m_exp[nm] = e;
       if (slot < 0) {
         m_loc[nm] = -1;
         loc_of[e] = B + nbyp;
-        ++nbyp;
       } else {
         s_tag[slot] = e;
         s_last[slot] = t;
@@ -123,8 +154,12 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
         m_loc[nm] = slot;
         loc_of[e] = slot;
       }
-      ++nm;
     }
+    if (slot < 0) ++nbyp;
+    ++nm;
+    __syncwarp();  // the next pick sees this slot taken
+  }
+  if (lane == 0) {
     s_out[0] = nm;
     a.step[a.layer] = t + 1;
     unsigned long long* c = a.counters + size_t(a.layer) * kCacheCounters;
@@ -134,8 +169,6 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
     atomicAdd(c + 4, static_cast<unsigned long long>(useful));
     a.pfmask[a.layer] = 0;
   }
-  cached = __shfl_sync(0xffffffffu, cached, 0);
-  pf = __shfl_sync(0xffffffffu, pf, 0);
   __syncwarp();
   // write back the state and publish the step's miss list and expert table (all lanes)
   for (int i = lane; i < B; i += 32) {
@@ -168,8 +201,9 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
 }
 
 // Prefetch decision (one warp). The lanes count how many predicted (token, k) entries name each
-// expert, touch the cached candidates and rank the uncached ones (warp max over packed keys);
-// lane 0 claims the slots in ascending id and the lanes write the fetch list.
+// expert, touch the cached candidates and rank the uncached ones (warp max over packed keys); the
+// loads then claim slots in ascending id (each slot a warp-wide choice) and the lanes write the
+// fetch list.
 __device__ inline void prefetch_warp(const PrefetchArgs& a) {
   __shared__ int cnt[kMaxE], rank[kMaxE];
   __shared__ int32_t s_tag[kMaxE];
@@ -240,30 +274,28 @@ __device__ inline void prefetch_warp(const PrefetchArgs& a) {
     load |= 1ull << (255u - (key & 255u));
   }
   __syncwarp();
-  if (lane == 0) {
-    unsigned long long pf = pf_in;
-    int nl = 0;
-    while (load) {
-      const int e = __ffsll(static_cast<long long>(load)) - 1;
-      load &= load - 1;
-      int slot = -1;
-      for (int sl = 0; sl < B; ++sl)
-        if (s_tag[sl] < 0) { slot = sl; break; }
-      if (slot < 0) {
-        for (int sl = 0; sl < B; ++sl) {
-          if (s_last[sl] >= t) continue;  // touched at this event: never a victim
-          if (slot < 0 || victim_before(a.policy, sl, slot, s_tag, s_last, s_ins, s_freq)) slot = sl;
-        }
-      }
-      if (slot < 0) continue;  // unreachable with n_max <= B; kept for safety
-      if (s_tag[slot] >= 0) pf &= ~(1ull << s_tag[slot]);
+  // slots for the loads, one at a time in ascending id (warp-parallel choice of each slot)
+  unsigned long long pf = pf_in;
+  int nl = 0;
+  while (load) {
+    const int e = __ffsll(static_cast<long long>(load)) - 1;
+    load &= load - 1;
+    const int slot = warp_pick_slot(a.policy, B, t, s_tag, s_last, s_ins, s_freq);
+    if (slot < 0) continue;  // unreachable with n_max <= B; kept for safety
+    const int old = s_tag[slot];
+    if (old >= 0) pf &= ~(1ull << old);
+    pf |= 1ull << e;
+    __syncwarp();  // every lane has read the slot before lane 0 rewrites it
+    if (lane == 0) {
       s_tag[slot] = e;
       s_last[slot] = t;
       s_ins[slot] = t;
-      pf |= 1ull << e;
       s_list[1 + nl] = e;
-      ++nl;
     }
+    ++nl;
+    __syncwarp();
+  }
+  if (lane == 0) {
     s_list[0] = nl;
     a.pfmask[a.layer] = pf;
     a.cancel[a.layer] = 0;
@@ -276,7 +308,6 @@ __device__ inline void prefetch_warp(const PrefetchArgs& a) {
     last[i] = s_last[i];
     ins[i] = s_ins[i];
   }
-  const int nl = s_list[0];
   for (int i = lane; i <= nl; i += 32) a.list[i] = s_list[i];
   for (int e = lane; e < E; e += 32) a.ptr_tab[e] = 0;
   __syncwarp();
