@@ -56,21 +56,34 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
                                 int rb, int ksplit) {
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
-  const int nseg = a.hdr->abort == 0 ? a.nseg : 0;
+  // every load first (abort flag, ready mask, offsets, block addresses: one round trip), then the
+  // abort flag applied
+  const int aborted = a.hdr->abort;
   const unsigned long long hits = a.ready ? *a.ready : 0ull;
+  int offv[3];
+  const char* blkv[3];
+#pragma unroll
   for (int j = 0; j < 3; ++j) {
     const int s = lane + 32 * j;
-    if (s <= nseg) it.off[s] = a.off[s];
+    offv[j] = s <= a.nseg ? a.off[s] : 0;
+    blkv[j] = s < a.nseg ? reinterpret_cast<const char*>(seg_block(a, s)) : nullptr;
+  }
+  const int nseg = aborted == 0 ? a.nseg : 0;
+#pragma unroll
+  for (int j = 0; j < 3; ++j) {
+    const int s = lane + 32 * j;
+    if (s <= nseg) it.off[s] = offv[j];
   }
   __syncwarp();
   bool bad = false;
   int key[3];  // token count of a segment with work, else -1
   unsigned work[3];
+#pragma unroll
   for (int j = 0; j < 3; ++j) {
     const int s = lane + 32 * j;
     key[j] = -1;
     if (s < nseg) {
-      const char* b = reinterpret_cast<const char*>(seg_block(a, s));
+      const char* b = blkv[j];
       it.blk[s] = b;
       const int n = it.off[s + 1] - it.off[s];
       if (n > 0 && seg_in_phase(a, s, hits)) {
