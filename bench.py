@@ -50,7 +50,7 @@ TRAFFIC = {
                     "profiles/dec_fused_kernel_decode.md"),
     "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", 1.0016,
                    "profiles/dec_fused_kernel_decode.md"),
-    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "71e2bb67dbc90a66", 0.9566,
+    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "ae0482332aaf7dee", 0.9558,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
 }
 
