@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", None,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e01b00e7fb48e6e5", None,
                      "profiles/dec_fused_kernel_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", None,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e01b00e7fb48e6e5", None,
                     "profiles/dec_fused_kernel_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "8952b420f1ec54fa", 1.0016,
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e01b00e7fb48e6e5", 1.0017,
                    "profiles/dec_fused_kernel_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "ae0482332aaf7dee", 0.9558,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
@@ -237,13 +237,16 @@ def unique_per_step(idx_steps):
 
 def decode_roofline(prof, U, steps, batch, shape, peaks):
     """HBM roofline of the decode FFN kernels. Algorithmic bytes per launch: the W1 and W3 rows
-    (GEMM13) or W2 rows (GEMM2) of every expert the step selected, read once, plus the token
-    activations in and out; the fused kernel (both GEMMs in one launch) reads all three. Returns
-    (dominant kernel's roofline dict, {kernel: GB/s})."""
-    sel = sum(U)
+    (GEMM13) or W2 rows (GEMM2) of every expert the step computes, read once (the routed experts
+    it selected and the shared experts, which every token uses), plus the token activations in and
+    out; the fused kernel (both GEMMs in one launch) reads all three. Returns (dominant kernel's
+    roofline dict, {kernel: GB/s})."""
+    S = shape.n_shared
+    sel = sum(U) + steps * S
     T, K, d, w = batch, shape.K, shape.d, shape.w
-    b13 = sel * 2 * w * d * 2 + steps * (T * d * 2 + T * K * w * 2)
-    b2 = sel * w * d * 2 + steps * T * K * (w * 2 + d * 4)
+    rows = T * (K + S)  # permuted rows per step: one per routed assignment and per shared expert
+    b13 = sel * 2 * w * d * 2 + steps * (T * d * 2 + rows * w * 2)
+    b2 = sel * w * d * 2 + steps * rows * (w * 2 + d * 4)
     alg = {"ffn13_decode": b13, "ffn2_decode": b2, "ffn_decode": b13 + b2}
     rates, best = {}, None
     for k, b in alg.items():
