@@ -60,9 +60,14 @@ def traffic_ratio(kernel):
 
     if kernel not in TRAFFIC:
         return None
-    src, digest, ratio, _ = TRAFFIC[kernel]
+    src, digest, ratio, summary = TRAFFIC[kernel]
     cur = hashlib.sha256(open(os.path.join(ROOT, src), "rb").read()).hexdigest()[:16]
-    return ratio if cur == digest else None
+    if cur != digest:
+        print(f"bench: {src} changed since the ncu capture in {summary} "
+              f"(sha {cur}, captured {digest}): traffic for {kernel} reported as null",
+              file=sys.stderr)
+        return None
+    return ratio
 
 
 # ------------------------------------------------------------------------------------------------
