@@ -264,7 +264,8 @@ mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, cons
  * step chose, reading the host memory directly over the host link; on compute_stream the
  * permutation and the FFN of the experts that were hits (and of the shared experts) run at the
  * same time; then compute_stream waits for the copies and computes the fetched experts and the
- * combine. Results equal mcft_moe_forward's with the same experts.
+ * combine. Results equal mcft_moe_forward's with the same experts, bit for bit (a decode work item
+ * has the same shape and summation order whichever launch computes its expert).
  * Section 3.1 Eq. topk (the layer); Section 1 and Section 3.1 "Preliminaries" (every miss is a fetch
  * from host memory).
  *   cache  created with host blocks (not accounting-only); its E and expert size match desc
