@@ -536,7 +536,11 @@ int decode_ksplit(int T) { return T <= 4 ? 8 : (T <= 16 ? 2 : 1); }
 // Row blocks per CTA item: the smallest RB in {1, 2, 4, 8} whose 8 / RB contraction slices give
 // every warp at least min_chunks chunks of 64 (while the rows still split into whole items). More
 // slices mean finer items and better balance; fewer mean longer, better pipelined loops.
+// At up to 4 tokens a launch is latency-bound (few items per CTA, each warp's chunks in series),
+// so GEMM13 items take half the minimum (finer items, each warp walking fewer chunks); beyond
+// that the longer loops pay. A function of the layer and the batch only, like every item shape.
 constexpr int kMinChunks = 8;
+constexpr int kMinChunksSmallBatch = 4;
 int rows_per_item(int rows, int contraction, int rows_per_warp, int min_chunks = kMinChunks) {
   const int nch = contraction / kChunk;
   int rb = 1;
@@ -553,7 +557,7 @@ cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int 
   // one CTA per SM slot, less the slots left to another kernel
   const int g13 = max(num_sms, num_sms * nb13 - reserved);
   const int g2 = max(num_sms, num_sms * nb2 - reserved);
-  const int rb13 = rows_per_item(a.w, a.d, kRows);
+  const int rb13 = rows_per_item(a.w, a.d, kRows, a.T <= 4 ? kMinChunksSmallBatch : kMinChunks);
   const int rb2 = rows_per_item(a.d, a.w / a.ksplit, kRows2);
   cudaError_t e = cudaSuccess;
   if (stages == 3 && a.done && a.lrank == 0) {
