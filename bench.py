@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
 # the source has changed since the capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e01b00e7fb48e6e5", None,
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None,
                      "profiles/dec_fused_kernel_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e01b00e7fb48e6e5", None,
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None,
                     "profiles/dec_fused_kernel_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e01b00e7fb48e6e5", 1.0017,
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", 1.0017,
                    "profiles/dec_fused_kernel_decode.md"),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "ae0482332aaf7dee", 0.9558,
               "profiles/fetch_kernel_mixtral_decode_b16.md"),
