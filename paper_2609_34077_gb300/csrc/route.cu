@@ -14,6 +14,8 @@
 // about one memory round trip instead of one per expert. Partial sums are reduced with shuffles
 // and added in shared memory in a fixed order; warp 0 ranks (two experts per lane, shuffle
 // arg-max) and writes idx / gate.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "internal.h"
 #include "route_warp.cuh"
@@ -21,7 +23,10 @@
 namespace mcft {
 namespace {
 
+namespace cg = cooperative_groups;
+
 constexpr int kWarps = 16;
+constexpr int kRouteCluster = 4;  // CTAs per token for routers of many experts
 
 template <typename TX>
 struct Chunk;  // 16 bytes of a row: 8 bf16 or 4 fp32
@@ -47,6 +52,37 @@ __host__ __device__ inline int route_parts(int E, int nchunk) {
   return p;
 }
 
+// One warp: the logit part of token row xrow over chunks [0, per_part) of expert row wp (16-byte
+// chunks, lane-strided, NCH chunks in flight per lane and pass, then a warp sum).
+template <typename TX, int NCH>
+__device__ __forceinline__ float router_dot(const char* xp, const char* wp, int per_part) {
+  using C = Chunk<TX>;
+  const int lane = threadIdx.x & 31;
+  float acc = 0.f;
+  for (int base = 0; base < per_part; base += 32 * NCH) {
+    uint4 xv[NCH], wv[NCH];
+#pragma unroll
+    for (int i = 0; i < NCH; ++i) {
+      const int c = base + i * 32 + lane;
+      if (c < per_part) {
+        xv[i] = ldg16(xp + size_t(c) * 16);
+        wv[i] = ldg16(wp + size_t(c) * 16);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < NCH; ++i) {
+      if (base + i * 32 + lane < per_part) {
+        float xf[C::n], wf[C::n];
+        C::unpack(xv[i], xf);
+        C::unpack(wv[i], wf);
+#pragma unroll
+        for (int j = 0; j < C::n; ++j) acc = fmaf(xf[j], wf[j], acc);
+      }
+    }
+  }
+  return warp_sum(acc);
+}
+
 // NCH = 16-byte chunks a lane keeps in flight per task and pass (2, 4 or 8).
 template <typename TX, int NCH>
 __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constant__ RouteArgs a) {
@@ -56,8 +92,7 @@ __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constan
   const int t = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E, d = a.d;
-  using C = Chunk<TX>;
-  const int nchunk = d / C::n;
+  const int nchunk = d / Chunk<TX>::n;
   const int parts = route_parts(E, nchunk);
   const int per_part = nchunk / parts;
 
@@ -68,29 +103,7 @@ __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constan
     const int e = task / parts, pt = task % parts;
     const char* xp = xrow + size_t(pt) * per_part * 16;
     const char* wp = wr + e * wrow + size_t(pt) * per_part * 16;
-    float acc = 0.f;
-    for (int base = 0; base < per_part; base += 32 * NCH) {
-      uint4 xv[NCH], wv[NCH];
-#pragma unroll
-      for (int i = 0; i < NCH; ++i) {
-        const int c = base + i * 32 + lane;
-        if (c < per_part) {
-          xv[i] = ldg16(xp + size_t(c) * 16);
-          wv[i] = ldg16(wp + size_t(c) * 16);
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < NCH; ++i) {
-        if (base + i * 32 + lane < per_part) {
-          float xf[C::n], wf[C::n];
-          C::unpack(xv[i], xf);
-          C::unpack(wv[i], wf);
-#pragma unroll
-          for (int j = 0; j < C::n; ++j) acc = fmaf(xf[j], wf[j], acc);
-        }
-      }
-    }
-    acc = warp_sum(acc);
+    const float acc = router_dot<TX, NCH>(xp, wp, per_part);
     if (lane == 0) part[e][pt] = acc;
   }
   __syncthreads();
@@ -105,12 +118,51 @@ __global__ void __launch_bounds__(kWarps * 32) route_kernel(const __grid_constan
   rank_and_gate_warp(a, zs, t);
 }
 
+// Routers of many experts (E >= 32, whole rows per task in route_kernel too): each token is one
+// 4-CTA thread-block cluster, one expert per warp instead of E / 16 in series, each logit computed
+// exactly as route_kernel computes it (router_dot over the whole row, then 0 + the logit, as its
+// sum over one part), written into the leader CTA's shared memory over distributed shared memory;
+// after one cluster barrier the leader's first warp ranks. The routing is bit-identical to
+// route_kernel's in a quarter of the serial dot products.
+template <typename TX, int NCH>
+__global__ void __cluster_dims__(kRouteCluster, 1, 1) __launch_bounds__(kWarps * 32)
+    route_cluster_kernel(const __grid_constant__ RouteArgs a) {
+  pdl_wait();
+  __shared__ float zs[kMaxE];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int crank = int(cluster.block_rank());
+  const int t = blockIdx.x / kRouteCluster;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int E = a.E, d = a.d;
+  const int nchunk = d / Chunk<TX>::n;
+  const char* xrow = reinterpret_cast<const char*>(a.x) + size_t(t) * d * sizeof(TX);
+  const char* wr = reinterpret_cast<const char*>(a.w_router);
+  const size_t wrow = size_t(d) * sizeof(TX);
+  float* lead = cluster.map_shared_rank(&zs[0], 0);
+  for (int e = crank * kWarps + warp; e < E; e += kRouteCluster * kWarps) {
+    const float acc = router_dot<TX, NCH>(xrow, wr + e * wrow, nchunk);
+    if (lane == 0) lead[e] = 0.f + acc;
+  }
+  cluster.sync();  // every logit is in the leader's shared memory
+  if (crank != 0 || warp != 0) return;
+  rank_and_gate_warp(a, zs, t);
+}
+
 template <typename TX>
 cudaError_t launch_typed(const RouteArgs& a, cudaStream_t s) {
   const int nchunk = a.d / Chunk<TX>::n;
   const int per_lane = (nchunk / route_parts(a.E, nchunk) + 31) / 32;  // chunks per lane and task
   dim3 grid(a.T), block(kWarps * 32);
   prof_begin(kProfRoute, s);
+  if (a.E >= 2 * kWarps) {  // whole rows per task: one cluster per token
+    const dim3 cgrid(a.T * kRouteCluster);
+    const cudaError_t e =
+        per_lane <= 2   ? launch_pdl(route_cluster_kernel<TX, 2>, cgrid, block, 0, s, a)
+        : per_lane <= 4 ? launch_pdl(route_cluster_kernel<TX, 4>, cgrid, block, 0, s, a)
+                        : launch_pdl(route_cluster_kernel<TX, 8>, cgrid, block, 0, s, a);
+    prof_end(kProfRoute, s);
+    return e != cudaSuccess ? e : cudaGetLastError();
+  }
   const cudaError_t e =
       per_lane <= 2   ? launch_pdl(route_kernel<TX, 2>, grid, block, 0, s, a)
       : per_lane <= 4 ? launch_pdl(route_kernel<TX, 4>, grid, block, 0, s, a)
