@@ -22,7 +22,7 @@
  *  - Calls are asynchronous on the given stream unless stated otherwise; a NULL stream is the
  *    legacy default stream.
  *  - Argument errors are found on the host and returned synchronously as MCFT_ERR_INVALID (or
- *    MCFT_ERR_UNSUPPORTED for shapes this build does not handle); nothing is launched then.
+ *    MCFT_ERR_UNSUPPORTED for shapes the library does not handle); nothing is launched then.
  *  - Errors found inside a kernel (an expert id out of range, a missing expert pointer, a wait that
  *    ran out of time) set a device error word and make the remaining kernels of that call skip
  *    their work; mcft_device_error() reads and clears it.
@@ -49,7 +49,7 @@ typedef enum {
   MCFT_ERR_OOM = 2,          /* a device or pinned host allocation failed */
   MCFT_ERR_CUDA = 3,         /* a CUDA runtime call failed; mcft_last_error() has the text */
   MCFT_ERR_TIMEOUT = 4,      /* a kernel's bounded wait ran out; the kernel returned early */
-  MCFT_ERR_UNSUPPORTED = 5   /* valid but outside what this build handles (e.g. E > 64) */
+  MCFT_ERR_UNSUPPORTED = 5   /* valid but outside what the library handles (e.g. E > 64) */
 } mcft_status;
 
 /* Routing rule. Section 3.1 Eq. topk / Section 3.2 Eq. stage1 / Section 3.2 Eq. inference. */
