@@ -603,6 +603,192 @@ def run_prefill(steps, warmup, seed, dev, peaks):
     return res
 
 
+def _flush_l2(buf):
+    buf.add_(1)  # writes 256 MB, twice the L2, so the next kernel starts from a cold L2
+
+
+def time_calls(fn, n, stream, flush=None):
+    """Mean device time (ms) of fn() over n calls, each bracketed by its own CUDA events on
+    `stream`; with `flush` given, the L2 is flushed before every call (outside the events)."""
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(n)]
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for a, b in evs:
+            if flush is not None:
+                _flush_l2(flush)
+            a.record(stream)
+            fn()
+            b.record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs) / n
+
+
+_BATCHES = {}
+
+
+def _masked_batch(sh, T, seed, dev):
+    """A fine-tuning batch under a hard mask keeping 75 % of the experts (compact ratio r = 75 %):
+    the mask, the kept experts' weights (others absent), x and the hard-mask routing. Built once
+    per shape and kept in _BATCHES for the LoRA and mask measurements (cleared by the caller)."""
+    key = (sh.name, T, seed, str(dev))
+    if key not in _BATCHES:
+        _BATCHES[key] = _make_masked_batch(sh, T, seed, dev)
+    return _BATCHES[key]
+
+
+def _make_masked_batch(sh, T, seed, dev):
+    from paper_2609_34077_gb300 import mcft as M
+
+    mask = I.keep_mask(seed, sh.E, sh.E * 3 // 4)
+    kept = [int(e) for e in np.nonzero(mask)[0]]
+    lw = I.layer_weights(seed, sh, experts=kept)
+    experts = [None if b is None else b.to(dev) for b in lw.experts]
+    shared = [b.to(dev) for b in lw.shared]
+    x = I.hidden_iid(seed, sh, T).to(dev)
+    desc = M.desc_of(sh)
+    idx, gate = M.mcft_route(desc, x, lw.router.to(dev), M.MCFT_ROUTE_HARD_MASK, mask=mask)
+    return desc, kept, experts, shared, x, idx, gate
+
+
+def run_lora(steps, warmup, seed, dev, peaks, rank=8, shapes=(I.MIXTRAL, I.DSV2_LITE), T=4096):
+    """The Stage-2 forward (experts of the fixed concentration set with rank-8 LoRA adapters,
+    alpha 16; the shared experts adapted too) against the plain forward on the same batch: T tokens
+    routed under a hard mask keeping 75 % of the experts. Both arms are timed in alternating
+    blocks with CUDA events, then one profiled pass of the LoRA arm gives its kernels' times."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    out = {}
+    stream = torch.cuda.current_stream(dev)
+    for sh in shapes:
+        desc, kept, experts, shared, x, idx, gate = _masked_batch(sh, T, seed, dev)
+        ad = [I.lora_block(seed, sh, e, rank).to(dev) if e in kept else None for e in range(sh.E)]
+        sad = [I.lora_block(seed, sh, ("shared", s), rank).to(dev) for s in range(sh.n_shared)]
+        ws = torch.empty(M.mcft_moe_workspace_size_lora(desc, rank, T), dtype=torch.uint8,
+                         device=dev)
+        y = torch.empty_like(x)
+        scale = 16.0 / rank
+
+        def plain(s):
+            M.mcft_moe_forward(desc, x, idx, gate, experts, shared, y=y, workspace=ws, stream=stream)
+
+        def lora(s):
+            M.mcft_moe_forward_lora(desc, x, idx, gate, experts, shared, ad, sad, rank, scale, y=y,
+                                    workspace=ws, stream=stream)
+
+        for s in range(warmup):
+            plain(s)
+            lora(s)
+        t_plain = t_lora = 0.0
+        blocks = 4
+        per = max(1, steps // blocks)
+        for _ in range(blocks):
+            t_plain += time_steps(plain, 0, per, stream)
+            t_lora += time_steps(lora, 0, per, stream)
+        n = blocks * per
+        profs = []
+        for fn in (plain, lora):
+            M.mcft_profile_reset()
+            M.mcft_profile_enable(True)
+            time_steps(fn, 0, n, stream)
+            M.mcft_profile_enable(False)
+            profs.append(M.mcft_profile_read())
+        prof_plain, prof = profs
+        M.mcft_device_error()
+        rows = T * (sh.K + sh.n_shared)  # permuted rows, all of them adapted
+        r, d, w = rank, sh.d, sh.w
+        # lora_down (two tcgen05 launches): every gathered row (x) and every h row read once,
+        # s [A1 x | A3 x] and s A2 h written in bf16
+        ld_bytes = rows * (d * 2 + 2 * r * 2) + rows * (w * 2 + r * 2)
+        f_base = 2.0 * rows * 3 * d * w
+        f_up = 2.0 * rows * (2 * w + d) * r  # the adapters' up projections (extra k-blocks)
+        f_down = 2.0 * rows * (2 * d + w) * r
+        nl, msl = prof.get("lora_down", (0, 0.0))
+        n13, ms13 = prof.get("gemm13_tc", (0, 0.0))
+        n2, ms2 = prof.get("gemm2_tc", (0, 0.0))
+        res = dict(workload=f"{sh.name} T={T} hard mask keep {len(kept)}/{sh.E}, rank {r} "
+                            f"adapters on the {len(kept)} kept and {sh.n_shared} shared experts",
+                   tokens_per_s=T * n / t_lora, tokens_per_s_plain=T * n / t_plain,
+                   ms_per_step=t_lora * 1e3 / n, ms_per_step_plain=t_plain * 1e3 / n,
+                   lora_overhead=t_lora / t_plain - 1.0,
+                   kernels={k: dict(launches=v[0], ms_per_step=round(v[1] / n, 4))
+                            for k, v in prof.items() if v[0]},
+                   kernels_plain={k: dict(launches=v[0], ms_per_step=round(v[1] / n, 4))
+                                  for k, v in prof_plain.items() if v[0]},
+                   gpu_launches_per_step=sum(v[0] for v in prof.values()) / n)
+        if nl and msl:
+            a = ld_bytes / (msl / n / 1e3) / 1e9
+            res["roofline_lora_down"] = dict(
+                bound="hbm", kernel="lora_down", achieved=a, peak=peaks["hbm"], unit="GB/s",
+                frac=a / peaks["hbm"], alg_bytes_per_step=ld_bytes, launches_per_step=nl / n,
+                note="x and h rows read once + bf16 U13 / U2 written; the adapters' A "
+                     "matrices are L2-resident")
+        if n13 and n2 and ms13 and ms2:
+            a = (f_base + f_up) / ((ms13 + ms2) / n / 1e3) / 1e12
+            res["roofline_gemm"] = dict(bound="tensor", kernel="gemm13_tc+gemm2_tc", achieved=a,
+                                        peak=peaks["bf16"], unit="TFLOP/s", frac=a / peaks["bf16"],
+                                        flop_per_step=f_base + f_up,
+                                        note="base GEMM flops + the adapters' up projections "
+                                             "(one extra k-block per adapted tile)")
+        res["adapter_flop_share"] = (f_up + f_down) / (f_base + f_up + f_down)
+        out[sh.name] = res
+        del ad, sad, ws, y
+        torch.cuda.empty_cache()
+    return out
+
+
+def run_mask(calls, warmup, seed, dev, peaks, T=4096):
+    """The Stage-1 mask machinery on a fine-tuning batch of T tokens per shape, each kernel timed
+    alone with the L2 flushed before every call: mcft_mask_sample for every layer at once
+    (compact ratio 75 %), mcft_gate_grad after the layer forward (HBM: the forward's fp32 expert
+    output rows and dL/dy), mcft_mask_grad for one layer (two small launches)."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    out = {}
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.zeros(64 << 20, dtype=torch.float32, device=dev)
+    for sh, L in ((I.MIXTRAL, 32), (I.DSV2_LITE, 26)):
+        desc, kept, experts, shared, x, idx, gate = _masked_batch(sh, T, seed, dev)
+        keep = len(kept)
+        g = np.random.default_rng(seed)
+        m_t = torch.from_numpy(g.standard_normal((L, sh.E)).astype(np.float32)).to(dev)
+        u = torch.from_numpy(I.uniforms(seed, (L, sh.E))).to(dev)
+        mask, pi = M.mcft_mask_sample(m_t, u, keep, stream=stream)
+        ws = torch.empty(M.mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=dev)
+        y = torch.empty_like(x)
+        M.mcft_moe_forward(desc, x, idx, gate, experts, shared, y=y, workspace=ws, stream=stream)
+        dy = I.hidden_iid(seed + 1, sh, T, tag="dy").to(dev)
+        dg = torch.empty((T, sh.K), dtype=torch.float32, device=dev)
+        dm = torch.empty(sh.E, dtype=torch.float32, device=dev)
+        dmt = torch.zeros(sh.E, dtype=torch.float32, device=dev)
+        fns = dict(
+            mask_sample=lambda: M.mcft_mask_sample(m_t, u, keep, stream=stream),
+            gate_grad=lambda: M.mcft_gate_grad(desc, dy, ws, dgate=dg, stream=stream),
+            mask_grad=lambda: M.mcft_mask_grad(desc, idx, gate, dg, pi[0], dm=dm, dm_tilde=dmt,
+                                               accumulate=True, stream=stream))
+        for f in fns.values():
+            for _ in range(warmup):
+                f()
+        us = {k: 1e3 * time_calls(f, calls, stream, flush) for k, f in fns.items()}
+        M.mcft_device_error()
+        rows = T * sh.K
+        gg_bytes = rows * sh.d * 4 + T * sh.d * 2 + rows * 4 * 2  # o rows, dy, pos in, dgate out
+        a = gg_bytes / (us["gate_grad"] / 1e6) / 1e9
+        out[sh.name] = dict(
+            workload=f"{sh.name} T={T}, {L} layers x {sh.E} experts, keep {keep}",
+            us_per_call={k: round(v, 2) for k, v in us.items()},
+            roofline_gate_grad=dict(bound="hbm", kernel="gate_grad", achieved=a, peak=peaks["hbm"],
+                                    unit="GB/s", frac=a / peaks["hbm"], alg_bytes=gg_bytes,
+                                    note="each routed row's fp32 expert output and its token's "
+                                         "dL/dy read once; L2 flushed before each call"),
+            mask_sample_note="one 32-thread block per layer: latency-bound, "
+                             f"{L * sh.E * (4 + 4 + 1 + 4)} bytes in total (m~, u in; mask, pi out)")
+        del ws, y, dy
+        torch.cuda.empty_cache()
+    del flush
+    return out
+
+
 # ------------------------------------------------------------------------------------------------
 # CPU oracle timing (the reported baseline, and the reference arm)
 
@@ -728,17 +914,37 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
     ap.add_argument("--case", choices=["decode16", "decode1", "ds_decode1", "ds_decode64", "prefill",
-                                       "fetch16"],
+                                       "fetch16", "lora", "mask"],
                     help="run only a few resident-expert forwards (for profiler captures)")
     ap.add_argument("--workload", default="layer",
-                    choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2"],
+                    choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2",
+                             "lora", "mask"],
                     help="layer: the single-layer decode line; stack-*: the full decode stack "
-                         "(layers on independent streams); chain-*: the chained stack")
+                         "(layers on independent streams); chain-*: the chained stack; lora: the "
+                         "Stage-2 LoRA forward against the plain forward (T = 4096); mask: the "
+                         "Stage-1 mask sampling and gradient kernels (T = 4096)")
     ap.add_argument("--prefetch", type=int, default=0,
                     help="chain workloads: experts prefetched per layer (0 = off)")
     ap.add_argument("--policy", default="LRU", choices=["LRU", "LFU", "FIFO"])
     ap.add_argument("--graph", action="store_true", help="stack workloads: replay a captured step")
     args = ap.parse_args()
+    if args.workload in ("lora", "mask") or args.case in ("lora", "mask"):
+        import __graft_entry__
+
+        __graft_entry__.build()
+        dev = torch.device("cuda", 0)
+        torch.cuda.set_device(dev)
+        peaks = load_peaks()
+        if args.case == "lora":  # a few Mixtral-shaped Stage-2 forwards (profiler captures)
+            res = run_lora(1, 1, 61, dev, peaks, shapes=(I.MIXTRAL,))
+        elif args.case == "mask":
+            res = run_mask(2, 1, 62, dev, peaks)
+        elif args.workload == "lora":
+            res = run_lora(args.steps, args.warmup, 61, dev, peaks)
+        else:
+            res = run_mask(args.steps, args.warmup, 62, dev, peaks)
+        print(json.dumps(res), flush=True)
+        return 0
     if args.workload != "layer":
         import __graft_entry__
 
@@ -857,6 +1063,10 @@ def main():
             del Ld
             torch.cuda.empty_cache()
         line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)
+        line["stage2_lora"] = run_lora(8, 3, seed + 4, dev, peaks)
+        line["stage1_mask"] = run_mask(20, 3, seed + 4, dev, peaks)
+        _BATCHES.clear()
+        torch.cuda.empty_cache()
     if rank == 0 and not args.no_cpu_baseline:
         tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0)
         line["cpu_baseline"] = dict(value=tps, unit="tokens/s", cores=_CORES, kind="oracle",

@@ -422,8 +422,10 @@ mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, cons
     la.K = desc->d;
     la.u = const_cast<float*>(fa.u13);
     la.ustride = 2 * lrank;
-    e = launch_lora_down(la, desc->dtype, 2 * lrank, L.mcap, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "LoRA kernel launch");
+    if (!L.tc) {  // the tcgen05 path projects the gathered rows instead, after the gather
+      e = launch_lora_down(la, desc->dtype, 2 * lrank, L.mcap, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "LoRA kernel launch");
+    }
   }
   auto ffn = [&](int stages) -> cudaError_t {
     if (L.tc) return launch_ffn_tc(fa, ws + L.xp, L.mcap, num_sms(), stream, stages);
@@ -434,10 +436,19 @@ mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, cons
     GatherArgs ga{x, perm, hdr, ws + L.xp, desc->d, L.mcap};
     e = launch_gather(ga, stream);
     if (e != cudaSuccess) return cuda_fail(e, "gather kernel launch");
+    if (lora) {  // U13, GEMM13, U2 (from h), GEMM2
+      e = launch_lora_down_tc(fa, ws + L.xp, L.mcap, num_sms(), stream, 1);
+      if (e == cudaSuccess) e = ffn(1);
+      if (e == cudaSuccess) e = launch_lora_down_tc(fa, ws + L.xp, L.mcap, num_sms(), stream, 2);
+      if (e == cudaSuccess) e = ffn(2);
+      if (e != cudaSuccess) return cuda_fail(e, "LoRA expert GEMM launch");
+    }
   }
-  e = ffn(lora ? 1 : 3);
-  if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
-  if (lora) {
+  if (!(lora && L.tc)) {
+    e = ffn(lora ? 1 : 3);
+    if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
+  }
+  if (lora && !L.tc) {
     // u2[q] = A2 h_q for every permuted row, then the down projection with its adapter
     const LoraOffsets lo = lora_offsets(desc->d, desc->w, lrank);
     la.in = fa.h;

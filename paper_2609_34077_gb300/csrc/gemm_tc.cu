@@ -6,6 +6,11 @@
 //           h[m, n0:n0+128] = bf16(silu(acc_gate) * acc_up)             (fused epilogue)
 //   GEMM2:  o[m, n0:n0+256] = h[m] . W2[n0:n0+256]^T                       (fp32 out)
 // both D = A B^T with A and B K-major bf16, fp32 accumulators in tensor memory.
+// With LoRA adapters (Section 3.2, Stage 2) every projection is W v + s B (A v). The down
+// projections are skinny GEMMs on the same kernel (N = 16 or 32 columns, bf16 out, scaled by s):
+//   DOWN13: U13[m] = s [A1 xp[m] | A3 xp[m]]    DOWN2: U2[m] = s A2 h[m]
+// and the up projections ride on the expert GEMMs as one extra k-block per adapted tile,
+// D += U B'^T, so the tensor cores add them to the accumulators and the epilogues are unchanged.
 //
 // One persistent CTA per SM, 6 warps:
 //   warp 0  - TMA producer (one thread): A tile 128x64 and B tile 256x64 per stage, 4 stages,
@@ -14,7 +19,8 @@
 //             tcgen05.mma (M=128, N=256, K=16) from one thread; tcgen05.commit frees a stage /
 //             publishes an accumulator;
 //   warps 2-5 - epilogue: tcgen05.ld of their 32-lane quarter, SwiGLU or fp32 store; they release
-//             the accumulator so the next tile's MMAs overlap this tile's epilogue.
+//             the accumulator so the next tile's MMAs overlap this tile's epilogue;
+//   warp 6  - with adapters only: writes each adapted tile's extra k-block (see LoraOps).
 // Tiles are walked m-fastest inside groups of m-tiles so concurrently running CTAs share weight
 // tiles (and the activation group) in L2. Every wait is bounded: after 2 s the kernel records
 // MCFT_ERR_TIMEOUT, stops issuing, waits (bounded) for its copies and MMAs in flight, frees TMEM
@@ -27,20 +33,15 @@
 namespace mcft {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int BM = 128, BN = 256, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = 2 * BN;
-constexpr int kThreads = 192;
+constexpr int kMaxStages = 8;
+constexpr int kThreads = 192;  // producer, MMA, 4 epilogue warps
+constexpr int kBuilderWarp = 6;  // with adapters: one more warp writes the extra k-blocks
+__host__ __device__ constexpr int threads_for(int lr) { return lr > 0 ? kThreads + 32 : kThreads; }
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
-enum { EPI_SWIGLU = 0, EPI_F32 = 1 };
-
-// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1),
-// B bf16 (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bit 17, M >> 4 at bit 24.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BN >> 3) << 17) |
-                            (uint32_t(BM >> 4) << 24);
+enum { EPI_SWIGLU = 0, EPI_F32 = 1, EPI_DOWN = 2 };
 
 struct TcParams {
   CUtensorMap tma_a;
@@ -51,33 +52,20 @@ struct TcParams {
   unsigned* err;
   uint32_t wmask[3];  // segments that have weights
   int nseg, kblocks, ntiles_n, ldo, b_half, group_m;
-  // LoRA (Stage 2): adapter block per segment (NULL: none), down-projections u [rows, ustride],
-  // element offsets of the up matrices (B1, B3 for GEMM13; B2 for GEMM2), scale alpha / r.
+  // LoRA (Stage 2): adapter block per segment (NULL: none); lug: the U operand rows (bf16;
+  // GEMM13 [rows, 2r] = s [A1 x | A3 x], GEMM2 [rows, r] = s A2 h); lb0 / lb1: element offsets
+  // of the up matrices (B1, B3 for GEMM13; B2 for GEMM2); lscale = s = alpha / r (DOWN scales
+  // its output by it). b3d: the DOWN B map is 3-D ([A1; A3] planes) rather than 2-D (A2).
   const char* lblk[kMaxSeg];
-  const float* lu;
-  int lustride;
+  const uint16_t* lug;
   size_t lb0, lb1;
   float lscale;
+  int b3d;
 };
 
-// s * <u, B[row]> for rank R (B rows of R bf16 values, u in registers).
-template <int R>
-__device__ __forceinline__ float lora_dot(const char* blk, size_t b_off, int row, const float* u,
-                                          float scale) {
-  const uint4* b = reinterpret_cast<const uint4*>(blk + (b_off + size_t(row) * R) * 2);
-  float acc = 0.f;
-#pragma unroll
-  for (int v = 0; v < R / 8; ++v) {
-    float w8[8];
-    unpack8(__ldg(b + v), w8);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) acc = fmaf(u[8 * v + i], w8[i], acc);
-  }
-  return scale * acc;
-}
-
 struct SmemCtl {
-  uint64_t full[STAGES], empty[STAGES], tfull[2], tempty[2], drain;
+  uint64_t full[kMaxStages], empty[kMaxStages], tfull[2], tempty[2], drain;
+  uint64_t bgo[2];  // with adapters: the producer hands the extra k-blocks' stages to the builder
   uint32_t tmem_base;
   int abort;
   int mt_total;
@@ -85,7 +73,24 @@ struct SmemCtl {
   int off[kMaxSeg + 1];
 };
 
-constexpr int kSmemBytes = STAGES * STAGE_BYTES + 1024 + int(sizeof(SmemCtl));
+// Geometry for an N-tile of NB columns: the expert GEMMs use NB = 256 (4 stages of 48 KB, two
+// 128 x 256 fp32 accumulators = all 512 TMEM columns); the adapter down projection NB = 2r
+// (8 stages of 18-20 KB, 32 or 64 TMEM columns).
+template <int NB>
+struct Tile {
+  static constexpr int B_BYTES = NB * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = NB >= 128 ? 4 : kMaxStages;
+  static constexpr int TMEM_COLS = 2 * NB < 32 ? 32 : 2 * NB;
+  // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1), B bf16
+  // (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                                    (uint32_t(NB >> 3) << 17) | (uint32_t(BM >> 4) << 24);
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + int(sizeof(SmemCtl));
+  static_assert(NB % 16 == 0 && NB >= 16 && NB <= 256, "M = 128 needs N a multiple of 16");
+  static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM allocation");
+  static_assert(SMEM <= 227 * 1024, "shared memory");
+};
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -149,6 +154,14 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
       : "memory");
 }
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
+                                            int c2, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
+      : "memory");
+}
 
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -165,11 +178,12 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
          (uint64_t(1) << 46) | (uint64_t(2) << 61);
 }
 
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc) {
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t acc) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(kIdesc), "r"(acc)
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
       : "memory");
 }
 
@@ -209,8 +223,93 @@ __device__ __forceinline__ int seg_of_row(const SmemCtl* c, int row) {
   return s;
 }
 
+// Whether an m-tile has work: always for the expert GEMMs; for the adapter down projection only
+// when its segment (expert) has an adapter.
+template <int EPI>
+__device__ __forceinline__ bool tile_live(const SmemCtl* c, const TcParams& p, int mt) {
+  if constexpr (EPI != EPI_DOWN) return true;
+  const int s = seg_of_row(c, mt * BM);
+  return ((p.wmask[s >> 5] >> (s & 31)) & 1u) != 0;
+}
+
+// The adapter operands of the extra k-block an adapted tile appends to its K loop (the up
+// projections on the tensor cores): D += U B'^T with
+//   GEMM13: U = [s A1 x | s A3 x] (K' = 2r), B' = [B1 rows | 0] for the gate half and
+//           [0 | B3 rows] for the up half (block-diagonal, so one pass of N = 256 adds both);
+//   GEMM2:  U = [s A2 h | 0], B' = [B2 rows | 0] (K' = r, zero-padded to 16).
+// U and the B rows are bf16 in global memory (U written by the down-projection kernel / by
+// GEMM13). The producer warp loads them into registers when it starts the tile, and writes them
+// into the stage's A and B regions in the 128-byte-swizzled K-major layout the TMA tiles use
+// (16-byte chunk c of row i at chunk c ^ (i % 8) of the row's 128 bytes) when the extra k-block's
+// stage is free. Only the first K' columns of the stage are written and read.
 template <int EPI, int LR>
-__global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+struct LoraOps {
+  static constexpr int KL = EPI == EPI_SWIGLU ? 2 * LR : (LR < 16 ? 16 : LR);  // K' of the block
+  static constexpr int UC = (EPI == EPI_SWIGLU ? 2 * LR : LR) / 8;  // data chunks of a U row
+  static constexpr int BC = LR / 8;                                 // data chunks of a B row
+  static constexpr int CH = KL / 8;                                 // chunks written per row
+  uint4 u[4][UC];  // tile rows 4 lane + i
+  uint4 b[8][BC];  // B' rows lane + 32 i
+
+  __device__ __forceinline__ void load(const TcParams& p, const char* lb, int mt, int nt,
+                                       int lane) {
+    const int ucols = EPI == EPI_SWIGLU ? 2 * LR : LR;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint4* src =
+          reinterpret_cast<const uint4*>(p.lug + (size_t(mt) * BM + 4 * lane + i) * ucols);
+#pragma unroll
+      for (int c = 0; c < UC; ++c) u[i][c] = __ldcg(src + c);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int j = lane + 32 * i;
+      size_t el;
+      if constexpr (EPI == EPI_SWIGLU)
+        el = j < BN / 2 ? p.lb0 + (size_t(nt) * (BN / 2) + j) * LR
+                        : p.lb1 + (size_t(nt) * (BN / 2) + j - BN / 2) * LR;
+      else
+        el = p.lb0 + (size_t(nt) * BN + j) * LR;
+      const uint4* src = reinterpret_cast<const uint4*>(lb + el * 2);
+#pragma unroll
+      for (int c = 0; c < BC; ++c) b[i][c] = __ldg(src + c);
+    }
+  }
+
+  __device__ __forceinline__ void store(uint8_t* sa, uint8_t* sb, int lane) const {
+    const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int row = 4 * lane + i;
+      uint4* dst = reinterpret_cast<uint4*>(sa + row * 128);
+#pragma unroll
+      for (int c = 0; c < CH; ++c) dst[c ^ (row & 7)] = c < UC ? u[i][c] : z;
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int row = lane + 32 * i;
+      uint4* dst = reinterpret_cast<uint4*>(sb + row * 128);
+      // GEMM13: gate rows hold B1 in chunks [0, BC), up rows B3 in chunks [BC, 2 BC)
+      const int c0 = EPI == EPI_SWIGLU && row >= BN / 2 ? BC : 0;  // i >= 4: known when unrolled
+#pragma unroll
+      for (int c = 0; c < CH; ++c) {
+        uint4 v = z;
+#pragma unroll
+        for (int e = 0; e < BC; ++e)
+          if (c == c0 + e) v = b[i][e];
+        dst[c ^ (row & 7)] = v;
+      }
+    }
+  }
+};
+
+template <int EPI, int LR, int NB>
+__global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+  using C = Tile<NB>;
+  constexpr int STAGES = C::STAGES, STAGE_BYTES = C::STAGE_BYTES, TMEM_COLS = C::TMEM_COLS;
+  constexpr int LRA = LR > 0 ? LR : 8;
+  using LOps = LoraOps<EPI, LRA>;
+  static_assert(LR == 0 || NB == BN, "adapters ride on the expert GEMMs");
   pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -223,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
     const int nseg = p.nseg;
     ctl->nseg = nseg;
     for (int s = 0; s <= nseg; ++s) ctl->off[s] = p.off[s];
-    for (int s = 0; s < nseg; ++s) {
+    for (int s = 0; s < nseg && EPI != EPI_DOWN; ++s) {  // no adapter: no down projection
       if (ctl->off[s + 1] > ctl->off[s] && !((p.wmask[s >> 5] >> (s & 31)) & 1u)) {
         set_error(p.err, kErrInvalid);  // a selected expert without weights
         const_cast<WsHeader*>(p.hdr)->abort = 1;  // later kernels of the call skip their work
@@ -241,6 +340,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
       mbar_init(&ctl->tempty[b], 4);
     }
     mbar_init(&ctl->drain, 1);
+    mbar_init(&ctl->bgo[0], 1);
+    mbar_init(&ctl->bgo[1], 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -262,40 +363,99 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
   volatile int* abort = &ctl->abort;
 
   if (warp == 0) {
+    // Producer: one thread issues the TMA copies. An adapted tile's extra k-block takes the next
+    // stage after its K loop: the producer waits for that stage like any other and hands it to
+    // the builder warp (bgo), which fills it. Every waiter thus waits on every phase of its
+    // barriers in order, which a parity wait needs (it is ambiguous two phases away).
     if (lane == 0 && int(blockIdx.x) < tiles) {
-      uint32_t it = 0;
+      uint32_t it = 0, nl = 0;
       for (int tile = blockIdx.x; tile < tiles && !*abort; tile += gridDim.x) {
         int mt, nt;
         tile_coords(tile, mt_total, ntn, p.group_m, mt, nt);
+        if (!tile_live<EPI>(ctl, p, mt)) continue;
         const int row0 = mt * BM;
-        const CUtensorMap* mb = &p.tma_b[seg_of_row(ctl, row0)];
-        const int yb0 = EPI == EPI_SWIGLU ? nt * (BN / 2) : nt * BN;
-        const int yb1 = EPI == EPI_SWIGLU ? p.b_half + nt * (BN / 2) : nt * BN + BN / 2;
+        const int sg = seg_of_row(ctl, row0);
+        const CUtensorMap* mb = &p.tma_b[sg];
+        const int yb0 = EPI == EPI_SWIGLU ? nt * (NB / 2) : nt * NB;
+        const int yb1 = EPI == EPI_SWIGLU ? p.b_half + nt * (NB / 2) : nt * NB + NB / 2;
         for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
           const int s = int(it % STAGES);
           if (!mbar_wait(&ctl->empty[s], ((it / STAGES) & 1u) ^ 1u, abort, p.err)) break;
           const uint32_t sa = base + uint32_t(s) * STAGE_BYTES, sb = sa + A_BYTES;
           mbar_expect_tx(&ctl->full[s], STAGE_BYTES);
           tma_load_2d(sa, &p.tma_a, kb * BK, row0, &ctl->full[s]);
-          tma_load_2d(sb, mb, kb * BK, yb0, &ctl->full[s]);
-          tma_load_2d(sb + B_BYTES / 2, mb, kb * BK, yb1, &ctl->full[s]);
+          if constexpr (EPI == EPI_DOWN) {
+            if (p.b3d)  // [A1; A3]: one box of r rows x 2 planes
+              tma_load_3d(sb, mb, kb * BK, 0, 0, &ctl->full[s]);
+            else        // A2: a box of NB rows, those past r zero-filled
+              tma_load_2d(sb, mb, kb * BK, 0, &ctl->full[s]);
+          } else {
+            tma_load_2d(sb, mb, kb * BK, yb0, &ctl->full[s]);
+            tma_load_2d(sb + C::B_BYTES / 2, mb, kb * BK, yb1, &ctl->full[s]);
+          }
+        }
+        if constexpr (LR > 0) {
+          if (p.lblk[sg] != nullptr && !*abort) {  // the extra k-block's stage, for the builder
+            const int s = int(it % STAGES);
+            if (!mbar_wait(&ctl->empty[s], ((it / STAGES) & 1u) ^ 1u, abort, p.err)) break;
+            mbar_arrive(&ctl->bgo[nl & 1u]);
+            ++nl;
+            ++it;
+          }
         }
       }
-      // Copies still in flight: the last STAGES issued ones (all consumed unless aborting).
+      // Stages still in flight: the last STAGES issued ones (all consumed unless aborting).
       const uint32_t n_tail = it < STAGES ? it : STAGES;
       for (uint32_t j = it - n_tail; j < it; ++j)
         mbar_wait_drain(&ctl->full[j % STAGES], (j / STAGES) & 1u, p.err);
     }
+  } else if (LR > 0 && warp == kBuilderWarp) {
+    // Builder (adapters only): walks the producer's tile sequence and counts its stages; for the
+    // n-th adapted tile it loads U and B' into registers when the tile starts, waits for the
+    // producer's n-th hand-off (bgo[n % 2]: at most two are outstanding, since the MMAs stop at
+    // the first unfilled stage and a tile has at least two TMA stages), writes the stage and
+    // marks it full. Lane 0 waits; the outcome is broadcast.
+    if (int(blockIdx.x) < tiles) {
+      uint32_t it = 0, nl = 0;
+      for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+        int mt, nt;
+        tile_coords(tile, mt_total, ntn, p.group_m, mt, nt);
+        const int sg = seg_of_row(ctl, mt * BM);
+        it += uint32_t(p.kblocks);
+        if (p.lblk[sg] == nullptr) continue;
+        LOps lops;
+        lops.load(p, p.lblk[sg], mt, nt, lane);
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait(&ctl->bgo[nl & 1u], (nl >> 1) & 1u, abort, p.err);
+        if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+        const int s = int(it % STAGES);
+        const uint32_t sa = base + uint32_t(s) * STAGE_BYTES, sb = sa + A_BYTES;
+        lops.store(smem_raw + (sa - raw), smem_raw + (sb - raw), lane);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // for the MMA reads
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ctl->full[s]);
+        ++nl;
+        ++it;
+      }
+    }
   } else if (warp == 1) {
     if (lane == 0 && int(blockIdx.x) < tiles) {
       uint32_t it = 0, lt = 0;
-      for (int tile = blockIdx.x; tile < tiles && !*abort; tile += gridDim.x, ++lt) {
+      for (int tile = blockIdx.x; tile < tiles && !*abort; tile += gridDim.x) {
+        bool lor = false;
+        if constexpr (EPI == EPI_DOWN || LR > 0) {
+          int mt, nt;
+          tile_coords(tile, mt_total, ntn, p.group_m, mt, nt);
+          if (!tile_live<EPI>(ctl, p, mt)) continue;
+          if constexpr (LR > 0) lor = p.lblk[seg_of_row(ctl, mt * BM)] != nullptr;
+        }
         const uint32_t b = lt & 1u;
         if (!mbar_wait(&ctl->tempty[b], ((lt >> 1) & 1u) ^ 1u, abort, p.err)) break;
         tc_fence_after();
-        const uint32_t dt = tmem + b * BN;
+        const uint32_t dt = tmem + b * NB;
         bool ok = true;
-        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+        const int nkb = p.kblocks + (lor ? 1 : 0);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
           const int s = int(it % STAGES);
           if (!mbar_wait(&ctl->full[s], (it / STAGES) & 1u, abort, p.err)) {
             ok = false;
@@ -304,103 +464,92 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_tc_kernel(const __grid_const
           tc_fence_after();
           const uint32_t sa = base + uint32_t(s) * STAGE_BYTES, sb = sa + A_BYTES;
           const uint64_t da = sw128_desc(sa), db = sw128_desc(sb);
+          if (LR == 0 || kb < p.kblocks) {
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K per step inside the swizzle atom
-            tc_mma(dt, da + uint64_t(2 * k), db + uint64_t(2 * k), (kb | k) != 0 ? 1u : 0u);
+            for (int k = 0; k < BK / 16; ++k)  // +32 bytes along K per step inside the swizzle atom
+              tc_mma(dt, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC,
+                     (kb | k) != 0 ? 1u : 0u);
+          } else {  // the adapters' up projections: D += U B'^T over K' columns
+#pragma unroll
+            for (int k = 0; k < LOps::KL / 16; ++k)
+              tc_mma(dt, da + uint64_t(2 * k), db + uint64_t(2 * k), C::IDESC, 1u);
+          }
           tc_commit(&ctl->empty[s]);
         }
         if (!ok) break;
         tc_commit(&ctl->tfull[b]);
+        ++lt;
       }
       tc_commit(&ctl->drain);  // arrives once every MMA issued above has completed
       mbar_wait_drain(&ctl->drain, 0, p.err);
     }
-  } else {
+  } else if (warp >= 2 && warp < 6) {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int row = q * 32 + lane;
     uint32_t lt = 0;
-    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++lt) {
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
       int mt, nt;
       tile_coords(tile, mt_total, ntn, p.group_m, mt, nt);
+      if (!tile_live<EPI>(ctl, p, mt)) continue;
       const uint32_t b = lt & 1u;
       int ok = 1;
       if (lane == 0) ok = mbar_wait(&ctl->tfull[b], (lt >> 1) & 1u, abort, p.err) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t taddr = tmem + b * BN + (uint32_t(q * 32) << 16);
+      const uint32_t taddr = tmem + b * NB + (uint32_t(q * 32) << 16);
       const size_t grow = size_t(mt) * BM + row;
-      // LoRA down-projections of this row (A1 x, A3 x) or (A2 h), kept in registers
-      constexpr int LRA = LR > 0 ? LR : 1;
-      float ua[LRA], ub[LRA];
-      const char* lb = nullptr;
-      if constexpr (LR > 0) {
-        lb = p.lblk[seg_of_row(ctl, mt * BM)];
-        if (lb) {
-          const float* uq = p.lu + grow * p.lustride;
-#pragma unroll
-          for (int j = 0; j < LR; ++j) {
-            ua[j] = uq[j];
-            ub[j] = EPI == EPI_SWIGLU ? uq[LR + j] : 0.f;
-          }
-        }
-      }
       if constexpr (EPI == EPI_SWIGLU) {
-        uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo + size_t(nt) * (BN / 2);
+        uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo + size_t(nt) * (NB / 2);
 #pragma unroll 1
-        for (int c = 0; c < BN / 2; c += 16) {
+        for (int c = 0; c < NB / 2; c += 16) {
           uint32_t g[16], u[16];
           tmem_ld16(taddr + c, g);
-          tmem_ld16(taddr + BN / 2 + c, u);
+          tmem_ld16(taddr + NB / 2 + c, u);
           tmem_ld_wait();
-          float gf[16], uf[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            gf[i] = __uint_as_float(g[i]);
-            uf[i] = __uint_as_float(u[i]);
-          }
-          if constexpr (LR > 0) {
-            if (lb) {  // + s B1 (A1 x), + s B3 (A3 x)
-              const int n0 = nt * (BN / 2) + c;
-#pragma unroll
-              for (int i = 0; i < 16; ++i) {
-                gf[i] += lora_dot<LR>(lb, p.lb0, n0 + i, ua, p.lscale);
-                uf[i] += lora_dot<LR>(lb, p.lb1, n0 + i, ub, p.lscale);
-              }
-            }
-          }
           uint32_t pk[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            pk[i] = pack2bf(silu(gf[2 * i]) * uf[2 * i], silu(gf[2 * i + 1]) * uf[2 * i + 1]);
+            pk[i] = pack2bf(silu(__uint_as_float(g[2 * i])) * __uint_as_float(u[2 * i]),
+                            silu(__uint_as_float(g[2 * i + 1])) * __uint_as_float(u[2 * i + 1]));
           uint4* dst = reinterpret_cast<uint4*>(out + c);
           dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
-      } else {
-        float* out = reinterpret_cast<float*>(p.out) + grow * p.ldo + size_t(nt) * BN;
-#pragma unroll 1
-        for (int c = 0; c < BN; c += 16) {
+      } else if constexpr (EPI == EPI_DOWN) {  // U = s (A v) in bf16, the first ldo columns
+        uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo;
+#pragma unroll
+        for (int c = 0; c < NB; c += 16) {
           uint32_t v[16];
           tmem_ld16(taddr + c, v);
           tmem_ld_wait();
-          float f[16];
+          uint32_t pk[8];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) f[i] = __uint_as_float(v[i]);
-          if constexpr (LR > 0) {
-            if (lb) {  // + s B2 (A2 h)
-#pragma unroll
-              for (int i = 0; i < 16; ++i) f[i] += lora_dot<LR>(lb, p.lb0, nt * BN + c + i, ua, p.lscale);
-            }
-          }
+          for (int i = 0; i < 8; ++i)
+            pk[i] = pack2bf(p.lscale * __uint_as_float(v[2 * i]),
+                            p.lscale * __uint_as_float(v[2 * i + 1]));
+          uint4* dst = reinterpret_cast<uint4*>(out + c);
+          dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          if (c + 16 <= p.ldo) dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        }
+      } else {
+        float* out = reinterpret_cast<float*>(p.out) + grow * p.ldo + size_t(nt) * NB;
+#pragma unroll 1
+        for (int c = 0; c < NB; c += 16) {
+          uint32_t v[16];
+          tmem_ld16(taddr + c, v);
+          tmem_ld_wait();
           float4* dst = reinterpret_cast<float4*>(out + c);
 #pragma unroll
-          for (int i = 0; i < 4; ++i) dst[i] = make_float4(f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
+          for (int i = 0; i < 4; ++i)
+            dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
+                                 __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl->tempty[b]);
+      ++lt;
     }
   }
 
@@ -445,20 +594,50 @@ bool encode_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The [A1; A3] rows of one adapter block as a 3-D map {d, r, 2}: plane 0 = A1 (element offset
+// 0), plane 1 = A3 (plane stride a3 elements); box 64 columns x r rows x 2 planes, so one load
+// fills the 2r rows of a down-projection B tile (A1 rows first), 128-byte swizzle.
+bool encode_adapter_a13(CUtensorMap* m, const void* blk, uint64_t d, uint32_t r, uint64_t a3) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(blk) & 15u) || ((d * 2) & 15u) || ((a3 * 2) & 15u))
+    return false;
+  const cuuint64_t dims[3] = {d, r, 2};
+  const cuuint64_t strides[2] = {d * 2, a3 * 2};
+  const cuuint32_t box[3] = {BK, r, 2};
+  const cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(blk), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// A2 of one adapter block, [r, w] row-major, as a 2-D map with a box of 64 columns x 16 rows:
+// for r = 8 the rows past r are outside the tensor and arrive as zeros (an N = 16 B tile).
+bool encode_adapter_a2(CUtensorMap* m, const void* a2, uint64_t w, uint32_t r) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || (reinterpret_cast<uintptr_t>(a2) & 15u) || ((w * 2) & 15u) || r > 16) return false;
+  const cuuint64_t dims[2] = {w, r};
+  const cuuint64_t strides[1] = {w * 2};
+  const cuuint32_t box[2] = {BK, 16};
+  const cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(a2), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int group_for(size_t a_tile_bytes) {
   const size_t budget = size_t(48) << 20;  // activation rows kept hot in L2 per group
   size_t g = budget / (a_tile_bytes ? a_tile_bytes : 1);
   return g < 1 ? 1 : int(g > 4096 ? 4096 : g);
 }
 
-template <int EPI, int LR>
-cudaError_t launch_one(const TcParams& p, int num_sms, cudaStream_t s) {
+template <int EPI, int LR, int NB>
+cudaError_t launch_one(const TcParams& p, int grid, cudaStream_t s) {
   static cudaError_t attr = cudaFuncSetAttribute(
-      gemm_tc_kernel<EPI, LR>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+      gemm_tc_kernel<EPI, LR, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, Tile<NB>::SMEM);
   if (attr != cudaSuccess) return attr;
-  const int kid = EPI == EPI_SWIGLU ? kProfGemm13 : kProfGemm2;
+  const int kid = EPI == EPI_SWIGLU ? kProfGemm13 : EPI == EPI_F32 ? kProfGemm2 : kProfLora;
   prof_begin(kid, s);
-  gemm_tc_kernel<EPI, LR><<<num_sms, kThreads, kSmemBytes, s>>>(p);
+  gemm_tc_kernel<EPI, LR, NB><<<grid, threads_for(LR), Tile<NB>::SMEM, s>>>(p);
   prof_end(kid, s);
   return cudaGetLastError();
 }
@@ -466,9 +645,9 @@ cudaError_t launch_one(const TcParams& p, int num_sms, cudaStream_t s) {
 template <int EPI>
 cudaError_t launch_rank(const TcParams& p, int rank, int num_sms, cudaStream_t s) {
   switch (rank) {
-    case 0: return launch_one<EPI, 0>(p, num_sms, s);
-    case 8: return launch_one<EPI, 8>(p, num_sms, s);
-    case 16: return launch_one<EPI, 16>(p, num_sms, s);
+    case 0: return launch_one<EPI, 0, BN>(p, num_sms, s);
+    case 8: return launch_one<EPI, 8, BN>(p, num_sms, s);
+    case 16: return launch_one<EPI, 16, BN>(p, num_sms, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -517,20 +696,54 @@ cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sm
       p13.lblk[sgi] = reinterpret_cast<const char*>(a.lblk[sgi]);
       p2.lblk[sgi] = p13.lblk[sgi];
     }
-    p13.lu = a.u13;
-    p13.lustride = 2 * a.lrank;
+    // U13 and U2 (bf16, from the down-projection launches) feed the extra k-blocks
+    p13.lug = reinterpret_cast<const uint16_t*>(a.u13);
     p13.lb0 = lo.b1;
     p13.lb1 = lo.b3;
-    p13.lscale = a.lscale;
-    p2.lu = a.u2;
-    p2.lustride = a.lrank;
+    p2.lug = reinterpret_cast<const uint16_t*>(a.u2);
     p2.lb0 = lo.b2;
-    p2.lscale = a.lscale;
   }
   cudaError_t e = cudaSuccess;
   if (stages & 1) e = launch_rank<EPI_SWIGLU>(p13, a.lrank, num_sms, s);
   if (e != cudaSuccess || !(stages & 2)) return e;
   return launch_rank<EPI_F32>(p2, a.lrank, num_sms, s);
+}
+
+cudaError_t launch_lora_down_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms,
+                                cudaStream_t s, int stage) {
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  const size_t d = size_t(a.d), w = size_t(a.w);
+  const int r = a.lrank;
+  if (r != 8 && r != 16) return cudaErrorInvalidValue;
+  const bool s13 = stage == 1;
+  const size_t K = s13 ? d : w;
+  if (!encode_2d(&p.tma_a, s13 ? xp : a.h, K, size_t(mcap))) return cudaErrorInvalidValue;
+  const LoraOffsets lo = lora_offsets(a.d, a.w, r);
+  for (int sgi = 0; sgi < a.nseg; ++sgi) {
+    const char* blk = reinterpret_cast<const char*>(a.lblk[sgi]);
+    if (!blk) continue;  // no adapter: the tile is skipped (its U rows are never read)
+    const bool ok = s13 ? encode_adapter_a13(&p.tma_b[sgi], blk, d, uint32_t(r), lo.a3)
+                        : encode_adapter_a2(&p.tma_b[sgi], blk + lo.a2 * 2, w, uint32_t(r));
+    if (!ok) return cudaErrorInvalidValue;
+    p.wmask[sgi >> 5] |= 1u << (sgi & 31);
+  }
+  p.off = a.off;
+  p.hdr = a.hdr;
+  p.err = a.err;
+  p.nseg = a.nseg;
+  p.b3d = s13 ? 1 : 0;
+  p.out = const_cast<float*>(s13 ? a.u13 : a.u2);  // bf16 [rows, 2r] / [rows, r]
+  p.lscale = a.lscale;
+  p.kblocks = int(K / BK);
+  p.ntiles_n = 1;
+  p.ldo = s13 ? 2 * r : r;
+  p.group_m = 1;
+  const int mtiles = (mcap + BM - 1) / BM;
+  const int grid = mtiles < num_sms ? (mtiles > 0 ? mtiles : 1) : num_sms;
+  // N = 2r for [A1; A3]; 16 for A2 (r = 8: rows 8-15 of the box are zero)
+  return s13 && r == 16 ? launch_one<EPI_DOWN, 0, 32>(p, grid, s)
+                        : launch_one<EPI_DOWN, 0, 16>(p, grid, s);
 }
 
 }  // namespace mcft

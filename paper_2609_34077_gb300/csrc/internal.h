@@ -154,7 +154,8 @@ struct FfnArgs {
   const unsigned long long* ready;
   int phase;
   // LoRA (Stage 2): adapter block of each segment (NULL: none), rank, scale alpha / r, and the
-  // down-projections u13 [mcap, 2r] (A1 x, A3 x) and u2 [mcap, r] (A2 h) from lora_down.
+  // down-projections u13 [mcap, 2r] (A1 x, A3 x) and u2 [mcap, r] (A2 h): fp32 from lora_down,
+  // or on the tcgen05 path bf16 and scaled by s (s [A1 x | A3 x], s A2 h).
   const void* lblk[72];
   int lrank;
   float lscale;
@@ -211,6 +212,11 @@ cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int
 int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
 cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
                           int stages = 3);
+// Down projections of the adapters for the tcgen05 path, on the tensor cores, bf16 out scaled by
+// s: stage 1: u13[q] = s [A1 xp[q] | A3 xp[q]] (N = 2r); stage 2: u2[q] = s A2 h[q] (N = 16),
+// for the rows of every segment with an adapter. The expert GEMMs add the up projections.
+cudaError_t launch_lora_down_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms,
+                                cudaStream_t s, int stage);
 
 struct CombineArgs {
   const float* o;

@@ -3,8 +3,9 @@
 //
 // Each adapted projection is W v + s B (A v) with A [r, in], B [out, r], s = alpha / r. The large
 // term W v runs in the expert GEMM / GEMV kernels, which also add s B u in their epilogues (r
-// multiply-adds per output); this kernel computes the small middle vectors u = A v for every
-// permuted row whose segment has an adapter:
+// multiply-adds per output). On the decode and fp32 paths this kernel computes the small middle
+// vectors u = A v for every permuted row whose segment has an adapter (the tcgen05 path projects
+// its gathered rows on the tensor cores and takes A2 h from GEMM13's epilogue instead):
 //   stage 13: u[q] = [A1 x ; A3 x]     (2r values; x = the row's token, or the gathered row)
 //   stage 2:  u[q] = A2 h_q            (r values; h = the SwiGLU activation of the row)
 // One warp per row: lanes walk the input in 16-byte chunks, each chunk is dotted with the R rows

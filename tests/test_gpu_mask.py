@@ -115,3 +115,30 @@ def test_stage1_step_end_to_end():
     assert np.all(dm.cpu().numpy()[ref_mask[0] == 0] == 0)
     scale = np.abs(dmt_ref).max()
     assert np.abs(dmt.cpu().double().numpy() - dmt_ref).max() <= 3e-2 * scale
+
+
+def test_gate_grad_mixtral_full_size_sampled():
+    """Gate gradients of a Mixtral-shaped fine-tuning batch of 4096 tokens (tcgen05 forward, the
+    size the bench times): 48 sampled tokens against the oracle's <dL/dy_t, F_e(x_t)>."""
+    sh, T = I.MIXTRAL, 4096
+    lw = weights(sh)
+    x = I.hidden_iid(83, sh, T)
+    ids = I.random_ids(83, 1, T, sh.K, sh.E, hot=range(6), p_hot=1.0)[0]
+    gate = np.random.default_rng(83).uniform(0.05, 1.0, (T, sh.K)).astype(np.float32)
+    desc = M.desc_of(sh)
+    ws = torch.empty(M.mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=DEV)
+    M.mcft_moe_forward(desc, x.to(DEV), torch.from_numpy(ids).to(DEV),
+                       torch.from_numpy(gate).to(DEV),
+                       [b.to(DEV) if e < 6 else None for e, b in enumerate(lw.experts)], workspace=ws)
+    dy = I.hidden_iid(84, sh, T, tag="dy")
+    dg = M.mcft_gate_grad(desc, dy.to(DEV), ws).cpu().double().numpy()
+    M.mcft_device_error()
+    rows = np.random.default_rng(83).choice(T, 48, replace=False)
+    ex = [tuple(f64(t) for t in I.split_expert(lw.experts[e], sh)) if e < 6 else None
+          for e in range(sh.E)]
+    xs = f64(x)[rows]
+    outs = np.stack([np.stack([oracle.ffn.expert(xs[i:i + 1], *ex[ids[t, k]])[0]
+                               for k in range(sh.K)]) for i, t in enumerate(rows)])
+    ref = oracle.mask.gate_grad(f64(dy)[rows], outs)
+    err = np.abs(dg[rows] - ref).max() / np.abs(ref).max()
+    assert err <= TOL_BF16, err
