@@ -8,12 +8,19 @@
 //   forward left in its workspace (summed over its partial planes). One warp per assignment.
 // mask_grad: dL/dm_e = sum over tokens t with e in A_t of g_{t,e} (dg_{t,e} - sum_i g_{t,i} dg_{t,i})
 //   for renormalised gates, g_{t,e} dg_{t,e} for plain gates (the gates of the active experts are
-//   computed from p * m with m = 1 on A); one CTA per expert, every thread walking a fixed stride of
-//   the assignments and a fixed-order tree reduction, so the sum is deterministic. Then
-//   dL/dm~ = (diag(pi) - pi pi^T) dL/dm (straight-through estimator and softmax Jacobian),
-//   optionally accumulated over several steps (the paper accumulates T steps per update).
+//   computed from p * m with m = 1 on A). One cluster of 8 CTAs: each CTA takes a contiguous
+//   share of the tokens, each lane one token at a time (its K contributions computed once), and
+//   the warp sums every expert's contributions with a butterfly; the warps' and then the CTAs'
+//   partials are added in a fixed order (the leader reads the others' shared memory), so the sum
+//   is deterministic. Then dL/dm~ = (diag(pi) - pi pi^T) dL/dm (straight-through estimator and
+//   softmax Jacobian), optionally accumulated over several steps (the paper accumulates T steps
+//   per update), in the same launch.
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "internal.h"
+
+namespace cg = cooperative_groups;
 
 namespace mcft {
 namespace {
@@ -123,44 +130,97 @@ __global__ void __launch_bounds__(256) gate_grad_kernel(const __grid_constant__ 
   }
 }
 
-__global__ void __launch_bounds__(256) mask_grad_kernel(const __grid_constant__ MaskGradArgs a) {
+constexpr int kGradCluster = 8, kGradWarps = 16;
+
+__global__ void __cluster_dims__(kGradCluster, 1, 1) __launch_bounds__(kGradWarps * 32)
+    mask_grad_kernel(const __grid_constant__ MaskGradArgs a) {
   pdl_wait();
-  __shared__ float part[256];
-  const int e = blockIdx.x, tid = threadIdx.x;
-  const int n = a.T * a.K;
-  float acc = 0.f;
-  for (int i = tid; i < n; i += blockDim.x) {
-    if (a.idx[i] != e) continue;
-    const int t = i / a.K;
-    const float g = a.gate[i], dg = a.dgate[i];
-    if (a.gate_mode == MCFT_GATE_RENORM) {
+  __shared__ float wpart[kGradWarps][kMaxE];
+  __shared__ float cpart[kMaxE];  // this CTA's share of dL/dm
+  cg::cluster_group cluster = cg::this_cluster();
+  const int crank = int(cluster.block_rank());
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int E = a.E, K = a.K, T = a.T;
+  const int per = (T + kGradCluster - 1) / kGradCluster;
+  const int t0 = crank * per, t1 = min(T, t0 + per);
+  float acc0 = 0.f, acc1 = 0.f;  // this warp's sums for experts lane and lane + 32
+  for (int base = t0 + warp * 32; base < t1; base += kGradWarps * 32) {
+    const int t = base + lane;
+    int ids[kMaxK];
+    float c[kMaxK];
+#pragma unroll
+    for (int k = 0; k < kMaxK; ++k) {
+      ids[k] = -1;
+      c[k] = 0.f;
+    }
+    if (t < t1) {
       float inner = 0.f;  // sum_i g_{t,i} dL/dg_{t,i}
-      for (int k = 0; k < a.K; ++k)
-        inner = fmaf(a.gate[size_t(t) * a.K + k], a.dgate[size_t(t) * a.K + k], inner);
-      acc += g * (dg - inner);
-    } else {
-      acc += g * dg;
+      for (int k = 0; k < K; ++k)
+        inner = fmaf(a.gate[size_t(t) * K + k], a.dgate[size_t(t) * K + k], inner);
+#pragma unroll
+      for (int k = 0; k < kMaxK; ++k) {
+        if (k < K) {
+          const float g = a.gate[size_t(t) * K + k], dg = a.dgate[size_t(t) * K + k];
+          ids[k] = a.idx[size_t(t) * K + k];
+          c[k] = a.gate_mode == MCFT_GATE_RENORM ? g * (dg - inner) : g * dg;
+        }
+      }
+    }
+    for (int e = 0; e < E; ++e) {
+      float v = 0.f;
+      bool has = false;
+#pragma unroll
+      for (int k = 0; k < kMaxK; ++k) {
+        if (ids[k] == e) {
+          v += c[k];
+          has = true;
+        }
+      }
+      if (!__any_sync(0xffffffffu, has)) continue;  // no token of this group picked e
+      v = warp_sum(v);
+      if (lane == (e & 31)) {
+        if (e < 32) acc0 += v;
+        else acc1 += v;
+      }
     }
   }
-  part[tid] = acc;
+  wpart[warp][lane] = acc0;
+  wpart[warp][lane + 32] = acc1;
   __syncthreads();
-  for (int s = 128; s > 0; s >>= 1) {
-    if (tid < s) part[tid] += part[tid + s];
-    __syncthreads();
+  if (threadIdx.x < E) {
+    float sum = 0.f;
+    for (int w = 0; w < kGradWarps; ++w) sum += wpart[w][threadIdx.x];
+    cpart[threadIdx.x] = sum;
   }
-  if (tid == 0) a.dm[e] = part[0];
-}
-
-__global__ void __launch_bounds__(32) mask_tilde_kernel(const __grid_constant__ MaskGradArgs a) {
-  pdl_wait();
-  const int lane = threadIdx.x, E = a.E;
-  float s = 0.f;
-  for (int e = lane; e < E; e += 32) s += a.pi[e] * a.dm[e];
-  s = warp_sum(s);  // pi . dL/dm
-  for (int e = lane; e < E; e += 32) {
-    const float v = a.pi[e] * (a.dm[e] - s);
-    a.dm_tilde[e] = a.accumulate ? a.dm_tilde[e] + v : v;
+  cluster.sync();  // every CTA's share is in its shared memory
+  if (crank == 0 && warp == 0) {
+    float dm[2] = {0.f, 0.f};
+    for (int r = 0; r < kGradCluster; ++r) {
+      const float* pr = cluster.map_shared_rank(&cpart[0], r);
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        if (lane + 32 * j < E) dm[j] += pr[lane + 32 * j];
+    }
+    float sp = 0.f;  // pi . dL/dm
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int e = lane + 32 * j;
+      if (e < E) {
+        a.dm[e] = dm[j];
+        sp += a.pi[e] * dm[j];
+      }
+    }
+    sp = warp_sum(sp);
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int e = lane + 32 * j;
+      if (e < E) {
+        const float v = a.pi[e] * (dm[j] - sp);
+        a.dm_tilde[e] = a.accumulate ? a.dm_tilde[e] + v : v;
+      }
+    }
   }
+  cluster.sync();  // the leader has read the other CTAs' shared memory
 }
 
 }  // namespace
@@ -180,10 +240,7 @@ cudaError_t launch_gate_grad(const GateGradArgs& a, int dtype, cudaStream_t s) {
 }
 
 cudaError_t launch_mask_grad(const MaskGradArgs& a, cudaStream_t s) {
-  mask_grad_kernel<<<a.E, 256, 0, s>>>(a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  mask_tilde_kernel<<<1, 32, 0, s>>>(a);
+  mask_grad_kernel<<<kGradCluster, kGradWarps * 32, 0, s>>>(a);
   return cudaGetLastError();
 }
 
