@@ -860,8 +860,8 @@ def _config(batch):
 def profile_case(case: str, dev) -> int:
     """A few forwards: the small launch sequences that ncu captures. decode16 / decode1:
     Mixtral-shaped decode at batch 16 / 1 with every expert resident (decode FFN); ds_decode1 /
-    ds_decode64: the same for the DeepSeek-V2-Lite shape at batch 1 / 64; prefill: T = 4096
-    tokens, hard mask keep 4 of 8 (tcgen05 GEMMs); fetch16: three decode steps at batch 16 through
+    ds_decode64: the same for the DeepSeek-V2-Lite shape at batch 1 / 64; prefill / ds_prefill:
+    T = 4096 tokens, hard mask keeping 4 of 8 / 48 of 64 (tcgen05 GEMMs); fetch16: three decode steps at batch 16 through
     the cache with the device-driven fetch (fetch kernel)."""
     from paper_2609_34077_gb300 import mcft as M
 
@@ -879,9 +879,9 @@ def profile_case(case: str, dev) -> int:
         print(json.dumps({"case": case, "fetches_per_step": per_step,
                           "fetch_bytes_per_step": [n * sh.expert_bytes for n in per_step]}))
         return 0
-    if case == "prefill":
+    if case in ("prefill", "ds_prefill"):  # Mixtral keeps 4 of 8, DeepSeek 48 of 64
         T, mode = 4096, M.MCFT_ROUTE_HARD_MASK
-        kw = dict(mask=I.keep_mask(7, sh.E, 4))
+        kw = dict(mask=I.keep_mask(7, sh.E, 4 if sh is I.MIXTRAL else sh.E * 3 // 4))
         keep = [int(e) for e in np.nonzero(kw["mask"])[0]]
         x = I.hidden_iid(7, sh, T).to(dev)
     else:
@@ -914,7 +914,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
     ap.add_argument("--case", choices=["decode16", "decode1", "ds_decode1", "ds_decode64", "prefill",
-                                       "fetch16", "lora", "mask"],
+                                       "ds_prefill", "fetch16", "lora", "mask"],
                     help="run only a few resident-expert forwards (for profiler captures)")
     ap.add_argument("--workload", default="layer",
                     choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2",

@@ -76,6 +76,13 @@ struct SmemCtl {
 // Geometry for an N-tile of NB columns: the expert GEMMs use NB = 256 (4 stages of 48 KB, two
 // 128 x 256 fp32 accumulators = all 512 TMEM columns); the adapter down projection NB = 2r
 // (8 stages of 18-20 KB, 32 or 64 TMEM columns).
+// Epilogue store staging of the expert GEMMs: each epilogue warp writes 32 rows x 128 bytes of its
+// output into shared memory (rows padded to 144 bytes: conflict-free 16-byte writes and reads),
+// then stores them as whole 128-byte row segments, four rows per instruction.
+constexpr int kOutRowBytes = 144;
+constexpr int kOutWarpBytes = 32 * kOutRowBytes;
+constexpr int kCtlBytes = (int(sizeof(SmemCtl)) + 15) / 16 * 16;
+
 template <int NB>
 struct Tile {
   static constexpr int B_BYTES = NB * BK * 2;
@@ -86,7 +93,8 @@ struct Tile {
   // (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                                     (uint32_t(NB >> 3) << 17) | (uint32_t(BM >> 4) << 24);
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + int(sizeof(SmemCtl));
+  static constexpr int OUT_STAGE = NB >= 128 ? 4 * kOutWarpBytes : 0;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + kCtlBytes + OUT_STAGE;
   static_assert(NB % 16 == 0 && NB >= 16 && NB <= 256, "M = 128 needs N a multiple of 16");
   static_assert((TMEM_COLS & (TMEM_COLS - 1)) == 0 && TMEM_COLS <= 512, "TMEM allocation");
   static_assert(SMEM <= 227 * 1024, "shared memory");
@@ -499,22 +507,37 @@ __global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __gri
       tc_fence_after();
       const uint32_t taddr = tmem + b * NB + (uint32_t(q * 32) << 16);
       const size_t grow = size_t(mt) * BM + row;
+      // this warp's staging rows; row r of the warp's quarter goes to global row grow0 + r
+      uint8_t* stg = reinterpret_cast<uint8_t*>(ctl) + kCtlBytes + q * kOutWarpBytes;
+      const size_t grow0 = size_t(mt) * BM + q * 32;
       if constexpr (EPI == EPI_SWIGLU) {
-        uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo + size_t(nt) * (NB / 2);
+        // two rounds of 64 h columns (128 bytes of bf16 per row)
 #pragma unroll 1
-        for (int c = 0; c < NB / 2; c += 16) {
-          uint32_t g[16], u[16];
-          tmem_ld16(taddr + c, g);
-          tmem_ld16(taddr + NB / 2 + c, u);
-          tmem_ld_wait();
-          uint32_t pk[8];
+        for (int c0 = 0; c0 < NB / 2; c0 += 64) {
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
-            pk[i] = pack2bf(silu(__uint_as_float(g[2 * i])) * __uint_as_float(u[2 * i]),
-                            silu(__uint_as_float(g[2 * i + 1])) * __uint_as_float(u[2 * i + 1]));
-          uint4* dst = reinterpret_cast<uint4*>(out + c);
-          dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          for (int c = 0; c < 64; c += 16) {
+            uint32_t g[16], u[16];
+            tmem_ld16(taddr + c0 + c, g);
+            tmem_ld16(taddr + NB / 2 + c0 + c, u);
+            tmem_ld_wait();
+            uint32_t pk[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              pk[i] = pack2bf(silu(__uint_as_float(g[2 * i])) * __uint_as_float(u[2 * i]),
+                              silu(__uint_as_float(g[2 * i + 1])) * __uint_as_float(u[2 * i + 1]));
+            uint4* sw = reinterpret_cast<uint4*>(stg + lane * kOutRowBytes + c * 2);
+            sw[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            sw[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
+          __syncwarp();
+          const size_t col = size_t(nt) * (NB / 2) + c0 + (lane & 7) * 8;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int r = 4 * i + (lane >> 3);
+            const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kOutRowBytes + (lane & 7) * 16);
+            *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.out) + (grow0 + r) * p.ldo + col) = v;
+          }
+          __syncwarp();
         }
       } else if constexpr (EPI == EPI_DOWN) {  // U = s (A v) in bf16, the first ldo columns
         uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo;
@@ -533,17 +556,27 @@ __global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __gri
           if (c + 16 <= p.ldo) dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
       } else {
-        float* out = reinterpret_cast<float*>(p.out) + grow * p.ldo + size_t(nt) * NB;
+        // eight rounds of 32 fp32 columns (128 bytes per row)
 #pragma unroll 1
-        for (int c = 0; c < NB; c += 16) {
-          uint32_t v[16];
-          tmem_ld16(taddr + c, v);
-          tmem_ld_wait();
-          float4* dst = reinterpret_cast<float4*>(out + c);
+        for (int c0 = 0; c0 < NB; c0 += 32) {
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
-                                 __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
+          for (int c = 0; c < 32; c += 16) {
+            uint32_t v[16];
+            tmem_ld16(taddr + c0 + c, v);
+            tmem_ld_wait();
+            uint4* sw = reinterpret_cast<uint4*>(stg + lane * kOutRowBytes + c * 4);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) sw[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          }
+          __syncwarp();
+          const size_t col = size_t(nt) * NB + c0 + (lane & 7) * 4;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int r = 4 * i + (lane >> 3);
+            const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kOutRowBytes + (lane & 7) * 16);
+            *reinterpret_cast<uint4*>(reinterpret_cast<float*>(p.out) + (grow0 + r) * p.ldo + col) = v;
+          }
+          __syncwarp();
         }
       }
       tc_fence_before();
@@ -624,8 +657,8 @@ bool encode_adapter_a2(CUtensorMap* m, const void* a2, uint64_t w, uint32_t r) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int group_for(size_t a_tile_bytes) {
-  const size_t budget = size_t(48) << 20;  // activation rows kept hot in L2 per group
+int group_for(size_t a_tile_bytes, size_t budget_mb) {
+  const size_t budget = budget_mb << 20;  // activation rows kept hot in L2 per group
   size_t g = budget / (a_tile_bytes ? a_tile_bytes : 1);
   return g < 1 ? 1 : int(g > 4096 ? 4096 : g);
 }
@@ -683,13 +716,15 @@ cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sm
   p13.ntiles_n = int(w / (BN / 2));
   p13.ldo = int(w);
   p13.b_half = int(w);
-  p13.group_m = group_for(size_t(BM) * d * 2);
+  // L2 budgets per group of m-tiles, from same-box sweeps of 6-48 MB over the Mixtral- and
+  // DeepSeek-V2-Lite-shaped T = 4096 layers (GEMM13 best at 24 MB, GEMM2 at 12 MB)
+  p13.group_m = group_for(size_t(BM) * d * 2, 24);
   p2.out = a.o;
   p2.kblocks = int(w / BK);
   p2.ntiles_n = int(d / BN);
   p2.ldo = int(d);
   p2.b_half = 0;
-  p2.group_m = group_for(size_t(BM) * w * 2);
+  p2.group_m = group_for(size_t(BM) * w * 2, 12);
   if (a.lrank > 0) {
     const LoraOffsets lo = lora_offsets(a.d, a.w, a.lrank);
     for (int sgi = 0; sgi < a.nseg; ++sgi) {
