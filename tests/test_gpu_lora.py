@@ -99,3 +99,41 @@ def test_lora_full_size(shape, T, n_rows):
                                shared_triples(lw, shape), lora=[split(b) for b in ad],
                                shared_lora=[split(b) for b in sad], lora_scale=2.0)
     check_output(y[torch.from_numpy(rows).to(DEV)], ref, TOL_BF16, f"{shape.name} T={T} lora")
+
+
+@pytest.mark.parametrize("shape,T", [(I.MIXTRAL, 4096), (I.DSV2_LITE, 4096), (I.DSV2_LITE, 64),
+                                     (BF_MIX, 300)],
+                         ids=["mixtral-T4096", "deepseek-T4096", "deepseek-b64", "small-T300"])
+@pytest.mark.parametrize("kind", ["zero-B", "no-adapter"])
+def test_lora_without_effect_equals_plain_forward_bitwise(shape, T, kind):
+    """Adapters whose up matrices are zero, or no adapter on any expert, add exact zeros: the
+    Stage-2 forward then equals the plain forward bit for bit. On the tcgen05 path this runs the
+    down projections, the builder warp's extra k-blocks and their hand-off, all adding 0."""
+    seed = 90 + T
+    lw = weights(shape)
+    kept = [int(e) for e in np.nonzero(I.keep_mask(seed, shape.E, shape.E * 3 // 4))[0]]
+    ids = I.random_ids(seed, 1, T, shape.K, shape.E, hot=kept, p_hot=1.0)[0]
+    gate = np.random.default_rng(seed).uniform(0.05, 1.0, (T, shape.K)).astype(np.float32)
+    x = I.hidden_iid(seed, shape, T).to(DEV)
+    idx, g = torch.from_numpy(ids).to(DEV), torch.from_numpy(gate).to(DEV)
+    experts = [lw.experts[e].to(DEV) if e in kept else None for e in range(shape.E)]
+    shared = [b.to(DEV) for b in lw.shared]
+
+    def zero_b(b):
+        b = b.clone()
+        for t, part in zip(I.split_lora(b, shape, 8), range(6)):
+            if part % 2 == 1:  # B1, B3, B2
+                t.zero_()
+        return b.to(DEV)
+
+    if kind == "zero-B":
+        ad = [zero_b(I.lora_block(seed, shape, e, 8)) if e in kept else None for e in range(shape.E)]
+        sad = [zero_b(I.lora_block(seed, shape, ("shared", s), 8)) for s in range(shape.n_shared)]
+    else:
+        ad = [None] * shape.E
+        sad = [None] * shape.n_shared
+    desc = M.desc_of(shape)
+    y_l = M.mcft_moe_forward_lora(desc, x, idx, g, experts, shared, ad, sad, 8, 2.0)
+    y_p = M.mcft_moe_forward(desc, x, idx, g, experts, shared)
+    M.mcft_device_error()
+    assert torch.equal(y_l, y_p), f"{shape.name} T={T} {kind}"
