@@ -94,6 +94,18 @@ __global__ void __launch_bounds__(32) mask_sample_kernel(const __grid_constant__
   }
 }
 
+// Four consecutive dL/dy values of a row (bf16 or fp32) as fp32.
+template <typename TY>
+__device__ __forceinline__ void load_dy4(const void* row, int c, float* dy) {
+  if constexpr (sizeof(TY) == 2) {
+    const uint2 v = *reinterpret_cast<const uint2*>(reinterpret_cast<const uint16_t*>(row) + c);
+    dy[0] = bf16lo(v.x); dy[1] = bf16hi(v.x); dy[2] = bf16lo(v.y); dy[3] = bf16hi(v.y);
+  } else {
+    const float4 v = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(row) + c);
+    dy[0] = v.x; dy[1] = v.y; dy[2] = v.z; dy[3] = v.w;
+  }
+}
+
 template <typename TY>
 __global__ void __launch_bounds__(256) gate_grad_kernel(const __grid_constant__ GateGradArgs a) {
   pdl_wait();
@@ -104,26 +116,45 @@ __global__ void __launch_bounds__(256) gate_grad_kernel(const __grid_constant__ 
     const int t = i / a.K;
     const size_t row = size_t(a.pos[i]) * a.d;
     float acc = 0.f;
-    for (int c = lane * 4; c < a.d; c += 128) {
-      float4 o = *reinterpret_cast<const float4*>(a.o + row + c);
-      for (int p = 1; p < a.ks; ++p) {
-        const float4 u = *reinterpret_cast<const float4*>(a.o + size_t(p) * a.o_plane + row + c);
-        o.x += u.x; o.y += u.y; o.z += u.z; o.w += u.w;
+    const void* dyrow = sizeof(TY) == 2
+        ? static_cast<const void*>(reinterpret_cast<const uint16_t*>(a.dy) + size_t(t) * a.d)
+        : static_cast<const void*>(reinterpret_cast<const float*>(a.dy) + size_t(t) * a.d);
+    if (a.ks == 1) {  // one plane (the tcgen05 path): 8 chunks in flight per lane, summed in order
+      for (int c0 = lane * 4; c0 < a.d; c0 += 128 * 8) {
+        float4 o[8];
+        float dy[8][4];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int c = c0 + 128 * j;
+          if (c < a.d) {
+            o[j] = __ldcs(reinterpret_cast<const float4*>(a.o + row + c));
+            load_dy4<TY>(dyrow, c, dy[j]);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (c0 + 128 * j < a.d) {
+            acc = fmaf(dy[j][0], o[j].x, acc);
+            acc = fmaf(dy[j][1], o[j].y, acc);
+            acc = fmaf(dy[j][2], o[j].z, acc);
+            acc = fmaf(dy[j][3], o[j].w, acc);
+          }
+        }
       }
-      float dy[4];
-      if constexpr (sizeof(TY) == 2) {
-        const uint2 v = *reinterpret_cast<const uint2*>(
-            reinterpret_cast<const uint16_t*>(a.dy) + size_t(t) * a.d + c);
-        dy[0] = bf16lo(v.x); dy[1] = bf16hi(v.x); dy[2] = bf16lo(v.y); dy[3] = bf16hi(v.y);
-      } else {
-        const float4 v = *reinterpret_cast<const float4*>(
-            reinterpret_cast<const float*>(a.dy) + size_t(t) * a.d + c);
-        dy[0] = v.x; dy[1] = v.y; dy[2] = v.z; dy[3] = v.w;
+    } else {
+      for (int c = lane * 4; c < a.d; c += 128) {
+        float4 o = *reinterpret_cast<const float4*>(a.o + row + c);
+        for (int p = 1; p < a.ks; ++p) {
+          const float4 u = *reinterpret_cast<const float4*>(a.o + size_t(p) * a.o_plane + row + c);
+          o.x += u.x; o.y += u.y; o.z += u.z; o.w += u.w;
+        }
+        float dy[4];
+        load_dy4<TY>(dyrow, c, dy);
+        acc = fmaf(dy[0], o.x, acc);
+        acc = fmaf(dy[1], o.y, acc);
+        acc = fmaf(dy[2], o.z, acc);
+        acc = fmaf(dy[3], o.w, acc);
       }
-      acc = fmaf(dy[0], o.x, acc);
-      acc = fmaf(dy[1], o.y, acc);
-      acc = fmaf(dy[2], o.z, acc);
-      acc = fmaf(dy[3], o.w, acc);
     }
     acc = warp_sum(acc);
     if (lane == 0) a.dgate[i] = acc;
