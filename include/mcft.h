@@ -144,9 +144,12 @@ mcft_status mcft_moe_forward(const mcft_layer_desc* desc, const void* x, int T, 
  *                3 r (d + w) elements, 16-byte aligned
  *   shared_lora  host array [n_shared], same layout (NULL entries allowed; NULL if n_shared = 0)
  *   lora_rank    8 or 16 (MCFT_ERR_UNSUPPORTED otherwise); lora_scale finite
- * The workspace needs mcft_moe_workspace_size_lora(desc, lora_rank, T) bytes. The down
- * projections A v run in a small kernel per stage; the up projections are added in the epilogue
- * of the expert GEMM / GEMV of every path. No dropout (a forward whose output is compared). */
+ * The workspace needs mcft_moe_workspace_size_lora(desc, lora_rank, T) bytes. On the tensor-core
+ * path (bf16, T > 64) the down projections are skinny GEMMs on the tensor cores and the up
+ * projections one extra k-block of each adapted tile of the expert GEMMs; on the decode and fp32
+ * paths a small kernel computes A v and the up projections are added as the expert GEMV finishes
+ * each output. Adapters that add nothing (B = 0, or none) give mcft_moe_forward's result bit for
+ * bit. No dropout (a forward whose output is compared). */
 mcft_status mcft_moe_workspace_size_lora(const mcft_layer_desc* desc, int lora_rank, int T_max,
                                          size_t* bytes);
 mcft_status mcft_moe_forward_lora(const mcft_layer_desc* desc, const void* x, int T,

@@ -12,7 +12,7 @@
 // and the up projections ride on the expert GEMMs as one extra k-block per adapted tile,
 // D += U B'^T, so the tensor cores add them to the accumulators and the epilogues are unchanged.
 //
-// One persistent CTA per SM, 6 warps:
+// One persistent CTA per SM, 6 warps (7 with adapters):
 //   warp 0  - TMA producer (one thread): A tile 128x64 and B tile 256x64 per stage, 4 stages,
 //             128-byte swizzle, one mbarrier with a transaction count per stage;
 //   warp 1  - allocates 512 TMEM columns (two 128x256 fp32 accumulators) and issues
