@@ -76,7 +76,7 @@ struct WsLayout {
   int pad;        // rows per segment are padded to a multiple of this (128 on the TC path)
   int mcap;       // capacity in permuted rows
   int ks;         // partial planes of o (contraction split of the decode GEMM2)
-  size_t hdr, cnt, off, pos, perm, done, xp, h, o, u13, u2, total;
+  size_t hdr, cnt, off, pos, perm, done, pscr, xp, h, o, u13, u2, total;
 };
 WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lrank = 0);
 
@@ -124,7 +124,10 @@ struct PermuteArgs {
   int* perm;   // [mcap] token of each permuted row, -1 for padding
   unsigned* err;
   int* done;   // [E+S + kClaimSlots] progress and claim counters of the fused decode FFN, zeroed here
+  int* scr;    // NULL, or kPermScrInts of scratch: large batches then permute in chunks
 };
+constexpr int kPermChunks = 256;  // most chunks of the large-batch permutation
+constexpr int kPermScrInts = kPermChunks * kMaxE + kPermChunks;
 cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s);
 
 struct GatherArgs {
