@@ -18,9 +18,12 @@
 //   warp 1  - allocates 512 TMEM columns (two 128x256 fp32 accumulators) and issues
 //             tcgen05.mma (M=128, N=256, K=16) from one thread; tcgen05.commit frees a stage /
 //             publishes an accumulator;
-//   warps 2-5 - epilogue: tcgen05.ld of their 32-lane quarter, SwiGLU or fp32 store; they release
-//             the accumulator so the next tile's MMAs overlap this tile's epilogue;
+//   warps 2-5 - epilogue: tcgen05.ld of their 32-lane quarter, SwiGLU or fp32, staged through
+//             shared memory and stored as whole 128-byte row segments; they release the
+//             accumulator so the next tile's MMAs overlap this tile's epilogue;
 //   warp 6  - with adapters only: writes each adapted tile's extra k-block (see LoraOps).
+// The down projections use the same roles with N = 16 or 32: 8 stages of 18-20 KB, 32 or 64 TMEM
+// columns, bf16 rows written directly.
 // Tiles are walked m-fastest inside groups of m-tiles so concurrently running CTAs share weight
 // tiles (and the activation group) in L2. Every wait is bounded: after 2 s the kernel records
 // MCFT_ERR_TIMEOUT, stops issuing, waits (bounded) for its copies and MMAs in flight, frees TMEM
