@@ -134,14 +134,15 @@ def test_ffn_empty_and_bad_ids():
     lw = weights(sh)
     desc = M.desc_of(sh)
     ex = [b.to(DEV) for b in lw.experts]
-    x = I.hidden_iid(12, sh, 100).to(DEV)
+    x = I.hidden_iid(12, sh, 3000).to(DEV)
     y0 = torch.empty((0, sh.d), dtype=torch.bfloat16, device=DEV)
     M.mcft_moe_forward(desc, x[:0], torch.empty((0, 2), dtype=torch.int32, device=DEV),
                        torch.empty((0, 2), device=DEV), ex, y=y0)
     M.mcft_device_error()
     # an id out of range: the device error word is set and y is left untouched (every decode
-    # kernel variant: 1, 16 and 64 tokens; and the tensor-core path)
-    for T in (1, 16, 64, 100):
+    # kernel variant: 1, 16 and 64 tokens; the tensor-core path; and 6000 assignments, which the
+    # chunked permutation handles)
+    for T in (1, 16, 64, 100, 3000):
         idx = torch.zeros((T, 2), dtype=torch.int32, device=DEV)
         idx[:, 1] = 1
         idx[T // 2, 1] = sh.E
@@ -152,7 +153,7 @@ def test_ffn_empty_and_bad_ids():
         assert ei.value.status == M.MCFT_ERR_INVALID
         assert torch.all(y == 7.0)
     # a selected expert with no weights
-    for T in (1, 16, 64, 100):
+    for T in (1, 16, 64, 100, 3000):
         idx = torch.zeros((T, 2), dtype=torch.int32, device=DEV)
         idx[:, 1] = 2
         missing = list(ex)
@@ -163,3 +164,16 @@ def test_ffn_empty_and_bad_ids():
             M.mcft_device_error()
         assert torch.all(y == 7.0)
     M.mcft_device_error()
+
+
+@pytest.mark.parametrize("shape,T", [(SMALL_BF16, 2049), (SMALL_BF16, 2500), (SMALL_DS, 700)],
+                         ids=["mix-4098", "mix-5000", "ds-4200"])
+def test_ffn_chunked_permutation(shape, T):
+    """Just above 4096 assignments the permutation runs in chunks (ragged: 820 to 1000
+    assignments each, shared-expert rows filled by every chunk's CTA); every output row matches
+    the oracle."""
+    lw = weights(shape)
+    x = I.hidden_iid(13, shape, T)
+    idx, gate = _routing(shape, T, 13, hot=range(shape.keep))
+    y = _forward(shape, x, idx, gate, lw)
+    check_output(y, _reference(shape, x, idx, gate, lw), TOL_BF16, f"{shape.name} T={T}")
