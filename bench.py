@@ -651,6 +651,20 @@ def _make_masked_batch(sh, T, seed, dev):
     return desc, kept, experts, shared, x, idx, gate
 
 
+def lora_work(shape, T, rank):
+    """Algorithmic work of a Stage-2 forward of T tokens, every permuted row adapted (rank r):
+    bytes of the two tcgen05 down projections (each gathered x row and each h row read once,
+    s [A1 x | A3 x] and s A2 h written in bf16) and FLOP of the base GEMMs, of the adapters' up
+    projections (the extra k-blocks) and of their down projections."""
+    rows = T * (shape.K + shape.n_shared)
+    r, d, w = rank, shape.d, shape.w
+    return dict(rows=rows,
+                down_bytes=rows * (d * 2 + 2 * r * 2) + rows * (w * 2 + r * 2),
+                base_flop=2.0 * rows * 3 * d * w,
+                up_flop=2.0 * rows * (2 * w + d) * r,
+                down_flop=2.0 * rows * (2 * d + w) * r)
+
+
 def run_lora(steps, warmup, seed, dev, peaks, rank=8, shapes=(I.MIXTRAL, I.DSV2_LITE), T=4096):
     """The Stage-2 forward (experts of the fixed concentration set with rank-8 LoRA adapters,
     alpha 16; the shared experts adapted too) against the plain forward on the same batch: T tokens
@@ -695,14 +709,10 @@ def run_lora(steps, warmup, seed, dev, peaks, rank=8, shapes=(I.MIXTRAL, I.DSV2_
             profs.append(M.mcft_profile_read())
         prof_plain, prof = profs
         M.mcft_device_error()
-        rows = T * (sh.K + sh.n_shared)  # permuted rows, all of them adapted
-        r, d, w = rank, sh.d, sh.w
-        # lora_down (two tcgen05 launches): every gathered row (x) and every h row read once,
-        # s [A1 x | A3 x] and s A2 h written in bf16
-        ld_bytes = rows * (d * 2 + 2 * r * 2) + rows * (w * 2 + r * 2)
-        f_base = 2.0 * rows * 3 * d * w
-        f_up = 2.0 * rows * (2 * w + d) * r  # the adapters' up projections (extra k-blocks)
-        f_down = 2.0 * rows * (2 * d + w) * r
+        wk = lora_work(sh, T, rank)
+        r = rank
+        ld_bytes, f_base, f_up, f_down = (wk["down_bytes"], wk["base_flop"], wk["up_flop"],
+                                          wk["down_flop"])
         nl, msl = prof.get("lora_down", (0, 0.0))
         n13, ms13 = prof.get("gemm13_tc", (0, 0.0))
         n2, ms2 = prof.get("gemm2_tc", (0, 0.0))

@@ -49,3 +49,16 @@ def test_traffic_ratio_is_null_for_a_changed_source(tmp_path, monkeypatch):
     digest = hashlib.sha256(b"kernel source").hexdigest()[:16]
     monkeypatch.setitem(bench.TRAFFIC, "k", ("k.cu", digest, 1.25, "profiles/k.md"))
     assert bench.traffic_ratio("k") == 1.25
+
+
+def test_lora_work_mixtral():
+    """Mixtral-shaped T = 4096, rank 8: 8192 permuted rows; the down projections read each 8 KB
+    x row and each 28 KB h row once and write 16 + 8 bf16 values; the base GEMMs are 2.886 TFLOP
+    and the adapters add 0.25 % (up) on the tensor cores."""
+    wk = bench.lora_work(I.MIXTRAL, 4096, 8)
+    assert wk["rows"] == 8192
+    assert wk["down_bytes"] == 8192 * (4096 * 2 + 32) + 8192 * (14336 * 2 + 16)
+    assert wk["base_flop"] == pytest.approx(2.886e12, rel=1e-3)
+    assert wk["up_flop"] / wk["base_flop"] == pytest.approx(8 * (2 * 14336 + 4096) / (3 * 4096 * 14336))
+    # DeepSeek: the two shared experts are adapted rows too
+    assert bench.lora_work(I.DSV2_LITE, 4096, 8)["rows"] == 4096 * 8
