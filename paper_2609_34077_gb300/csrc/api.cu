@@ -116,7 +116,7 @@ WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lran
   L.pos = o;  o = align256(o + sizeof(int) * size_t(T) * K);
   L.perm = o; o = align256(o + sizeof(int) * size_t(L.mcap));
   L.done = o; o = align256(o + sizeof(int) * (nseg + kClaimSlots));
-  L.pscr = o; o = align256(o + (T * K > 4096 ? sizeof(int) * kPermScrInts : 0));
+  L.pscr = o; o = align256(o + (T * K > kPermSingleMax ? sizeof(int) * kPermScrInts : 0));
   L.xp = o;   o = align256(o + (L.tc ? size_t(L.mcap) * d * 2 : 0));
   L.h = o;    o = align256(o + size_t(L.mcap) * w * (dtype == MCFT_BF16 ? 2 : 4));
   L.o = o;    o = align256(o + size_t(L.ks) * L.mcap * d * 4);
@@ -378,7 +378,7 @@ mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, cons
 
   int* done = reinterpret_cast<int*>(ws + L.done);
   PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err, done,
-                 T * K > 4096 ? reinterpret_cast<int*>(ws + L.pscr) : nullptr};
+                 T * K > kPermSingleMax ? reinterpret_cast<int*>(ws + L.pscr) : nullptr};
   cudaError_t e = launch_permute(pa, stream);
   if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
 

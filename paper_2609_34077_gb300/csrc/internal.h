@@ -126,7 +126,8 @@ struct PermuteArgs {
   int* done;   // [E+S + kClaimSlots] progress and claim counters of the fused decode FFN, zeroed here
   int* scr;    // NULL, or kPermScrInts of scratch: large batches then permute in chunks
 };
-constexpr int kPermChunks = 256;  // most chunks of the large-batch permutation
+constexpr int kPermChunks = 256;      // most chunks of the large-batch permutation
+constexpr int kPermSingleMax = 4096;  // up to this many assignments one CTA permutes (faster)
 constexpr int kPermScrInts = kPermChunks * kMaxE + kPermChunks;
 cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s);
 

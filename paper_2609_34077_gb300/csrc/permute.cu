@@ -144,7 +144,6 @@ __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant
 // kChunk assignments. The scratch holds, per chunk, its per-expert counts (turned into the
 // chunk's first position inside each expert) and whether it saw an invalid id.
 constexpr int kChunk = 1024;
-constexpr int kSingleMax = 4 * kChunk;  // up to this many assignments the single CTA is faster
 
 __device__ __forceinline__ int* chunk_row(const PermuteArgs& a, int c) { return a.scr + c * kMaxE; }
 __device__ __forceinline__ int* chunk_bad(const PermuteArgs& a) { return a.scr + kPermChunks * kMaxE; }
@@ -248,7 +247,7 @@ cudaError_t launch_permute(const PermuteArgs& a, cudaStream_t s) {
   const int n = a.T * a.K;
   prof_begin(kProfPermute, s);
   cudaError_t e;
-  if (a.scr == nullptr || n <= kSingleMax) {
+  if (a.scr == nullptr || n <= kPermSingleMax) {
     e = launch_pdl(permute_kernel, dim3(1), dim3(kThreads), 0, s, a);
   } else {
     int nchunks = (n + kChunk - 1) / kChunk;
