@@ -747,6 +747,13 @@ def run_lora(steps, warmup, seed, dev, peaks, rank=8, shapes=(I.MIXTRAL, I.DSV2_
     return out
 
 
+def gate_grad_bytes(shape, T):
+    """Algorithmic bytes of one gate-gradient call: each routed row's fp32 expert output read
+    once, dL/dy read once per token (bf16), the permuted row index read and dL/dg written."""
+    rows = T * shape.K
+    return rows * shape.d * 4 + T * shape.d * 2 + rows * 4 * 2
+
+
 def run_mask(calls, warmup, seed, dev, peaks, T=4096):
     """The Stage-1 mask machinery on a fine-tuning batch of T tokens per shape, each kernel timed
     alone with the L2 flushed before every call: mcft_mask_sample for every layer at once
@@ -781,8 +788,7 @@ def run_mask(calls, warmup, seed, dev, peaks, T=4096):
                 f()
         us = {k: 1e3 * time_calls(f, calls, stream, flush) for k, f in fns.items()}
         M.mcft_device_error()
-        rows = T * sh.K
-        gg_bytes = rows * sh.d * 4 + T * sh.d * 2 + rows * 4 * 2  # o rows, dy, pos in, dgate out
+        gg_bytes = gate_grad_bytes(sh, T)
         a = gg_bytes / (us["gate_grad"] / 1e6) / 1e9
         out[sh.name] = dict(
             workload=f"{sh.name} T={T}, {L} layers x {sh.E} experts, keep {keep}",

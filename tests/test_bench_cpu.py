@@ -62,3 +62,11 @@ def test_lora_work_mixtral():
     assert wk["up_flop"] / wk["base_flop"] == pytest.approx(8 * (2 * 14336 + 4096) / (3 * 4096 * 14336))
     # DeepSeek: the two shared experts are adapted rows too
     assert bench.lora_work(I.DSV2_LITE, 4096, 8)["rows"] == 4096 * 8
+
+
+def test_gate_grad_bytes():
+    """Mixtral-shaped T = 4096: 8192 fp32 rows of 16 KB, 4096 bf16 dL/dy rows of 8 KB, ids and
+    gradients: 167.8 MB, the figure the ncu capture reads back."""
+    b = bench.gate_grad_bytes(I.MIXTRAL, 4096)
+    assert b == 8192 * 4096 * 4 + 4096 * 4096 * 2 + 8192 * 8
+    assert b / 1e6 == pytest.approx(167.84, abs=0.01)
