@@ -27,6 +27,10 @@
  *    ran out of time) set a device error word and make the remaining kernels of that call skip
  *    their work; mcft_device_error() reads and clears it.
  *  - No call throws; mcft_last_error() returns a message for the calling thread's last error.
+ *  - The library keeps, per device, the device addresses of its own static device arrays (the
+ *    error word, the scratch of mcft_moe_forward_noalloc), looked up on first use. A
+ *    cudaDeviceReset() destroys the context those addresses belong to: after one, no mcft call may
+ *    be made on that device in the same process, and handles created before it are invalid.
  *  - Layouts are row-major. dtype MCFT_BF16 means bf16 x, weights and y (fp32 accumulation);
  *    MCFT_F32 means fp32 everywhere (CUDA-core arithmetic, no TF32).
  */
@@ -167,8 +171,10 @@ mcft_status mcft_moe_forward_lora(const mcft_layer_desc* desc, const void* x, in
  * the library (held by every GPU that loads it, until exit), enough for decode calls of up to 64
  * tokens of the Mixtral- and DeepSeek-V2-Lite-shaped layers; a call needing more returns
  * MCFT_ERR_UNSUPPORTED (use mcft_moe_forward). The first call on a device looks up the array's
- * device address; make it before any stream capture. All calls share the array: calls whose
- * kernels overlap on the GPU race and must be serialised by the caller. Allocates nothing. */
+ * device address; make it before any stream capture. The address is kept for the life of the
+ * process, so after a cudaDeviceReset() this entry point must not be called on that device again.
+ * All calls share the array: calls whose kernels overlap on the GPU race and must be serialised by
+ * the caller. Allocates nothing. */
 mcft_status mcft_moe_forward_noalloc(const mcft_layer_desc* desc, const void* x, int T,
                                      const int32_t* idx, const float* gate,
                                      const void* const* experts, const void* const* shared,

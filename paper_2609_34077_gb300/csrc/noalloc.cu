@@ -13,7 +13,9 @@
 // calls are rejected with MCFT_ERR_UNSUPPORTED. In host code the array's name is only a host-side
 // stand-in, so the device address is looked up once per device with cudaGetSymbolAddress, with
 // that device current, on the first call made on it (make that first call before any stream
-// capture). Every call shares the array and it keeps the last call's contents: nothing in it needs
+// capture). The looked-up address is kept for the life of the process: after a cudaDeviceReset
+// the context it belonged to is gone, and this entry point must not be called on that device
+// again. Every call shares the array and it keeps the last call's contents: nothing in it needs
 // to start at zero (the first kernel of a call writes the header and offsets the later kernels
 // read), but calls whose kernels overlap on the GPU (different streams, or different host threads)
 // race on it and must be serialised by the caller. This entry point calls no cudaMalloc,

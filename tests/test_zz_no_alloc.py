@@ -4,9 +4,10 @@ Some callers cannot allocate device memory when they run a layer: a plugin insid
 that owns every device allocation through its own pool, or a decode loop that cannot take an
 allocation's implicit synchronisation. mcft_moe_forward_noalloc serves them from a fixed scratch
 array inside the library instead of a caller-provided workspace. These tests check that two calls
-in a row (the array keeps the previous call's contents) give the outputs of the workspace entry
-point, within the bf16 output tolerance the other parity tests use, and that a call needing more
-scratch than the array holds is refused. This file is collected last on purpose.
+in a row (the array keeps the previous call's contents) give exactly the bits of the workspace
+entry point (both run the same kernels with the same workspace layout, so any difference, even in
+the low bits, would mean stale scratch leaking into a call), and that a call needing more scratch
+than the array holds is refused. This file is collected last on purpose.
 """
 import numpy as np
 import pytest
@@ -41,6 +42,7 @@ def test_noalloc_matches_workspace_forward_two_calls(shape, T):
         y_ref = M.mcft_moe_forward(desc, x, idx, gate, experts, shared)
         y = M.mcft_moe_forward_noalloc(desc, x, idx, gate, experts, shared)
         M.mcft_device_error()
+        assert torch.equal(y, y_ref), f"{shape.name} call {call}: outputs differ from the workspace call"
         check_output(y, f64(y_ref), TOL_BF16, f"{shape.name} call {call}")
 
 
