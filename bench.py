@@ -40,18 +40,14 @@ from paper_2609_34077_gb300 import inputs as I  # noqa: E402
 STREAM_STEPS = 512
 METRIC = "masked MoE layer tokens/s"
 
-# DRAM traffic per launch / algorithmic bytes, from one ncu capture of the kernel (summary and
-# command in profiles/), keyed by the first 16 hex digits of the kernel source's sha256: when
-# the source has changed since the capture, the bench reports traffic as null.
+# DRAM traffic per launch / algorithmic bytes, from one ncu capture of the kernel, keyed by the
+# first 16 hex digits of the kernel source's sha256: when the source has changed since the
+# capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None,
-                     "profiles/dec_fused_kernel_decode.md"),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None,
-                    "profiles/dec_fused_kernel_decode.md"),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", 1.0017,
-                   "profiles/dec_fused_kernel_decode.md"),
-    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "ae0482332aaf7dee", 0.9558,
-              "profiles/fetch_kernel_mixtral_decode_b16.md"),
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None),
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None),
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", 1.0017),
+    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "ae0482332aaf7dee", 0.9558),
 }
 
 
@@ -60,10 +56,10 @@ def traffic_ratio(kernel):
 
     if kernel not in TRAFFIC:
         return None
-    src, digest, ratio, summary = TRAFFIC[kernel]
+    src, digest, ratio = TRAFFIC[kernel]
     cur = hashlib.sha256(open(os.path.join(ROOT, src), "rb").read()).hexdigest()[:16]
     if cur != digest:
-        print(f"bench: {src} changed since the ncu capture in {summary} "
+        print(f"bench: {src} changed since the ncu capture of {kernel} "
               f"(sha {cur}, captured {digest}): traffic for {kernel} reported as null",
               file=sys.stderr)
         return None
@@ -179,14 +175,23 @@ class DecodeLayer:
         self.x = self.x_host.to(dev)
         self.wr = self.lw.router.to(dev)
         self.shared = [b.to(dev) for b in self.lw.shared]
-        self.cache = M.mcft_cache_create(1, shape.E, shape.cache_slots, shape.expert_bytes,
-                                         self.lw.experts, max_assign=batch * shape.K)
+        self.cache = None
+        self.new_cache()
         self.ws = torch.empty(M.mcft_moe_workspace_size(self.desc, batch), dtype=torch.uint8, device=dev)
         self.idx = torch.empty((STREAM_STEPS, batch, shape.K), dtype=torch.int32, device=dev)
         self.gate = torch.empty((STREAM_STEPS, batch, shape.K), dtype=torch.float32, device=dev)
         self.y = torch.empty((batch, shape.d), dtype=torch.bfloat16, device=dev)
         self.compute = torch.cuda.current_stream(dev)
         self.copy = torch.cuda.Stream(dev)
+
+    def new_cache(self):
+        """Replace the expert cache by an empty one (same slots, policy and host pool)."""
+        torch.cuda.synchronize(self.dev)
+        if self.cache is not None:
+            self.M.mcft_cache_destroy(self.cache)
+        self.cache = self.M.mcft_cache_create(1, self.shape.E, self.shape.cache_slots,
+                                              self.shape.expert_bytes, self.lw.experts,
+                                              max_assign=self.batch * self.shape.K)
 
     def step(self, s, x=None, path="device"):
         """One decode step. path "device": the cache step's kernel publishes the expert table and
@@ -221,19 +226,50 @@ def time_steps(fn, first, steps, stream):
 
 
 def host_link_probe(dev, nbytes):
-    """Pinned host -> device copy bandwidth (GB/s), best of 10."""
+    """Pinned host -> device bandwidth (GB/s) of nbytes by two methods: the copy engines (one
+    copy, and the same bytes split into 2 and 4 concurrent copies on separate streams) and SM
+    loads (the fetch kernel's copy loop, mcft_host_copy, on 38 / 76 / 152 CTAs); best of 10 (one
+    copy) or 5 (the others). Returns the rates and their best."""
+    from paper_2609_34077_gb300 import mcft as M
+
     src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
     dst = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-    best = 0.0
-    for _ in range(10):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
-        dst.copy_(src, non_blocking=True)
-        b.record()
-        torch.cuda.synchronize()
-        best = max(best, nbytes / (a.elapsed_time(b) / 1e3) / 1e9)
+    cur = torch.cuda.current_stream(dev)
+    res = {}
+
+    def best_of(reps, enqueue):
+        best = 0.0
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(cur)
+            enqueue(a)
+            b.record(cur)
+            torch.cuda.synchronize()
+            best = max(best, nbytes / (a.elapsed_time(b) / 1e3) / 1e9)
+        return best
+
+    for n in (1, 2, 4):
+        streams = [torch.cuda.Stream(dev) for _ in range(n)]
+        chunk = -(-nbytes // n)
+
+        def copies(start, streams=streams, chunk=chunk):
+            for i, st in enumerate(streams):
+                st.wait_event(start)
+                with torch.cuda.stream(st):
+                    dst[i * chunk:(i + 1) * chunk].copy_(src[i * chunk:(i + 1) * chunk],
+                                                         non_blocking=True)
+            for st in streams:
+                cur.wait_stream(st)
+
+        res[f"copy_engine_{n}_streams_gbs"] = best_of(10 if n == 1 else 5, copies)
+    for blocks in (38, 76, 152):
+        res[f"sm_loads_{blocks}_ctas_gbs"] = best_of(
+            5, lambda start, blocks=blocks: M.mcft_host_copy(dst, src, blocks, stream=cur))
+    M.mcft_device_error()
+    res["best_gbs"] = max(res.values())
     del src, dst
-    return best
+    return res
 
 
 def unique_per_step(idx_steps):
@@ -273,81 +309,111 @@ def decode_roofline(prof, U, steps, batch, shape, peaks):
     return roof, rates
 
 
-def run_decode(shape, batch, steps, warmup, seed, dev, peaks, path="device", clocks=None,
-               world=1):
-    """Decode `steps` timed steps of one layer (after `warmup`), kernels timed with CUDA events.
-    Returns (layer, result dict, elapsed seconds of this rank, clock summary)."""
-    from paper_2609_34077_gb300 import mcft as M
+def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks=None, world=1):
+    """One measured pass over the decode steps [first, first + steps) of layer L.
 
-    L = DecodeLayer(shape, batch, seed, dev)
-    for s in range(warmup):
+    The pass starts from an empty cache and runs the untimed steps 0 .. first - 1 first, so every
+    pass makes the same cache decisions and moves the same bytes over the same steps. With
+    `profile` the library brackets each kernel with CUDA events (per-kernel times; a pass of its
+    own, so the instrumentation never touches the headline time). With `e2e` every step also copies
+    its hidden states from pinned host memory to the device and its output back to pinned host
+    memory, on the compute stream inside the timed region. Returns (elapsed seconds, (hits,
+    fetches, bypass) over the timed steps, per-kernel profile or None, bytes copied per step)."""
+    M = L.M
+    L.new_cache()
+    for s in range(first):
         L.step(s, path=path)
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
-    h0, f0, b0 = M.mcft_cache_stats(L.cache, 0)
-    M.mcft_profile_reset()
-    M.mcft_profile_enable(True)
+    c0 = M.mcft_cache_stats(L.cache, 0)
+    io_bytes = (0, 0)
+    if e2e:
+        xd = torch.empty((L.batch, L.shape.d), dtype=torch.bfloat16, device=L.dev)
+        y_host = torch.empty((L.batch, L.shape.d), dtype=torch.bfloat16).pin_memory()
+
+        def fn(s):
+            xd.copy_(L.x_host[s % STREAM_STEPS], non_blocking=True)
+            y = L.step(s, x=xd, path=path)
+            y_host.copy_(y, non_blocking=True)
+
+        io_bytes = (xd.numel() * 2, y_host.numel() * 2)
+    else:
+        def fn(s):
+            L.step(s, path=path)
+    if profile:
+        M.mcft_profile_reset()
+        M.mcft_profile_enable(True)
     if clocks is not None:
         with clocks:
-            elapsed = time_steps(lambda s: L.step(s, path=path), warmup, steps, L.compute)
+            elapsed = time_steps(fn, first, steps, L.compute)
     else:
-        elapsed = time_steps(lambda s: L.step(s, path=path), warmup, steps, L.compute)
-    M.mcft_profile_enable(False)
+        elapsed = time_steps(fn, first, steps, L.compute)
+    prof = None
+    if profile:
+        M.mcft_profile_enable(False)
+        prof = M.mcft_profile_read()
     if world > 1:
         torch.distributed.barrier()
-    prof = M.mcft_profile_read()
     M.mcft_device_error()
-    h1, f1, b1 = M.mcft_cache_stats(L.cache, 0)
-    pos = [(s % STREAM_STEPS) for s in range(warmup, warmup + steps)]
+    c1 = M.mcft_cache_stats(L.cache, 0)
+    return elapsed, tuple(int(b - a) for a, b in zip(c0, c1)), prof, io_bytes
+
+
+def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world=1, e2e=False):
+    """Decode `steps` timed steps of one layer after `warmup` untimed ones, in four measured passes
+    over the same steps from the same cache state (decode_pass), after one untimed pass:
+      1. the headline time: device-driven fetch, no instrumentation (clocks sampled here);
+      2. with `e2e`: the same with host <-> device copies of each step's inputs and output;
+      3. the same as 1 with per-kernel CUDA events (kernel times, launches, FFN and fetch rooflines);
+      4. the host-driven fetch (host reads the miss list, copy engine), kernels timed: the expert
+         FFN then runs alone on the GPU.
+    Returns (result dict, GPU routing ids [512, batch, K] on the host, elapsed seconds of pass 1)."""
+    L = DecodeLayer(shape, batch, seed, dev)
+    # an untimed pass over the same steps first: the first reads of the pinned host pool map its
+    # pages for the device, which later passes (and any long-running decode) no longer pay
+    decode_pass(L, warmup, steps)
+    elapsed, cnt, _, _ = decode_pass(L, warmup, steps, clocks=clocks, world=world)
+    passes = {"timed": cnt}
+    e2e_res = None
+    if e2e:
+        el_e, cnt_e, _, (bi, bo) = decode_pass(L, warmup, steps, e2e=True)
+        passes["e2e"] = cnt_e
+        e2e_res = dict(value=batch * steps / el_e, elapsed_s=el_e, unit="tokens/s", h2d_bytes_per_step=bi,
+                       d2h_bytes_per_step=bo, ms_per_step=el_e * 1e3 / steps,
+                       steps="the same decode steps as value, from the same cache state")
+    el_p, cnt_p, prof, _ = decode_pass(L, warmup, steps, profile=True)
+    passes["profiled"] = cnt_p
+    el_h, cnt_h, hprof, _ = decode_pass(L, warmup, steps, path="host", profile=True)
+    passes["host_fetch"] = cnt_h
+    pos = [s % STREAM_STEPS for s in range(warmup, warmup + steps)]
     U = unique_per_step([L.idx[p] for p in pos])
-    hits, fetches, byp = h1 - h0, f1 - f0, b1 - b0
+    hits, fetches, byp = cnt
     roof, rates = decode_roofline(prof, U, steps, batch, shape, peaks)
+    roof_alone, rates_alone = decode_roofline(hprof, U, steps, batch, shape, peaks)
     fetch_bytes = fetches * shape.expert_bytes / steps
     out = dict(
         tokens_per_s=batch * steps / elapsed, ms_per_step=elapsed * 1e3 / steps, steps=steps,
-        fetch_path=path, hits=hits, fetches=fetches, bypass=byp,
+        warmup=warmup, fetch_path="device", hits=hits, fetches=fetches, bypass=byp,
         fetches_per_step=fetches / steps, fetches_per_token=fetches / (steps * batch),
         hit_rate=hits / max(1, hits + fetches), mean_experts_per_step=float(np.mean(U)),
         fetch_bytes_per_step=fetch_bytes,
+        passes_same_decisions=all(c == cnt for c in passes.values()),
+        profiled_ms_per_step=el_p * 1e3 / steps,
         kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
-        gpu_launches=int(sum(v[0] for v in prof.values() if v[0])), roofline=roof, kernel_gbs=rates,
-        kernel_ms_per_step=sum(v[1] for k, v in prof.items() if k != "fetch") / steps,
+        gpu_launches=int(sum(v[0] for v in prof.values() if v[0])), roofline=roof,
+        kernel_gbs=rates, kernel_ms_per_step=sum(v[1] for k, v in prof.items() if k != "fetch") / steps,
+        roofline_alone=dict(roof_alone or {}, note="same FFN kernel in the host-driven step, "
+                            "where it runs alone"),
+        host_fetch_path=dict(tokens_per_s=batch * steps / el_h, ms_per_step=el_h * 1e3 / steps,
+                             kernel_gbs=rates_alone),
     )
-    return L, out, elapsed
-
-
-def alone_roofline(L, shape, batch, steps, first, peaks):
-    """The same decode steps with the host-driven fetch (the host reads the miss list, the copy
-    engine moves the experts): the expert FFN then runs alone on the GPU. Returns its roofline."""
-    from paper_2609_34077_gb300 import mcft as M
-
-    M.mcft_profile_reset()
-    M.mcft_profile_enable(True)
-    time_steps(lambda s: L.step(s, path="host"), first, steps, L.compute)
-    M.mcft_profile_enable(False)
-    prof = M.mcft_profile_read()
-    pos = [s % STREAM_STEPS for s in range(first, first + steps)]
-    roof, _ = decode_roofline(prof, unique_per_step([L.idx[p] for p in pos]), steps, batch, shape,
-                              peaks)
-    return dict(roof or {}, note="same FFN kernel in the host-driven step, where it runs alone")
-
-
-def run_decode_e2e(L, steps, first):
-    """Same decode steps through the public calls with the hidden states in pinned host memory:
-    each step copies its inputs host -> device and its output device -> host."""
-    xd = torch.empty((L.batch, L.shape.d), dtype=torch.bfloat16, device=L.dev)
-    y_host = torch.empty((L.batch, L.shape.d), dtype=torch.bfloat16).pin_memory()
-
-    def step(s):
-        xd.copy_(L.x_host[s % STREAM_STEPS], non_blocking=True)
-        y = L.step(s, x=xd)
-        y_host.copy_(y, non_blocking=True)
-
-    elapsed = time_steps(step, first, steps, L.compute)
-    nb = L.batch * L.shape.d * 2
-    return dict(value=L.batch * steps / elapsed, unit="tokens/s", h2d_bytes_per_step=nb,
-                d2h_bytes_per_step=nb)
+    if e2e_res is not None:
+        out["e2e"] = e2e_res
+    idx_host = L.idx.cpu().numpy()
+    del L
+    torch.cuda.empty_cache()
+    return out, idx_host, elapsed
 
 
 class DecodeStack:
@@ -841,6 +907,96 @@ def oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0, lw=None, warmu
             return batch * n / el, n
 
 
+def oracle_fetch_check(shape, batch, seed, idx_gpu, first, steps):
+    """Checks a decode run's routing and fetch counts against the CPU oracle (the metric's
+    "fetches/token exact"): the oracle routes every stream position the run used (fp64, Eq.
+    inference with the run's prior), the GPU's ids are compared with it token by token, and two
+    oracle caches (Section 4.1 LRU) replay steps 0 .. first + steps - 1, one on the oracle's ids and
+    one on the GPU's. Returns the counts over the timed steps [first, first + steps): tokens routed,
+    near ties (relative gap between the K-th and (K+1)-th score below 1e-4), tokens whose ids differ
+    from the oracle's (inside / outside the near-tie band) and hits and fetches of both replays."""
+    import oracle
+
+    n = first + steps
+    xs = I.ar1_streams(seed, shape, STREAM_STEPS, batch)
+    wr = I.router_weight(seed, shape).double().numpy()
+    prior = I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep))
+    ref = {}
+    for p in sorted({s % STREAM_STEPS for s in range(n)}):
+        ref[p] = oracle.routing.route(xs[p].double().numpy(), wr, shape.K,
+                                      oracle.routing.MODE_SOFT_PRIOR, shape.gate, prior=prior)
+    near = near_order = diff_in = diff_out = 0
+    c_ref = oracle.cache.SlotCache(shape.E, shape.cache_slots, "LRU")
+    c_gpu = oracle.cache.SlotCache(shape.E, shape.cache_slots, "LRU")
+    tot = dict(oracle_hits=0, oracle_fetches=0, replay_hits=0, replay_fetches=0)
+    for s in range(n):
+        p = s % STREAM_STEPS
+        r, g = ref[p], idx_gpu[p]
+        ho, fo, _, _ = c_ref.step(r["idx"])
+        hg, fg, _, _ = c_gpu.step(g)
+        if s < first:
+            continue
+        tot["oracle_hits"] += ho
+        tot["oracle_fetches"] += fo
+        tot["replay_hits"] += hg
+        tot["replay_fetches"] += fg
+        nk = r["gap_k"] < 1e-4
+        ni = r["gap_in"] < 1e-4
+        near += int(nk.sum())
+        near_order += int((ni & ~nk).sum())
+        differ = np.any(g != r["idx"], axis=1)
+        diff_in += int((differ & (nk | ni)).sum())
+        diff_out += int((differ & ~(nk | ni)).sum())
+    return dict(tokens=steps * batch, near_tie_tokens=near, near_tie_rule="(s_K - s_K+1) / s_K < 1e-4",
+                order_only_near_ties=near_order, ids_differ_in_band=diff_in,
+                ids_differ_outside_band=diff_out, **tot)
+
+
+def fetch_verdict(chk, gpu_hits, gpu_fetches):
+    """fetches_exact: the GPU's counted hits and fetches over the timed steps equal the oracle's
+    (routing and cache both from the oracle); cache_exact: they equal the oracle cache's on the
+    GPU's own ids (the cache decision alone, independent of near ties in routing)."""
+    chk = dict(chk, gpu_hits=gpu_hits, gpu_fetches=gpu_fetches)
+    chk["cache_exact"] = (gpu_hits, gpu_fetches) == (chk["replay_hits"], chk["replay_fetches"])
+    chk["fetches_exact"] = (gpu_hits, gpu_fetches) == (chk["oracle_hits"], chk["oracle_fetches"])
+    chk["routing_exact_outside_band"] = chk["ids_differ_outside_band"] == 0
+    return chk
+
+
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the platform string)."""
+    import platform
+
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().lower().startswith("model name"):
+                return ln.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for ln in open("/proc/cpuinfo"):
+            if ln.lower().startswith("model name"):
+                return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.processor() or platform.machine()
+
+
+def oracle_timing_one_thread(shape, batch, seed, budget_s):
+    """The same oracle timing in a fresh interpreter whose BLAS uses one thread. Returns
+    (tokens/s, timed steps) or None if the child failed."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    cmd = [sys.executable, os.path.abspath(__file__), "--oracle-timing",
+           json.dumps(dict(shape=shape.name, batch=batch, seed=seed, budget_s=budget_s))]
+    try:
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=budget_s + 300)
+        d = json.loads(r.stdout.strip().splitlines()[-1])
+        return d["tokens_per_s"], d["steps"]
+    except (OSError, subprocess.SubprocessError, ValueError, IndexError, KeyError):
+        return None
+
+
 def reference_arm(args, rank, world):
     """The reference arm: there is no reference implementation to run (the paper ships no code),
     so this times the CPU oracle as it stands on the host cores, on the same workload, metric and
@@ -858,6 +1014,7 @@ def reference_arm(args, rank, world):
                 scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
                 config=_config(batch),
                 cpu_baseline=dict(value=tps, unit="tokens/s", cores=_CORES, kind="oracle",
+                                  cpu_model=cpu_model(),
                                   sample=f"{n} decode steps x batch {batch} of the same stream "
                                          f"after {args.warmup} untimed (fp64 numpy)"),
                 e2e=dict(value=tps, unit="tokens/s", h2d_bytes_per_step=0, d2h_bytes_per_step=0))
@@ -943,7 +1100,14 @@ def main():
                     help="chain workloads: experts prefetched per layer (0 = off)")
     ap.add_argument("--policy", default="LRU", choices=["LRU", "LFU", "FIFO"])
     ap.add_argument("--graph", action="store_true", help="stack workloads: replay a captured step")
+    ap.add_argument("--oracle-timing", help=argparse.SUPPRESS)  # child of oracle_timing_one_thread
     args = ap.parse_args()
+    if args.oracle_timing:
+        o = json.loads(args.oracle_timing)
+        sh = {s_.name: s_ for s_ in (I.MIXTRAL, I.DSV2_LITE)}[o["shape"]]
+        tps, n = oracle_decode_tokens_per_s(sh, o["batch"], o["seed"], budget_s=o["budget_s"])
+        print(json.dumps(dict(tokens_per_s=tps, steps=n)), flush=True)
+        return 0
     if args.workload in ("lora", "mask") or args.case in ("lora", "mask"):
         import __graft_entry__
 
@@ -1009,34 +1173,27 @@ def main():
     shape, batch = I.MIXTRAL, args.batch
 
     clk = ClockSampler(local)
-    L, d, elapsed = run_decode(shape, batch, args.steps, args.warmup, seed, dev, peaks,
-                               path="device", clocks=clk, world=world)
+    d, idx_main, elapsed = run_decode(shape, batch, args.steps, args.warmup, seed, dev, peaks,
+                                      clocks=clk, world=world, e2e=True)
     max_el, tokens = aggregate(elapsed, batch * args.steps, world)
-    first = args.warmup + args.steps
-    e2e = run_decode_e2e(L, args.steps, first)
-    # the same steps with the host-driven fetch (host reads the miss list, copy engine): the
-    # expert FFN then runs alone on the GPU
-    first += args.steps
-    M.mcft_profile_reset()
-    M.mcft_profile_enable(True)
-    host_el = time_steps(lambda s: L.step(s, path="host"), first, args.steps, L.compute)
-    M.mcft_profile_enable(False)
-    hprof = M.mcft_profile_read()
-    hpos = [s % STREAM_STEPS for s in range(first, first + args.steps)]
-    host_roof, host_rates = decode_roofline(hprof, unique_per_step([L.idx[p] for p in hpos]),
-                                            args.steps, batch, shape, peaks)
     link = host_link_probe(dev, shape.expert_bytes)
     ms = max_el * 1e3 / args.steps
     # the dominant kernel of the device-driven step is the fetch: bound by the host link
     nf, msf = d["kernels"].get("fetch", {}).get("launches", 0), d["kernels"].get("fetch", {}).get("ms", 0.0)
     fetched = d["fetch_bytes_per_step"] * args.steps
     fetch_roof = dict(bound="host-link", kernel="fetch", unit="GB/s",
-                      achieved=fetched / (msf / 1e3) / 1e9 if msf else None, peak=link,
-                      peak_source="pinned host-to-device copy probe in this run (352 MB, best of 10)",
+                      achieved=fetched / (msf / 1e3) / 1e9 if msf else None, peak=link["best_gbs"],
+                      peak_source="best pinned host-to-device rate of the link probes in this run "
+                                  "(352 MB: copy engines with 1, 2, 4 concurrent copies; SM loads "
+                                  "on 38, 76, 152 CTAs)",
                       traffic=(traffic_ratio("fetch") * fetched / max(1, nf)
                                if traffic_ratio("fetch") else None),
-                      alg_bytes_per_launch=fetched / max(1, nf), launches=nf)
-    fetch_roof["frac"] = fetch_roof["achieved"] / link if msf else None
+                      alg_bytes_per_launch=fetched / max(1, nf), launches=nf,
+                      timed_in="the profiled pass over the same steps (kernel CUDA events)")
+    fetch_roof["frac"] = fetch_roof["achieved"] / link["best_gbs"] if msf else None
+    e2e = dict(d["e2e"])
+    el_e2e, tok_e2e = aggregate(e2e.pop("elapsed_s"), batch * args.steps, world)
+    e2e["value"] = tok_e2e / el_e2e
     line = dict(
         metric=METRIC, value=tokens / max_el, unit="tokens/s", n_gpus=world, steps=args.steps,
         warmup=args.warmup, ms_per_step=ms, higher_is_better=True,
@@ -1044,50 +1201,67 @@ def main():
         roofline=fetch_roof,
         roofline_ffn=dict(d["roofline"] or {}, note="decode FFN inside the device-driven step, "
                           "sharing SMs and HBM with the concurrent fetch kernel"),
-        roofline_ffn_alone=dict(host_roof or {}, note="same kernel in the host-driven step, "
-                                "where it runs alone"),
+        roofline_ffn_alone=d["roofline_alone"],
         kernel_gbs=d["kernel_gbs"],
-        e2e=e2e, gpu_launches=d["gpu_launches"], clocks=clk.summary(), kernels=d["kernels"],
+        e2e=e2e, gpu_launches=d["gpu_launches"],
+        gpu_launches_note="kernels launched by the same steps in the profiled pass",
+        clocks=clk.summary(), kernels=d["kernels"],
+        timing=dict(value="CUDA events around the timed steps, no per-kernel instrumentation",
+                    profiled_ms_per_step=d["profiled_ms_per_step"],
+                    passes_same_decisions=d["passes_same_decisions"]),
         cache=dict(policy="LRU", hits=d["hits"], fetches=d["fetches"], bypass=d["bypass"],
                    fetches_per_step=d["fetches_per_step"], fetches_per_token=d["fetches_per_token"],
                    hit_rate=d["hit_rate"], mean_experts_per_step=d["mean_experts_per_step"]),
         fetch=dict(path="device-driven (fetch kernel on a copy stream, overlapped with the hit "
                         "experts' FFN)",
-                   bytes_per_step=d["fetch_bytes_per_step"], host_link_probe_gbs=link,
-                   link_roofline_ms_per_step=d["fetch_bytes_per_step"] / (link * 1e9) * 1e3,
-                   link_frac=(d["fetch_bytes_per_step"] / (ms / 1e3)) / (link * 1e9),
+                   bytes_per_step=d["fetch_bytes_per_step"], host_link_probe=link,
+                   link_roofline_ms_per_step=d["fetch_bytes_per_step"] / (link["best_gbs"] * 1e9) * 1e3,
+                   link_frac=(d["fetch_bytes_per_step"] / (ms / 1e3)) / (link["best_gbs"] * 1e9),
                    kernel_ms_per_step=d["kernel_ms_per_step"]),
-        host_fetch_path=dict(tokens_per_s=batch * args.steps / host_el,
-                             ms_per_step=host_el * 1e3 / args.steps, kernel_gbs=host_rates),
+        host_fetch_path=d["host_fetch_path"],
     )
-    del L
-    torch.cuda.empty_cache()
+    runs = {"mixtral_b%d" % batch: (shape, batch, seed, idx_main, args.steps, d)}
     if not args.no_extra:
         nb1 = min(args.steps, 256)
-        Lb, b1, _ = run_decode(shape, 1, nb1, args.warmup, seed + 1, dev, peaks)
+        b1, idx_b1, _ = run_decode(shape, 1, nb1, args.warmup, seed + 1, dev, peaks)
         b1.pop("kernels", None)
-        b1["roofline_alone"] = alone_roofline(Lb, shape, 1, nb1, args.warmup + nb1, peaks)
         line["batch1"] = b1
-        del Lb
-        for bsz in (1, 64):
+        runs["mixtral_b1"] = (shape, 1, seed + 1, idx_b1, nb1, b1)
+        for bsz in (1, 8, 64):
             nds = min(args.steps, 128)
-            Ld, ds, _ = run_decode(I.DSV2_LITE, bsz, nds, args.warmup, seed + 3, dev, peaks)
+            ds, idx_ds, _ = run_decode(I.DSV2_LITE, bsz, nds, args.warmup, seed + 3, dev, peaks)
             ds.pop("kernels", None)
-            ds["roofline_alone"] = alone_roofline(Ld, I.DSV2_LITE, bsz, nds, args.warmup + nds,
-                                                  peaks)
             line[f"dsv2_b{bsz}"] = ds
-            del Ld
-            torch.cuda.empty_cache()
+            runs[f"dsv2_b{bsz}"] = (I.DSV2_LITE, bsz, seed + 3, idx_ds, nds, ds)
         line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)
         line["stage2_lora"] = run_lora(8, 3, seed + 4, dev, peaks)
         line["stage1_mask"] = run_mask(20, 3, seed + 4, dev, peaks)
         _BATCHES.clear()
         torch.cuda.empty_cache()
     if rank == 0 and not args.no_cpu_baseline:
+        # the oracle as a checker of the timed steps: routing (near ties counted) and fetch counts
+        checks = {}
+        for name, (sh, bsz, sd, idx_h, n, res) in runs.items():
+            chk = fetch_verdict(oracle_fetch_check(sh, bsz, sd, idx_h, args.warmup, n),
+                                res["hits"], res["fetches"])
+            checks[name] = chk
+            if name == "mixtral_b%d" % batch:
+                line["cache"]["oracle_check"] = chk
+            else:
+                line["batch1" if name == "mixtral_b1" else name]["oracle_check"] = chk
+        line["fetches_exact"] = all(c["fetches_exact"] for c in checks.values())
+        line["cache_exact"] = all(c["cache_exact"] for c in checks.values())
+        line["near_tie_tokens"] = {k: c["near_tie_tokens"] for k, c in checks.items()}
+        # the oracle as the timed baseline: all cores, then one thread in a fresh interpreter
         tps, n = oracle_decode_tokens_per_s(shape, batch, seed, budget_s=12.0)
+        one = oracle_timing_one_thread(shape, batch, seed, 12.0)
         line["cpu_baseline"] = dict(value=tps, unit="tokens/s", cores=_CORES, kind="oracle",
+                                    cpu_model=cpu_model(),
                                     sample=f"{n} decode steps x batch {batch} of the same stream "
-                                           "(fp64 numpy, BLAS threads = cores)")
+                                           "(fp64 numpy, BLAS threads = cores)",
+                                    one_thread=(dict(value=one[0], unit="tokens/s", cores=1,
+                                                     sample=f"{one[1]} decode steps x batch {batch}")
+                                                if one else None))
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

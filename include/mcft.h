@@ -232,6 +232,18 @@ mcft_status mcft_cache_step(mcft_cache* cache, int layer, const int32_t* idx, in
 mcft_status mcft_fetch_experts(mcft_cache* cache, int layer, mcft_stream_t compute_stream,
                                mcft_stream_t copy_stream, const void** expert_ptrs);
 
+/* mcft_host_copy: copy `bytes` from pinned host memory to device memory with the device-driven
+ * fetch's copy loop (64 KB pieces, 16-byte loads, four in flight per thread) on a grid of `blocks`
+ * CTAs of 256 threads. The paper has no counterpart: offloaded decoding is bound by this host link
+ * (Section 1), and this call measures what SM loads get from it at a chosen grid size, beside the
+ * copy engines. host_src: host memory the device can address (pinned memory, or any host memory
+ * on a system whose GPU reads pageable memory, such as a Grace-based node); dst: device memory;
+ * both 16-byte aligned; bytes a multiple of 16; 1 <= blocks <= 65535. MCFT_ERR_INVALID for a
+ * pointer that is NULL or misaligned, for a host_src the device cannot address, for
+ * bytes % 16 != 0 or a bad block count. Asynchronous on `stream`. */
+mcft_status mcft_host_copy(void* dst, const void* host_src, size_t bytes, int blocks,
+                           mcft_stream_t stream);
+
 /* ---------------------------------------------------------------------------------------------
  * Stage-1 mask machinery (Section 3.2 "Stage 1" Eq. stage1 and "Mask optimization" Eq. ste).
  *

@@ -644,6 +644,24 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
   return MCFT_OK;
 }
 
+mcft_status mcft_host_copy(void* dst, const void* host_src, size_t bytes, int blocks,
+                           mcft_stream_t stream) {
+  if (!dst || !host_src) return fail(MCFT_ERR_INVALID, "NULL pointer");
+  if ((reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(host_src)) % 16)
+    return fail(MCFT_ERR_INVALID, "pointers must be 16-byte aligned");
+  if (bytes % 16) return fail(MCFT_ERR_INVALID, "bytes = %zu is not a multiple of 16", bytes);
+  if (blocks < 1 || blocks > 65535) return fail(MCFT_ERR_INVALID, "blocks = %d out of range", blocks);
+  if (bytes == 0) return MCFT_OK;
+  void* src = nullptr;
+  if (cudaHostGetDevicePointer(&src, const_cast<void*>(host_src), 0) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(MCFT_ERR_INVALID, "host_src is not host memory the device can address");
+  }
+  const cudaError_t e = launch_host_copy(dst, src, bytes, blocks, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "host copy kernel launch");
+  return MCFT_OK;
+}
+
 mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_stream,
                                mcft_stream_t copy_stream, const void** expert_ptrs) {
   mcft::NvtxRange nvtx_range("mcft_fetch_experts");

@@ -42,6 +42,21 @@ __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ Pr
   prefetch_warp(a);
 }
 
+// One 64 KB piece [w0, w1) of a copy, in 16-byte words: each thread keeps four loads in flight
+// before it stores them, so a CTA has 64 KB of reads outstanding on the host link.
+__device__ __forceinline__ void copy_piece(const uint4* src, uint4* dst, size_t w0, size_t w1) {
+  const size_t stride = blockDim.x;
+  for (size_t w = w0 + threadIdx.x; w < w1; w += 4 * stride) {
+    uint4 v[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (w + j * stride < w1) v[j] = src[w + j * stride];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (w + j * stride < w1) dst[w + j * stride] = v[j];
+  }
+}
+
 // Copy the missed experts' blocks host -> device with 16-byte loads over the host link. Work
 // units are 64 KB pieces of the missed blocks, spread over the grid.
 __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ FetchArgs a) {
@@ -64,16 +79,20 @@ __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ Fetc
     const size_t w0 = (u % per) * piece;
     const size_t w1 = w0 + piece < words ? w0 + piece : words;
     if (a.moved && threadIdx.x == 0) atomicAdd(a.moved, (unsigned long long)(w1 - w0) * 16ull);
-    const size_t stride = blockDim.x;
-    for (size_t w = w0 + threadIdx.x; w < w1; w += 4 * stride) {
-      uint4 v[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (w + j * stride < w1) v[j] = src[w + j * stride];
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (w + j * stride < w1) dst[w + j * stride] = v[j];
-    }
+    copy_piece(src, dst, w0, w1);
+  }
+}
+
+// A plain copy of `words` 16-byte words from device-visible host memory with the fetch kernel's
+// pieces and load loop: measures what SM loads get from the host link at a given grid size.
+__global__ void __launch_bounds__(256) host_copy_kernel(const uint4* __restrict__ src,
+                                                        uint4* __restrict__ dst, size_t words) {
+  pdl_wait();
+  const size_t piece = 4096;
+  const size_t units = (words + piece - 1) / piece;
+  for (size_t u = blockIdx.x; u < units; u += gridDim.x) {
+    const size_t w0 = u * piece;
+    copy_piece(src, dst, w0, w0 + piece < words ? w0 + piece : words);
   }
 }
 
@@ -84,6 +103,14 @@ cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool pr
   prof_begin(kid, s);
   fetch_kernel<<<blocks, 256, 0, s>>>(a);
   prof_end(kid, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_host_copy(void* dst, const void* src, size_t bytes, int blocks, cudaStream_t s) {
+  prof_begin(kProfHostCopy, s);
+  host_copy_kernel<<<blocks, 256, 0, s>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst),
+                                          bytes / 16);
+  prof_end(kProfHostCopy, s);
   return cudaGetLastError();
 }
 

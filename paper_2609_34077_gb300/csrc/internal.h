@@ -294,6 +294,8 @@ struct FetchArgs {
   unsigned long long* moved;          // prefetch fetches: bytes copied (accumulated), else NULL
 };
 cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch = false);
+// Plain copy from device-visible host memory with the fetch kernel's load loop (bytes % 16 == 0).
+cudaError_t launch_host_copy(void* dst, const void* src, size_t bytes, int blocks, cudaStream_t s);
 
 // Fused decode prologue of one chained-stack layer at batch 1 (prologue.cu): residual update and
 // RMSNorm, routing of layer l, cache step of layer l, prediction and prefetch event of layer l+1,
@@ -386,7 +388,7 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
        kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfNorm,
-       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfDecFused, kProfCount };
+       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfDecFused, kProfHostCopy, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

@@ -33,6 +33,7 @@ SIGNATURES = {
     "mcft_cache_create": (_i, [_i, _i, _i, _sz, _vp, _i, _i, C.POINTER(_vp)]),
     "mcft_cache_step": (_i, [_vp, _i, _vp, _i, _i, _vp]),
     "mcft_fetch_experts": (_i, [_vp, _i, _vp, _vp, _vp]),
+    "mcft_host_copy": (_i, [_vp, _vp, _sz, _i, _vp]),
     "mcft_moe_forward_cached": (_i, [_vp, _vp, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _sz, _vp, _vp]),
     "mcft_mask_sample": (_i, [_vp, _vp, _i, _i, _i, _vp, _vp, _vp]),
     "mcft_gate_grad": (_i, [_vp, _vp, _i, _vp, _sz, _vp, _vp]),
@@ -271,6 +272,15 @@ def mcft_fetch_experts(cache: Cache, layer, compute_stream=None, copy_stream=Non
     _check(lib().mcft_fetch_experts(C.c_void_p(cache.handle), layer, _stream(compute_stream),
                                     _stream(copy_stream), C.cast(out, C.c_void_p)))
     return [v or 0 for v in out]
+
+
+def mcft_host_copy(dst, host_src, blocks, stream=None):
+    """Copy the pinned host tensor host_src into the device tensor dst (same byte size) with the
+    fetch kernel's copy loop on `blocks` CTAs."""
+    nbytes = host_src.numel() * host_src.element_size()
+    assert dst.numel() * dst.element_size() == nbytes, "dst and host_src differ in size"
+    _check(lib().mcft_host_copy(_ptr(dst), _ptr(host_src), nbytes, int(blocks), _stream(stream)))
+    return dst
 
 
 def mcft_moe_forward_cached(desc: LayerDesc, x, idx, gate, cache: Cache, layer, shared=(), y=None,

@@ -76,3 +76,10 @@ def test_host_validation_without_gpu(libpath):
     assert L.mcft_cache_create(1, 8, 0, 0, None, 2, 0, C.byref(h)) == mcft.MCFT_ERR_INVALID
     assert L.mcft_cache_create(1, 8, 4, 0, None, 2, 7, C.byref(h)) == mcft.MCFT_ERR_INVALID
     assert b"policy" in L.mcft_last_error()
+    # host copy probe: alignment, size and grid are checked before any CUDA call
+    assert L.mcft_host_copy(None, C.c_void_p(16), 16, 1, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_host_copy(C.c_void_p(16), C.c_void_p(24), 16, 1, None) == mcft.MCFT_ERR_INVALID
+    assert b"aligned" in L.mcft_last_error()
+    assert L.mcft_host_copy(C.c_void_p(16), C.c_void_p(32), 40, 1, None) == mcft.MCFT_ERR_INVALID
+    assert b"multiple of 16" in L.mcft_last_error()
+    assert L.mcft_host_copy(C.c_void_p(16), C.c_void_p(32), 64, 0, None) == mcft.MCFT_ERR_INVALID

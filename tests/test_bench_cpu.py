@@ -2,6 +2,7 @@
 every weight byte of the experts the step computes (the routed experts it selected and the shared
 experts, which every token uses) plus the activations, and the achieved rate is those bytes over
 the measured kernel time."""
+import numpy as np
 import pytest
 
 import bench
@@ -42,12 +43,12 @@ def test_decode_roofline_counts_shared_experts(shape, T, U):
 def test_traffic_ratio_is_null_for_a_changed_source(tmp_path, monkeypatch):
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     (tmp_path / "k.cu").write_text("kernel source")
-    monkeypatch.setitem(bench.TRAFFIC, "k", ("k.cu", "0" * 16, 1.0, "profiles/k.md"))
+    monkeypatch.setitem(bench.TRAFFIC, "k", ("k.cu", "0" * 16, 1.0))
     assert bench.traffic_ratio("k") is None
     import hashlib
 
     digest = hashlib.sha256(b"kernel source").hexdigest()[:16]
-    monkeypatch.setitem(bench.TRAFFIC, "k", ("k.cu", digest, 1.25, "profiles/k.md"))
+    monkeypatch.setitem(bench.TRAFFIC, "k", ("k.cu", digest, 1.25))
     assert bench.traffic_ratio("k") == 1.25
 
 
@@ -70,3 +71,47 @@ def test_gate_grad_bytes():
     b = bench.gate_grad_bytes(I.MIXTRAL, 4096)
     assert b == 8192 * 4096 * 4 + 4096 * 4096 * 2 + 8192 * 8
     assert b / 1e6 == pytest.approx(167.84, abs=0.01)
+
+
+def _oracle_ids(shape, batch, seed, n):
+    import oracle
+
+    xs = I.ar1_streams(seed, shape, bench.STREAM_STEPS, batch)
+    wr = I.router_weight(seed, shape).double().numpy()
+    prior = I.prior_from_mask(I.keep_mask(seed, shape.E, shape.keep))
+    idx = np.zeros((bench.STREAM_STEPS, batch, shape.K), np.int32)
+    for p in range(n):
+        idx[p] = oracle.routing.route(xs[p].double().numpy(), wr, shape.K,
+                                      oracle.routing.MODE_SOFT_PRIOR, shape.gate, prior=prior)["idx"]
+    return idx
+
+
+def test_oracle_fetch_check_counts_and_flags():
+    """The bench's fetches-exact check: the oracle's own ids pass with matching counts; a changed
+    id outside a near tie is reported, and counts that differ from the replay are not exact."""
+    import oracle
+
+    shape, batch, seed, first, steps = I.DSV2_LITE, 2, 5, 4, 12
+    idx = _oracle_ids(shape, batch, seed, first + steps)
+    chk = bench.oracle_fetch_check(shape, batch, seed, idx, first, steps)
+    assert chk["tokens"] == steps * batch and chk["ids_differ_outside_band"] == 0
+    assert (chk["oracle_hits"], chk["oracle_fetches"]) == (chk["replay_hits"], chk["replay_fetches"])
+    # counts taken independently: a fresh LRU over the same ids
+    c = oracle.cache.SlotCache(shape.E, shape.cache_slots, "LRU")
+    h = f = 0
+    for s in range(first + steps):
+        hs, fs, _, _ = c.step(idx[s])
+        if s >= first:
+            h, f = h + hs, f + fs
+    ok = bench.fetch_verdict(chk, h, f)
+    assert ok["fetches_exact"] and ok["cache_exact"] and ok["routing_exact_outside_band"]
+    assert not bench.fetch_verdict(chk, h, f + 1)["fetches_exact"]
+    # plant a different expert for one token of a timed step (not a near tie): flagged
+    bad = idx.copy()
+    t_pos = first + 3
+    row = bad[t_pos, 0]
+    row[-1] = next(e for e in range(shape.E) if e not in row)
+    chk2 = bench.oracle_fetch_check(shape, batch, seed, bad, first, steps)
+    assert chk2["ids_differ_outside_band"] + chk2["ids_differ_in_band"] == 1
+    assert not bench.fetch_verdict(chk2, h, f)["routing_exact_outside_band"] or \
+        chk2["ids_differ_in_band"] == 1

@@ -84,6 +84,20 @@ def test_cache_fetch_copies_expert_bytes():
     M.mcft_device_error()
 
 
+@pytest.mark.parametrize("nbytes,blocks", [(16, 1), (65536, 1), (65536 + 48, 3),
+                                           (5 * 65536 + 16 * 77, 38), (17301504, 152)])
+def test_host_copy_moves_every_byte(nbytes, blocks):
+    """The link probe's SM-load copy: whole and ragged 64 KB pieces, grids smaller and larger than
+    the piece count; the bytes after the copied range stay untouched."""
+    g = torch.Generator().manual_seed(nbytes)
+    src = torch.randint(0, 256, (nbytes,), generator=g, dtype=torch.uint8).pin_memory()
+    dst = torch.full((nbytes + 64,), 0xAB, dtype=torch.uint8, device=DEV)
+    M.mcft_host_copy(dst[:nbytes], src, blocks)
+    torch.cuda.synchronize()
+    assert torch.equal(dst[:nbytes].cpu(), src)
+    assert bool((dst[nbytes:] == 0xAB).all())
+
+
 @pytest.mark.parametrize("policy", ["LRU", "LFU", "FIFO"])
 def test_cache_export_import_resume(policy):
     """Run N steps == run n steps, export, import into a fresh cache, run the other N - n."""
