@@ -36,6 +36,12 @@ __device__ __forceinline__ uint4 ldg16(const void* p) {
   return __ldg(reinterpret_cast<const uint4*>(p));
 }
 
+// Ask L2 to fetch [p, p + bytes) from memory (no destination; p 16-byte aligned, bytes a multiple
+// of 16): one instruction puts a whole tile's reads in flight.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 // 16-byte load through L2 only (coherent with stores of other CTAs of the same kernel that were
 // published with a fence: no stale L1 line can be returned).
 __device__ __forceinline__ uint4 ldcg16(const void* p) {
@@ -80,6 +86,16 @@ __device__ __forceinline__ uint16_t f2bf(float f) {
 
 __device__ __forceinline__ uint32_t pack2bf(float a, float b) {
   return uint32_t(f2bf(a)) | (uint32_t(f2bf(b)) << 16);
+}
+
+// D += A B on the tensor cores, one warp: A 16 x 16 bf16 (row), B 16 x 8 bf16 (col), D fp32.
+__device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
 __device__ __forceinline__ float silu(float u) { return u / (1.0f + expf(-u)); }

@@ -150,15 +150,6 @@ __device__ __forceinline__ int dec_pos(const DecItems& it, int item) {
   return lo;
 }
 
-__device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
-                                         uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
 // A lane of quad position c holds elements 8c..8c+7 (lo) and 32+8c..32+8c+7 (hi) of a 64-wide
 // chunk. MMA step j (0..3) uses 32-bit words 2j and 2j+1 of (lo, hi): for each c these are 4
 // elements, and over the 4 lanes of the quad and the 4 steps every element is used exactly once.

@@ -54,6 +54,8 @@ struct RouteArgs {
   unsigned* err;
 };
 cudaError_t launch_route(const RouteArgs& a, int dtype, cudaStream_t s);
+// bf16 calls of more tokens than this route in 16-token tensor-core tiles (route.cu).
+constexpr int kRouteTileMinT = 64;
 
 // Header at the start of the forward workspace.
 // Work-claim counters of the fused decode FFN that follow the per-segment progress counters in

@@ -1,4 +1,5 @@
-// Router GEMV + mask / prior + Top-K + gate softmax, one CTA per token.
+// Router GEMV + mask / prior + Top-K + gate softmax: one CTA per token at decode sizes, tiles of
+// 16 tokens on the tensor cores at prefill sizes (route_tile_kernel, bf16).
 //
 // z = W x (Section 3.1); the score is z (plain Top-K, Eq. topk), z restricted to m_e = 1 (hard
 // mask, Eq. stage1) or z_e + log pi_e (soft prior, Eq. inference: log(p_e pi_e) = z_e + log pi_e
@@ -15,6 +16,8 @@
 // and added in shared memory in a fixed order; warp 0 ranks (two experts per lane, shuffle
 // arg-max) and writes idx / gate.
 #include <cooperative_groups.h>
+
+#include <type_traits>
 
 #include "common.cuh"
 #include "internal.h"
@@ -148,12 +151,123 @@ __global__ void __cluster_dims__(kRouteCluster, 1, 1) __launch_bounds__(kWarps *
   rank_and_gate_warp(a, zs, t);
 }
 
+// Prefill-sized bf16 calls (T > kRouteTileMinT): the router is a skinny GEMM z[T, E] = x W^T,
+// bound by reading x once. One CTA of 8 warps takes 16 tokens; the logits come from mma.sync
+// m16n8k16 (bf16 products, exact in fp32, fp32 accumulation). The CTA's 16 token rows are one
+// contiguous block of x, which the CTA first asks L2 to fetch whole (bulk L2 prefetches), so the
+// warps' loads that follow find their lines in L2 or already on the way. Warp w takes contraction
+// slice w of 8 for all NTW 8-expert column tiles (NTW = ceil(E / 8) rounded up to a power of two;
+// rows past E read as zero), U 32-element chunks per pass with every load of a pass issued before
+// its MMAs, so a warp's chain of dependent memory round trips is (d / 256) / U passes long. A lane
+// of quad position c loads 16 bytes (elements 8c..8c+7 of a chunk) of token rows g and g + 8 and
+// of expert row g of each tile, and feeds words 0-1 to one MMA and words 2-3 to the next: the
+// contraction order inside a chunk is permuted identically for x and W, so every product is
+// formed exactly once. The 8 slices are summed in shared memory in slice order and each warp then
+// ranks two tokens with the same warp function as the per-token kernel. The fp32 order differs
+// from route_kernel's by rounding only (about 1e-7 relative), far inside the near-tie band of the
+// routing contract.
+constexpr int kTileTokens = 16;
+constexpr int kTileWarps = 8;
+constexpr size_t kTilePrefetch = 32768;  // bytes per L2 prefetch instruction
+
+template <int NTW, int U>
+__global__ void __launch_bounds__(kTileWarps * 32, 2)
+    route_tile_kernel(const __grid_constant__ RouteArgs a) {
+  pdl_wait();
+  __shared__ float part[kTileWarps][kTileTokens][kMaxE + 1];
+  __shared__ float zs[kTileTokens][kMaxE];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, c = lane & 3;
+  const int E = a.E, d = a.d;
+  const int t0 = blockIdx.x * kTileTokens;
+  const size_t row = size_t(d) * 2;
+  {  // the tile's token rows are one contiguous block: have L2 fetch all of it at once
+    const size_t bytes = size_t(min(kTileTokens, a.T - t0)) * row;
+    const char* base = static_cast<const char*>(a.x) + size_t(t0) * row;
+    for (size_t o = size_t(threadIdx.x) * kTilePrefetch; o < bytes; o += blockDim.x * kTilePrefetch)
+      prefetch_l2_bulk(base + o, uint32_t(min(kTilePrefetch, bytes - o)));
+  }
+  const int nch = d / 32;
+  const int c0 = warp * nch / kTileWarps, c1 = (warp + 1) * nch / kTileWarps;
+  const bool ok0 = t0 + g < a.T, ok1 = t0 + g + 8 < a.T;
+  // rows past the last token or expert read a valid row and are zeroed before use
+  const char* xa = static_cast<const char*>(a.x) + size_t(ok0 ? t0 + g : 0) * row + c * 16;
+  const char* xb = static_cast<const char*>(a.x) + size_t(ok1 ? t0 + g + 8 : 0) * row + c * 16;
+  const char* wr = static_cast<const char*>(a.w_router) + c * 16;
+  float acc[NTW][4];
+#pragma unroll
+  for (int j = 0; j < NTW; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  auto wrow = [&](int j) { return wr + size_t(j * 8 + g < E ? j * 8 + g : 0) * row; };
+  auto pass = [&](int ch, auto nchunks) {
+    constexpr int n = decltype(nchunks)::value;
+    uint4 va[n], vb[n], vw[n][NTW];
+#pragma unroll
+    for (int i = 0; i < n; ++i) {
+      const size_t o = size_t(ch + i) * 64;
+      va[i] = ldg16(xa + o);
+      vb[i] = ldg16(xb + o);
+#pragma unroll
+      for (int j = 0; j < NTW; ++j) vw[i][j] = ldg16(wrow(j) + o);
+    }
+#pragma unroll
+    for (int i = 0; i < n; ++i) {
+      if (!ok0) va[i] = zero;
+      if (!ok1) vb[i] = zero;
+#pragma unroll
+      for (int j = 0; j < NTW; ++j) {
+        if (j * 8 + g >= E) vw[i][j] = zero;
+        mma16816(acc[j], va[i].x, vb[i].x, va[i].y, vb[i].y, vw[i][j].x, vw[i][j].y);
+        mma16816(acc[j], va[i].z, vb[i].z, va[i].w, vb[i].w, vw[i][j].z, vw[i][j].w);
+      }
+    }
+  };
+  int ch = c0;
+  for (; ch + U <= c1; ch += U) pass(ch, std::integral_constant<int, U>{});
+  for (; ch < c1; ++ch) pass(ch, std::integral_constant<int, 1>{});
+  // C fragment of tile j: rows g and g + 8 (tokens), columns 2c and 2c + 1 (experts of the tile)
+#pragma unroll
+  for (int j = 0; j < NTW; ++j) {
+    const int e0 = j * 8 + 2 * c;
+    part[warp][g][e0] = acc[j][0];
+    part[warp][g][e0 + 1] = acc[j][1];
+    part[warp][g + 8][e0] = acc[j][2];
+    part[warp][g + 8][e0 + 1] = acc[j][3];
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < kTileTokens * E; i += blockDim.x) {
+    const int t = i / E, e = i % E;
+    float v = part[0][t][e];
+#pragma unroll
+    for (int k = 1; k < kTileWarps; ++k) v += part[k][t][e];
+    zs[t][e] = v;
+  }
+  __syncthreads();
+  for (int t = warp; t < kTileTokens; t += kTileWarps)
+    if (t0 + t < a.T) rank_and_gate_warp(a, zs[t], t0 + t);
+}
+
+cudaError_t launch_route_tile(const RouteArgs& a, cudaStream_t s) {
+  const dim3 grid((a.T + kTileTokens - 1) / kTileTokens), block(kTileWarps * 32);
+  const int nt = (a.E + 7) / 8;
+  // chunks per pass: about 24 16-byte loads in flight per lane
+  if (nt == 1) return launch_pdl(route_tile_kernel<1, 8>, grid, block, 0, s, a);
+  if (nt == 2) return launch_pdl(route_tile_kernel<2, 6>, grid, block, 0, s, a);
+  if (nt <= 4) return launch_pdl(route_tile_kernel<4, 4>, grid, block, 0, s, a);
+  return launch_pdl(route_tile_kernel<8, 2>, grid, block, 0, s, a);
+}
+
 template <typename TX>
 cudaError_t launch_typed(const RouteArgs& a, cudaStream_t s) {
   const int nchunk = a.d / Chunk<TX>::n;
   const int per_lane = (nchunk / route_parts(a.E, nchunk) + 31) / 32;  // chunks per lane and task
   dim3 grid(a.T), block(kWarps * 32);
   prof_begin(kProfRoute, s);
+  if (sizeof(TX) == 2 && a.T > kRouteTileMinT) {  // prefill-sized: tensor-core tiles of 16 tokens
+    const cudaError_t e = launch_route_tile(a, s);
+    prof_end(kProfRoute, s);
+    return e != cudaSuccess ? e : cudaGetLastError();
+  }
   if (a.E >= 2 * kWarps) {  // whole rows per task: one cluster per token
     const dim3 cgrid(a.T * kRouteCluster);
     const cudaError_t e =

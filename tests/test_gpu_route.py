@@ -36,7 +36,7 @@ def _run(shape, x, mode, **kw):
 
 @pytest.mark.parametrize("shape", [I.TINY, I.MIXTRAL, I.DSV2_LITE], ids=lambda s: s.name)
 @pytest.mark.parametrize("mode", list(MODES.values()), ids=list(MODES))
-@pytest.mark.parametrize("T", [1, 16, 64, 333])
+@pytest.mark.parametrize("T", [1, 16, 64, 65, 333])
 def test_route_parity(shape, mode, T):
     x = I.hidden_iid(1, shape, T)
     kw = _mode_args(shape, mode)
@@ -55,6 +55,19 @@ def test_route_prefill_full_size_hard_mask():
     flagged, swapped = check_routing(idx, gate, ref, sh.gate)
     assert flagged < 4096 // 100
     assert np.all(kw["mask"][idx.cpu().numpy()] == 1)
+
+
+def test_route_prefill_full_size_dsv2_soft_prior():
+    """DeepSeek-V2-Lite-shaped T = 4096 (the tensor-core tiles: 8 column tiles of 8 experts, one
+    warp each, over the whole contraction), soft prior of a keep-16-of-64 mask, plus a ragged
+    tail of 4096 + 7 tokens in top-k mode."""
+    sh = I.DSV2_LITE
+    for T, mode in ((4096, M.MCFT_ROUTE_SOFT_PRIOR), (4103, M.MCFT_ROUTE_TOPK)):
+        x = I.hidden_iid(5, sh, T)
+        kw = _mode_args(sh, mode, seed=5)
+        idx, gate, ref = _run(sh, x, mode, **kw)
+        flagged, swapped = check_routing(idx, gate, ref, sh.gate)
+        assert flagged < T // 100
 
 
 @pytest.mark.parametrize("shape,batch", [(I.MIXTRAL, 16), (I.DSV2_LITE, 64)], ids=["mixtral-b16", "dsv2-b64"])
