@@ -426,6 +426,24 @@ void mcft_stack_destroy(mcft_stack* stack);
 mcft_status mcft_device_error(mcft_stream_t stream);
 
 /* ---------------------------------------------------------------------------------------------
+ * Failure injection for tests (no counterpart in the paper). Sets, for the whole process:
+ *   fail_pinned_allocs   the next n pinned host allocations of the library fail as if the runtime
+ *                        were out of memory (mcft_cache_create then returns MCFT_ERR_OOM and
+ *                        frees everything it had allocated);
+ *   fail_expert_copies   the next n host-to-device expert copies of mcft_fetch_experts fail as if
+ *                        the runtime had refused them (MCFT_ERR_CUDA; the slots that step was
+ *                        filling then hold undefined bytes: destroy the cache or import a state);
+ *   wait_limit_ns        the limit of the decode FFN's bounded waits (0 = the default, 2 s);
+ *   withhold_gemm13      nonzero: the fused decode FFN skips its GEMM13 items, so every GEMM2
+ *                        item's wait for its segment runs out after wait_limit_ns; the call then
+ *                        sets MCFT_ERR_TIMEOUT in the device error word and leaves y untouched.
+ * Nothing here makes a kernel fault or wait without a limit. mcft_test_inject(0, 0, 0, 0) restores
+ * normal operation. Not synchronised with calls running on other threads. MCFT_ERR_INVALID for a
+ * negative count. */
+mcft_status mcft_test_inject(int fail_pinned_allocs, int fail_expert_copies,
+                             unsigned long long wait_limit_ns, int withhold_gemm13);
+
+/* ---------------------------------------------------------------------------------------------
  * Kernel timing (no counterpart in the paper; used to measure the path). While enabled, every
  * kernel the library launches is bracketed by two CUDA events on its stream.
  * mcft_profile_read synchronises the recorded events and returns, per kernel of the library, its

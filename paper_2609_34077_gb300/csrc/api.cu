@@ -6,6 +6,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -41,6 +42,41 @@ mcft_status cuda_fail(cudaError_t e, const char* where) {
   } while (0)
 
 __device__ unsigned g_device_error;  // one per device that loads the library
+
+// Test hooks (mcft_test_inject): how many of the next pinned host allocations and host-driven
+// expert copies fail as if the runtime had refused them, the decode FFN's wait limit, and whether
+// the decode FFN withholds its GEMM13 items. All zero (off) unless a test sets them.
+std::atomic<int> g_inject_pinned{0}, g_inject_copy{0}, g_inject_withhold{0};
+std::atomic<unsigned long long> g_inject_wait_ns{0};
+
+// Consume one injected failure from counter n: true while it is positive.
+bool take_injected(std::atomic<int>& n) {
+  int v = n.load();
+  while (v > 0)
+    if (n.compare_exchange_weak(v, v - 1)) return true;
+  return false;
+}
+
+cudaError_t host_alloc_mapped(void** p, size_t bytes) {
+  if (take_injected(g_inject_pinned)) return cudaErrorMemoryAllocation;
+  return cudaHostAlloc(p, bytes, cudaHostAllocMapped);
+}
+
+cudaError_t expert_copy(void* dst, const void* src, size_t bytes, cudaStream_t s) {
+  if (take_injected(g_inject_copy)) return cudaErrorUnknown;
+  return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, s);
+}
+
+}  // namespace
+
+unsigned long long test_wait_limit_ns() {
+  const unsigned long long v = g_inject_wait_ns.load();
+  return v ? v : 2000000000ull;
+}
+
+bool test_withhold_gemm13() { return g_inject_withhold.load() != 0; }
+
+namespace {
 
 constexpr int kMaxDevices = 64;
 
@@ -235,6 +271,17 @@ mcft_status enqueue_prefetch_fetches(mcft_cache* c, cudaStream_t copy) {
 extern "C" {
 
 int mcft_version(void) { return 200; }
+
+mcft_status mcft_test_inject(int fail_pinned_allocs, int fail_expert_copies,
+                             unsigned long long wait_limit_ns, int withhold_gemm13) {
+  if (fail_pinned_allocs < 0 || fail_expert_copies < 0)
+    return fail(MCFT_ERR_INVALID, "failure counts must be >= 0");
+  g_inject_pinned.store(fail_pinned_allocs);
+  g_inject_copy.store(fail_expert_copies);
+  g_inject_wait_ns.store(wait_limit_ns);
+  g_inject_withhold.store(withhold_gemm13 ? 1 : 0);
+  return MCFT_OK;
+}
 
 const char* mcft_last_error(void) { return g_last_error.c_str(); }
 
@@ -577,7 +624,8 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   MCFT_CACHE_CUDA(cudaMemset(c->d_freq, 0, sizeof(int64_t) * L * E));
   MCFT_CACHE_CUDA(cudaMemset(c->d_step, 0, sizeof(int64_t) * L));
   MCFT_CACHE_CUDA(cudaMemset(c->d_cnt, 0, sizeof(unsigned long long) * L * kCacheCounters));
-  MCFT_CACHE_CUDA(cudaHostAlloc(&c->h_miss, sizeof(int32_t) * L * c->miss_stride, cudaHostAllocMapped));
+  MCFT_CACHE_CUDA(host_alloc_mapped(reinterpret_cast<void**>(&c->h_miss),
+                                    sizeof(int32_t) * L * c->miss_stride));
   memset(c->h_miss, 0, sizeof(int32_t) * L * c->miss_stride);
   MCFT_CACHE_CUDA(cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->d_miss), c->h_miss, 0));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_miss_dev, sizeof(int32_t) * L * c->miss_stride));
@@ -690,8 +738,8 @@ mcft_status mcft_fetch_experts(mcft_cache* c, int layer, mcft_stream_t compute_s
       const int e = m_exp[i];
       if (e < 0 || e >= E) return fail(MCFT_ERR_INVALID, "corrupt miss list");
       const char* dst = loc_ptr(c, layer, loc_of[e]);
-      MCFT_CUDA(cudaMemcpyAsync(const_cast<char*>(dst), c->host_experts[size_t(layer) * E + e],
-                                c->expert_bytes, cudaMemcpyHostToDevice, copy_stream));
+      MCFT_CUDA(expert_copy(const_cast<char*>(dst), c->host_experts[size_t(layer) * E + e],
+                            c->expert_bytes, copy_stream));
     }
     MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
     MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));

@@ -438,13 +438,13 @@ __global__ void __launch_bounds__(kWarps * 32, 2) dec2_kernel(const __grid_const
   for (int item = blockIdx.x; item < it.total; item += gridDim.x) run2_item<MAXNG>(a, it, item, red);
 }
 
-constexpr uint64_t kSegWaitNs = 2000000000ull;
 // the fused kernel holds both GEMMs' code, so it keeps double-buffered loads only where both fit
 // the register budget without spills (see -Xptxas -v)
 constexpr bool kFusedDB = false;
 
 // Bounded wait (one thread) until segment s has `need` finished GEMM13 items; false (and the call
-// aborted, so later waits return at once) if 2 s pass or the call is already aborting.
+// aborted, so later waits return at once) if a.wait_ns pass (2 s unless a test shortened it) or
+// the call is already aborting.
 __device__ bool wait_segment(const FfnArgs& a, int s, int need) {
   const volatile int* p = a.done + s;
   const volatile int* abort = &a.hdr->abort;
@@ -452,7 +452,7 @@ __device__ bool wait_segment(const FfnArgs& a, int s, int need) {
     const uint64_t t0 = globaltimer_ns();
     while (*p < need) {
       if (*abort) return false;
-      if (globaltimer_ns() - t0 > kSegWaitNs) {
+      if (globaltimer_ns() - t0 > a.wait_ns) {
         set_error(a.err, kErrTimeout);
         const_cast<WsHeader*>(a.hdr)->abort = 1;
         return false;
@@ -495,10 +495,12 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
     int next = 0;
     if (threadIdx.x == 0) next = atomicAdd(a.done + a.nseg + a.phase, 1);
     if (item < it13.total) {
-      const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, red);
-      __threadfence();  // this CTA's h rows, before the segment's count moves
-      __syncthreads();
-      if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
+      if (!a.withhold13) {  // (a test withholds GEMM13 items to make the GEMM2 waits run out)
+        const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, red);
+        __threadfence();  // this CTA's h rows, before the segment's count moves
+        __syncthreads();
+        if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
+      }
     } else {
       const int i2 = item - it13.total;
       // every segment with work has w / (16 rb) GEMM13 items
@@ -573,8 +575,11 @@ cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int 
   return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages,
+cudaError_t launch_ffn_decode(const FfnArgs& args, int num_sms, cudaStream_t s, int stages,
                               int reserved) {
+  FfnArgs a = args;
+  a.wait_ns = test_wait_limit_ns();
+  a.withhold13 = test_withhold_gemm13() ? 1 : 0;
   // a segment holds at most T tokens (routed experts: distinct per token; shared: all T)
   if (a.T <= 8) return launch_decode_ng<1>(a, num_sms, s, stages, reserved);
   if (a.T <= 16) return launch_decode_ng<2>(a, num_sms, s, stages, reserved);

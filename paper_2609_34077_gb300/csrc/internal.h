@@ -171,7 +171,15 @@ struct FfnArgs {
   // phase), all zeroed by the permutation of the call: they let one fused decode launch hand out
   // its items dynamically and start a segment's GEMM2 as soon as that segment's h is written
   int* done;
+  // Limit of the fused decode FFN's bounded waits (ns), and a test switch that makes it skip its
+  // GEMM13 items so that those waits run out (set by launch_ffn_decode from the test hooks).
+  unsigned long long wait_ns;
+  int withhold13;
 };
+
+// Test hooks (mcft_test_inject in api.cu); all off by default.
+unsigned long long test_wait_limit_ns();  // the decode FFN's wait limit (default 2 s)
+bool test_withhold_gemm13();              // skip the decode FFN's GEMM13 items
 
 // s * sum_j u[j] B[row][j] for a LoRA up-projection B [rows, r] (layer dtype TW).
 template <typename TW>

@@ -54,6 +54,7 @@ SIGNATURES = {
     "mcft_cache_import": (_i, [_vp, _vp, _sz, _vp]),
     "mcft_cache_destroy": (None, [_vp]),
     "mcft_device_error": (_i, [_vp]),
+    "mcft_test_inject": (_i, [_i, _i, C.c_ulonglong, _i]),
     "mcft_profile_enable": (_i, [_i]),
     "mcft_profile_reset": (_i, []),
     "mcft_profile_read": (_i, [_i, _vp, _vp, _vp, C.POINTER(_i)]),
@@ -424,6 +425,13 @@ def mcft_cache_import(cache: Cache, state: bytes, stream=None):
     buf = C.create_string_buffer(state, len(state))
     _check(lib().mcft_cache_import(C.c_void_p(cache.handle), C.cast(buf, C.c_void_p), len(state),
                                    _stream(stream)))
+
+
+def mcft_test_inject(fail_pinned_allocs=0, fail_expert_copies=0, wait_limit_ns=0,
+                     withhold_gemm13=False):
+    """Failure injection for tests (all zero: normal operation)."""
+    _check(lib().mcft_test_inject(int(fail_pinned_allocs), int(fail_expert_copies),
+                                  int(wait_limit_ns), 1 if withhold_gemm13 else 0))
 
 
 def mcft_profile_enable(on: bool = True):

@@ -83,3 +83,12 @@ def test_host_validation_without_gpu(libpath):
     assert L.mcft_host_copy(C.c_void_p(16), C.c_void_p(32), 40, 1, None) == mcft.MCFT_ERR_INVALID
     assert b"multiple of 16" in L.mcft_last_error()
     assert L.mcft_host_copy(C.c_void_p(16), C.c_void_p(32), 64, 0, None) == mcft.MCFT_ERR_INVALID
+
+
+def test_test_inject_validation_without_gpu(libpath):
+    from paper_2609_34077_gb300 import mcft
+
+    L = mcft.lib()
+    assert L.mcft_test_inject(-1, 0, 0, 0) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_test_inject(0, -2, 0, 0) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_test_inject(0, 0, 0, 0) == mcft.MCFT_OK

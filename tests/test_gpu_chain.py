@@ -228,3 +228,64 @@ def test_stack_invalid():
                                 T_max=1)
     with pytest.raises(M.MCFTError):  # T > T_max
         M.mcft_stack_step(stack, torch.zeros((2, shape.d), device=DEV))
+
+
+def teacher_forced(shape, L, T, steps, seed):
+    """The chain layer by layer through the unfused calls (mcft_residual_rmsnorm -> mcft_route ->
+    mcft_moe_forward), each layer checked against the oracle applied to the GPU's own stream and
+    normalised input: the residual add is exact in fp32, u_l is the oracle's RMSNorm of the GPU's
+    x_l rounded once to bf16, the routing of u_l meets the paper-level near-tie rule (1e-4) with
+    gates within 1e-4, and the layer output is within 2e-2 of the oracle's layer on the GPU's u_l,
+    at every depth (the drift of a free-running chain is taken out of the comparison).
+    Returns the number of near-tie tokens seen."""
+    from tests.gpu_helpers import TOL_BF16, check_output, check_routing
+
+    st = _stack(shape, L, seed, False)
+    lws, _, _ = _pool(shape, seed, L, False)
+    experts = [b.to(DEV) for b in lws[0].experts]  # every layer aliases layer 0's expert blocks
+    desc = M.desc_of(shape)
+    x0 = I.residual_stream(seed, shape, steps, T)
+    flagged_total = 0
+    for s in range(steps):
+        x = x0[s].to(DEV).clone()
+        y_prev = None
+        for l in range(L):
+            ly = st["layers"][l]
+            x_before = x.cpu().numpy().copy()
+            u = M.mcft_residual_rmsnorm(desc, x, y=y_prev, gamma=st["gammas"][l], eps=shape.norm_eps)
+            xs = x.cpu().numpy()
+            if y_prev is not None:  # x_l = x_{l-1} + y_{l-1}, one fp32 add per element
+                want = (x_before + y_prev.cpu().float().numpy()).astype(np.float32)
+                assert np.array_equal(xs, want), f"step {s} layer {l}: residual add"
+            uh = u.cpu().double().numpy()
+            u_ref = oracle.stack.rmsnorm(xs.astype(np.float64), ly["gamma"], shape.norm_eps)
+            nerr = (np.abs(uh - u_ref).max(axis=1) / np.abs(u_ref).max(axis=1)).max()
+            assert nerr <= 2.0 ** -8, f"step {s} layer {l}: RMSNorm error {nerr:.3e}"
+            idx, gate = M.mcft_route(desc, u, st["routers"][l], M.MCFT_ROUTE_SOFT_PRIOR,
+                                     prior=st["priors"][l])
+            r = oracle.stack.route_layer(uh, ly, shape.K, shape.gate)
+            flagged, _ = check_routing(idx, gate, r, shape.gate)
+            flagged_total += flagged
+            y = M.mcft_moe_forward(desc, u, idx, gate, experts, st["shared"][l])
+            M.mcft_device_error()
+            gi = idx.cpu().numpy()
+            pa = np.take_along_axis(r["p"], gi.astype(np.int64), axis=1)
+            g_ref = pa / pa.sum(axis=1, keepdims=True) if shape.gate == I.GATE_RENORM else pa
+            yref = oracle.ffn.moe_layer(uh, gi, g_ref, ly["experts"], ly["shared"])
+            check_output(y, yref, TOL_BF16, f"step {s} layer {l}")
+            y_prev = y
+    return flagged_total
+
+
+@pytest.mark.parametrize("T", [1, 2])
+def test_chain_mixtral_32_layers_teacher_forced(T):
+    """32 Mixtral-shaped layers (the depth where the free-running chain needs a 0.15 band), each
+    layer at the paper-level rule on the GPU's own input."""
+    flagged = teacher_forced(I.MIXTRAL, 32, T, steps=3, seed=61)
+    assert flagged <= 32 * 3 * T // 50
+
+
+@pytest.mark.parametrize("T", [1, 4])
+def test_chain_deepseek_26_layers_teacher_forced(T):
+    flagged = teacher_forced(I.DSV2_LITE, 26, T, steps=3, seed=62)
+    assert flagged <= 26 * 3 * T // 50

@@ -141,3 +141,48 @@ def test_cached_forward_equals_plain_forward_bitwise(shape, T):
         assert torch.equal(y_c, y_p), f"step {s}"
     M.mcft_device_error()
     assert M.mcft_cache_stats(cache, 0)[1] > 0  # the stream did fetch
+
+
+def _prefill_full(shape, keep, seed):
+    """The masked fine-tuning / prefill forward at full size: T = 4096 tokens routed by mcft_route
+    under a hard mask keeping `keep` experts, then mcft_moe_forward (tcgen05 grouped GEMMs),
+    against the oracle on every one of the 4096 rows."""
+    T = 4096
+    mask = I.keep_mask(seed, shape.E, keep)
+    kept = [int(e) for e in np.nonzero(mask)[0]]
+    lw = I.layer_weights(seed, shape, experts=kept)
+    desc = M.desc_of(shape)
+    x = I.hidden_iid(seed, shape, T)
+    xd = x.to(DEV)
+    idx, gate = M.mcft_route(desc, xd, lw.router.to(DEV), M.MCFT_ROUTE_HARD_MASK, mask=mask)
+    y = M.mcft_moe_forward(desc, xd, idx, gate, [None if b is None else b.to(DEV) for b in lw.experts],
+                           [b.to(DEV) for b in lw.shared])
+    M.mcft_device_error()
+    ref = oracle.routing.route(f64(x), f64(lw.router), shape.K, M.MCFT_ROUTE_HARD_MASK, shape.gate,
+                               mask=mask)
+    from tests.gpu_helpers import check_routing
+
+    flagged, _ = check_routing(idx, gate, ref, shape.gate)
+    assert flagged < T // 100
+    gi = idx.cpu().numpy()
+    assert np.all(mask[gi] == 1)
+    # the layer for the experts the GPU chose (the oracle's own set outside near ties), with the
+    # oracle's gates for them (from its p)
+    pa = np.take_along_axis(ref["p"], gi.astype(np.int64), axis=1)
+    g_ref = pa / pa.sum(axis=1, keepdims=True) if shape.gate == I.GATE_RENORM else pa
+    yref = oracle.ffn.moe_layer(f64(x), gi, g_ref, expert_triples(lw, shape), shared_triples(lw, shape))
+    row, fro = check_output(y, yref, TOL_BF16, f"{shape.name} prefill T={T}, every row")
+    assert fro < TOL_BF16
+    return row, fro
+
+
+def test_prefill_mixtral_full_size_every_row():
+    """Mixtral-shaped, T = 8 x 512 = 4096, hard mask keeping 4 of 8 experts (unbalanced loads:
+    8192 assignments over the 4 kept experts, each padded to 128-row tiles)."""
+    _prefill_full(I.MIXTRAL, 4, seed=90)
+
+
+def test_prefill_deepseek_full_size_every_row():
+    """DeepSeek-V2-Lite-shaped, T = 4096, 64 routed experts (hard mask keeping 48) plus the 2
+    shared experts on every token: 24576 routed and 8192 shared rows through the grouped GEMMs."""
+    _prefill_full(I.DSV2_LITE, 48, seed=91)
