@@ -36,12 +36,6 @@ __device__ __forceinline__ uint4 ldg16(const void* p) {
   return __ldg(reinterpret_cast<const uint4*>(p));
 }
 
-// Ask L2 to fetch [p, p + bytes) from memory (no destination; p 16-byte aligned, bytes a multiple
-// of 16): one instruction puts a whole tile's reads in flight.
-__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
-
 // 16-byte load through L2 only (coherent with stores of other CTAs of the same kernel that were
 // published with a fence: no stale L1 line can be returned).
 __device__ __forceinline__ uint4 ldcg16(const void* p) {

@@ -153,9 +153,7 @@ __global__ void __cluster_dims__(kRouteCluster, 1, 1) __launch_bounds__(kWarps *
 
 // Prefill-sized bf16 calls (T > kRouteTileMinT): the router is a skinny GEMM z[T, E] = x W^T,
 // bound by reading x once. One CTA of 8 warps takes 16 tokens; the logits come from mma.sync
-// m16n8k16 (bf16 products, exact in fp32, fp32 accumulation). The CTA's 16 token rows are one
-// contiguous block of x, which the CTA first asks L2 to fetch whole (bulk L2 prefetches), so the
-// warps' loads that follow find their lines in L2 or already on the way. Warp w takes contraction
+// m16n8k16 (bf16 products, exact in fp32, fp32 accumulation). Warp w takes contraction
 // slice w of 8 for all NTW 8-expert column tiles (NTW = ceil(E / 8) rounded up to a power of two;
 // rows past E read as zero), U 32-element chunks per pass with every load of a pass issued before
 // its MMAs, so a warp's chain of dependent memory round trips is (d / 256) / U passes long. A lane
@@ -168,7 +166,6 @@ __global__ void __cluster_dims__(kRouteCluster, 1, 1) __launch_bounds__(kWarps *
 // routing contract.
 constexpr int kTileTokens = 16;
 constexpr int kTileWarps = 8;
-constexpr size_t kTilePrefetch = 32768;  // bytes per L2 prefetch instruction
 
 template <int NTW, int U>
 __global__ void __launch_bounds__(kTileWarps * 32, 2)
@@ -181,12 +178,6 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2)
   const int E = a.E, d = a.d;
   const int t0 = blockIdx.x * kTileTokens;
   const size_t row = size_t(d) * 2;
-  {  // the tile's token rows are one contiguous block: have L2 fetch all of it at once
-    const size_t bytes = size_t(min(kTileTokens, a.T - t0)) * row;
-    const char* base = static_cast<const char*>(a.x) + size_t(t0) * row;
-    for (size_t o = size_t(threadIdx.x) * kTilePrefetch; o < bytes; o += blockDim.x * kTilePrefetch)
-      prefetch_l2_bulk(base + o, uint32_t(min(kTilePrefetch, bytes - o)));
-  }
   const int nch = d / 32;
   const int c0 = warp * nch / kTileWarps, c1 = (warp + 1) * nch / kTileWarps;
   const bool ok0 = t0 + g < a.T, ok1 = t0 + g + 8 < a.T;
