@@ -44,10 +44,10 @@ METRIC = "masked MoE layer tokens/s"
 # first 16 hex digits of the kernel source's sha256: when the source has changed since the
 # capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", None),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "c9700da601f8ebb6", 1.0017),
-    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "ae0482332aaf7dee", 0.9558),
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e965b486ab27bed2", None),
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e965b486ab27bed2", None),
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e965b486ab27bed2", 1.0017),
+    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "980d86643d8088ca", 0.9559),
 }
 
 
