@@ -86,6 +86,8 @@ int current_device() {
   return dev;
 }
 
+}  // namespace
+
 int num_sms() {
   static int cache[kMaxDevices] = {0};
   const int dev = current_device();
@@ -96,6 +98,8 @@ int num_sms() {
   if (dev < kMaxDevices) cache[dev] = n;
   return n;
 }
+
+namespace {
 
 size_t align256(size_t v) { return (v + 255) & ~size_t(255); }
 

@@ -54,6 +54,7 @@ struct RouteArgs {
   unsigned* err;
 };
 cudaError_t launch_route(const RouteArgs& a, int dtype, cudaStream_t s);
+int num_sms();  // SMs of the current device (looked up once per device)
 // bf16 calls of more tokens than this route in 16-token tensor-core tiles (route.cu).
 constexpr int kRouteTileMinT = 64;
 

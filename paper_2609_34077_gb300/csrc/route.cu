@@ -152,8 +152,10 @@ __global__ void __cluster_dims__(kRouteCluster, 1, 1) __launch_bounds__(kWarps *
 }
 
 // Prefill-sized bf16 calls (T > kRouteTileMinT): the router is a skinny GEMM z[T, E] = x W^T,
-// bound by reading x once. One CTA of 8 warps takes 16 tokens; the logits come from mma.sync
-// m16n8k16 (bf16 products, exact in fp32, fp32 accumulation). Warp w takes contraction
+// bound by reading x once. A CTA of 8 warps takes up to 16 tokens; the logits come from mma.sync
+// m16n8k16 (bf16 products, exact in fp32, fp32 accumulation). The tokens are spread evenly over
+// two CTAs per SM (at most 16 per CTA, the MMA's rows; rows past a CTA's tokens read as zero), so
+// no SM streams twice the rows of another. Warp w takes contraction
 // slice w of 8 for all NTW 8-expert column tiles (NTW = ceil(E / 8) rounded up to a power of two;
 // rows past E read as zero), U 32-element chunks per pass with every load of a pass issued before
 // its MMAs, so a warp's chain of dependent memory round trips is (d / 256) / U passes long. A lane
@@ -169,18 +171,18 @@ constexpr int kTileWarps = 8;
 
 template <int NTW, int U>
 __global__ void __launch_bounds__(kTileWarps * 32, 2)
-    route_tile_kernel(const __grid_constant__ RouteArgs a) {
+    route_tile_kernel(const __grid_constant__ RouteArgs a, int tpc) {
   pdl_wait();
   __shared__ float part[kTileWarps][kTileTokens][kMaxE + 1];
   __shared__ float zs[kTileTokens][kMaxE];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
   const int E = a.E, d = a.d;
-  const int t0 = blockIdx.x * kTileTokens;
+  const int t0 = blockIdx.x * tpc, t1 = min(a.T, t0 + tpc);  // this CTA's tokens
   const size_t row = size_t(d) * 2;
   const int nch = d / 32;
   const int c0 = warp * nch / kTileWarps, c1 = (warp + 1) * nch / kTileWarps;
-  const bool ok0 = t0 + g < a.T, ok1 = t0 + g + 8 < a.T;
+  const bool ok0 = t0 + g < t1, ok1 = t0 + g + 8 < t1;
   // rows past the last token or expert read a valid row and are zeroed before use
   const char* xa = static_cast<const char*>(a.x) + size_t(ok0 ? t0 + g : 0) * row + c * 16;
   const char* xb = static_cast<const char*>(a.x) + size_t(ok1 ? t0 + g + 8 : 0) * row + c * 16;
@@ -235,17 +237,20 @@ __global__ void __launch_bounds__(kTileWarps * 32, 2)
   }
   __syncthreads();
   for (int t = warp; t < kTileTokens; t += kTileWarps)
-    if (t0 + t < a.T) rank_and_gate_warp(a, zs[t], t0 + t);
+    if (t0 + t < t1) rank_and_gate_warp(a, zs[t], t0 + t);
 }
 
-cudaError_t launch_route_tile(const RouteArgs& a, cudaStream_t s) {
-  const dim3 grid((a.T + kTileTokens - 1) / kTileTokens), block(kTileWarps * 32);
+cudaError_t launch_route_tile(const RouteArgs& a, int num_sms, cudaStream_t s) {
+  // tokens per CTA: the T tokens spread evenly over two CTAs per SM (at most 16, the MMA's rows)
+  const int slots = 2 * num_sms;
+  const int tpc = min(kTileTokens, max(1, (a.T + slots - 1) / slots));
+  const dim3 grid((a.T + tpc - 1) / tpc), block(kTileWarps * 32);
   const int nt = (a.E + 7) / 8;
   // chunks per pass: about 24 16-byte loads in flight per lane
-  if (nt == 1) return launch_pdl(route_tile_kernel<1, 8>, grid, block, 0, s, a);
-  if (nt == 2) return launch_pdl(route_tile_kernel<2, 6>, grid, block, 0, s, a);
-  if (nt <= 4) return launch_pdl(route_tile_kernel<4, 4>, grid, block, 0, s, a);
-  return launch_pdl(route_tile_kernel<8, 2>, grid, block, 0, s, a);
+  if (nt == 1) return launch_pdl(route_tile_kernel<1, 8>, grid, block, 0, s, a, tpc);
+  if (nt == 2) return launch_pdl(route_tile_kernel<2, 6>, grid, block, 0, s, a, tpc);
+  if (nt <= 4) return launch_pdl(route_tile_kernel<4, 4>, grid, block, 0, s, a, tpc);
+  return launch_pdl(route_tile_kernel<8, 2>, grid, block, 0, s, a, tpc);
 }
 
 template <typename TX>
@@ -255,7 +260,7 @@ cudaError_t launch_typed(const RouteArgs& a, cudaStream_t s) {
   dim3 grid(a.T), block(kWarps * 32);
   prof_begin(kProfRoute, s);
   if (sizeof(TX) == 2 && a.T > kRouteTileMinT) {  // prefill-sized: tensor-core tiles of 16 tokens
-    const cudaError_t e = launch_route_tile(a, s);
+    const cudaError_t e = launch_route_tile(a, num_sms(), s);
     prof_end(kProfRoute, s);
     return e != cudaSuccess ? e : cudaGetLastError();
   }
