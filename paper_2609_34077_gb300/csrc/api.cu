@@ -189,9 +189,6 @@ struct mcft_cache {
   int32_t* d_miss_dev = nullptr;            // device-memory copy [L][miss_stride]
   unsigned long long* d_ptr_tab = nullptr;  // [L*E] block address of each selected expert
   unsigned long long* d_ready = nullptr;    // [L] hit mask of the last step
-  unsigned long long* d_stream = nullptr;   // [L] miss mask of the last step
-  unsigned* d_landed = nullptr;  // [L][E][ppe] epoch stamps of the demand fetch's landed pieces
-  int ppe = 0;                   // fetch pieces per expert block
   unsigned long long* d_host_src = nullptr; // [L*E] device-visible addresses of the host blocks
   unsigned long long* d_pfmask = nullptr;   // [L] experts loaded by a prefetch since the last step
   unsigned long long* d_pf_cancel = nullptr;  // [L] prefetched experts the next step dropped
@@ -225,8 +222,6 @@ void cache_free(mcft_cache* c) {
   cudaFree(c->d_miss_dev);
   cudaFree(c->d_ptr_tab);
   cudaFree(c->d_ready);
-  cudaFree(c->d_stream);
-  cudaFree(c->d_landed);
   cudaFree(c->d_host_src);
   cudaFree(c->d_pfmask);
   cudaFree(c->d_pf_cancel);
@@ -643,16 +638,10 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   MCFT_CACHE_CUDA(cudaMemset(c->d_ptr_tab, 0, sizeof(unsigned long long) * L * E));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_ready, sizeof(unsigned long long) * L));
   MCFT_CACHE_CUDA(cudaMemset(c->d_ready, 0, sizeof(unsigned long long) * L));
-  MCFT_CACHE_CUDA(cudaMalloc(&c->d_stream, sizeof(unsigned long long) * L));
-  MCFT_CACHE_CUDA(cudaMemset(c->d_stream, 0, sizeof(unsigned long long) * L));
   if (host_experts) {
     c->host_experts.assign(host_experts, host_experts + size_t(L) * E);
     c->n_staging = stg;
     MCFT_CACHE_CUDA(cudaMalloc(&c->d_slots, expert_bytes * size_t(L) * B));
-    // stamps start below every epoch (steps count from 1)
-    c->ppe = int((expert_bytes + kFetchPiece - 1) / kFetchPiece);
-    MCFT_CACHE_CUDA(cudaMalloc(&c->d_landed, sizeof(unsigned) * size_t(L) * E * c->ppe));
-    MCFT_CACHE_CUDA(cudaMemset(c->d_landed, 0, sizeof(unsigned) * size_t(L) * E * c->ppe));
     if (stg > 0) MCFT_CACHE_CUDA(cudaMalloc(&c->d_staging, expert_bytes * size_t(stg)));
     // device-visible addresses of the pinned host blocks, for the device-driven fetch
     std::vector<unsigned long long> src(size_t(L) * E);
@@ -698,7 +687,7 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
                   c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
                   c->d_miss + size_t(layer) * c->miss_stride,
                   c->d_miss_dev + size_t(layer) * c->miss_stride,
-                  c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer, c->d_stream + layer,
+                  c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer,
                   c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                   c->d_staging, c->expert_bytes, device_error_word()};
   cudaError_t e = launch_cache_step(a, stream);
@@ -953,25 +942,17 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
     st = enqueue_prefetch_fetches(c, copy_stream);
     if (st != MCFT_OK) return st;
   }
-  // Small bf16 decode batches stream the misses behind their fetch: the fetch kernel stamps each
-  // piece it has written, and the FFN's first launch computes the misses with the hits, each of
-  // their items waiting for the pieces it reads, so their FFN runs while the rest of the step's
-  // bytes are still on the host link.
-  const bool streaming = L.decode && T <= kStreamMaxT && c->d_landed != nullptr;
-  unsigned* landed = streaming ? c->d_landed + size_t(layer) * E * c->ppe : nullptr;
   // 1. the missed experts stream in on the copy stream, after this layer's cache step
   MCFT_CUDA(cudaStreamWaitEvent(copy_stream, c->ev_step[layer], 0));
   FetchArgs fe{c->d_miss_dev + size_t(layer) * c->miss_stride, c->d_host_src + size_t(layer) * E,
-               c->d_ptr_tab + size_t(layer) * E, c->expert_bytes, nullptr, nullptr, landed,
-               c->d_step + layer, c->ppe};
+               c->d_ptr_tab + size_t(layer) * E, c->expert_bytes, nullptr, nullptr};
   cudaError_t e = launch_fetch(fe, fetch_blocks(), copy_stream);
   if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
   // Experts a prefetch of this layer is still bringing in are not in the step's ready mask: the
   // FFN computes them in phase 2, after compute_stream waits for ev_copy, which follows their
   // fetch on this copy stream.
-  const bool pf_landing = c->pf_state[layer] == 2;
-  if (pf_landing) c->pf_state[layer] = 0;
+  if (c->pf_state[layer] == 2) c->pf_state[layer] = 0;
   // 1b. prefetches decided for later layers stream in behind this layer's misses
   int queued = 0;
   for (int l = 0; l < c->L; ++l) queued += c->pf_state[l] == 1 ? 1 : 0;
@@ -1003,18 +984,10 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   fa.err = err;
   fa.wtab = c->d_ptr_tab + size_t(layer) * E;
   fa.ready = c->d_ready + layer;
-  if (streaming) {
-    fa.stream = c->d_stream + layer;
-    fa.landed = landed;
-    fa.epoch = c->d_step + layer;
-    fa.ppe = c->ppe;
-  }
   // A fetch kernel running alongside keeps its SM slots: this layer's misses (or an earlier
   // prefetch still on the copy stream) during phase 1; during phase 2, which starts after the
-  // misses have landed, only prefetches queued behind them at 1b. When streaming, phase 2 is left
-  // out unless a prefetch of this layer may still be landing.
+  // misses have landed, only prefetches queued behind them at 1b.
   for (int phase = 1; phase <= 2; ++phase) {
-    if (phase == 2 && streaming && !pf_landing) break;
     fa.phase = phase;
     if (phase == 2) MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
     const int reserved = phase == 1 || queued > 0 ? fetch_blocks() : 0;
@@ -1025,10 +998,6 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S, L.ks, fa.o_plane};
   e = launch_combine(ca, desc->dtype, compute_stream);
   if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
-  // without phase 2 the compute stream has not waited for the copy stream yet: work issued on it
-  // after this call must find the step's fetch complete (the FFN saw every piece land, but the
-  // fetch kernel may still be exiting)
-  if (streaming && !pf_landing) MCFT_CUDA(cudaStreamWaitEvent(compute_stream, c->ev_copy, 0));
   return MCFT_OK;
 }
 
@@ -1085,7 +1054,7 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
                           c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
                           c->d_miss + size_t(layer) * c->miss_stride,
                           c->d_miss_dev + size_t(layer) * c->miss_stride,
-                          c->d_ptr_tab + size_t(layer) * E, c->d_ready + layer, c->d_stream + layer,
+                          c->d_ptr_tab + size_t(layer) * E, c->d_ready + layer,
                           c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                           c->d_staging, c->expert_bytes, err};
   a.do_prefetch = do_pf ? 1 : 0;
@@ -1209,9 +1178,6 @@ mcft_status mcft_cache_import(mcft_cache* c, const void* buf, size_t bytes, mcft
     MCFT_CUDA(cudaMemcpyAsync(part.dst, p, part.n, cudaMemcpyHostToDevice, stream));
     p += part.n;
   }
-  // landed stamps may carry the epochs of steps taken after the exported state: clear them
-  if (c->d_landed)
-    MCFT_CUDA(cudaMemsetAsync(c->d_landed, 0, sizeof(unsigned) * size_t(c->L) * c->E * c->ppe, stream));
   MCFT_CUDA(cudaStreamSynchronize(stream));
   return MCFT_OK;
 }

@@ -62,8 +62,7 @@ __device__ __forceinline__ void copy_piece(const uint4* src, uint4* dst, size_t 
 __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ FetchArgs a) {
   pdl_wait();
   const int n = a.miss[0];
-  const unsigned epoch = a.landed ? static_cast<unsigned>(*a.epoch) : 0u;
-  const size_t words = a.bytes / 16, piece = kFetchPiece / 16;
+  const size_t words = a.bytes / 16, piece = 4096;
   const size_t per = (words + piece - 1) / piece;
   const size_t units = size_t(n) * per;
   for (size_t u = blockIdx.x; u < units; u += gridDim.x) {
@@ -81,12 +80,6 @@ __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ Fetc
     const size_t w1 = w0 + piece < words ? w0 + piece : words;
     if (a.moved && threadIdx.x == 0) atomicAdd(a.moved, (unsigned long long)(w1 - w0) * 16ull);
     copy_piece(src, dst, w0, w1);
-    if (a.landed) {  // stamp the piece once every thread's stores of it are visible device-wide
-      __threadfence();
-      __syncthreads();
-      if (threadIdx.x == 0)
-        *reinterpret_cast<volatile unsigned*>(a.landed + size_t(e) * a.ppe + u % per) = epoch;
-    }
   }
 }
 

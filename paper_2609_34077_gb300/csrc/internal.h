@@ -176,21 +176,7 @@ struct FfnArgs {
   // GEMM13 items so that those waits run out (set by launch_ffn_decode from the test hooks).
   unsigned long long wait_ns;
   int withhold13;
-  // Experts streamed behind their fetch (cached forward, bf16 decode): stream has bit e set when
-  // expert e is copied by the step's demand fetch kernel, which stamps each kFetchPiece-byte piece
-  // of it in landed [E][ppe] with the step's epoch (*epoch, the layer's step count after its cache
-  // step) once the piece's bytes are written; the FFN computes such an expert in the same launch
-  // as the hits, each item waiting (bounded) for the pieces it reads. NULL landed: no streaming.
-  const unsigned long long* stream;
-  const unsigned* landed;
-  const int64_t* epoch;
-  int ppe;
 };
-
-// Bytes per work unit of the device-driven fetch: the granule of its landed stamps.
-constexpr size_t kFetchPiece = 65536;
-// Cached decode forwards of up to this many tokens stream their misses behind the fetch.
-constexpr int kStreamMaxT = 16;
 
 // Test hooks (mcft_test_inject in api.cu); all off by default.
 unsigned long long test_wait_limit_ns();  // the decode FFN's wait limit (default 2 s)
@@ -226,16 +212,10 @@ __device__ __forceinline__ float lora_up<float>(const void* blk, size_t b_off, i
 __device__ __forceinline__ const void* seg_block(const FfnArgs& a, int s) {
   return (a.wtab && s < a.E) ? reinterpret_cast<const void*>(a.wtab[s]) : a.wblk[s];
 }
-// Phase 1 computes the hit and shared experts and the experts streamed behind their fetch, phase 2
-// the others (experts a prefetch is still bringing in; without streaming, also the misses).
-__device__ __forceinline__ bool seg_streamed(const FfnArgs& a, int s, unsigned long long stream) {
-  return a.landed != nullptr && s < a.E && ((stream >> s) & 1ull);
-}
-__device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned long long hits,
-                                             unsigned long long stream = 0) {
+__device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned long long hits) {
   if (a.phase == 0) return true;
-  const bool first = s >= a.E || ((hits >> s) & 1ull) || seg_streamed(a, s, stream);
-  return a.phase == 1 ? first : !first;
+  const bool hit = s >= a.E || ((hits >> s) & 1ull);
+  return a.phase == 1 ? hit : !hit;
 }
 // stages: bit 0 = GEMM13 (+ SwiGLU), bit 1 = GEMM2
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s,
@@ -282,8 +262,6 @@ struct CacheStepArgs {
   int32_t* miss_dev;  // device copy of the same list (read by the fetch kernel)
   unsigned long long* ptr_tab;  // device [E]: block address of each selected expert, else 0
   unsigned long long* ready;    // device: bit e set when expert e was a hit at this step
-  unsigned long long* stream;   // device: bit e set when expert e is a miss of this step (copied
-                                // by the step's demand fetch); NULL: not published
   const char* slots;            // this layer's first slot block (NULL in accounting mode)
   const char* staging;          // bypass staging blocks
   size_t expert_bytes;
@@ -325,9 +303,6 @@ struct FetchArgs {
   size_t bytes;                       // per expert block, multiple of 16
   const unsigned long long* cancel;   // prefetch fetches: experts to stop copying, else NULL
   unsigned long long* moved;          // prefetch fetches: bytes copied (accumulated), else NULL
-  unsigned* landed;                   // demand fetches: [E][ppe] piece stamps (NULL: none)
-  const int64_t* epoch;               // the stamp: the layer's step count after its cache step
-  int ppe;                            // pieces per expert block
 };
 cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch = false);
 // Plain copy from device-visible host memory with the fetch kernel's load loop (bytes % 16 == 0).
