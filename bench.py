@@ -309,6 +309,20 @@ def decode_roofline(prof, U, steps, batch, shape, peaks):
     return roof, rates
 
 
+# Launches that move experts over the host link in a device-driven step: the fetch kernel on the
+# copy stream (batches of more than 16 tokens, or a prefetch in flight), or the decode FFN launch
+# that fetches its own misses (smaller batches).
+FETCHING = ("fetch", "ffn_decode_fetch")
+
+
+def fetching_kernel(kernels):
+    """Name of the launch that fetched the misses in a profiled device-driven pass."""
+    for k in FETCHING:
+        if kernels.get(k, {}).get("launches", 0):
+            return k
+    return None
+
+
 def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks=None, world=1):
     """One measured pass over the decode steps [first, first + steps) of layer L.
 
@@ -402,7 +416,9 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world
         profiled_ms_per_step=el_p * 1e3 / steps,
         kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
         gpu_launches=int(sum(v[0] for v in prof.values() if v[0])), roofline=roof,
-        kernel_gbs=rates, kernel_ms_per_step=sum(v[1] for k, v in prof.items() if k != "fetch") / steps,
+        kernel_gbs=rates,
+        kernel_ms_per_step=sum(v[1] for k, v in prof.items() if k not in FETCHING) / steps,
+        fetch_launch_ms_per_step=sum(v[1] for k, v in prof.items() if k in FETCHING) / steps,
         roofline_alone=dict(roof_alone or {}, note="same FFN kernel in the host-driven step, "
                             "where it runs alone"),
         host_fetch_path=dict(tokens_per_s=batch * steps / el_h, ms_per_step=el_h * 1e3 / steps,
@@ -1178,16 +1194,17 @@ def main():
     max_el, tokens = aggregate(elapsed, batch * args.steps, world)
     link = host_link_probe(dev, shape.expert_bytes)
     ms = max_el * 1e3 / args.steps
-    # the dominant kernel of the device-driven step is the fetch: bound by the host link
-    nf, msf = d["kernels"].get("fetch", {}).get("launches", 0), d["kernels"].get("fetch", {}).get("ms", 0.0)
+    # the dominant kernel of the device-driven step is the one that fetches: bound by the host link
+    fk = fetching_kernel(d["kernels"]) or "fetch"
+    nf, msf = d["kernels"].get(fk, {}).get("launches", 0), d["kernels"].get(fk, {}).get("ms", 0.0)
     fetched = d["fetch_bytes_per_step"] * args.steps
-    fetch_roof = dict(bound="host-link", kernel="fetch", unit="GB/s",
+    fetch_roof = dict(bound="host-link", kernel=fk, unit="GB/s",
                       achieved=fetched / (msf / 1e3) / 1e9 if msf else None, peak=link["best_gbs"],
                       peak_source="best pinned host-to-device rate of the link probes in this run "
                                   "(352 MB: copy engines with 1, 2, 4 concurrent copies; SM loads "
                                   "on 38, 76, 152 CTAs)",
-                      traffic=(traffic_ratio("fetch") * fetched / max(1, nf)
-                               if traffic_ratio("fetch") else None),
+                      traffic=(traffic_ratio(fk) * fetched / max(1, nf)
+                               if traffic_ratio(fk) else None),
                       alg_bytes_per_launch=fetched / max(1, nf), launches=nf,
                       timed_in="the profiled pass over the same steps (kernel CUDA events)")
     fetch_roof["frac"] = fetch_roof["achieved"] / link["best_gbs"] if msf else None
@@ -1199,8 +1216,11 @@ def main():
         warmup=args.warmup, ms_per_step=ms, higher_is_better=True,
         scaling="weak", vs_baseline=None, dtype="bf16", data="synthetic", config=_config(batch),
         roofline=fetch_roof,
-        roofline_ffn=dict(d["roofline"] or {}, note="decode FFN inside the device-driven step, "
-                          "sharing SMs and HBM with the concurrent fetch kernel"),
+        roofline_ffn=(dict(d["roofline"], note="decode FFN inside the device-driven step, sharing SMs "
+                                               "and HBM with the concurrent fetch kernel")
+                      if d["roofline"] else
+                      dict(note="the step's FFN runs in the launch that fetches its misses, which "
+                                "the host link bounds: see roofline and roofline_ffn_alone")),
         roofline_ffn_alone=d["roofline_alone"],
         kernel_gbs=d["kernel_gbs"],
         e2e=e2e, gpu_launches=d["gpu_launches"],
@@ -1212,12 +1232,15 @@ def main():
         cache=dict(policy="LRU", hits=d["hits"], fetches=d["fetches"], bypass=d["bypass"],
                    fetches_per_step=d["fetches_per_step"], fetches_per_token=d["fetches_per_token"],
                    hit_rate=d["hit_rate"], mean_experts_per_step=d["mean_experts_per_step"]),
-        fetch=dict(path="device-driven (fetch kernel on a copy stream, overlapped with the hit "
-                        "experts' FFN)",
+        fetch=dict(path="device-driven: batches of up to 16 tokens fetch in the FFN's own launch "
+                        "(its first 38 CTAs copy the misses piece by piece while the others compute "
+                        "the hits, and each missed expert's items start as their pieces land); "
+                        "larger batches run a fetch kernel on a copy stream beside the hits' FFN",
                    bytes_per_step=d["fetch_bytes_per_step"], host_link_probe=link,
                    link_roofline_ms_per_step=d["fetch_bytes_per_step"] / (link["best_gbs"] * 1e9) * 1e3,
                    link_frac=(d["fetch_bytes_per_step"] / (ms / 1e3)) / (link["best_gbs"] * 1e9),
-                   kernel_ms_per_step=d["kernel_ms_per_step"]),
+                   kernel_ms_per_step=d["kernel_ms_per_step"],
+                   fetch_launch_ms_per_step=d["fetch_launch_ms_per_step"]),
         host_fetch_path=d["host_fetch_path"],
     )
     runs = {"mixtral_b%d" % batch: (shape, batch, seed, idx_main, args.steps, d)}

@@ -280,13 +280,18 @@ mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, cons
 /* mcft_moe_forward_cached: mcft_moe_forward for a decode step of `layer` whose experts come from
  * the cache, with the fetch driven by the device and overlapped with compute; no host round trip.
  * Call it after mcft_cache_step(cache, layer, idx, ...) on compute_stream, instead of
- * mcft_fetch_experts + mcft_moe_forward. On copy_stream (after that cache step) a kernel copies
- * every missed expert's block from pinned host memory into the slot or staging buffer the cache
- * step chose, reading the host memory directly over the host link; on compute_stream the
- * permutation and the FFN of the experts that were hits (and of the shared experts) run at the
- * same time; then compute_stream waits for the copies and computes the fetched experts and the
- * combine. Results equal mcft_moe_forward's with the same experts, bit for bit (a decode work item
- * has the same shape and summation order whichever launch computes its expert).
+ * mcft_fetch_experts + mcft_moe_forward. Every missed expert's block is copied from pinned host
+ * memory into the slot or staging buffer the cache step chose, by SM loads over the host link:
+ *  - bf16, T <= 16, and no prefetch of any layer in flight: in the FFN's own launch on
+ *    compute_stream, whose first CTAs copy the misses piece by piece while the others compute the
+ *    hits (and shared experts); a missed expert's work items start as the pieces they read land,
+ *    so its FFN runs while the rest of the step's bytes are still on the host link (copy_stream is
+ *    not used);
+ *  - otherwise: on copy_stream (after that cache step) a fetch kernel copies them while the
+ *    permutation and the FFN of the hits run on compute_stream; then compute_stream waits for the
+ *    copies and computes the fetched experts.
+ * Then the combine. Results equal mcft_moe_forward's with the same experts, bit for bit (a decode
+ * work item has the same shape and summation order whichever launch computes its expert).
  * Section 3.1 Eq. topk (the layer); Section 1 and Section 3.1 "Preliminaries" (every miss is a fetch
  * from host memory).
  *   cache  created with host blocks (not accounting-only); its E and expert size match desc

@@ -189,6 +189,9 @@ struct mcft_cache {
   int32_t* d_miss_dev = nullptr;            // device-memory copy [L][miss_stride]
   unsigned long long* d_ptr_tab = nullptr;  // [L*E] block address of each selected expert
   unsigned long long* d_ready = nullptr;    // [L] hit mask of the last step
+  unsigned long long* d_stream = nullptr;   // [L] miss mask of the last step
+  unsigned* d_landed = nullptr;  // [L][E][ppe] epoch stamps of the demand fetch's landed pieces
+  int ppe = 0;                   // fetch pieces per expert block
   unsigned long long* d_host_src = nullptr; // [L*E] device-visible addresses of the host blocks
   unsigned long long* d_pfmask = nullptr;   // [L] experts loaded by a prefetch since the last step
   unsigned long long* d_pf_cancel = nullptr;  // [L] prefetched experts the next step dropped
@@ -222,6 +225,8 @@ void cache_free(mcft_cache* c) {
   cudaFree(c->d_miss_dev);
   cudaFree(c->d_ptr_tab);
   cudaFree(c->d_ready);
+  cudaFree(c->d_stream);
+  cudaFree(c->d_landed);
   cudaFree(c->d_host_src);
   cudaFree(c->d_pfmask);
   cudaFree(c->d_pf_cancel);
@@ -638,10 +643,16 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
   MCFT_CACHE_CUDA(cudaMemset(c->d_ptr_tab, 0, sizeof(unsigned long long) * L * E));
   MCFT_CACHE_CUDA(cudaMalloc(&c->d_ready, sizeof(unsigned long long) * L));
   MCFT_CACHE_CUDA(cudaMemset(c->d_ready, 0, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMalloc(&c->d_stream, sizeof(unsigned long long) * L));
+  MCFT_CACHE_CUDA(cudaMemset(c->d_stream, 0, sizeof(unsigned long long) * L));
   if (host_experts) {
     c->host_experts.assign(host_experts, host_experts + size_t(L) * E);
     c->n_staging = stg;
     MCFT_CACHE_CUDA(cudaMalloc(&c->d_slots, expert_bytes * size_t(L) * B));
+    // stamps start below every epoch (steps count from 1)
+    c->ppe = int((expert_bytes + kFetchPiece - 1) / kFetchPiece);
+    MCFT_CACHE_CUDA(cudaMalloc(&c->d_landed, sizeof(unsigned) * size_t(L) * E * c->ppe));
+    MCFT_CACHE_CUDA(cudaMemset(c->d_landed, 0, sizeof(unsigned) * size_t(L) * E * c->ppe));
     if (stg > 0) MCFT_CACHE_CUDA(cudaMalloc(&c->d_staging, expert_bytes * size_t(stg)));
     // device-visible addresses of the pinned host blocks, for the device-driven fetch
     std::vector<unsigned long long> src(size_t(L) * E);
@@ -687,7 +698,7 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
                   c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
                   c->d_miss + size_t(layer) * c->miss_stride,
                   c->d_miss_dev + size_t(layer) * c->miss_stride,
-                  c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer,
+                  c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer, c->d_stream + layer,
                   c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                   c->d_staging, c->expert_bytes, device_error_word()};
   cudaError_t e = launch_cache_step(a, stream);
@@ -936,6 +947,58 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   int* perm = reinterpret_cast<int*>(ws + L.perm);
   int* done = reinterpret_cast<int*>(ws + L.done);
   unsigned* err = device_error_word();
+  // Small bf16 decode batches with no prefetch in flight (for any layer) fetch in the FFN's own
+  // launch: its first fetch_blocks() CTAs copy the misses piece by piece and stamp each piece,
+  // and the launch computes the misses with the hits, each of their items waiting for the pieces
+  // it reads, so their FFN runs while the rest of the step's bytes are still on the host link and
+  // no second launch waits for the copy. Otherwise a fetch kernel on the copy stream moves the
+  // misses (behind this layer's prefetch, ahead of later layers') and a second FFN launch computes
+  // them after it.
+  int pf_any = 0;
+  for (int l = 0; l < c->L; ++l) pf_any += c->pf_state[l] != 0 ? 1 : 0;
+  const bool own_fetch = L.decode && T <= kStreamMaxT && c->d_landed != nullptr && pf_any == 0;
+  cudaError_t e = cudaSuccess;
+  if (own_fetch) {
+    if (!permuted) {
+      PermuteArgs pa{idx, T, K, E, S, L.pad, L.mcap, hdr, cnt, off, pos, perm, err, done};
+      e = launch_permute(pa, compute_stream);
+      if (e != cudaSuccess) return cuda_fail(e, "permute kernel launch");
+    }
+    FfnArgs fa{};
+    fa.x = x;
+    fa.off = off;
+    fa.perm = perm;
+    fa.hdr = hdr;
+    fa.done = done;
+    for (int s = 0; s < S; ++s) fa.wblk[E + s] = shared[s];
+    fa.h = ws + L.h;
+    fa.o = reinterpret_cast<float*>(ws + L.o);
+    fa.o_plane = size_t(L.mcap) * desc->d;
+    fa.ksplit = L.ks;
+    fa.T = T;
+    fa.d = desc->d;
+    fa.w = desc->w;
+    fa.nseg = E + S;
+    fa.E = E;
+    fa.err = err;
+    fa.wtab = c->d_ptr_tab + size_t(layer) * E;
+    fa.ready = c->d_ready + layer;
+    fa.phase = 1;  // hits, shared experts and the misses it fetches
+    fa.stream = c->d_stream + layer;
+    fa.landed = c->d_landed + size_t(layer) * E * c->ppe;
+    fa.epoch = c->d_step + layer;
+    fa.ppe = c->ppe;
+    fa.fmiss = c->d_miss_dev + size_t(layer) * c->miss_stride;
+    fa.fsrc = c->d_host_src + size_t(layer) * E;
+    fa.fbytes = c->expert_bytes;
+    fa.nfetch = fetch_blocks();
+    e = launch_ffn_decode(fa, num_sms(), compute_stream, 3, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "expert FFN launch");
+    CombineArgs ca{fa.o, gate, pos, off, hdr, y, T, desc->d, K, E, S, L.ks, fa.o_plane};
+    e = launch_combine(ca, desc->dtype, compute_stream);
+    if (e != cudaSuccess) return cuda_fail(e, "combine kernel launch");
+    return MCFT_OK;
+  }
   // 0. a prefetch of this layer decided before the step lands first (it may target the slots the
   //    step's misses overwrite)
   if (c->pf_state[layer] == 1) {
@@ -946,7 +1009,7 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   MCFT_CUDA(cudaStreamWaitEvent(copy_stream, c->ev_step[layer], 0));
   FetchArgs fe{c->d_miss_dev + size_t(layer) * c->miss_stride, c->d_host_src + size_t(layer) * E,
                c->d_ptr_tab + size_t(layer) * E, c->expert_bytes, nullptr, nullptr};
-  cudaError_t e = launch_fetch(fe, fetch_blocks(), copy_stream);
+  e = launch_fetch(fe, fetch_blocks(), copy_stream);
   if (e != cudaSuccess) return cuda_fail(e, "fetch kernel launch");
   MCFT_CUDA(cudaEventRecord(c->ev_copy, copy_stream));
   // Experts a prefetch of this layer is still bringing in are not in the step's ready mask: the
@@ -1054,7 +1117,7 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
                           c->d_freq, c->d_step, c->d_cnt, c->d_pfmask, c->d_pf_cancel,
                           c->d_miss + size_t(layer) * c->miss_stride,
                           c->d_miss_dev + size_t(layer) * c->miss_stride,
-                          c->d_ptr_tab + size_t(layer) * E, c->d_ready + layer,
+                          c->d_ptr_tab + size_t(layer) * E, c->d_ready + layer, c->d_stream + layer,
                           c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                           c->d_staging, c->expert_bytes, err};
   a.do_prefetch = do_pf ? 1 : 0;
@@ -1178,6 +1241,9 @@ mcft_status mcft_cache_import(mcft_cache* c, const void* buf, size_t bytes, mcft
     MCFT_CUDA(cudaMemcpyAsync(part.dst, p, part.n, cudaMemcpyHostToDevice, stream));
     p += part.n;
   }
+  // landed stamps may carry the epochs of steps taken after the exported state: clear them
+  if (c->d_landed)
+    MCFT_CUDA(cudaMemsetAsync(c->d_landed, 0, sizeof(unsigned) * size_t(c->L) * c->E * c->ppe, stream));
   MCFT_CUDA(cudaStreamSynchronize(stream));
   return MCFT_OK;
 }

@@ -42,27 +42,12 @@ __global__ void __launch_bounds__(32) prefetch_kernel(const __grid_constant__ Pr
   prefetch_warp(a);
 }
 
-// One 64 KB piece [w0, w1) of a copy, in 16-byte words: each thread keeps four loads in flight
-// before it stores them, so a CTA has 64 KB of reads outstanding on the host link.
-__device__ __forceinline__ void copy_piece(const uint4* src, uint4* dst, size_t w0, size_t w1) {
-  const size_t stride = blockDim.x;
-  for (size_t w = w0 + threadIdx.x; w < w1; w += 4 * stride) {
-    uint4 v[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (w + j * stride < w1) v[j] = src[w + j * stride];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      if (w + j * stride < w1) dst[w + j * stride] = v[j];
-  }
-}
-
 // Copy the missed experts' blocks host -> device with 16-byte loads over the host link. Work
 // units are 64 KB pieces of the missed blocks, spread over the grid.
 __global__ void __launch_bounds__(256) fetch_kernel(const __grid_constant__ FetchArgs a) {
   pdl_wait();
   const int n = a.miss[0];
-  const size_t words = a.bytes / 16, piece = 4096;
+  const size_t words = a.bytes / 16, piece = kFetchPiece / 16;
   const size_t per = (words + piece - 1) / piece;
   const size_t units = size_t(n) * per;
   for (size_t u = blockIdx.x; u < units; u += gridDim.x) {

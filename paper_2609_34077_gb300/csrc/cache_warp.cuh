@@ -82,6 +82,7 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
       a.miss_out[0] = 0;
       a.miss_dev[0] = 0;
       *a.ready = 0;
+      if (a.stream) *a.stream = 0;
     }
     for (int e = lane; e < E; e += 32) a.ptr_tab[e] = 0;
     __threadfence_system();
@@ -194,7 +195,11 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) hitbits |= __shfl_xor_sync(0xffffffffu, hitbits, o);
-  if (lane == 0) *a.ready = hitbits;
+  if (lane == 0) {
+    *a.ready = hitbits;
+    // the misses, which this step's demand fetch copies (none without slots)
+    if (a.stream) *a.stream = a.slots ? (mine & ~cached) : 0ull;
+  }
   // No fence: the FFN and fetch kernels read these after a kernel boundary (or an event), the host
   // after synchronising on one; the running fetch kernel that polls the cancel mask only needs the
   // write to arrive, in any order.

@@ -82,6 +82,21 @@ __device__ __forceinline__ uint32_t pack2bf(float a, float b) {
   return uint32_t(f2bf(a)) | (uint32_t(f2bf(b)) << 16);
 }
 
+// One piece [w0, w1) of a host-to-device copy, in 16-byte words, by the whole CTA: each thread
+// keeps four loads in flight before it stores them (64 KB outstanding per 256-thread CTA).
+__device__ __forceinline__ void copy_piece(const uint4* src, uint4* dst, size_t w0, size_t w1) {
+  const size_t stride = blockDim.x;
+  for (size_t w = w0 + threadIdx.x; w < w1; w += 4 * stride) {
+    uint4 v[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (w + j * stride < w1) v[j] = src[w + j * stride];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (w + j * stride < w1) dst[w + j * stride] = v[j];
+  }
+}
+
 // D += A B on the tensor cores, one warp: A 16 x 16 bf16 (row), B 16 x 8 bf16 (col), D fp32.
 __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {

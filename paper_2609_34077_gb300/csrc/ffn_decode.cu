@@ -38,6 +38,8 @@ constexpr int kMaxNG = kPassTokens / 8;
 
 struct DecItems {
   int npos, total, ksplit, rb;  // rb: row blocks per item
+  unsigned long long stream;    // segments streamed behind their fetch (seg_streamed)
+  unsigned epoch;               // the stamp their landed pieces carry
   int off[kMaxSeg + 1];    // by segment: permuted-row offsets
   const char* blk[kMaxSeg];
   int seg[kMaxSeg];        // by position in the work list: segment
@@ -48,8 +50,9 @@ struct DecItems {
 // s = lane, lane + 32, lane + 64): for every non-empty segment of the phase, its rows in items of
 // rb blocks of rows_per_block rows, times ksplit contraction parts; segments in decreasing order
 // of their token counts (ties by index), so that the items that take longest (segments that need
-// a second pass or more MMA columns) are handed out first and the last ones are short. Only
-// segments with work get a position. The item shape depends on the layer and the batch only, not
+// a second pass or more MMA columns) are handed out first and the last ones are short; segments
+// streamed behind their fetch come after all the others (their items wait for bytes still on the
+// host link). Only segments with work get a position. The item shape depends on the layer and the batch only, not
 // on which segments a launch computes, so an output is bit-identical whichever phase of a cached
 // forward computes it. The caller synchronises the block before reading the list.
 __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int rows_per_block,
@@ -60,6 +63,8 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
   // abort flag applied
   const int aborted = a.hdr->abort;
   const unsigned long long hits = a.ready ? *a.ready : 0ull;
+  const unsigned long long stream = a.landed && a.stream ? *a.stream : 0ull;
+  const unsigned epoch = a.landed ? static_cast<unsigned>(*a.epoch) : 0u;
   int offv[3];
   const char* blkv[3];
 #pragma unroll
@@ -76,7 +81,9 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
   }
   __syncwarp();
   bool bad = false;
-  int key[3];  // token count of a segment with work, else -1
+  // key of a segment with work (else -1): its token count, raised by 2^20 unless it is streamed
+  // behind its fetch, so that the streamed segments' items come last
+  int key[3];
   unsigned work[3];
 #pragma unroll
   for (int j = 0; j < 3; ++j) {
@@ -86,9 +93,9 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
       const char* b = blkv[j];
       it.blk[s] = b;
       const int n = it.off[s + 1] - it.off[s];
-      if (n > 0 && seg_in_phase(a, s, hits)) {
+      if (n > 0 && seg_in_phase(a, s, hits, stream)) {
         if (b == nullptr) bad = true;  // a selected expert without weights
-        else key[j] = n;
+        else key[j] = n + (seg_streamed(a, s, stream) ? 0 : (1 << 20));
       }
     }
     work[j] = __ballot_sync(full, key[j] >= 0);
@@ -135,6 +142,8 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
     it.ksplit = ksplit;
     it.rb = rb;
     it.total = base;
+    it.stream = stream;
+    it.epoch = epoch;
   }
 }
 
@@ -203,7 +212,15 @@ __device__ __forceinline__ void warp_slice(int nch, int parts, int part, int& c0
 // GEMM13 + SwiGLU for RB blocks of 16 rows starting at r0 and n <= 32 tokens of one segment
 // starting at permuted row q0; warp w owns row block w / KS and contraction slice w % KS.
 // red: shared scratch [kWarps][kMaxNG][8][32] floats.
-template <int NG, bool DB>
+// COH: weight loads through L2 only (ld.global.cg) for a block that a fetch kernel running beside
+// this launch wrote; otherwise streaming non-coherent loads. Both read the same bytes.
+template <bool COH>
+__device__ __forceinline__ uint4 ldw16(const void* p) {
+  if constexpr (COH) return ldcg16(p);
+  else return ld_stream16(p);
+}
+
+template <int NG, bool DB, bool COH = false>
 __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, const void* lblk,
                                            int r0, int q0, int n, int RB, int KS, float* red) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -232,10 +249,10 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
   // one chunk's weights: W1 rows g / g+8 (lo, hi halves), then W3's
   auto load = [&](uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
-    v[0] = ld_stream16(w1g + k); v[1] = ld_stream16(w1g + k + 64);
-    v[2] = ld_stream16(w1h + k); v[3] = ld_stream16(w1h + k + 64);
-    v[4] = ld_stream16(w3g + k); v[5] = ld_stream16(w3g + k + 64);
-    v[6] = ld_stream16(w3h + k); v[7] = ld_stream16(w3h + k + 64);
+    v[0] = ldw16<COH>(w1g + k); v[1] = ldw16<COH>(w1g + k + 64);
+    v[2] = ldw16<COH>(w1h + k); v[3] = ldw16<COH>(w1h + k + 64);
+    v[4] = ldw16<COH>(w3g + k); v[5] = ldw16<COH>(w3g + k + 64);
+    v[6] = ldw16<COH>(w3h + k); v[7] = ldw16<COH>(w3h + k + 64);
   };
   auto compute = [&](const uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
@@ -294,7 +311,7 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
 // share the h fragments, so each lane keeps 8 weight loads in flight per chunk), contraction part
 // kp of ks, and n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part.
 // red: shared scratch [kWarps][kMaxNG][8][32] floats. Output plane kp of o.
-template <int NG, bool DB>
+template <int NG, bool DB, bool COH = false>
 __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, const void* lblk,
                                           int r0, int q0, int n, int kp, int ks, int RB, int KS,
                                           float* red) {
@@ -325,10 +342,10 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
   // one chunk's weights: tile 0 rows g / g+8 (lo, hi halves), then tile 1's
   auto load = [&](uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
-    v[0] = ld_stream16(wg + k); v[1] = ld_stream16(wg + k + 64);
-    v[2] = ld_stream16(wh + k); v[3] = ld_stream16(wh + k + 64);
-    v[4] = ld_stream16(vg + k); v[5] = ld_stream16(vg + k + 64);
-    v[6] = ld_stream16(vh + k); v[7] = ld_stream16(vh + k + 64);
+    v[0] = ldw16<COH>(wg + k); v[1] = ldw16<COH>(wg + k + 64);
+    v[2] = ldw16<COH>(wh + k); v[3] = ldw16<COH>(wh + k + 64);
+    v[4] = ldw16<COH>(vg + k); v[5] = ldw16<COH>(vg + k + 64);
+    v[6] = ldw16<COH>(vh + k); v[7] = ldw16<COH>(vh + k + 64);
   };
   auto compute = [&](const uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
@@ -378,7 +395,7 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
 // kernel, so the small-batch kernels keep the registers for double-buffered loads.
 // One GEMM13 work item (RB blocks of 16 rows of one segment, all its tokens in passes of at most
 // 8 * MAXNG); returns the segment.
-template <int MAXNG, bool DBOK = true>
+template <int MAXNG, bool DBOK = true, bool COH = false>
 __device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, int item,
                                           float* red) {
   const int RB = it.rb, KS = kWarps / RB;
@@ -389,16 +406,16 @@ __device__ __forceinline__ int run13_item(const FfnArgs& a, const DecItems& it, 
   // passes of at most 8 * MAXNG tokens; a later pass re-reads the rows from L2, not HBM
   for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
     const int n = min(8 * MAXNG, it.off[s + 1] - q0);
-    if (n <= 8) dec13_item<1, DBOK && MAXNG <= 2>(a, blk, lblk, r0, q0, n, RB, KS, red);
+    if (n <= 8) dec13_item<1, DBOK && MAXNG <= 2, COH>(a, blk, lblk, r0, q0, n, RB, KS, red);
     else if (MAXNG == 2 || n <= 16)
-      dec13_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, RB, KS, red);
-    else dec13_item<MAXNG, false>(a, blk, lblk, r0, q0, n, RB, KS, red);
+      dec13_item<(MAXNG >= 2 ? 2 : 1), false, COH>(a, blk, lblk, r0, q0, n, RB, KS, red);
+    else dec13_item<MAXNG, false, COH>(a, blk, lblk, r0, q0, n, RB, KS, red);
   }
   return s;
 }
 
 // One GEMM2 work item (RB blocks of 32 rows of W2 of one segment, one contraction part).
-template <int MAXNG, bool DBOK = true>
+template <int MAXNG, bool DBOK = true, bool COH = false>
 __device__ __forceinline__ void run2_item(const FfnArgs& a, const DecItems& it, int item,
                                           float* red) {
   const int RB = it.rb, KS = kWarps / RB;
@@ -409,10 +426,12 @@ __device__ __forceinline__ void run2_item(const FfnArgs& a, const DecItems& it, 
   const void* lblk = a.lrank ? a.lblk[s] : nullptr;
   for (int q0 = it.off[s]; q0 < it.off[s + 1]; q0 += 8 * MAXNG) {
     const int n = min(8 * MAXNG, it.off[s + 1] - q0);
-    if (n <= 8) dec2_item<1, DBOK && MAXNG <= 2>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+    if (n <= 8)
+      dec2_item<1, DBOK && MAXNG <= 2, COH>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
     else if (MAXNG == 2 || n <= 16)
-      dec2_item<(MAXNG >= 2 ? 2 : 1), false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
-    else dec2_item<MAXNG, false>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
+      dec2_item<(MAXNG >= 2 ? 2 : 1), false, COH>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS,
+                                                   red);
+    else dec2_item<MAXNG, false, COH>(a, blk, lblk, r0, q0, n, kp, it.ksplit, RB, KS, red);
   }
 }
 
@@ -464,6 +483,31 @@ __device__ bool wait_segment(const FfnArgs& a, int s, int need) {
   return true;
 }
 
+// Bounded wait (one thread) until every fetch piece of expert e's block that [off, off + len)
+// touches carries this step's stamp, i.e. its bytes have landed; false (and the call aborted) if
+// a.wait_ns pass or the call is already aborting.
+__device__ bool wait_landed(const FfnArgs& a, unsigned epoch, int e, size_t off, size_t len) {
+  const volatile unsigned* f = a.landed + size_t(e) * a.ppe;
+  const volatile int* abort = &a.hdr->abort;
+  const size_t p1 = (off + len - 1) / kFetchPiece;
+  uint64_t t0 = 0;
+  for (size_t p = off / kFetchPiece; p <= p1; ++p) {
+    while (f[p] != epoch) {
+      if (*abort) return false;
+      const uint64_t now = globaltimer_ns();
+      if (t0 == 0) t0 = now;
+      else if (now - t0 > a.wait_ns) {
+        set_error(a.err, kErrTimeout);
+        const_cast<WsHeader*>(a.hdr)->abort = 1;
+        return false;
+      }
+      __nanosleep(256);
+    }
+  }
+  __threadfence();
+  return true;
+}
+
 // GEMM13 and GEMM2 of a decode call in one launch. The work list is every GEMM13 item, then every
 // GEMM2 item; CTAs claim items from a counter in the workspace (one atomic per item, issued for the
 // next item while the current one runs), so CTAs that finish early take more and the launch ends
@@ -473,17 +517,52 @@ __device__ bool wait_segment(const FfnArgs& a, int s, int need) {
 // done, then reads h through L2. The waits always end: every GEMM13 item precedes every GEMM2 item
 // in the claim order, so when a GEMM2 item is claimed its segment's GEMM13 items have all been
 // claimed, each by a CTA that is running and finishes it without waiting on anything.
+// A launch that fetches its own misses (a.nfetch > 0) first hands out fetcher roles: the first
+// a.nfetch CTAs to take a role copy the step's missed blocks from host memory piece by piece
+// (pieces claimed from a second counter, each stamped once written and fenced), then claim FFN
+// items like the others. An item of a missed expert waits (bounded) for the stamps of the pieces
+// it reads. Those waits end too: a CTA that holds an FFN item took its role after the a.nfetch
+// fetchers took theirs, so every fetcher is running, and fetchers wait on nothing until all
+// pieces are copied.
 template <int MAXNG>
 __global__ void __launch_bounds__(kWarps * 32, 2)
     dec_fused_kernel(const __grid_constant__ FfnArgs a, int RB13, int RB2) {
+  // streaming behind the fetch is compiled into the kernels of up to kStreamMaxT tokens (the
+  // host only asks for it there)
+  constexpr bool kStreams = 8 * MAXNG <= kStreamMaxT;
   pdl_wait();
   __shared__ DecItems it13, it2;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
-  __shared__ int s_next, s_ok;
+  __shared__ int s_next, s_ok, s_role;
   const int warp = threadIdx.x >> 5;
   if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1);
   else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit);
-  else if (threadIdx.x == 64) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
+  else if (threadIdx.x == 64) s_role = a.nfetch > 0 ? atomicAdd(a.done + a.nseg + 4, 1) : a.nfetch;
+  __syncthreads();
+  if constexpr (kStreams) {
+    if (s_role < a.nfetch) {  // fetcher: copy pieces of the missed blocks until none are left
+      const int nm = a.fmiss[0];  // copied even if the call aborts: the cache holds them now
+      const size_t words = a.fbytes / 16, piece = kFetchPiece / 16;
+      const int per = int((words + piece - 1) / piece);
+      const unsigned epoch = it13.epoch;
+      for (;;) {
+        if (threadIdx.x == 0) s_ok = atomicAdd(a.done + a.nseg + 5, 1);
+        __syncthreads();
+        const int u = s_ok;
+        __syncthreads();
+        if (u >= nm * per) break;
+        const int e = a.fmiss[1 + u / per];
+        const size_t w0 = size_t(u % per) * piece, w1 = w0 + piece < words ? w0 + piece : words;
+        copy_piece(reinterpret_cast<const uint4*>(a.fsrc[e]), reinterpret_cast<uint4*>(a.wtab[e]),
+                   w0, w1);
+        __threadfence();  // every thread's stores of the piece, before its stamp
+        __syncthreads();
+        if (threadIdx.x == 0)
+          *reinterpret_cast<volatile unsigned*>(a.landed + size_t(e) * a.ppe + u % per) = epoch;
+      }
+    }
+  }
+  if (threadIdx.x == 0) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
   __syncthreads();
   // Only the next claim stays live across an item body (the item index is consumed at its start;
   // the bounds are re-read from shared memory). Thread 0 issues the claim before the body and
@@ -496,19 +575,56 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
     if (threadIdx.x == 0) next = atomicAdd(a.done + a.nseg + a.phase, 1);
     if (item < it13.total) {
       if (!a.withhold13) {  // (a test withholds GEMM13 items to make the GEMM2 waits run out)
-        const int s = run13_item<MAXNG, kFusedDB>(a, it13, item, red);
-        __threadfence();  // this CTA's h rows, before the segment's count moves
-        __syncthreads();
-        if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
+        const int p = dec_pos(it13, item), s = it13.seg[p];
+        const bool streamed = kStreams && seg_streamed(a, s, it13.stream);
+        int ok = 1;
+        if (streamed) {  // the item's rows of W1 and of W3 must have landed
+          if (threadIdx.x == 0) {
+            const size_t rowb = size_t(a.d) * 2, r0 = size_t(item - it13.first[p]) * kRows * it13.rb;
+            const size_t n = size_t(kRows) * it13.rb * rowb;
+            s_ok = wait_landed(a, it13.epoch, s, r0 * rowb, n) &&
+                   wait_landed(a, it13.epoch, s, (a.w + r0) * rowb, n);
+          }
+          __syncthreads();
+          ok = s_ok;
+        }
+        if (ok) {
+          if constexpr (kStreams) {
+            if (streamed) run13_item<MAXNG, kFusedDB, true>(a, it13, item, red);
+            else run13_item<MAXNG, kFusedDB>(a, it13, item, red);
+          } else {
+            run13_item<MAXNG, kFusedDB>(a, it13, item, red);
+          }
+          __threadfence();  // this CTA's h rows, before the segment's count moves
+          __syncthreads();
+          if (threadIdx.x == 0) atomicAdd(a.done + s, 1);
+        }
       }
     } else {
       const int i2 = item - it13.total;
-      // every segment with work has w / (16 rb) GEMM13 items
-      if (threadIdx.x == 0)
-        s_ok = wait_segment(a, it2.seg[dec_pos(it2, i2)], a.w / (kRows * it13.rb)) ? 1 : 0;
+      const int p = dec_pos(it2, i2), s = it2.seg[p];
+      const bool streamed = kStreams && seg_streamed(a, s, it2.stream);
+      // every segment with work has w / (16 rb) GEMM13 items; a streamed segment's item also
+      // waits for its rows of W2
+      if (threadIdx.x == 0) {
+        bool ok = wait_segment(a, s, a.w / (kRows * it13.rb));
+        if (ok && streamed) {
+          const size_t rowb = size_t(a.w) * 2;
+          const size_t r0 = size_t((i2 - it2.first[p]) / it2.ksplit) * kRows2 * it2.rb;
+          ok = wait_landed(a, it2.epoch, s, size_t(2) * a.w * a.d * 2 + r0 * rowb,
+                           size_t(kRows2) * it2.rb * rowb);
+        }
+        s_ok = ok ? 1 : 0;
+      }
       __syncthreads();
-      const int ok = s_ok;
-      if (ok) run2_item<MAXNG, kFusedDB>(a, it2, i2, red);
+      if (s_ok) {
+        if constexpr (kStreams) {
+          if (streamed) run2_item<MAXNG, kFusedDB, true>(a, it2, i2, red);
+          else run2_item<MAXNG, kFusedDB>(a, it2, i2, red);
+        } else {
+          run2_item<MAXNG, kFusedDB>(a, it2, i2, red);
+        }
+      }
     }
     if (threadIdx.x == 0) s_next = next;
     __syncthreads();
@@ -557,9 +673,10 @@ cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int 
     // both GEMMs in one launch with claimed items
     static const int nbf = blocks_per_sm(reinterpret_cast<const void*>(dec_fused_kernel<MAXNG>));
     const int gf = max(num_sms, num_sms * nbf - reserved);
-    prof_begin(kProfDecFused, s);
+    const int kid = a.nfetch > 0 ? kProfDecFetch : kProfDecFused;  // fetching its own misses
+    prof_begin(kid, s);
     e = launch_pdl(dec_fused_kernel<MAXNG>, dim3(gf), dim3(kWarps * 32), 0, s, a, rb13, rb2);
-    prof_end(kProfDecFused, s);
+    prof_end(kid, s);
     return e != cudaSuccess ? e : cudaGetLastError();
   }
   if (stages & 1) {

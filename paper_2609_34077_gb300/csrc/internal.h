@@ -61,7 +61,9 @@ constexpr int kRouteTileMinT = 64;
 // Header at the start of the forward workspace.
 // Work-claim counters of the fused decode FFN that follow the per-segment progress counters in
 // the workspace: one per FFN phase (0 all segments, 1 hits, 2 misses).
-constexpr int kClaimSlots = 4;
+// slots 0-2: the claim counters of phases 0-2; slot 4: fetcher roles and slot 5: fetch pieces of
+// a decode launch that fetches its own misses (FfnArgs::nfetch)
+constexpr int kClaimSlots = 6;
 
 struct WsHeader {
   int abort;     // set when a kernel of this call found bad data; later kernels skip their work
@@ -176,7 +178,28 @@ struct FfnArgs {
   // GEMM13 items so that those waits run out (set by launch_ffn_decode from the test hooks).
   unsigned long long wait_ns;
   int withhold13;
+  // A decode launch that fetches its own misses (cached forward, small bf16 batches, no prefetch
+  // in flight): its first nfetch CTAs to start copy the step's missed expert blocks (miss list
+  // fmiss, device-visible host blocks fsrc [E], destinations wtab [E], fbytes each) piece by
+  // piece, stamping each kFetchPiece-byte piece in landed [E][ppe] with the step's epoch (*epoch,
+  // the layer's step count after its cache step) once its bytes are written, then join the FFN.
+  // stream has bit e set when expert e is such a miss: the launch computes those experts with the
+  // hits, each of their items waiting (bounded) for the pieces it reads, so their FFN runs while
+  // the rest of the step's bytes are still on the host link. nfetch = 0: no fetch, no streaming.
+  const unsigned long long* stream;
+  unsigned* landed;
+  const int64_t* epoch;
+  int ppe;
+  const int32_t* fmiss;
+  const unsigned long long* fsrc;
+  size_t fbytes;
+  int nfetch;
 };
+
+// Bytes per work unit of the device-driven fetch: the granule of its landed stamps.
+constexpr size_t kFetchPiece = 65536;
+// Cached decode forwards of up to this many tokens stream their misses behind the fetch.
+constexpr int kStreamMaxT = 16;
 
 // Test hooks (mcft_test_inject in api.cu); all off by default.
 unsigned long long test_wait_limit_ns();  // the decode FFN's wait limit (default 2 s)
@@ -212,10 +235,16 @@ __device__ __forceinline__ float lora_up<float>(const void* blk, size_t b_off, i
 __device__ __forceinline__ const void* seg_block(const FfnArgs& a, int s) {
   return (a.wtab && s < a.E) ? reinterpret_cast<const void*>(a.wtab[s]) : a.wblk[s];
 }
-__device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned long long hits) {
+// Phase 1 computes the hit and shared experts and the experts streamed behind their fetch, phase 2
+// the others (experts a prefetch is still bringing in; without streaming, also the misses).
+__device__ __forceinline__ bool seg_streamed(const FfnArgs& a, int s, unsigned long long stream) {
+  return a.landed != nullptr && s < a.E && ((stream >> s) & 1ull);
+}
+__device__ __forceinline__ bool seg_in_phase(const FfnArgs& a, int s, unsigned long long hits,
+                                             unsigned long long stream = 0) {
   if (a.phase == 0) return true;
-  const bool hit = s >= a.E || ((hits >> s) & 1ull);
-  return a.phase == 1 ? hit : !hit;
+  const bool first = s >= a.E || ((hits >> s) & 1ull) || seg_streamed(a, s, stream);
+  return a.phase == 1 ? first : !first;
 }
 // stages: bit 0 = GEMM13 (+ SwiGLU), bit 1 = GEMM2
 cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStream_t s,
@@ -262,6 +291,8 @@ struct CacheStepArgs {
   int32_t* miss_dev;  // device copy of the same list (read by the fetch kernel)
   unsigned long long* ptr_tab;  // device [E]: block address of each selected expert, else 0
   unsigned long long* ready;    // device: bit e set when expert e was a hit at this step
+  unsigned long long* stream;   // device: bit e set when expert e is a miss of this step (copied
+                                // by the step's demand fetch); NULL: not published
   const char* slots;            // this layer's first slot block (NULL in accounting mode)
   const char* staging;          // bypass staging blocks
   size_t expert_bytes;
@@ -399,7 +430,8 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
 // Kernel timing (profile.cu): event pairs around each launch while mcft_profile_enable(1) is on.
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
        kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfNorm,
-       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfDecFused, kProfHostCopy, kProfCount };
+       kProfPrefetch, kProfPfFetch, kProfPrologue, kProfDecFused, kProfHostCopy, kProfDecFetch,
+       kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 
