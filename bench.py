@@ -1058,14 +1058,15 @@ def profile_case(case: str, dev) -> int:
     desc = M.desc_of(sh)
     if case == "fetch16":  # decode steps with the cache and the device-driven fetch
         L = DecodeLayer(sh, 16, 7, dev)
-        per_step = []
+        per_step, experts = [], []
         for s in range(3):
             before = M.mcft_cache_stats(L.cache, 0)[1]
             L.step(s, path="device")
             torch.cuda.synchronize()
             per_step.append(M.mcft_cache_stats(L.cache, 0)[1] - before)
+            experts.append(len(torch.unique(L.idx[s])))
         M.mcft_device_error()
-        print(json.dumps({"case": case, "fetches_per_step": per_step,
+        print(json.dumps({"case": case, "fetches_per_step": per_step, "experts_per_step": experts,
                           "fetch_bytes_per_step": [n * sh.expert_bytes for n in per_step]}))
         return 0
     if case in ("prefill", "ds_prefill"):  # Mixtral keeps 4 of 8, DeepSeek 48 of 64
