@@ -44,10 +44,12 @@ METRIC = "masked MoE layer tokens/s"
 # first 16 hex digits of the kernel source's sha256: when the source has changed since the
 # capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e965b486ab27bed2", None),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e965b486ab27bed2", None),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "e965b486ab27bed2", 1.0017),
-    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "980d86643d8088ca", 0.9559),
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "be7009c604060157", None),
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "be7009c604060157", None),
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "be7009c604060157", 1.0016),
+    # DRAM traffic / (weights of the step's experts read once + activations + fetched bytes written)
+    "ffn_decode_fetch": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "be7009c604060157", 0.902),
+    "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "68e0415de46353e9", 0.9253),
 }
 
 
@@ -276,18 +278,27 @@ def unique_per_step(idx_steps):
     return [len(torch.unique(i)) for i in idx_steps]
 
 
-def decode_roofline(prof, U, steps, batch, shape, peaks):
-    """HBM roofline of the decode FFN kernels. Algorithmic bytes per launch: the W1 and W3 rows
-    (GEMM13) or W2 rows (GEMM2) of every expert the step computes, read once (the routed experts
-    it selected and the shared experts, which every token uses), plus the token activations in and
-    out; the fused kernel (both GEMMs in one launch) reads all three. Returns (dominant kernel's
-    roofline dict, {kernel: GB/s})."""
+def decode_alg_bytes(U, steps, batch, shape):
+    """Algorithmic DRAM bytes of the decode FFN over `steps` steps (U: distinct routed experts of
+    each step): the W1 and W3 rows (GEMM13) and the W2 rows (GEMM2) of every expert the step
+    computes (its routed experts and the shared experts, which every token uses), read once, plus
+    the token activations in and out. Returns (GEMM13 bytes, GEMM2 bytes)."""
     S = shape.n_shared
     sel = sum(U) + steps * S
     T, K, d, w = batch, shape.K, shape.d, shape.w
     rows = T * (K + S)  # permuted rows per step: one per routed assignment and per shared expert
     b13 = sel * 2 * w * d * 2 + steps * (T * d * 2 + rows * w * 2)
     b2 = sel * w * d * 2 + steps * rows * (w * 2 + d * 4)
+    return b13, b2
+
+
+def decode_roofline(prof, U, steps, batch, shape, peaks):
+    """HBM roofline of the decode FFN kernels. Algorithmic bytes per launch: the W1 and W3 rows
+    (GEMM13) or W2 rows (GEMM2) of every expert the step computes, read once (the routed experts
+    it selected and the shared experts, which every token uses), plus the token activations in and
+    out; the fused kernel (both GEMMs in one launch) reads all three. Returns (dominant kernel's
+    roofline dict, {kernel: GB/s})."""
+    b13, b2 = decode_alg_bytes(U, steps, batch, shape)
     alg = {"ffn13_decode": b13, "ffn2_decode": b2, "ffn_decode": b13 + b2}
     rates, best = {}, None
     for k, b in alg.items():
@@ -406,6 +417,7 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world
     roof, rates = decode_roofline(prof, U, steps, batch, shape, peaks)
     roof_alone, rates_alone = decode_roofline(hprof, U, steps, batch, shape, peaks)
     fetch_bytes = fetches * shape.expert_bytes / steps
+    b13, b2 = decode_alg_bytes(U, steps, batch, shape)
     out = dict(
         tokens_per_s=batch * steps / elapsed, ms_per_step=elapsed * 1e3 / steps, steps=steps,
         warmup=warmup, fetch_path="device", hits=hits, fetches=fetches, bypass=byp,
@@ -413,6 +425,7 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world
         hit_rate=hits / max(1, hits + fetches), mean_experts_per_step=float(np.mean(U)),
         fetch_bytes_per_step=fetch_bytes,
         passes_same_decisions=all(c == cnt for c in passes.values()),
+        ffn_dram_bytes_per_step=(b13 + b2) / steps,
         profiled_ms_per_step=el_p * 1e3 / steps,
         kernels={k: dict(launches=v[0], ms=round(v[1], 4)) for k, v in prof.items() if v[0]},
         gpu_launches=int(sum(v[0] for v in prof.values() if v[0])), roofline=roof,
@@ -1050,14 +1063,15 @@ def profile_case(case: str, dev) -> int:
     """A few forwards: the small launch sequences that ncu captures. decode16 / decode1:
     Mixtral-shaped decode at batch 16 / 1 with every expert resident (decode FFN); ds_decode1 /
     ds_decode64: the same for the DeepSeek-V2-Lite shape at batch 1 / 64; prefill / ds_prefill:
-    T = 4096 tokens, hard mask keeping 4 of 8 / 48 of 64 (tcgen05 GEMMs); fetch16: three decode steps at batch 16 through
-    the cache with the device-driven fetch (fetch kernel)."""
+    T = 4096 tokens, hard mask keeping 4 of 8 / 48 of 64 (tcgen05 GEMMs); fetch16 / ds_fetch64:
+    three decode steps (Mixtral-shaped batch 16 / DeepSeek-shaped batch 64) through the cache with
+    the device-driven fetch (the FFN launch that fetches its own misses / the fetch kernel)."""
     from paper_2609_34077_gb300 import mcft as M
 
     sh = I.DSV2_LITE if case.startswith("ds_") else I.MIXTRAL
     desc = M.desc_of(sh)
-    if case == "fetch16":  # decode steps with the cache and the device-driven fetch
-        L = DecodeLayer(sh, 16, 7, dev)
+    if case in ("fetch16", "ds_fetch64"):  # decode steps with the cache, device-driven fetch
+        L = DecodeLayer(sh, 16 if case == "fetch16" else 64, 7, dev)
         per_step, experts = [], []
         for s in range(3):
             before = M.mcft_cache_stats(L.cache, 0)[1]
@@ -1104,7 +1118,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
     ap.add_argument("--case", choices=["decode16", "decode1", "ds_decode1", "ds_decode64", "prefill",
-                                       "ds_prefill", "fetch16", "lora", "mask"],
+                                       "ds_prefill", "fetch16", "ds_fetch64", "lora", "mask"],
                     help="run only a few resident-expert forwards (for profiler captures)")
     ap.add_argument("--workload", default="layer",
                     choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2",
@@ -1204,11 +1218,15 @@ def main():
                       peak_source="best pinned host-to-device rate of the link probes in this run "
                                   "(352 MB: copy engines with 1, 2, 4 concurrent copies; SM loads "
                                   "on 38, 76, 152 CTAs)",
-                      traffic=(traffic_ratio(fk) * fetched / max(1, nf)
-                               if traffic_ratio(fk) else None),
+                      traffic=None, traffic_vs=None,
                       alg_bytes_per_launch=fetched / max(1, nf), launches=nf,
                       timed_in="the profiled pass over the same steps (kernel CUDA events)")
     fetch_roof["frac"] = fetch_roof["achieved"] / link["best_gbs"] if msf else None
+    if traffic_ratio(fk):  # DRAM bytes per launch, from the ncu capture's ratio
+        dram_alg = fetched / max(1, nf)
+        if fk == "ffn_decode_fetch":  # it also reads the step's expert weights
+            dram_alg += d["ffn_dram_bytes_per_step"] * args.steps / max(1, nf)
+        fetch_roof.update(traffic=traffic_ratio(fk) * dram_alg, traffic_vs=dram_alg)
     e2e = dict(d["e2e"])
     el_e2e, tok_e2e = aggregate(e2e.pop("elapsed_s"), batch * args.steps, world)
     e2e["value"] = tok_e2e / el_e2e
