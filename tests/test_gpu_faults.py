@@ -99,3 +99,42 @@ def test_decode_ffn_wait_runs_out(T):
     ref = oracle.ffn.moe_layer(f64(x), ids, gate.cpu().double().numpy(), expert_triples(lw, sh),
                                shared_triples(lw, sh))
     check_output(y, ref, TOL_BF16, f"after the timeout, T={T}")
+
+
+def test_cached_forward_wait_runs_out_and_the_cache_stays_whole():
+    """The cached forward at batch 1 fetches its misses in the FFN's own launch. With GEMM13 items
+    withheld and a 1 ms wait limit, that launch's GEMM2 waits run out: MCFT_ERR_TIMEOUT, y untouched.
+    Its fetchers still copy every missed block (the cache already counts them as resident), so the
+    following steps, with injection off, equal the plain forward bit for bit."""
+    sh = SMALL_DS
+    lw = I.layer_weights(96, sh, pin=True)
+    desc = M.desc_of(sh)
+    cache = M.mcft_cache_create(1, sh.E, sh.cache_slots, sh.expert_bytes, lw.experts, max_assign=sh.K)
+    experts = [b.to(DEV) for b in lw.experts]
+    shared = [b.to(DEV) for b in lw.shared]
+    ws = torch.empty(M.mcft_moe_workspace_size(desc, 1), dtype=torch.uint8, device=DEV)
+    compute, copy = torch.cuda.Stream(), torch.cuda.Stream()
+    ids = I.random_ids(96, 6, 1, sh.K, sh.E, hot=range(sh.keep), p_hot=0.7)
+    for s in range(6):
+        x = I.hidden_iid(97 + s, sh, 1).to(DEV)
+        idx = torch.from_numpy(ids[s]).to(DEV)
+        gate = torch.full((1, sh.K), 0.25, device=DEV)
+        y = torch.full((1, sh.d), 7.0, dtype=torch.bfloat16, device=DEV)
+        torch.cuda.synchronize()
+        M.mcft_cache_step(cache, 0, idx, stream=compute)
+        if s == 0:
+            M.mcft_test_inject(wait_limit_ns=1_000_000, withhold_gemm13=True)
+        M.mcft_moe_forward_cached(desc, x, idx, gate, cache, 0, shared, y=y, workspace=ws,
+                                  compute_stream=compute, copy_stream=copy)
+        M.mcft_test_inject()
+        compute.synchronize()
+        if s == 0:
+            with pytest.raises(M.MCFTError) as ei:
+                M.mcft_device_error()
+            assert ei.value.status == M.MCFT_ERR_TIMEOUT
+            assert torch.all(y == 7.0)
+            continue
+        M.mcft_device_error()
+        y_ref = M.mcft_moe_forward(desc, x, idx, gate, experts, shared)
+        assert torch.equal(y, y_ref), f"step {s}"
+    assert M.mcft_cache_stats(cache, 0)[1] > sh.K  # the stream kept fetching

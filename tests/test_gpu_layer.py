@@ -186,3 +186,31 @@ def test_prefill_deepseek_full_size_every_row():
     """DeepSeek-V2-Lite-shaped, T = 4096, 64 routed experts (hard mask keeping 48) plus the 2
     shared experts on every token: 24576 routed and 8192 shared rows through the grouped GEMMs."""
     _prefill_full(I.DSV2_LITE, 48, seed=91)
+
+
+@pytest.mark.parametrize("T,fetching", [(1, "ffn_decode_fetch"), (16, "ffn_decode_fetch"),
+                                        (17, "fetch"), (40, "fetch")])
+def test_cached_forward_fetches_in_the_ffn_launch_up_to_16_tokens(T, fetching):
+    """Which launch moves the misses: up to 16 tokens (with no prefetch in flight) the decode FFN
+    launch itself, above that the fetch kernel on the copy stream beside a two-phase FFN."""
+    shape = SMALL_DS
+    desc = M.desc_of(shape)
+    lw = I.layer_weights(85, shape, pin=True)
+    cache = M.mcft_cache_create(1, shape.E, shape.cache_slots, shape.expert_bytes, lw.experts,
+                                max_assign=T * shape.K)
+    shared = [b.to(DEV) for b in lw.shared]
+    x = I.hidden_iid(86, shape, T).to(DEV)
+    idx = torch.from_numpy(I.random_ids(85, 1, T, shape.K, shape.E, hot=range(shape.keep))[0]).to(DEV)
+    gate = torch.full((T, shape.K), 0.2, device=DEV)
+    torch.cuda.synchronize()
+    M.mcft_profile_reset()
+    M.mcft_profile_enable(True)
+    M.mcft_cache_step(cache, 0, idx)
+    M.mcft_moe_forward_cached(desc, x, idx, gate, cache, 0, shared, copy_stream=torch.cuda.Stream())
+    M.mcft_profile_enable(False)
+    prof = {k: v[0] for k, v in M.mcft_profile_read().items() if v[0]}
+    M.mcft_device_error()
+    assert prof.get(fetching, 0) == 1, prof
+    other = "fetch" if fetching == "ffn_decode_fetch" else "ffn_decode_fetch"
+    assert prof.get(other, 0) == 0, prof
+    assert prof.get("ffn_decode", 0) == (0 if fetching == "ffn_decode_fetch" else 2), prof
