@@ -524,12 +524,14 @@ __device__ bool wait_landed(const FfnArgs& a, unsigned epoch, int e, size_t off,
 // it reads. Those waits end too: a CTA that holds an FFN item took its role after the a.nfetch
 // fetchers took theirs, so every fetcher is running, and fetchers wait on nothing until all
 // pieces are copied.
-template <int MAXNG>
+// FETCH: the build for launches that fetch their own misses (a.nfetch > 0); the plain build
+// carries none of that code.
+template <int MAXNG, bool FETCH>
 __global__ void __launch_bounds__(kWarps * 32, 2)
     dec_fused_kernel(const __grid_constant__ FfnArgs a, int RB13, int RB2) {
-  // streaming behind the fetch is compiled into the kernels of up to kStreamMaxT tokens (the
-  // host only asks for it there)
-  constexpr bool kStreams = 8 * MAXNG <= kStreamMaxT;
+  // fetching and streaming are compiled into the kernels of up to kStreamMaxT tokens (the host
+  // only asks for them there)
+  constexpr bool kStreams = FETCH && 8 * MAXNG <= kStreamMaxT;
   pdl_wait();
   __shared__ DecItems it13, it2;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
@@ -537,10 +539,14 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   const int warp = threadIdx.x >> 5;
   if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1);
   else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit);
-  else if (threadIdx.x == 64) s_role = a.nfetch > 0 ? atomicAdd(a.done + a.nseg + 4, 1) : a.nfetch;
+  else if (threadIdx.x == 64) {
+    // without fetchers the first claim goes out now, beside the work-list build
+    if (kStreams) s_role = atomicAdd(a.done + a.nseg + 4, 1);
+    else s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
+  }
   __syncthreads();
   if constexpr (kStreams) {
-    if (s_role < a.nfetch) {  // fetcher: copy pieces of the missed blocks until none are left
+    if (s_role < a.nfetch) {  // fetcher: copy the missed blocks' pieces until none are left
       const int nm = a.fmiss[0];  // copied even if the call aborts: the cache holds them now
       const size_t words = a.fbytes / 16, piece = kFetchPiece / 16;
       const int per = int((words + piece - 1) / piece);
@@ -562,8 +568,10 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
       }
     }
   }
-  if (threadIdx.x == 0) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
-  __syncthreads();
+  if constexpr (kStreams) {  // a fetcher claims its first item only once the pieces are all taken
+    if (threadIdx.x == 0) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
+    __syncthreads();
+  }
   // Only the next claim stays live across an item body (the item index is consumed at its start;
   // the bounds are re-read from shared memory). Thread 0 issues the claim before the body and
   // publishes it after, so the atomic's round trip overlaps warp 0's weight loads.
@@ -671,12 +679,21 @@ cudaError_t launch_decode_ng(const FfnArgs& a, int num_sms, cudaStream_t s, int 
   cudaError_t e = cudaSuccess;
   if (stages == 3 && a.done && a.lrank == 0) {
     // both GEMMs in one launch with claimed items
-    static const int nbf = blocks_per_sm(reinterpret_cast<const void*>(dec_fused_kernel<MAXNG>));
+    static const int nbf =
+        blocks_per_sm(reinterpret_cast<const void*>(dec_fused_kernel<MAXNG, false>));
     const int gf = max(num_sms, num_sms * nbf - reserved);
-    const int kid = a.nfetch > 0 ? kProfDecFetch : kProfDecFused;  // fetching its own misses
-    prof_begin(kid, s);
-    e = launch_pdl(dec_fused_kernel<MAXNG>, dim3(gf), dim3(kWarps * 32), 0, s, a, rb13, rb2);
-    prof_end(kid, s);
+    if constexpr (8 * MAXNG <= kStreamMaxT) {
+      if (a.nfetch > 0) {  // fetching its own misses
+        prof_begin(kProfDecFetch, s);
+        e = launch_pdl(dec_fused_kernel<MAXNG, true>, dim3(gf), dim3(kWarps * 32), 0, s, a, rb13,
+                       rb2);
+        prof_end(kProfDecFetch, s);
+        return e != cudaSuccess ? e : cudaGetLastError();
+      }
+    }
+    prof_begin(kProfDecFused, s);
+    e = launch_pdl(dec_fused_kernel<MAXNG, false>, dim3(gf), dim3(kWarps * 32), 0, s, a, rb13, rb2);
+    prof_end(kProfDecFused, s);
     return e != cudaSuccess ? e : cudaGetLastError();
   }
   if (stages & 1) {
