@@ -48,7 +48,7 @@ TRAFFIC = {
     "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "569c2d91706ff439", None),
     "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "569c2d91706ff439", 1.0016),
     # DRAM traffic / (weights of the step's experts read once + activations + fetched bytes written)
-    "ffn_decode_fetch": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "569c2d91706ff439", 0.902),
+    "ffn_decode_fetch": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "569c2d91706ff439", 0.933),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "68e0415de46353e9", 0.9253),
 }
 
