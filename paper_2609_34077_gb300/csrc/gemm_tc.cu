@@ -606,6 +606,8 @@ bool encode_adapter_a2(CUtensorMap* m, const void* a2, uint64_t w, uint32_t r) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+constexpr size_t kSmallSegGroupMB = 2;  // group budget when routed experts have few m-tiles
+
 int group_for(size_t a_tile_bytes, size_t budget_mb) {
   const size_t budget = budget_mb << 20;  // activation rows kept hot in L2 per group
   size_t g = budget / (a_tile_bytes ? a_tile_bytes : 1);
@@ -665,15 +667,21 @@ cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sm
   p13.ntiles_n = int(w / (BN / 2));
   p13.ldo = int(w);
   p13.b_half = int(w);
-  // L2 budgets per group of m-tiles, from same-box sweeps of 6-48 MB over the Mixtral- and
-  // DeepSeek-V2-Lite-shaped T = 4096 layers (GEMM13 best at 24 MB, GEMM2 at 12 MB)
-  p13.group_m = group_for(size_t(BM) * d * 2, 24);
+  // L2 budgets per group of m-tiles, from same-box sweeps over the Mixtral- and
+  // DeepSeek-V2-Lite-shaped T = 4096 layers: with several m-tiles per routed expert (Mixtral)
+  // GEMM13 is best at 24 MB and GEMM2 at 12 MB; with fewer than four on average (DeepSeek-V2-Lite:
+  // 64 experts) small groups of about one expert's rows win (GEMM13 0.55 -> 0.60 of peak)
+  // routed rows T * K: the permuted rows less the shared experts' and the segment padding
+  const size_t routed = size_t(mcap) - size_t(a.T) * (a.nseg - a.E) - size_t(a.nseg) * (BM - 1);
+  const bool small_segs = routed < size_t(4) * BM * a.E;
+  const size_t mb13 = small_segs ? kSmallSegGroupMB : 24, mb2 = small_segs ? kSmallSegGroupMB : 12;
+  p13.group_m = group_for(size_t(BM) * d * 2, mb13);
   p2.out = a.o;
   p2.kblocks = int(w / BK);
   p2.ntiles_n = int(d / BN);
   p2.ldo = int(d);
   p2.b_half = 0;
-  p2.group_m = group_for(size_t(BM) * w * 2, 12);
+  p2.group_m = group_for(size_t(BM) * w * 2, mb2);
   if (a.lrank > 0) {
     const LoraOffsets lo = lora_offsets(a.d, a.w, a.lrank);
     for (int sgi = 0; sgi < a.nseg; ++sgi) {
