@@ -8,7 +8,9 @@
 //    (GEMM2, two MMA tiles sharing the activation fragments), of one segment; its 8 warps are
 //    RB x KS (KS = 8 / RB contraction slices per row block, chosen so every warp walks at least 8
 //    chunks), each walking its slice 64 elements at a time; in each load instruction the 4 lanes
-//    of a quad read 64 contiguous bytes of one row;
+//    of a quad read 64 contiguous bytes of one row; slice k holds chunks k, k + KS, k + 2 KS, ...,
+//    so at each step the KS warps of a row block read KS adjacent chunks (KS x 128 contiguous
+//    bytes of every row) rather than KS chunks far apart;
 //  * the 16 x 64 weight slab is the A operand of four m16n8k16 MMAs (the contraction order inside
 //    a 64-wide chunk is permuted identically for A and B, which leaves every dot product intact);
 //    the B operand is 8 tokens of the segment, so one A fragment serves up to 32 tokens per pass
@@ -175,27 +177,28 @@ __device__ __forceinline__ uint32_t word(const uint4& lo, const uint4& hi, int i
   }
 }
 
-// Walk chunks [c0, c1): load(buf, ch) issues a chunk's weight loads, compute(buf, ch) consumes
-// them. With DB the next chunk's loads are issued before the current chunk's MMAs (two register
+// Walk chunks c0, c0 + step, ... below c1: load(buf, ch) issues a chunk's weight loads,
+// compute(buf, ch) consumes them. With DB the next chunk's loads are issued before the current chunk's MMAs (two register
 // buffers, unrolled by two so nothing is copied), so a warp keeps one chunk in flight while it
 // computes; without DB each chunk is loaded, then consumed (token groups of more than 8, and any
 // group in the kernel compiled for 32-token passes, whose accumulators need the registers).
 template <bool DB, typename Load, typename Compute>
-__device__ __forceinline__ void stream_chunks(int c0, int c1, Load&& load, Compute&& compute) {
+__device__ __forceinline__ void stream_chunks(int c0, int c1, int step, Load&& load,
+                                              Compute&& compute) {
   uint4 va[8];
   if constexpr (DB) {
     uint4 vb[8];
     if (c0 < c1) load(va, c0);
     int ch = c0;
-    for (; ch + 1 < c1; ch += 2) {
-      load(vb, ch + 1);
+    for (; ch + step < c1; ch += 2 * step) {
+      load(vb, ch + step);
       compute(va, ch);
-      if (ch + 2 < c1) load(va, ch + 2);
-      compute(vb, ch + 1);
+      if (ch + 2 * step < c1) load(va, ch + 2 * step);
+      compute(vb, ch + step);
     }
     if (ch < c1) compute(va, ch);
   } else {
-    for (int ch = c0; ch < c1; ++ch) {
+    for (int ch = c0; ch < c1; ch += step) {
       load(va, ch);
       compute(va, ch);
     }
@@ -210,7 +213,8 @@ __device__ __forceinline__ void warp_slice(int nch, int parts, int part, int& c0
 }
 
 // GEMM13 + SwiGLU for RB blocks of 16 rows starting at r0 and n <= 32 tokens of one segment
-// starting at permuted row q0; warp w owns row block w / KS and contraction slice w % KS.
+// starting at permuted row q0; warp w owns row block w / KS and contraction slice w % KS
+// (chunks w % KS, w % KS + KS, ...).
 // red: shared scratch [kWarps][kMaxNG][8][32] floats.
 // COH: weight loads through L2 only (ld.global.cg) for a block that a fetch kernel running beside
 // this launch wrote; otherwise streaming non-coherent loads. Both read the same bytes.
@@ -244,8 +248,7 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
 #pragma unroll
     for (int i = 0; i < 4; ++i) accg[G][i] = accu[G][i] = 0.f;
 
-  int c0, c1;
-  warp_slice(int(rowb / (kChunk * 2)), KS, warp % KS, c0, c1);
+  const int nch = int(rowb / (kChunk * 2));
   // one chunk's weights: W1 rows g / g+8 (lo, hi halves), then W3's
   auto load = [&](uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
@@ -269,7 +272,7 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
       }
     }
   };
-  stream_chunks<DB>(c0, c1, load, compute);
+  stream_chunks<DB>(warp % KS, nch, KS, load, compute);
 #pragma unroll
   for (int G = 0; G < NG; ++G)
 #pragma unroll
@@ -309,7 +312,8 @@ __device__ __forceinline__ void dec13_item(const FfnArgs& a, const char* blk, co
 
 // GEMM2 for RB blocks of 32 output rows of W2 starting at r0 (two 16-row MMA tiles per warp that
 // share the h fragments, so each lane keeps 8 weight loads in flight per chunk), contraction part
-// kp of ks, and n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part.
+// kp of ks, and n <= 32 tokens; warp w owns row block w / KS and slice w % KS of the part (its
+// chunks w % KS, w % KS + KS, ...).
 // red: shared scratch [kWarps][kMaxNG][8][32] floats. Output plane kp of o.
 template <int NG, bool DB, bool COH = false>
 __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, const void* lblk,
@@ -336,9 +340,8 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[G][i] = 0.f;
 
-  int p0, p1, c0, c1;
+  int p0, p1;
   warp_slice(int(rowb / (kChunk * 2)), ks, kp, p0, p1);
-  warp_slice(p1 - p0, KS, warp % KS, c0, c1);
   // one chunk's weights: tile 0 rows g / g+8 (lo, hi halves), then tile 1's
   auto load = [&](uint4* v, int ch) {
     const size_t k = size_t(ch) * kChunk * 2;
@@ -363,7 +366,7 @@ __device__ __forceinline__ void dec2_item(const FfnArgs& a, const char* blk, con
       }
     }
   };
-  stream_chunks<DB>(p0 + c0, p0 + c1, load, compute);
+  stream_chunks<DB>(p0 + warp % KS, p1, KS, load, compute);
 #pragma unroll
   for (int G = 0; G < NG; ++G)
 #pragma unroll
