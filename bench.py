@@ -695,6 +695,28 @@ def run_prefill(steps, warmup, seed, dev, peaks):
                                unit="TFLOP/s", frac=a13 / peak, flop_per_launch=f13)
         res["gemm2_tflops"] = a2
         res["gemm_frac_of_peak"] = (f13 + f2) / ((ms13 / n13 + ms2 / n2) / 1e3) / 1e12 / peak
+    # the same steps on CTA-pair tiles (mcft_set_tc_tiles), for comparison with the default tiles
+    M.mcft_set_tc_tiles(M.MCFT_TC_TILES_CTA_PAIR)
+    try:
+        ws = torch.empty(M.mcft_moe_workspace_size(desc, T), dtype=torch.uint8, device=dev)
+        for s in range(warmup):
+            step(s)
+        M.mcft_profile_reset()
+        M.mcft_profile_enable(True)
+        el_p = time_steps(step, 0, steps, stream)
+        M.mcft_profile_enable(False)
+        pp = M.mcft_profile_read()
+        M.mcft_device_error()
+    finally:
+        M.mcft_profile_enable(False)
+        M.mcft_set_tc_tiles(M.MCFT_TC_TILES_ONE_CTA)
+    (p13, t13), (p2, t2) = pp["gemm13_tc_pair"], pp["gemm2_tc_pair"]
+    if t13 and t2:
+        res["cta_pair_tiles"] = dict(
+            note="same steps with mcft_set_tc_tiles(CTA_PAIR): 256 x 256 tiles on 2-CTA clusters",
+            ms_per_step=el_p * 1e3 / steps, gemm13_us=t13 / p13 * 1e3, gemm2_us=t2 / p2 * 1e3,
+            gemm13_frac=f13 / (t13 / p13 / 1e3) / 1e12 / peak,
+            gemm2_frac=f2 / (t2 / p2 / 1e3) / 1e12 / peak)
     return res
 
 
@@ -1063,7 +1085,8 @@ def profile_case(case: str, dev) -> int:
     """A few forwards: the small launch sequences that ncu captures. decode16 / decode1:
     Mixtral-shaped decode at batch 16 / 1 with every expert resident (decode FFN); ds_decode1 /
     ds_decode64: the same for the DeepSeek-V2-Lite shape at batch 1 / 64; prefill / ds_prefill:
-    T = 4096 tokens, hard mask keeping 4 of 8 / 48 of 64 (tcgen05 GEMMs); fetch16 / ds_fetch64:
+    T = 4096 tokens, hard mask keeping 4 of 8 / 48 of 64 (tcgen05 GEMMs; prefill_pair: the Mixtral
+    case on CTA-pair tiles); fetch16 / ds_fetch64:
     three decode steps (Mixtral-shaped batch 16 / DeepSeek-shaped batch 64) through the cache with
     the device-driven fetch (the FFN launch that fetches its own misses / the fetch kernel)."""
     from paper_2609_34077_gb300 import mcft as M
@@ -1083,6 +1106,9 @@ def profile_case(case: str, dev) -> int:
         print(json.dumps({"case": case, "fetches_per_step": per_step, "experts_per_step": experts,
                           "fetch_bytes_per_step": [n * sh.expert_bytes for n in per_step]}))
         return 0
+    if case == "prefill_pair":  # the prefill case on CTA-pair tiles
+        M.mcft_set_tc_tiles(M.MCFT_TC_TILES_CTA_PAIR)
+        case = "prefill"
     if case in ("prefill", "ds_prefill"):  # Mixtral keeps 4 of 8, DeepSeek 48 of 64
         T, mode = 4096, M.MCFT_ROUTE_HARD_MASK
         kw = dict(mask=I.keep_mask(7, sh.E, 4 if sh is I.MIXTRAL else sh.E * 3 // 4))
@@ -1118,7 +1144,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extra", action="store_true", help="skip the batch-1 and prefill extras")
     ap.add_argument("--case", choices=["decode16", "decode1", "ds_decode1", "ds_decode64", "prefill",
-                                       "ds_prefill", "fetch16", "ds_fetch64", "lora", "mask"],
+                                       "prefill_pair", "ds_prefill", "fetch16", "ds_fetch64", "lora",
+                                       "mask"],
                     help="run only a few resident-expert forwards (for profiler captures)")
     ap.add_argument("--workload", default="layer",
                     choices=["layer", "stack-mixtral", "stack-dsv2", "chain-mixtral", "chain-dsv2",

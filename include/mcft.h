@@ -449,6 +449,23 @@ mcft_status mcft_test_inject(int fail_pinned_allocs, int fail_expert_copies,
                              unsigned long long wait_limit_ns, int withhold_gemm13);
 
 /* ---------------------------------------------------------------------------------------------
+ * Tensor-core tile shape of the expert GEMMs (Section 3.1's F(x) for the large-batch forward; no
+ * counterpart in the paper: a choice of kernel). Process-wide, read when a call lays out its
+ * workspace, so set it before sizing workspaces (mcft_moe_workspace_size) and keep it while they
+ * are in use: a workspace sized under one setting may be too small under the other, which the
+ * forward then rejects with MCFT_ERR_INVALID.
+ *   MCFT_TC_TILES_ONE_CTA   (default) 128 x 256 tiles, one CTA per SM, segments padded to 128
+ *                           rows;
+ *   MCFT_TC_TILES_CTA_PAIR  256 x 256 tiles on pairs of CTAs (cta_group::2 MMAs issued by one CTA
+ *                           of a 2-CTA cluster over both CTAs' shared memory), segments padded to
+ *                           256 rows, for layers without adapters whose routed experts average at
+ *                           least 512 rows (others keep the one-CTA tiles). Outputs equal the
+ *                           one-CTA tiles' bit for bit.
+ * MCFT_ERR_INVALID for another mode. */
+typedef enum { MCFT_TC_TILES_ONE_CTA = 0, MCFT_TC_TILES_CTA_PAIR = 1 } mcft_tc_tiles;
+mcft_status mcft_set_tc_tiles(int mode);
+
+/* ---------------------------------------------------------------------------------------------
  * Kernel timing (no counterpart in the paper; used to measure the path). While enabled, every
  * kernel the library launches is bracketed by two CUDA events on its stream.
  * mcft_profile_read synchronises the recorded events and returns, per kernel of the library, its

@@ -47,6 +47,8 @@ __device__ unsigned g_device_error;  // one per device that loads the library
 // expert copies fail as if the runtime had refused them, the decode FFN's wait limit, and whether
 // the decode FFN withholds its GEMM13 items. All zero (off) unless a test sets them.
 std::atomic<int> g_inject_pinned{0}, g_inject_copy{0}, g_inject_withhold{0};
+// Expert-GEMM tile shape (mcft_set_tc_tiles): MCFT_TC_TILES_ONE_CTA unless set.
+std::atomic<int> g_tc_tiles{MCFT_TC_TILES_ONE_CTA};
 std::atomic<unsigned long long> g_inject_wait_ns{0};
 
 // Consume one injected failure from counter n: true while it is positive.
@@ -146,7 +148,9 @@ WsLayout ws_layout(int d, int E, int K, int w, int S, int dtype, int T, int lran
   L.tc = dtype == MCFT_BF16 && T > 64 && d % 256 == 0 && w % 128 == 0;
   L.decode = !L.tc && dtype == MCFT_BF16;
   L.ks = L.decode ? decode_ksplit(T) : 1;
-  L.pad = L.tc ? 128 : 1;
+  L.pad = !L.tc ? 1
+          : g_tc_tiles.load() == MCFT_TC_TILES_CTA_PAIR && tc_pair_tiles(T, K, E, lrank) ? 256
+                                                                                       : 128;
   const int nseg = E + S;
   L.mcap = T * K + S * T + (L.tc ? nseg * (L.pad - 1) : 0);
   size_t o = 0;
@@ -289,6 +293,13 @@ mcft_status mcft_test_inject(int fail_pinned_allocs, int fail_expert_copies,
   g_inject_copy.store(fail_expert_copies);
   g_inject_wait_ns.store(wait_limit_ns);
   g_inject_withhold.store(withhold_gemm13 ? 1 : 0);
+  return MCFT_OK;
+}
+
+mcft_status mcft_set_tc_tiles(int mode) {
+  if (mode != MCFT_TC_TILES_ONE_CTA && mode != MCFT_TC_TILES_CTA_PAIR)
+    return fail(MCFT_ERR_INVALID, "tile mode %d is neither one-CTA (0) nor CTA-pair (1)", mode);
+  g_tc_tiles.store(mode);
   return MCFT_OK;
 }
 
@@ -486,7 +497,7 @@ mcft_status forward_impl(const mcft_layer_desc* desc, const void* x, int T, cons
     }
   }
   auto ffn = [&](int stages) -> cudaError_t {
-    if (L.tc) return launch_ffn_tc(fa, ws + L.xp, L.mcap, num_sms(), stream, stages);
+    if (L.tc) return launch_ffn_tc(fa, ws + L.xp, L.mcap, L.pad, num_sms(), stream, stages);
     if (L.decode) return launch_ffn_decode(fa, num_sms(), stream, stages);
     return launch_ffn_rowwise(fa, desc->dtype, num_sms(), stream, stages);
   };

@@ -164,6 +164,99 @@ __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// ---- CTA pairs (cta_group::2): one MMA of M = 256 over the shared memory of two CTAs ----
+// Rank 0 of a 2-CTA cluster (the leader) issues the MMAs; each CTA holds 128 rows of A, 128 rows
+// of B (its half of N) and its 128 accumulator rows in its own TMEM, at the same offsets.
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared variable in cluster CTA `rank` (shared::cluster window).
+__device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" :::
+                   "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cl(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded waits with cluster-scope acquire (the pair's barriers also complete from the peer CTA):
+// false if the kernel is aborting or 2 s passed (then MCFT_ERR_TIMEOUT and the abort flag).
+__device__ inline bool mbar_wait_cl(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                    unsigned* err) {
+  if (mbar_try_wait_cl(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait_cl(bar, parity)) return true;
+    if ((i & 31) == 0) {
+      if (*abort) return false;
+      if (globaltimer_ns() - t0 > kTimeoutNs) {
+        *abort = 1;
+        set_error(err, kErrTimeout);
+        return false;
+      }
+    }
+  }
+}
+__device__ inline bool mbar_wait_drain_cl(uint64_t* bar, uint32_t parity, unsigned* err) {
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait_cl(bar, parity)) {
+    if (globaltimer_ns() - t0 > kTimeoutNs) {
+      set_error(err, kErrTimeout);
+      return false;
+    }
+  }
+  return true;
+}
+// TMA tile load into this CTA's shared memory whose completion is counted on an mbarrier of
+// either CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int c0,
+                                                 int c1, uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void tc_mma_pair(uint32_t d_tmem, uint64_t a, uint64_t b,
+                                            uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// Arrives on the mbarrier at this offset in both CTAs of the pair once the leader's MMAs issued
+// so far have completed.
+__device__ __forceinline__ void tc_commit_pair_both(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)), "h"(static_cast<unsigned short>(3))
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
 // Tile -> (m-tile, n-tile): groups of group_m m-tiles; inside a group, n-major then m.
 __device__ __forceinline__ void tile_coords(int tile, int mt_total, int ntn, int G, int& mt,
                                             int& nt) {
@@ -259,6 +352,67 @@ struct LoraOps {
     }
   }
 };
+
+// Epilogue of one expert-GEMM tile for the 32 accumulator rows of an epilogue warp (TMEM lane
+// quarter at taddr, output rows grow0 .. grow0 + 31, n-tile nt): SwiGLU to bf16 h (GEMM13) or fp32
+// (GEMM2), staged through the warp's shared rows stg and stored as whole 128-byte row segments.
+template <int EPI, int NB>
+__device__ __forceinline__ void store_tile(const TcParams& p, uint8_t* stg, uint32_t taddr,
+                                           size_t grow0, int nt, int lane) {
+  if constexpr (EPI == EPI_SWIGLU) {
+    // two rounds of 64 h columns (128 bytes of bf16 per row)
+#pragma unroll 1
+    for (int c0 = 0; c0 < NB / 2; c0 += 64) {
+#pragma unroll
+      for (int c = 0; c < 64; c += 16) {
+        uint32_t g[16], u[16];
+        tmem_ld16(taddr + c0 + c, g);
+        tmem_ld16(taddr + NB / 2 + c0 + c, u);
+        tmem_ld_wait();
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          pk[i] = pack2bf(silu(__uint_as_float(g[2 * i])) * __uint_as_float(u[2 * i]),
+                          silu(__uint_as_float(g[2 * i + 1])) * __uint_as_float(u[2 * i + 1]));
+        uint4* sw = reinterpret_cast<uint4*>(stg + lane * kOutRowBytes + c * 2);
+        sw[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        sw[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      }
+      __syncwarp();
+      const size_t col = size_t(nt) * (NB / 2) + c0 + (lane & 7) * 8;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = 4 * i + (lane >> 3);
+        const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kOutRowBytes + (lane & 7) * 16);
+        *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.out) + (grow0 + r) * p.ldo + col) = v;
+      }
+      __syncwarp();
+    }
+  } else {
+    // eight rounds of 32 fp32 columns (128 bytes per row)
+#pragma unroll 1
+    for (int c0 = 0; c0 < NB; c0 += 32) {
+#pragma unroll
+      for (int c = 0; c < 32; c += 16) {
+        uint32_t v[16];
+        tmem_ld16(taddr + c0 + c, v);
+        tmem_ld_wait();
+        uint4* sw = reinterpret_cast<uint4*>(stg + lane * kOutRowBytes + c * 4);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) sw[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      }
+      __syncwarp();
+      const size_t col = size_t(nt) * NB + c0 + (lane & 7) * 4;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = 4 * i + (lane >> 3);
+        const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kOutRowBytes + (lane & 7) * 16);
+        *reinterpret_cast<uint4*>(reinterpret_cast<float*>(p.out) + (grow0 + r) * p.ldo + col) = v;
+      }
+      __syncwarp();
+    }
+  }
+}
 
 template <int EPI, int LR, int NB>
 __global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
@@ -459,36 +613,7 @@ __global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __gri
       // this warp's staging rows; row r of the warp's quarter goes to global row grow0 + r
       uint8_t* stg = reinterpret_cast<uint8_t*>(ctl) + kCtlBytes + q * kOutWarpBytes;
       const size_t grow0 = size_t(mt) * BM + q * 32;
-      if constexpr (EPI == EPI_SWIGLU) {
-        // two rounds of 64 h columns (128 bytes of bf16 per row)
-#pragma unroll 1
-        for (int c0 = 0; c0 < NB / 2; c0 += 64) {
-#pragma unroll
-          for (int c = 0; c < 64; c += 16) {
-            uint32_t g[16], u[16];
-            tmem_ld16(taddr + c0 + c, g);
-            tmem_ld16(taddr + NB / 2 + c0 + c, u);
-            tmem_ld_wait();
-            uint32_t pk[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-              pk[i] = pack2bf(silu(__uint_as_float(g[2 * i])) * __uint_as_float(u[2 * i]),
-                              silu(__uint_as_float(g[2 * i + 1])) * __uint_as_float(u[2 * i + 1]));
-            uint4* sw = reinterpret_cast<uint4*>(stg + lane * kOutRowBytes + c * 2);
-            sw[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            sw[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          }
-          __syncwarp();
-          const size_t col = size_t(nt) * (NB / 2) + c0 + (lane & 7) * 8;
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int r = 4 * i + (lane >> 3);
-            const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kOutRowBytes + (lane & 7) * 16);
-            *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.out) + (grow0 + r) * p.ldo + col) = v;
-          }
-          __syncwarp();
-        }
-      } else if constexpr (EPI == EPI_DOWN) {  // U = s (A v) in bf16, the first ldo columns
+      if constexpr (EPI == EPI_DOWN) {  // U = s (A v) in bf16, the first ldo columns
         uint16_t* out = reinterpret_cast<uint16_t*>(p.out) + grow * p.ldo;
 #pragma unroll
         for (int c = 0; c < NB; c += 16) {
@@ -505,28 +630,7 @@ __global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __gri
           if (c + 16 <= p.ldo) dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
       } else {
-        // eight rounds of 32 fp32 columns (128 bytes per row)
-#pragma unroll 1
-        for (int c0 = 0; c0 < NB; c0 += 32) {
-#pragma unroll
-          for (int c = 0; c < 32; c += 16) {
-            uint32_t v[16];
-            tmem_ld16(taddr + c0 + c, v);
-            tmem_ld_wait();
-            uint4* sw = reinterpret_cast<uint4*>(stg + lane * kOutRowBytes + c * 4);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) sw[i] = make_uint4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-          }
-          __syncwarp();
-          const size_t col = size_t(nt) * NB + c0 + (lane & 7) * 4;
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int r = 4 * i + (lane >> 3);
-            const uint4 v = *reinterpret_cast<const uint4*>(stg + r * kOutRowBytes + (lane & 7) * 16);
-            *reinterpret_cast<uint4*>(reinterpret_cast<float*>(p.out) + (grow0 + r) * p.ldo + col) = v;
-          }
-          __syncwarp();
-        }
+        store_tile<EPI, NB>(p, stg, taddr, grow0, nt, lane);
       }
       tc_fence_before();
       __syncwarp();
@@ -541,6 +645,184 @@ __global__ void __launch_bounds__(threads_for(LR), 1) gemm_tc_kernel(const __gri
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                  "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// The expert GEMMs on CTA pairs: tiles of 256 rows x 256 columns, one MMA of M = 256 per K step
+// issued by the pair's leader over both CTAs' shared memory. Each CTA loads its 128 activation
+// rows and its half of the tile's 256 weight rows (GEMM13: rank 0 the W1 rows, rank 1 the W3
+// rows, i.e. the gate and up halves of N; GEMM2: 128 consecutive W2 rows each), so every weight
+// element is read from shared memory once for the rows of both CTAs: a third less shared-memory
+// traffic per MMA than the one-CTA tiles, and half the weight tiles fetched from L2 per tile row.
+// Roles as in gemm_tc_kernel, 6 stages of 32 KB:
+//   warp 0 (both CTAs) - TMA producer; the loads of both CTAs complete on the leader's full[s],
+//             on which the leader expects the pair's bytes; each CTA waits on its own empty[s];
+//   warp 1 - allocates the pair's TMEM (both CTAs); in the leader, issues the MMAs, whose commits
+//             arrive on empty[s] and tfull[b] of both CTAs;
+//   warps 2-5 (both CTAs) - epilogue of the CTA's 128 rows of the tile; they release the
+//             accumulator on the leader's tempty[b] (eight arrivals: four warps per CTA).
+// Segments are padded to 256 rows. Every wait is bounded. The leader drains its last stages'
+// copies (both CTAs' bytes), the peer waits (bounded) until its last stages were consumed, and
+// both CTAs leave through one cluster barrier after the leader's MMAs have completed, so neither
+// exits while the other may still read its shared memory or arrive on its barriers.
+constexpr int kPairRows = 2 * BM;
+constexpr int kPairStages = 6;
+constexpr int kPairStageBytes = A_BYTES + (BN / 2) * BK * 2;  // 128 activation + 128 weight rows
+constexpr int kPairTmemCols = 2 * BN;                          // two 128 x 256 accumulators
+constexpr uint32_t kPairIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BN >> 3) << 17) |
+                                (uint32_t(kPairRows >> 4) << 24);
+constexpr int kPairSmem = kPairStages * kPairStageBytes + 1024 + kCtlBytes + 4 * kOutWarpBytes;
+static_assert(kPairSmem <= 227 * 1024, "shared memory");
+static_assert(kPairStages <= kMaxStages, "stage barriers");
+
+template <int EPI>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    gemm_tc_pair_kernel(const __grid_constant__ TcParams p) {
+  pdl_wait();
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;  // the same offsets in both CTAs
+  SmemCtl* ctl =
+      reinterpret_cast<SmemCtl*>(smem_raw + (base - raw) + kPairStages * kPairStageBytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+
+  if (threadIdx.x == 0) {
+    // both CTAs find the same offsets and the same abort decision
+    int abort = p.hdr->abort;
+    const int nseg = p.nseg;
+    ctl->nseg = nseg;
+    for (int s = 0; s <= nseg; ++s) ctl->off[s] = p.off[s];
+    for (int s = 0; s < nseg; ++s) {
+      if (ctl->off[s + 1] > ctl->off[s] && !((p.wmask[s >> 5] >> (s & 31)) & 1u)) {
+        set_error(p.err, kErrInvalid);  // a selected expert without weights
+        const_cast<WsHeader*>(p.hdr)->abort = 1;
+        abort = 1;
+      }
+    }
+    ctl->abort = abort;
+    ctl->mt_total = abort ? 0 : ctl->off[nseg] / kPairRows;
+    for (int s = 0; s < kPairStages; ++s) {
+      mbar_init(&ctl->full[s], 1);
+      mbar_init(&ctl->empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&ctl->tfull[b], 1);
+      mbar_init(&ctl->tempty[b], 8);
+    }
+    mbar_init(&ctl->drain, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&ctl->tmem_base)),
+                 "r"(kPairTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  cluster_sync();  // barriers initialised and TMEM allocated in both CTAs
+  tc_fence_after();
+
+  const uint32_t tmem = ctl->tmem_base;
+  const int mt_total = ctl->mt_total;  // 256-row tiles
+  const int ntn = p.ntiles_n;
+  const int tiles = mt_total * ntn;
+  const int cid = int(blockIdx.x >> 1), ncl = int(gridDim.x >> 1);  // pair, pairs
+  volatile int* abort = &ctl->abort;
+
+  if (warp == 0) {
+    if (lane == 0 && cid < tiles) {
+      uint32_t it = 0;
+      for (int tile = cid; tile < tiles && !*abort; tile += ncl) {
+        int mt, nt;
+        tile_coords(tile, mt_total, ntn, p.group_m, mt, nt);
+        const CUtensorMap* mb = &p.tma_b[seg_of_row(ctl, mt * kPairRows)];
+        const int row0 = mt * kPairRows + int(rank) * BM;
+        const int yb = EPI == EPI_SWIGLU ? int(rank) * p.b_half + nt * (BN / 2)
+                                         : nt * BN + int(rank) * (BN / 2);
+        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+          const int s = int(it % kPairStages);
+          if (!mbar_wait_cl(&ctl->empty[s], ((it / kPairStages) & 1u) ^ 1u, abort, p.err)) break;
+          const uint32_t sa = base + uint32_t(s) * kPairStageBytes, sb = sa + A_BYTES;
+          const uint32_t fb = peer_addr(&ctl->full[s], 0);
+          if (leader) mbar_expect_tx(&ctl->full[s], 2 * kPairStageBytes);
+          tma_load_2d_pair(sa, &p.tma_a, kb * BK, row0, fb);
+          tma_load_2d_pair(sb, mb, kb * BK, yb, fb);
+        }
+      }
+      // Stages still in flight: the leader waits for their bytes (both CTAs'), the peer until
+      // the leader's MMAs consumed them; after the first wait that runs out (an aborted pair,
+      // 2 s: nothing is in flight any more) the rest are skipped.
+      const uint32_t n_tail = it < kPairStages ? it : kPairStages;
+      for (uint32_t j = it - n_tail; j < it; ++j) {
+        uint64_t* bar = leader ? &ctl->full[j % kPairStages] : &ctl->empty[j % kPairStages];
+        if (!mbar_wait_drain_cl(bar, (j / kPairStages) & 1u, p.err)) break;
+      }
+    }
+  } else if (warp == 1) {
+    if (leader && lane == 0 && cid < tiles) {
+      uint32_t it = 0, lt = 0;
+      for (int tile = cid; tile < tiles && !*abort; tile += ncl) {
+        const uint32_t b = lt & 1u;
+        if (!mbar_wait_cl(&ctl->tempty[b], ((lt >> 1) & 1u) ^ 1u, abort, p.err)) break;
+        tc_fence_after();
+        const uint32_t dt = tmem + b * BN;
+        bool ok = true;
+        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+          const int s = int(it % kPairStages);
+          if (!mbar_wait_cl(&ctl->full[s], (it / kPairStages) & 1u, abort, p.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = base + uint32_t(s) * kPairStageBytes, sb = sa + A_BYTES;
+          const uint64_t da = sw128_desc(sa), db = sw128_desc(sb);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma_pair(dt, da + uint64_t(2 * k), db + uint64_t(2 * k), kPairIdesc,
+                        (kb | k) != 0 ? 1u : 0u);
+          tc_commit_pair_both(&ctl->empty[s]);
+        }
+        if (!ok) break;
+        tc_commit_pair_both(&ctl->tfull[b]);
+        ++lt;
+      }
+      tc_commit_pair(&ctl->drain);  // arrives once every MMA issued above has completed
+      mbar_wait_drain_cl(&ctl->drain, 0, p.err);
+    }
+  } else if (warp >= 2 && warp < 6) {
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    uint8_t* stg = reinterpret_cast<uint8_t*>(ctl) + kCtlBytes + q * kOutWarpBytes;
+    uint32_t lt = 0;
+    for (int tile = cid; tile < tiles; tile += ncl) {
+      int mt, nt;
+      tile_coords(tile, mt_total, ntn, p.group_m, mt, nt);
+      const uint32_t b = lt & 1u;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait_cl(&ctl->tfull[b], (lt >> 1) & 1u, abort, p.err) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem + b * BN + (uint32_t(q * 32) << 16);
+      const size_t grow0 = size_t(mt) * kPairRows + rank * BM + q * 32;
+      store_tile<EPI, BN>(p, stg, taddr, grow0, nt, lane);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(peer_addr(&ctl->tempty[b], 0));
+      ++lt;
+    }
+  }
+
+  tc_fence_before();
+  cluster_sync();  // the leader's MMAs drained, every copy landed, both epilogues done
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kPairTmemCols)
                  : "memory");
   }
 }
@@ -607,6 +889,9 @@ bool encode_adapter_a2(CUtensorMap* m, const void* a2, uint64_t w, uint32_t r) {
 }
 
 constexpr size_t kSmallSegGroupMB = 2;  // group budget when routed experts have few m-tiles
+// With CTA-pair tiles selected, layers whose routed experts average at least this many rows run
+// on pairs (segments padded to 256 rows); with fewer the extra padding would dominate.
+constexpr int kPairMinRows = 512;
 
 int group_for(size_t a_tile_bytes, size_t budget_mb) {
   const size_t budget = budget_mb << 20;  // activation rows kept hot in L2 per group
@@ -626,6 +911,33 @@ cudaError_t launch_one(const TcParams& p, int grid, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+// One pair per two SMs that can hold one at a time (one CTA per SM): a persistent grid of pairs
+// that all run at once, so no pair's tiles wait for another pair to exit.
+template <int EPI>
+cudaError_t launch_pair(const TcParams& p, int num_sms, cudaStream_t s) {
+  static cudaError_t attr = cudaFuncSetAttribute(
+      gemm_tc_pair_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+  if (attr != cudaSuccess) return attr;
+  static const int pairs = [num_sms] {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(num_sms & ~1));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kPairSmem;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_pair_kernel<EPI>, &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    return n;
+  }();
+  if (pairs < 1) return cudaErrorInvalidConfiguration;
+  const int kid = EPI == EPI_SWIGLU ? kProfGemm13Pair : kProfGemm2Pair;
+  prof_begin(kid, s);
+  gemm_tc_pair_kernel<EPI><<<2 * pairs, kThreads, kPairSmem, s>>>(p);
+  prof_end(kid, s);
+  return cudaGetLastError();
+}
+
 template <int EPI>
 cudaError_t launch_rank(const TcParams& p, int rank, int num_sms, cudaStream_t s) {
   switch (rank) {
@@ -638,8 +950,14 @@ cudaError_t launch_rank(const TcParams& p, int rank, int num_sms, cudaStream_t s
 
 }  // namespace
 
-cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
-                          int stages) {
+bool tc_pair_tiles(int T, int K, int E, int lrank) {
+  return lrank == 0 && size_t(T) * K >= size_t(kPairMinRows) * E;
+}
+
+cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int pad, int num_sms,
+                          cudaStream_t s, int stages) {
+  const bool pair = pad == kPairRows;
+  if (pair ? a.lrank != 0 : pad != BM) return cudaErrorInvalidValue;
   TcParams p13, p2;
   memset(&p13, 0, sizeof(p13));
   memset(&p2, 0, sizeof(p2));
@@ -672,16 +990,16 @@ cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sm
   // GEMM13 is best at 24 MB and GEMM2 at 12 MB; with fewer than four on average (DeepSeek-V2-Lite:
   // 64 experts) small groups of about one expert's rows win (GEMM13 0.55 -> 0.60 of peak)
   // routed rows T * K: the permuted rows less the shared experts' and the segment padding
-  const size_t routed = size_t(mcap) - size_t(a.T) * (a.nseg - a.E) - size_t(a.nseg) * (BM - 1);
+  const size_t routed = size_t(mcap) - size_t(a.T) * (a.nseg - a.E) - size_t(a.nseg) * (pad - 1);
   const bool small_segs = routed < size_t(4) * BM * a.E;
   const size_t mb13 = small_segs ? kSmallSegGroupMB : 24, mb2 = small_segs ? kSmallSegGroupMB : 12;
-  p13.group_m = group_for(size_t(BM) * d * 2, mb13);
+  p13.group_m = group_for(size_t(pad) * d * 2, mb13);
   p2.out = a.o;
   p2.kblocks = int(w / BK);
   p2.ntiles_n = int(d / BN);
   p2.ldo = int(d);
   p2.b_half = 0;
-  p2.group_m = group_for(size_t(BM) * w * 2, mb2);
+  p2.group_m = group_for(size_t(pad) * w * 2, mb2);
   if (a.lrank > 0) {
     const LoraOffsets lo = lora_offsets(a.d, a.w, a.lrank);
     for (int sgi = 0; sgi < a.nseg; ++sgi) {
@@ -696,9 +1014,11 @@ cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sm
     p2.lb0 = lo.b2;
   }
   cudaError_t e = cudaSuccess;
-  if (stages & 1) e = launch_rank<EPI_SWIGLU>(p13, a.lrank, num_sms, s);
+  if (stages & 1)
+    e = pair ? launch_pair<EPI_SWIGLU>(p13, num_sms, s)
+             : launch_rank<EPI_SWIGLU>(p13, a.lrank, num_sms, s);
   if (e != cudaSuccess || !(stages & 2)) return e;
-  return launch_rank<EPI_F32>(p2, a.lrank, num_sms, s);
+  return pair ? launch_pair<EPI_F32>(p2, num_sms, s) : launch_rank<EPI_F32>(p2, a.lrank, num_sms, s);
 }
 
 cudaError_t launch_lora_down_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms,

@@ -78,7 +78,8 @@ struct WsLayout {
   int lrank;      // LoRA rank (0: no adapters)
   bool tc;        // tensor-core path (bf16, large T)
   bool decode;    // bf16 decode path (T <= 64)
-  int pad;        // rows per segment are padded to a multiple of this (128 on the TC path)
+  int pad;        // rows per segment are padded to a multiple of this (TC path: 128, or 256
+                  // for CTA-pair tiles)
   int mcap;       // capacity in permuted rows
   int ks;         // partial planes of o (contraction split of the decode GEMM2)
   size_t hdr, cnt, off, pos, perm, done, pscr, xp, h, o, u13, u2, total;
@@ -254,8 +255,11 @@ cudaError_t launch_ffn_rowwise(const FfnArgs& a, int dtype, int num_sms, cudaStr
 cudaError_t launch_ffn_decode(const FfnArgs& a, int num_sms, cudaStream_t s, int stages = 3,
                               int reserved = 0);  // bf16, T <= 64
 int decode_ksplit(int T);  // contraction split of the decode GEMM2 for T tokens
-cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int num_sms, cudaStream_t s,
-                          int stages = 3);
+// pad: rows per segment of the permutation, 128 (one-CTA tiles) or 256 (CTA-pair tiles, which
+// tc_pair_tiles chooses for layers without adapters whose routed experts average >= 512 rows).
+cudaError_t launch_ffn_tc(const FfnArgs& a, const void* xp, int mcap, int pad, int num_sms,
+                          cudaStream_t s, int stages = 3);
+bool tc_pair_tiles(int T, int K, int E, int lrank);
 // Down projections of the adapters for the tcgen05 path, on the tensor cores, bf16 out scaled by
 // s: stage 1: u13[q] = s [A1 xp[q] | A3 xp[q]] (N = 2r); stage 2: u2[q] = s A2 h[q] (N = 16),
 // for the rows of every segment with an adapter. The expert GEMMs add the up projections.
@@ -431,7 +435,7 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
 enum { kProfRoute, kProfCache, kProfPermute, kProfGather, kProfFfn13, kProfFfn2, kProfGemm13,
        kProfGemm2, kProfCombine, kProfDec13, kProfDec2, kProfFetch, kProfLora, kProfNorm,
        kProfPrefetch, kProfPfFetch, kProfPrologue, kProfDecFused, kProfHostCopy, kProfDecFetch,
-       kProfCount };
+       kProfGemm13Pair, kProfGemm2Pair, kProfCount };
 void prof_begin(int kid, cudaStream_t s);
 void prof_end(int kid, cudaStream_t s);
 

@@ -16,7 +16,7 @@ const char* const kNames[kProfCount] = {
     "route",     "cache_step", "permute", "gather",       "ffn13_rowwise", "ffn2_rowwise",
     "gemm13_tc", "gemm2_tc",   "combine", "ffn13_decode", "ffn2_decode", "fetch", "lora_down",
     "rmsnorm",   "prefetch",   "fetch_prefetch", "prologue", "ffn_decode", "host_copy",
-    "ffn_decode_fetch"};
+    "ffn_decode_fetch", "gemm13_tc_pair", "gemm2_tc_pair"};
 
 struct Pending {
   int kid;

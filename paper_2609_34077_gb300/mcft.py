@@ -56,6 +56,7 @@ SIGNATURES = {
     "mcft_device_error": (_i, [_vp]),
     "mcft_test_inject": (_i, [_i, _i, C.c_ulonglong, _i]),
     "mcft_profile_enable": (_i, [_i]),
+    "mcft_set_tc_tiles": (_i, [_i]),
     "mcft_profile_reset": (_i, []),
     "mcft_profile_read": (_i, [_i, _vp, _vp, _vp, C.POINTER(_i)]),
     "mcft_last_error": (C.c_char_p, []),
@@ -432,6 +433,15 @@ def mcft_test_inject(fail_pinned_allocs=0, fail_expert_copies=0, wait_limit_ns=0
     """Failure injection for tests (all zero: normal operation)."""
     _check(lib().mcft_test_inject(int(fail_pinned_allocs), int(fail_expert_copies),
                                   int(wait_limit_ns), 1 if withhold_gemm13 else 0))
+
+
+MCFT_TC_TILES_ONE_CTA, MCFT_TC_TILES_CTA_PAIR = 0, 1
+
+
+def mcft_set_tc_tiles(mode: int):
+    """Expert-GEMM tile shape for the tensor-core forward (process-wide; set before sizing
+    workspaces): MCFT_TC_TILES_ONE_CTA (default) or MCFT_TC_TILES_CTA_PAIR."""
+    _check(lib().mcft_set_tc_tiles(int(mode)))
 
 
 def mcft_profile_enable(on: bool = True):

@@ -92,3 +92,39 @@ def test_test_inject_validation_without_gpu(libpath):
     assert L.mcft_test_inject(-1, 0, 0, 0) == mcft.MCFT_ERR_INVALID
     assert L.mcft_test_inject(0, -2, 0, 0) == mcft.MCFT_ERR_INVALID
     assert L.mcft_test_inject(0, 0, 0, 0) == mcft.MCFT_OK
+
+
+def test_tc_tile_mode_without_gpu(libpath):
+    """mcft_set_tc_tiles: only the two modes; under CTA-pair tiles a layer whose routed experts
+    average >= 512 rows pads its segments to 256 rows (a larger workspace), a smaller one keeps
+    the one-CTA layout, and a layer with adapters always does."""
+    import ctypes as C
+    from paper_2609_34077_gb300 import inputs as I
+    from paper_2609_34077_gb300 import mcft
+
+    L = mcft.lib()
+    assert L.mcft_set_tc_tiles(2) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_set_tc_tiles(-1) == mcft.MCFT_ERR_INVALID
+    desc = mcft.desc_of(I.MIXTRAL)
+
+    def size(T):
+        n = C.c_size_t(0)
+        assert L.mcft_moe_workspace_size(C.byref(desc), T, C.byref(n)) == mcft.MCFT_OK
+        return n.value
+
+    def size_lora(T):
+        n = C.c_size_t(0)
+        assert L.mcft_moe_workspace_size_lora(C.byref(desc), 8, T, C.byref(n)) == mcft.MCFT_OK
+        return n.value
+
+    try:
+        one = {T: size(T) for T in (1024, 2048, 4096)}
+        one_lora = size_lora(4096)
+        assert L.mcft_set_tc_tiles(mcft.MCFT_TC_TILES_CTA_PAIR) == mcft.MCFT_OK
+        pair = {T: size(T) for T in (1024, 2048, 4096)}
+        assert size_lora(4096) == one_lora
+    finally:
+        assert L.mcft_set_tc_tiles(mcft.MCFT_TC_TILES_ONE_CTA) == mcft.MCFT_OK
+    assert pair[1024] == one[1024]  # 2048 assignments over 8 experts: 256 rows each
+    assert pair[2048] > one[2048] and pair[4096] > one[4096]
+    assert size(4096) == one[4096]
