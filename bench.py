@@ -385,6 +385,20 @@ def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks
     return elapsed, tuple(int(b - a) for a, b in zip(c0, c1)), prof, io_bytes
 
 
+def step_floor(d, link_gbs, hbm_gbs):
+    """Lower bounds of a device-driven decode step from its own byte counts (per-step means): the
+    host link moving the step's misses (the FFN of the hits and of streamed misses can run under
+    it), and that plus the missed experts' FFN read at HBM speed after their bytes land; each no
+    less than the step's FFN bytes at HBM speed. Fractions are bound / measured step time."""
+    ms = d["ms_per_step"]
+    fb, ffn = d["fetch_bytes_per_step"], d["ffn_dram_bytes_per_step"]
+    hbm_ms = ffn / (hbm_gbs * 1e9) * 1e3
+    link_ms = max(fb / (link_gbs * 1e9) * 1e3, hbm_ms)
+    both_ms = max(fb / (link_gbs * 1e9) * 1e3 + fb / (hbm_gbs * 1e9) * 1e3, hbm_ms)
+    return dict(link_ms=link_ms, link_plus_miss_ffn_ms=both_ms, frac_of_link=link_ms / ms,
+                frac_of_link_plus_miss_ffn=both_ms / ms, link_gbs=link_gbs, hbm_gbs=hbm_gbs)
+
+
 def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world=1, e2e=False):
     """Decode `steps` timed steps of one layer after `warmup` untimed ones, in four measured passes
     over the same steps from the same cache state (decode_pass), after one untimed pass:
@@ -1286,7 +1300,8 @@ def main():
                    link_roofline_ms_per_step=d["fetch_bytes_per_step"] / (link["best_gbs"] * 1e9) * 1e3,
                    link_frac=(d["fetch_bytes_per_step"] / (ms / 1e3)) / (link["best_gbs"] * 1e9),
                    kernel_ms_per_step=d["kernel_ms_per_step"],
-                   fetch_launch_ms_per_step=d["fetch_launch_ms_per_step"]),
+                   fetch_launch_ms_per_step=d["fetch_launch_ms_per_step"],
+                   step_floor=step_floor(d, link["best_gbs"], peaks["hbm"])),
         host_fetch_path=d["host_fetch_path"],
     )
     runs = {"mixtral_b%d" % batch: (shape, batch, seed, idx_main, args.steps, d)}
@@ -1294,12 +1309,14 @@ def main():
         nb1 = min(args.steps, 256)
         b1, idx_b1, _ = run_decode(shape, 1, nb1, args.warmup, seed + 1, dev, peaks)
         b1.pop("kernels", None)
+        b1["step_floor"] = step_floor(b1, link["best_gbs"], peaks["hbm"])
         line["batch1"] = b1
         runs["mixtral_b1"] = (shape, 1, seed + 1, idx_b1, nb1, b1)
         for bsz in (1, 8, 64):
             nds = min(args.steps, 128)
             ds, idx_ds, _ = run_decode(I.DSV2_LITE, bsz, nds, args.warmup, seed + 3, dev, peaks)
             ds.pop("kernels", None)
+            ds["step_floor"] = step_floor(ds, link["best_gbs"], peaks["hbm"])
             line[f"dsv2_b{bsz}"] = ds
             runs[f"dsv2_b{bsz}"] = (I.DSV2_LITE, bsz, seed + 3, idx_ds, nds, ds)
         line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)

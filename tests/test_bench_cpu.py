@@ -115,3 +115,19 @@ def test_oracle_fetch_check_counts_and_flags():
     assert chk2["ids_differ_outside_band"] + chk2["ids_differ_in_band"] == 1
     assert not bench.fetch_verdict(chk2, h, f)["routing_exact_outside_band"] or \
         chk2["ids_differ_in_band"] == 1
+
+
+def test_step_floor_bounds():
+    """The step floors: link time of the misses (or the FFN bytes at HBM speed, whichever is
+    larger), and that plus the misses' FFN; fractions of the measured step."""
+    import bench
+
+    d = dict(ms_per_step=0.150, fetch_bytes_per_step=24.0e6, ffn_dram_bytes_per_step=138.0e6)
+    f = bench.step_floor(d, 200.0, 6000.0)
+    assert abs(f["link_ms"] - 0.120) < 1e-9
+    assert abs(f["link_plus_miss_ffn_ms"] - 0.124) < 1e-9
+    assert abs(f["frac_of_link"] - 0.8) < 1e-9
+    # no misses: the FFN at HBM speed is the bound
+    d0 = dict(ms_per_step=0.030, fetch_bytes_per_step=0.0, ffn_dram_bytes_per_step=138.0e6)
+    f0 = bench.step_floor(d0, 200.0, 6000.0)
+    assert abs(f0["link_ms"] - 0.023) < 1e-9 and f0["link_ms"] == f0["link_plus_miss_ffn_ms"]
