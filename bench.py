@@ -334,7 +334,8 @@ def fetching_kernel(kernels):
     return None
 
 
-def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks=None, world=1):
+def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks=None, world=1,
+                record=None):
     """One measured pass over the decode steps [first, first + steps) of layer L.
 
     The pass starts from an empty cache and runs the untimed steps 0 .. first - 1 first, so every
@@ -343,7 +344,9 @@ def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks
     own, so the instrumentation never touches the headline time). With `e2e` every step also copies
     its hidden states from pinned host memory to the device and its output back to pinned host
     memory, on the compute stream inside the timed region. Returns (elapsed seconds, (hits,
-    fetches, bypass) over the timed steps, per-kernel profile or None, bytes copied per step)."""
+    fetches, bypass) over the timed steps, per-kernel profile or None, bytes copied per step).
+    With `record` (a list; untimed passes only) each step is synchronised and its fetch count
+    appended."""
     M = L.M
     L.new_cache()
     for s in range(first):
@@ -366,6 +369,11 @@ def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks
     else:
         def fn(s):
             L.step(s, path=path)
+    if record is not None:
+        def fn(s, step=fn):
+            before = M.mcft_cache_stats(L.cache, 0)[1]
+            step(s)
+            record.append(int(M.mcft_cache_stats(L.cache, 0)[1] - before))
     if profile:
         M.mcft_profile_reset()
         M.mcft_profile_enable(True)
@@ -386,17 +394,28 @@ def decode_pass(L, first, steps, path="device", profile=False, e2e=False, clocks
 
 
 def step_floor(d, link_gbs, hbm_gbs):
-    """Lower bounds of a device-driven decode step from its own byte counts (per-step means): the
-    host link moving the step's misses (the FFN of the hits and of streamed misses can run under
-    it), and that plus the missed experts' FFN read at HBM speed after their bytes land; each no
-    less than the step's FFN bytes at HBM speed. Fractions are bound / measured step time."""
+    """Lower bounds of a device-driven decode step from its own byte counts: the host link moving
+    the step's misses (the FFN of the hits and of streamed misses can run under it), and that plus
+    the missed experts' FFN read at HBM speed after their bytes land; each no less than the step's
+    FFN bytes at HBM speed. From per-step means (link_ms, ...), and, with `per_step` counts in d,
+    as the mean over steps of each step's own bound (step_ms, ...: tighter, since a step without
+    a miss still streams its FFN). Fractions are bound / measured step time."""
     ms = d["ms_per_step"]
     fb, ffn = d["fetch_bytes_per_step"], d["ffn_dram_bytes_per_step"]
-    hbm_ms = ffn / (hbm_gbs * 1e9) * 1e3
-    link_ms = max(fb / (link_gbs * 1e9) * 1e3, hbm_ms)
-    both_ms = max(fb / (link_gbs * 1e9) * 1e3 + fb / (hbm_gbs * 1e9) * 1e3, hbm_ms)
-    return dict(link_ms=link_ms, link_plus_miss_ffn_ms=both_ms, frac_of_link=link_ms / ms,
-                frac_of_link_plus_miss_ffn=both_ms / ms, link_gbs=link_gbs, hbm_gbs=hbm_gbs)
+    lk, hb = link_gbs * 1e6, hbm_gbs * 1e6  # bytes per ms
+    link_ms = max(fb / lk, ffn / hb)
+    both_ms = max(fb / lk + fb / hb, ffn / hb)
+    out = dict(link_ms=link_ms, link_plus_miss_ffn_ms=both_ms, frac_of_link=link_ms / ms,
+               frac_of_link_plus_miss_ffn=both_ms / ms, link_gbs=link_gbs, hbm_gbs=hbm_gbs)
+    ps = d.get("per_step")
+    if ps and ps["fetches"] and len(ps["fetches"]) == len(ps["ffn_bytes"]):
+        eb = ps["expert_bytes"]
+        one = [max(f * eb / lk, b / hb) for f, b in zip(ps["fetches"], ps["ffn_bytes"])]
+        two = [max(f * eb / lk + f * eb / hb, b / hb) for f, b in zip(ps["fetches"], ps["ffn_bytes"])]
+        out.update(step_ms=sum(one) / len(one), step_plus_miss_ffn_ms=sum(two) / len(two),
+                   frac_of_step=sum(one) / len(one) / ms,
+                   frac_of_step_plus_miss_ffn=sum(two) / len(two) / ms)
+    return out
 
 
 def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world=1, e2e=False):
@@ -410,8 +429,10 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world
     Returns (result dict, GPU routing ids [512, batch, K] on the host, elapsed seconds of pass 1)."""
     L = DecodeLayer(shape, batch, seed, dev)
     # an untimed pass over the same steps first: the first reads of the pinned host pool map its
-    # pages for the device, which later passes (and any long-running decode) no longer pay
-    decode_pass(L, warmup, steps)
+    # pages for the device, which later passes (and any long-running decode) no longer pay; it
+    # records each step's fetches (every pass makes the same decisions)
+    per_step_fetches = []
+    decode_pass(L, warmup, steps, record=per_step_fetches)
     elapsed, cnt, _, _ = decode_pass(L, warmup, steps, clocks=clocks, world=world)
     passes = {"timed": cnt}
     e2e_res = None
@@ -433,6 +454,8 @@ def run_decode(shape, batch, steps, warmup, seed, dev, peaks, clocks=None, world
     fetch_bytes = fetches * shape.expert_bytes / steps
     b13, b2 = decode_alg_bytes(U, steps, batch, shape)
     out = dict(
+        per_step=dict(fetches=per_step_fetches, experts=U, expert_bytes=shape.expert_bytes,
+                      ffn_bytes=[sum(decode_alg_bytes([u], 1, batch, shape)) for u in U]),
         tokens_per_s=batch * steps / elapsed, ms_per_step=elapsed * 1e3 / steps, steps=steps,
         warmup=warmup, fetch_path="device", hits=hits, fetches=fetches, bypass=byp,
         fetches_per_step=fetches / steps, fetches_per_token=fetches / (steps * batch),
@@ -1310,6 +1333,7 @@ def main():
         b1, idx_b1, _ = run_decode(shape, 1, nb1, args.warmup, seed + 1, dev, peaks)
         b1.pop("kernels", None)
         b1["step_floor"] = step_floor(b1, link["best_gbs"], peaks["hbm"])
+        b1.pop("per_step", None)
         line["batch1"] = b1
         runs["mixtral_b1"] = (shape, 1, seed + 1, idx_b1, nb1, b1)
         for bsz in (1, 8, 64):
@@ -1317,6 +1341,7 @@ def main():
             ds, idx_ds, _ = run_decode(I.DSV2_LITE, bsz, nds, args.warmup, seed + 3, dev, peaks)
             ds.pop("kernels", None)
             ds["step_floor"] = step_floor(ds, link["best_gbs"], peaks["hbm"])
+            ds.pop("per_step", None)
             line[f"dsv2_b{bsz}"] = ds
             runs[f"dsv2_b{bsz}"] = (I.DSV2_LITE, bsz, seed + 3, idx_ds, nds, ds)
         line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)

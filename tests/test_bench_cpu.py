@@ -131,3 +131,20 @@ def test_step_floor_bounds():
     d0 = dict(ms_per_step=0.030, fetch_bytes_per_step=0.0, ffn_dram_bytes_per_step=138.0e6)
     f0 = bench.step_floor(d0, 200.0, 6000.0)
     assert abs(f0["link_ms"] - 0.023) < 1e-9 and f0["link_ms"] == f0["link_plus_miss_ffn_ms"]
+
+
+def test_step_floor_per_step_is_tighter():
+    """With per-step fetch counts the floor is the mean of each step's own bound: one step that
+    fetches and three that only stream their FFN bound the steps more tightly than the averages."""
+    import bench
+
+    eb, ffn = 352321536, 704.6e6
+    d = dict(ms_per_step=0.5, fetch_bytes_per_step=eb / 4, ffn_dram_bytes_per_step=ffn,
+             per_step=dict(fetches=[1, 0, 0, 0], experts=[2] * 4, expert_bytes=eb,
+                           ffn_bytes=[ffn] * 4))
+    f = bench.step_floor(d, 200.0, 6000.0)
+    link = eb / 200e6  # ms for one expert over the link
+    hbm = ffn / 6000e6
+    assert abs(f["step_ms"] - (link + 3 * hbm) / 4) < 1e-12
+    assert abs(f["step_plus_miss_ffn_ms"] - (link + eb / 6000e6 + 3 * hbm) / 4) < 1e-12
+    assert f["step_ms"] > f["link_ms"]
