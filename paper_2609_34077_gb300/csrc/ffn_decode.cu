@@ -58,7 +58,7 @@ struct DecItems {
 // on which segments a launch computes, so an output is bit-identical whichever phase of a cached
 // forward computes it. The caller synchronises the block before reading the list.
 __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int rows_per_block,
-                                int rb, int ksplit) {
+                                int rb, int ksplit, bool blk_ready = false) {
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   // every load first (abort flag, ready mask, offsets, block addresses: one round trip), then the
@@ -73,7 +73,8 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
   for (int j = 0; j < 3; ++j) {
     const int s = lane + 32 * j;
     offv[j] = s <= a.nseg ? a.off[s] : 0;
-    blkv[j] = s < a.nseg ? reinterpret_cast<const char*>(seg_block(a, s)) : nullptr;
+    blkv[j] = s >= a.nseg ? nullptr
+              : blk_ready ? it.blk[s] : reinterpret_cast<const char*>(seg_block(a, s));
   }
   const int nseg = aborted == 0 ? a.nseg : 0;
 #pragma unroll
@@ -146,6 +147,19 @@ __device__ void build_dec_items(DecItems& it, const FfnArgs& a, int rows, int ro
     it.total = base;
     it.stream = stream;
     it.epoch = epoch;
+  }
+}
+
+// Threads t0 .. t0 + kMaxSeg - 1 of the block fill the segment block table of both work lists,
+// one entry each. The fused kernel does this before its grid-dependency wait: the table comes from
+// the kernel parameters and the cache's device table, written before the previous launch (the
+// permutation, which lets this launch start early) began.
+__device__ __forceinline__ void fill_blk(DecItems& x, DecItems& y, const FfnArgs& a, int t0) {
+  const int s = int(threadIdx.x) - t0;
+  if (s >= 0 && s < kMaxSeg) {
+    const char* b = s < a.nseg ? reinterpret_cast<const char*>(seg_block(a, s)) : nullptr;
+    x.blk[s] = b;
+    y.blk[s] = b;
   }
 }
 
@@ -535,13 +549,17 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   // fetching and streaming are compiled into the kernels of up to kStreamMaxT tokens (the host
   // only asks for them there)
   constexpr bool kStreams = FETCH && 8 * MAXNG <= kStreamMaxT;
-  pdl_wait();
   __shared__ DecItems it13, it2;
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
   __shared__ int s_next, s_ok, s_role;
   const int warp = threadIdx.x >> 5;
-  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1);
-  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit);
+  // before the grid-dependency wait (the permutation lets this launch start while it runs): the
+  // segment block table, whose sources were all written before the permutation began
+  fill_blk(it13, it2, a, 64);
+  __syncthreads();
+  pdl_wait();
+  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1, true);
+  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit, true);
   else if (threadIdx.x == 64) {
     // without fetchers the first claim goes out now, beside the work-list build
     if (kStreams) s_role = atomicAdd(a.done + a.nseg + 4, 1);

@@ -107,6 +107,9 @@ __device__ void fill_rows(const PermuteArgs& a, const int* offs, const int* len_
 // One CTA for the whole call (decode batches: a few microseconds).
 __global__ void __launch_bounds__(kThreads) permute_kernel(const __grid_constant__ PermuteArgs a) {
   pdl_wait();
+  // the next launch (the decode FFN) may start now: before its own wait it reads only what was
+  // written before this kernel started (its parameters, the cache's expert table)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   __shared__ int hist[kMaxSeg];
   __shared__ int run[kMaxE];
   __shared__ int offs[kMaxSeg + 1];
