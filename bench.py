@@ -778,6 +778,39 @@ def time_calls(fn, n, stream, flush=None):
     return sum(a.elapsed_time(b) for a, b in evs) / n
 
 
+def run_read_probe(dev, peaks, reps=5):
+    """One launch of the decode FFN's grid reading the decode FFN's weight bytes with no
+    computation (mcft_read_probe): as one contiguous stream and with the FFN's own load pattern,
+    the L2 flushed before each call, for the expert bytes of DeepSeek-shaped batch 1 (8 experts,
+    138.4 MB) and Mixtral-shaped batch 1 / 16 (2 / 8 experts). What a launch of that shape reads
+    at all, beside the FFN's roofline against the copy peak."""
+    from paper_2609_34077_gb300 import mcft as M
+
+    flush = torch.zeros(64 << 20, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    blocks = 2 * torch.cuda.get_device_properties(dev).multi_processor_count
+    sink = torch.zeros(1, dtype=torch.int32, device=dev)
+    out = {}
+    for name, sh, n_exp in (("dsv2_b1", I.DSV2_LITE, 8), ("mixtral_b1", I.MIXTRAL, 2),
+                            ("mixtral_b16", I.MIXTRAL, 8)):
+        nbytes = n_exp * sh.expert_bytes
+        buf = torch.empty(nbytes // 2, dtype=torch.bfloat16, device=dev)
+        res = dict(bytes=nbytes, row_bytes=sh.d * 2, blocks=blocks)
+        for pattern, key in ((0, "contiguous"), (1, "ffn_pattern")):
+            f = lambda: M.mcft_read_probe(buf, pattern, row_bytes=sh.d * 2, blocks=blocks, sink=sink,
+                                          stream=stream)
+            f()
+            ms = time_calls(f, reps, stream, flush=flush)
+            gbs = nbytes / (ms / 1e3) / 1e9
+            res[key] = dict(us=ms * 1e3, gbs=gbs, frac_of_copy_peak=gbs / peaks["hbm"])
+        M.mcft_device_error()
+        out[name] = res
+        del buf
+    del flush
+    torch.cuda.empty_cache()
+    return out
+
+
 _BATCHES = {}
 
 
@@ -1347,6 +1380,7 @@ def main():
         line["prefill"] = run_prefill(max(5, min(20, args.steps // 10)), 3, seed + 2, dev, peaks)
         line["stage2_lora"] = run_lora(8, 3, seed + 4, dev, peaks)
         line["stage1_mask"] = run_mask(20, 3, seed + 4, dev, peaks)
+        line["read_probe"] = run_read_probe(dev, peaks)
         _BATCHES.clear()
         torch.cuda.empty_cache()
     if rank == 0 and not args.no_cpu_baseline:

@@ -244,6 +244,21 @@ mcft_status mcft_fetch_experts(mcft_cache* cache, int layer, mcft_stream_t compu
 mcft_status mcft_host_copy(void* dst, const void* host_src, size_t bytes, int blocks,
                            mcft_stream_t stream);
 
+/* mcft_read_probe: read `bytes` of device memory in one launch of `blocks` CTAs of 256 threads,
+ * with no computation on the data, to measure what a launch of the decode FFN's shape reads at
+ * all (no counterpart in the paper; the decode FFN of Section 3.1's experts streams the selected
+ * experts' weights once). pattern 0: one contiguous stream, grid-strided, eight 16-byte loads in
+ * flight per thread. pattern 1: exactly the decode FFN's weight loads: items of 32 rows of
+ * row_bytes (16 W1 rows, then 16 W3 rows) strided over the grid; warp w of a CTA reads the
+ * 128-byte chunks w, w + 8, ... of every row of its item, eight 16-byte loads per lane per step.
+ * Every 32-bit word is read once; *sink is XORed with the XOR of all of them (so it equals the
+ * buffer's XOR if it started at 0).
+ *   buf  device memory, 16-byte aligned; bytes a multiple of 16 (pattern 0) or of 32 * row_bytes
+ *        (pattern 1, row_bytes a positive multiple of 128); sink device, one unsigned;
+ *   1 <= blocks <= 65535. MCFT_ERR_INVALID otherwise. Asynchronous on `stream`. */
+mcft_status mcft_read_probe(const void* buf, size_t bytes, int pattern, int row_bytes, int blocks,
+                            unsigned* sink, mcft_stream_t stream);
+
 /* ---------------------------------------------------------------------------------------------
  * Stage-1 mask machinery (Section 3.2 "Stage 1" Eq. stage1 and "Mask optimization" Eq. ste).
  *

@@ -718,6 +718,22 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
   return MCFT_OK;
 }
 
+mcft_status mcft_read_probe(const void* buf, size_t bytes, int pattern, int row_bytes, int blocks,
+                            unsigned* sink, mcft_stream_t stream) {
+  if (!buf || !sink) return fail(MCFT_ERR_INVALID, "NULL pointer");
+  if (reinterpret_cast<uintptr_t>(buf) % 16) return fail(MCFT_ERR_INVALID, "buf must be 16-byte aligned");
+  if (pattern != 0 && pattern != 1) return fail(MCFT_ERR_INVALID, "pattern %d is not 0 or 1", pattern);
+  if (blocks < 1 || blocks > 65535) return fail(MCFT_ERR_INVALID, "blocks = %d out of range", blocks);
+  if (pattern == 0 && bytes % 16) return fail(MCFT_ERR_INVALID, "bytes = %zu is not a multiple of 16", bytes);
+  if (pattern == 1 && (row_bytes <= 0 || row_bytes % 128 || bytes % (size_t(32) * row_bytes)))
+    return fail(MCFT_ERR_INVALID, "pattern 1 needs row_bytes a positive multiple of 128 and bytes "
+                "a multiple of 32 rows");
+  if (bytes == 0) return MCFT_OK;
+  const cudaError_t e = launch_read_probe(buf, bytes, pattern, row_bytes, blocks, sink, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "read probe launch");
+  return MCFT_OK;
+}
+
 mcft_status mcft_host_copy(void* dst, const void* host_src, size_t bytes, int blocks,
                            mcft_stream_t stream) {
   if (!dst || !host_src) return fail(MCFT_ERR_INVALID, "NULL pointer");

@@ -342,6 +342,9 @@ struct FetchArgs {
 cudaError_t launch_fetch(const FetchArgs& a, int blocks, cudaStream_t s, bool prefetch = false);
 // Plain copy from device-visible host memory with the fetch kernel's load loop (bytes % 16 == 0).
 cudaError_t launch_host_copy(void* dst, const void* src, size_t bytes, int blocks, cudaStream_t s);
+// mcft_read_probe's kernels (csrc/probe.cu): pattern 0 contiguous, 1 the decode FFN's loads.
+cudaError_t launch_read_probe(const void* buf, size_t bytes, int pattern, int row_bytes,
+                              int blocks, unsigned* sink, cudaStream_t s);
 
 // Fused decode prologue of one chained-stack layer at batch 1 (prologue.cu): residual update and
 // RMSNorm, routing of layer l, cache step of layer l, prediction and prefetch event of layer l+1,

@@ -57,6 +57,7 @@ SIGNATURES = {
     "mcft_test_inject": (_i, [_i, _i, C.c_ulonglong, _i]),
     "mcft_profile_enable": (_i, [_i]),
     "mcft_set_tc_tiles": (_i, [_i]),
+    "mcft_read_probe": (_i, [_vp, _sz, _i, _i, _i, _vp, _vp]),
     "mcft_profile_reset": (_i, []),
     "mcft_profile_read": (_i, [_i, _vp, _vp, _vp, C.POINTER(_i)]),
     "mcft_last_error": (C.c_char_p, []),
@@ -283,6 +284,20 @@ def mcft_host_copy(dst, host_src, blocks, stream=None):
     assert dst.numel() * dst.element_size() == nbytes, "dst and host_src differ in size"
     _check(lib().mcft_host_copy(_ptr(dst), _ptr(host_src), nbytes, int(blocks), _stream(stream)))
     return dst
+
+
+def mcft_read_probe(buf, pattern, row_bytes=4096, blocks=None, sink=None, stream=None):
+    """Read the device tensor buf in one launch (pattern 0: contiguous; 1: the decode FFN's weight
+    loads over rows of row_bytes) with no computation; returns sink (an int32 device tensor of one
+    element, XORed with the XOR of every 32-bit word read)."""
+    nbytes = buf.numel() * buf.element_size()
+    if blocks is None:
+        blocks = 2 * torch.cuda.get_device_properties(buf.device).multi_processor_count
+    if sink is None:
+        sink = torch.zeros(1, dtype=torch.int32, device=buf.device)
+    _check(lib().mcft_read_probe(_ptr(buf), nbytes, int(pattern), int(row_bytes), int(blocks),
+                                 _ptr(sink), _stream(stream)))
+    return sink
 
 
 def mcft_moe_forward_cached(desc: LayerDesc, x, idx, gate, cache: Cache, layer, shared=(), y=None,

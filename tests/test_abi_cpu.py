@@ -128,3 +128,20 @@ def test_tc_tile_mode_without_gpu(libpath):
     assert pair[1024] == one[1024]  # 2048 assignments over 8 experts: 256 rows each
     assert pair[2048] > one[2048] and pair[4096] > one[4096]
     assert size(4096) == one[4096]
+
+
+def test_read_probe_validation_without_gpu(libpath):
+    import ctypes as C
+    from paper_2609_34077_gb300 import mcft
+
+    L = mcft.lib()
+    buf, sink = C.c_void_p(4096), C.c_void_p(64)
+    assert L.mcft_read_probe(None, 16, 0, 0, 1, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 16, 0, 0, 1, None, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(C.c_void_p(4100), 16, 0, 0, 1, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 16, 2, 0, 1, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 24, 0, 0, 1, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 32 * 4096, 1, 100, 1, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 32 * 4096 + 16, 1, 4096, 1, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 16, 0, 0, 0, sink, None) == mcft.MCFT_ERR_INVALID
+    assert L.mcft_read_probe(buf, 0, 0, 0, 1, sink, None) == mcft.MCFT_OK  # nothing to read
