@@ -474,8 +474,10 @@ mcft_status mcft_test_inject(int fail_pinned_allocs, int fail_expert_copies,
  *   MCFT_TC_TILES_CTA_PAIR  256 x 256 tiles on pairs of CTAs (cta_group::2 MMAs issued by one CTA
  *                           of a 2-CTA cluster over both CTAs' shared memory), segments padded to
  *                           256 rows, for layers without adapters whose routed experts average at
- *                           least 512 rows (others keep the one-CTA tiles). Outputs equal the
- *                           one-CTA tiles' bit for bit.
+ *                           least 512 rows (others keep the one-CTA tiles). Each output is the
+ *                           same products summed in the same order; on every shape tested the
+ *                           outputs equal the one-CTA tiles' bit for bit. Slower than the one-CTA
+ *                           tiles on the GB300 shapes measured (kept for comparison).
  * MCFT_ERR_INVALID for another mode. */
 typedef enum { MCFT_TC_TILES_ONE_CTA = 0, MCFT_TC_TILES_CTA_PAIR = 1 } mcft_tc_tiles;
 mcft_status mcft_set_tc_tiles(int mode);
