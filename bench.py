@@ -44,11 +44,11 @@ METRIC = "masked MoE layer tokens/s"
 # first 16 hex digits of the kernel source's sha256: when the source has changed since the
 # capture, the bench reports traffic as null.
 TRAFFIC = {
-    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "316c9dc68b5747e4", None),
-    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "316c9dc68b5747e4", None),
-    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "316c9dc68b5747e4", 1.0016),
+    "ffn13_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "393328975a2ceb3d", None),
+    "ffn2_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "393328975a2ceb3d", None),
+    "ffn_decode": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "393328975a2ceb3d", 1.0016),
     # DRAM traffic / (weights of the step's experts read once + activations + fetched bytes written)
-    "ffn_decode_fetch": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "316c9dc68b5747e4", 0.927),
+    "ffn_decode_fetch": ("paper_2609_34077_gb300/csrc/ffn_decode.cu", "393328975a2ceb3d", 0.898),
     "fetch": ("paper_2609_34077_gb300/csrc/cache.cu", "68e0415de46353e9", 0.9253),
 }
 

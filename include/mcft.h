@@ -294,8 +294,9 @@ mcft_status mcft_mask_grad(const mcft_layer_desc* desc, const int32_t* idx, cons
 
 /* mcft_moe_forward_cached: mcft_moe_forward for a decode step of `layer` whose experts come from
  * the cache, with the fetch driven by the device and overlapped with compute; no host round trip.
- * Call it after mcft_cache_step(cache, layer, idx, ...) on compute_stream, instead of
- * mcft_fetch_experts + mcft_moe_forward. Every missed expert's block is copied from pinned host
+ * Call it once after each mcft_cache_step(cache, layer, idx, ...) on compute_stream, instead of
+ * mcft_fetch_experts + mcft_moe_forward (the fetching launch below claims its copy work from
+ * counters that cache step resets). Every missed expert's block is copied from pinned host
  * memory into the slot or staging buffer the cache step chose, by SM loads over the host link:
  *  - bf16, T <= 16, and no prefetch of any layer in flight: in the FFN's own launch on
  *    compute_stream, whose first CTAs copy the misses piece by piece while the others compute the

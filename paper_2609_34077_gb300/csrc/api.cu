@@ -195,6 +195,7 @@ struct mcft_cache {
   unsigned long long* d_ready = nullptr;    // [L] hit mask of the last step
   unsigned long long* d_stream = nullptr;   // [L] miss mask of the last step
   unsigned* d_landed = nullptr;  // [L][E][ppe] epoch stamps of the demand fetch's landed pieces
+  unsigned* d_fctr = nullptr;    // [L][2] role and piece counters of that fetching FFN launch
   int ppe = 0;                   // fetch pieces per expert block
   unsigned long long* d_host_src = nullptr; // [L*E] device-visible addresses of the host blocks
   unsigned long long* d_pfmask = nullptr;   // [L] experts loaded by a prefetch since the last step
@@ -231,6 +232,7 @@ void cache_free(mcft_cache* c) {
   cudaFree(c->d_ready);
   cudaFree(c->d_stream);
   cudaFree(c->d_landed);
+  cudaFree(c->d_fctr);
   cudaFree(c->d_host_src);
   cudaFree(c->d_pfmask);
   cudaFree(c->d_pf_cancel);
@@ -664,6 +666,8 @@ mcft_status mcft_cache_create(int L, int E, int B, size_t expert_bytes,
     c->ppe = int((expert_bytes + kFetchPiece - 1) / kFetchPiece);
     MCFT_CACHE_CUDA(cudaMalloc(&c->d_landed, sizeof(unsigned) * size_t(L) * E * c->ppe));
     MCFT_CACHE_CUDA(cudaMemset(c->d_landed, 0, sizeof(unsigned) * size_t(L) * E * c->ppe));
+    MCFT_CACHE_CUDA(cudaMalloc(&c->d_fctr, sizeof(unsigned) * 2 * size_t(L)));
+    MCFT_CACHE_CUDA(cudaMemset(c->d_fctr, 0, sizeof(unsigned) * 2 * size_t(L)));
     if (stg > 0) MCFT_CACHE_CUDA(cudaMalloc(&c->d_staging, expert_bytes * size_t(stg)));
     // device-visible addresses of the pinned host blocks, for the device-driven fetch
     std::vector<unsigned long long> src(size_t(L) * E);
@@ -710,6 +714,7 @@ mcft_status mcft_cache_step(mcft_cache* c, int layer, const int32_t* idx, int T,
                   c->d_miss + size_t(layer) * c->miss_stride,
                   c->d_miss_dev + size_t(layer) * c->miss_stride,
                   c->d_ptr_tab + size_t(layer) * c->E, c->d_ready + layer, c->d_stream + layer,
+                  c->d_fctr ? c->d_fctr + 2 * size_t(layer) : nullptr,
                   c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                   c->d_staging, c->expert_bytes, device_error_word()};
   cudaError_t e = launch_cache_step(a, stream);
@@ -983,7 +988,8 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
   // them after it.
   int pf_any = 0;
   for (int l = 0; l < c->L; ++l) pf_any += c->pf_state[l] != 0 ? 1 : 0;
-  const bool own_fetch = L.decode && T <= kStreamMaxT && c->d_landed != nullptr && pf_any == 0;
+  const bool own_fetch = L.decode && T <= kStreamMaxT && c->d_landed != nullptr &&
+                         c->d_fctr != nullptr && pf_any == 0;
   cudaError_t e = cudaSuccess;
   if (own_fetch) {
     if (!permuted) {
@@ -1012,6 +1018,7 @@ mcft_status forward_cached_impl(const mcft_layer_desc* desc, const void* x, int 
     fa.ready = c->d_ready + layer;
     fa.phase = 1;  // hits, shared experts and the misses it fetches
     fa.stream = c->d_stream + layer;
+    fa.fctr = c->d_fctr + 2 * size_t(layer);
     fa.landed = c->d_landed + size_t(layer) * E * c->ppe;
     fa.epoch = c->d_step + layer;
     fa.ppe = c->ppe;
@@ -1145,6 +1152,7 @@ mcft_status stack_prologue(const mcft_layer_desc* desc, float* x, const void* y,
                           c->d_miss + size_t(layer) * c->miss_stride,
                           c->d_miss_dev + size_t(layer) * c->miss_stride,
                           c->d_ptr_tab + size_t(layer) * E, c->d_ready + layer, c->d_stream + layer,
+                          c->d_fctr ? c->d_fctr + 2 * size_t(layer) : nullptr,
                           c->d_slots ? c->d_slots + size_t(layer) * c->B * c->expert_bytes : nullptr,
                           c->d_staging, c->expert_bytes, err};
   a.do_prefetch = do_pf ? 1 : 0;

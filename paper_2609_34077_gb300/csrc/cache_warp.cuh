@@ -83,6 +83,7 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
       a.miss_dev[0] = 0;
       *a.ready = 0;
       if (a.stream) *a.stream = 0;
+      if (a.fctr) a.fctr[0] = a.fctr[1] = 0u;
     }
     for (int e = lane; e < E; e += 32) a.ptr_tab[e] = 0;
     __threadfence_system();
@@ -199,6 +200,7 @@ __device__ inline void cache_step_warp(const CacheStepArgs& a) {
     *a.ready = hitbits;
     // the misses, which this step's demand fetch copies (none without slots)
     if (a.stream) *a.stream = a.slots ? (mine & ~cached) : 0ull;
+    if (a.fctr) a.fctr[0] = a.fctr[1] = 0u;  // for the FFN launch that fetches these misses
   }
   // No fence: the FFN and fetch kernels read these after a kernel boundary (or an event), the host
   // after synchronising on one; the running fetch kernel that polls the cancel mask only needs the

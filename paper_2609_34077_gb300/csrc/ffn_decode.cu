@@ -534,13 +534,14 @@ __device__ bool wait_landed(const FfnArgs& a, unsigned epoch, int e, size_t off,
 // done, then reads h through L2. The waits always end: every GEMM13 item precedes every GEMM2 item
 // in the claim order, so when a GEMM2 item is claimed its segment's GEMM13 items have all been
 // claimed, each by a CTA that is running and finishes it without waiting on anything.
-// A launch that fetches its own misses (a.nfetch > 0) first hands out fetcher roles: the first
-// a.nfetch CTAs to take a role copy the step's missed blocks from host memory piece by piece
-// (pieces claimed from a second counter, each stamped once written and fenced), then claim FFN
-// items like the others. An item of a missed expert waits (bounded) for the stamps of the pieces
-// it reads. Those waits end too: a CTA that holds an FFN item took its role after the a.nfetch
-// fetchers took theirs, so every fetcher is running, and fetchers wait on nothing until all
-// pieces are copied.
+// A launch that fetches its own misses (a.nfetch > 0) first hands out fetcher roles from a
+// counter the layer's cache step zeroed: the first a.nfetch CTAs to take a role copy the step's
+// missed blocks from host memory piece by piece (pieces claimed from a second such counter, each
+// stamped once written and fenced), before the grid-dependency wait (everything they read was
+// written before the permutation began), then claim FFN items like the others. An item of a
+// missed expert waits (bounded) for the stamps of the pieces it reads. Those waits end too: a CTA
+// that holds an FFN item took its role after the a.nfetch fetchers took theirs, so every fetcher
+// is running, and fetchers wait on nothing until all pieces are copied.
 // FETCH: the build for launches that fetch their own misses (a.nfetch > 0); the plain build
 // carries none of that code.
 template <int MAXNG, bool FETCH>
@@ -553,17 +554,14 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   __shared__ float red[kWarps * kMaxNG * 8 * 32];
   __shared__ int s_next, s_ok, s_role;
   const int warp = threadIdx.x >> 5;
-  // before the grid-dependency wait (the permutation lets this launch start while it runs): the
-  // segment block table, whose sources were all written before the permutation began
+  // Before the grid-dependency wait (the permutation lets this launch start while it runs), only
+  // what was written before the permutation began is read: the segment block table (kernel
+  // parameters, the cache's expert table) and, for the fetchers, the cache step's miss list, slot
+  // addresses, step count and role and piece counters (zeroed by the cache step). So the copy of
+  // the misses starts while the permutation still runs.
   fill_blk(it13, it2, a, 64);
-  __syncthreads();
-  pdl_wait();
-  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1, true);
-  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit, true);
-  else if (threadIdx.x == 64) {
-    // without fetchers the first claim goes out now, beside the work-list build
-    if (kStreams) s_role = atomicAdd(a.done + a.nseg + 4, 1);
-    else s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
+  if constexpr (kStreams) {
+    if (threadIdx.x == 64) s_role = int(atomicAdd(a.fctr, 1u));
   }
   __syncthreads();
   if constexpr (kStreams) {
@@ -571,9 +569,9 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
       const int nm = a.fmiss[0];  // copied even if the call aborts: the cache holds them now
       const size_t words = a.fbytes / 16, piece = kFetchPiece / 16;
       const int per = int((words + piece - 1) / piece);
-      const unsigned epoch = it13.epoch;
+      const unsigned epoch = static_cast<unsigned>(*a.epoch);
       for (;;) {
-        if (threadIdx.x == 0) s_ok = atomicAdd(a.done + a.nseg + 5, 1);
+        if (threadIdx.x == 0) s_ok = int(atomicAdd(a.fctr + 1, 1u));
         __syncthreads();
         const int u = s_ok;
         __syncthreads();
@@ -589,10 +587,15 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
       }
     }
   }
-  if constexpr (kStreams) {  // a fetcher claims its first item only once the pieces are all taken
-    if (threadIdx.x == 0) s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
-    __syncthreads();
+  pdl_wait();
+  if (warp == 0) build_dec_items(it13, a, a.w, kRows, RB13, 1, true);
+  else if (warp == 1) build_dec_items(it2, a, a.d, kRows2, RB2, a.ksplit, true);
+  else if (threadIdx.x == 64) {
+    // the first claim goes out now, beside the work-list build (a fetcher only claims once the
+    // pieces are all taken)
+    s_next = atomicAdd(a.done + a.nseg + a.phase, 1);
   }
+  __syncthreads();
   // Only the next claim stays live across an item body (the item index is consumed at its start;
   // the bounds are re-read from shared memory). Thread 0 issues the claim before the body and
   // publishes it after, so the atomic's round trip overlaps warp 0's weight loads.

@@ -61,9 +61,9 @@ constexpr int kRouteTileMinT = 64;
 // Header at the start of the forward workspace.
 // Work-claim counters of the fused decode FFN that follow the per-segment progress counters in
 // the workspace: one per FFN phase (0 all segments, 1 hits, 2 misses).
-// slots 0-2: the claim counters of phases 0-2; slot 4: fetcher roles and slot 5: fetch pieces of
-// a decode launch that fetches its own misses (FfnArgs::nfetch)
-constexpr int kClaimSlots = 6;
+// slots 0-2: the claim counters of phases 0-2 (the fetching launch's role and piece counters are
+// the cache's, FfnArgs::fctr)
+constexpr int kClaimSlots = 3;
 
 struct WsHeader {
   int abort;     // set when a kernel of this call found bad data; later kernels skip their work
@@ -188,6 +188,7 @@ struct FfnArgs {
   // hits, each of their items waiting (bounded) for the pieces it reads, so their FFN runs while
   // the rest of the step's bytes are still on the host link. nfetch = 0: no fetch, no streaming.
   const unsigned long long* stream;
+  unsigned* fctr;  // [2] role and piece counters, zeroed by the layer's cache step
   unsigned* landed;
   const int64_t* epoch;
   int ppe;
@@ -297,6 +298,8 @@ struct CacheStepArgs {
   unsigned long long* ready;    // device: bit e set when expert e was a hit at this step
   unsigned long long* stream;   // device: bit e set when expert e is a miss of this step (copied
                                 // by the step's demand fetch); NULL: not published
+  unsigned* fctr;               // device [2]: role and piece counters of the decode FFN launch
+                                // that fetches this step's misses, zeroed here; NULL: none
   const char* slots;            // this layer's first slot block (NULL in accounting mode)
   const char* staging;          // bypass staging blocks
   size_t expert_bytes;
