@@ -108,9 +108,9 @@ def test_ffn_deepseek_decode_full_size(batch):
     check_output(y, _reference(sh, x, idx, gate, lw), TOL_BF16, f"deepseek decode b={batch}")
 
 
-def test_ffn_mixtral_prefill_full_size_sampled():
-    """T = 4096 tokens, hard mask keeping 4 of 8 experts (unbalanced loads): every output row is
-    finite, and 64 sampled rows match the oracle."""
+def test_ffn_mixtral_prefill_full_size():
+    """T = 4096 tokens, hard mask keeping 4 of 8 experts, seeded ids folded onto the kept set
+    (unbalanced loads): every output row matches the oracle."""
     sh = I.MIXTRAL
     lw = weights(sh)
     T = 4096
@@ -124,9 +124,7 @@ def test_ffn_mixtral_prefill_full_size_sampled():
             idx[t, 1] = int(kept[(list(kept).index(int(idx[t, 0])) + 1) % len(kept)])
     y = _forward(sh, x, idx, gate, lw)
     assert torch.isfinite(y.float()).all()
-    rows = np.random.default_rng(11).choice(T, 64, replace=False)
-    ref = _reference(sh, x, idx, gate, lw, rows=rows)
-    check_output(y[torch.from_numpy(rows).to(DEV)], ref, TOL_BF16, "mixtral prefill sampled")
+    check_output(y, _reference(sh, x, idx, gate, lw), TOL_BF16, "mixtral prefill, every row")
 
 
 def test_ffn_empty_and_bad_ids():
